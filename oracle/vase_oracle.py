@@ -1,0 +1,253 @@
+"""Plain fp64 CPU oracle of one VaSE eviction step (arXiv 2606.03928).
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+CPU-baseline / reference legs of ``bench.py`` may import this module.  The
+product path (the CUDA library and its Python binding) never calls it and
+shares no code with it.
+
+Every step follows the paper's definitions in the paper's order, one unit at a
+time, where a *unit* is one (layer, sequence, KV head):
+
+* attention weights of a window query over all N = K + B cached keys -- Eq. (1), Sec. 2;
+* the SnapKV score, the mean of those weights over the window queries, with
+  average pooling and non-causal cached queries -- Eq. (2) and its footnote, Sec. 2;
+* the value magnitude Range(v) -- Eq. (5), Sec. 3.1 -- and the L2 / Var variants -- App. A;
+* VaSE-AttnV: reserve the buffer R_B and the N_v largest-Range candidates R_V,
+  then fill the K - |R| remaining slots by weighted sampling without
+  replacement with weights proportional to the pooled score -- Sec. 3.2;
+* the deterministic "+V without sampling" ablation -- Sec. 4.1;
+* VaSE-DKV: the CurDKV product of key and value leverage scores under a
+  Gaussian projection G_t ~ N(0, 1/r) that is redrawn every eviction round,
+  then the top K - B candidates -- Eq. (4), Sec. 2 and Sec. 3.2;
+* the periodic-eviction framing (protect the B most recent tokens, keep
+  exactly K of the K + B cached tokens) -- Sec. 2, "Periodic eviction".
+
+Readings where the paper is silent (each is listed with its reason in the
+design notes of the repository):
+
+* GQA: the window rows of a KV head are the W cached queries of each of its
+  G query heads; the score is the mean over all G*W rows.
+* Window: W is its own parameter (the paper sets W = B); the divisor is G*W.
+* Pooling: odd kernel kappa, stride 1, zero padding, divisor kappa, along the
+  slot axis over all N slots, before restricting to candidates.
+* Weighted sampling without replacement is successive sampling (draw one
+  token with probability proportional to the remaining weights, remove it,
+  repeat).  It is realised as the exponential race: keep the m largest
+  alpha_i / E_i with E_i = -ln u_i (Efraimidis and Spirakis, 2006), which has
+  the same joint law.  The tests pin that equivalence by exact enumeration.
+* Ties in any ranking go to the lower slot (the older token).
+* Noise: u_i comes from Philox4x32-10 (Salmon et al., SC'11) with key
+  (seed_lo, seed_hi) and counter (position, round, layer | tag << 24,
+  seq * Hkv + head); tag 0 = selection noise, tag 1 = DKV Gaussian.
+  u = (2 * (x >> 9) + 1) * 2**-24 from word 0, exact in fp32 and fp64.
+  Gaussian entries use Box-Muller (1958) on words 0 and 1 with counter
+  word 0 = a * r + b; the fixed-G (CurDKV) option puts 0 in the round word.
+* DKV has no value reservation; the value awareness is the value leverage.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+
+# ----------------------------------------------------------------------------
+# Philox4x32-10 (Salmon, Moraes, Dror, Shaw: "Parallel random numbers: as easy
+# as 1, 2, 3", SC'11): two 32x32->64 multiplies per round, the Weyl key
+# schedule, ten rounds.
+# ----------------------------------------------------------------------------
+
+_MASK32 = np.uint64(0xFFFFFFFF)
+_PHILOX_M0 = np.uint64(0xD2511F53)
+_PHILOX_M1 = np.uint64(0xCD9E8D57)
+_PHILOX_W0 = np.uint64(0x9E3779B9)
+_PHILOX_W1 = np.uint64(0xBB67AE85)
+
+TAG_SELECT = 0
+TAG_DKV = 1
+
+
+def philox4x32_10(c0, c1, c2, c3, k0, k1):
+    """Philox4x32 with 10 rounds on arrays of 32-bit counters; returns 4 uint32 arrays."""
+    c0, c1, c2, c3 = (np.asarray(c, dtype=np.uint64) & _MASK32 for c in (c0, c1, c2, c3))
+    c0, c1, c2, c3 = np.broadcast_arrays(c0, c1, c2, c3)
+    k0 = np.uint64(int(k0) & 0xFFFFFFFF)
+    k1 = np.uint64(int(k1) & 0xFFFFFFFF)
+    for _ in range(10):
+        p0 = _PHILOX_M0 * c0
+        p1 = _PHILOX_M1 * c2
+        hi0, lo0 = p0 >> np.uint64(32), p0 & _MASK32
+        hi1, lo1 = p1 >> np.uint64(32), p1 & _MASK32
+        c0, c1, c2, c3 = hi1 ^ c1 ^ k0, lo1, hi0 ^ c3 ^ k1, lo0
+        k0 = (k0 + _PHILOX_W0) & _MASK32
+        k1 = (k1 + _PHILOX_W1) & _MASK32
+    return tuple(x.astype(np.uint32) for x in (c0, c1, c2, c3))
+
+
+def uniform_open01(word):
+    """Map a 32-bit word to u = (2 * (x >> 9) + 1) * 2**-24, strictly inside (0, 1)."""
+    x = np.asarray(word, dtype=np.uint64) >> np.uint64(9)
+    return (2.0 * x.astype(np.float64) + 1.0) * 2.0 ** -24
+
+
+def _noise_key(seed):
+    seed = int(seed) & 0xFFFFFFFFFFFFFFFF
+    return seed & 0xFFFFFFFF, seed >> 32
+
+
+def selection_uniforms(seed, layer, seq, head, num_kv_heads, rnd, positions):
+    """u_i for the sampling race of one unit, keyed by each token's stream position."""
+    k0, k1 = _noise_key(seed)
+    pos = np.asarray(positions, dtype=np.int64).astype(np.uint64)
+    w0, _, _, _ = philox4x32_10(pos, rnd, (layer | (TAG_SELECT << 24)), seq * num_kv_heads + head, k0, k1)
+    return uniform_open01(w0)
+
+
+def gaussian_projection(seed, layer, seq, head, num_kv_heads, rnd, d, r, fixed_g=False):
+    """G in R^{d x r} with i.i.d. N(0, 1/r) entries -- Eq. (4), Sec. 2; redrawn per round -- Sec. 3.2.
+
+    Entry (a, b) takes Philox counter (a * r + b, round, layer | 1 << 24, seq * Hkv + head)
+    and Box-Muller on words 0 and 1: z = sqrt(-2 ln u1) cos(2 pi u2).
+    """
+    k0, k1 = _noise_key(seed)
+    idx = np.arange(d * r, dtype=np.uint64)
+    rr = 0 if fixed_g else rnd
+    w0, w1, _, _ = philox4x32_10(idx, rr, (layer | (TAG_DKV << 24)), seq * num_kv_heads + head, k0, k1)
+    u1 = uniform_open01(w0)
+    u2 = uniform_open01(w1)
+    z = np.sqrt(-2.0 * np.log(u1)) * np.cos(2.0 * np.pi * u2)
+    return (z / np.sqrt(r)).reshape(d, r)
+
+
+# ----------------------------------------------------------------------------
+# bf16 widening (exact) -- inputs arrive as raw bf16 bit patterns.
+# ----------------------------------------------------------------------------
+
+def bf16_bits_to_f64(bits):
+    b = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return b.view(np.float32).astype(np.float64)
+
+
+# ----------------------------------------------------------------------------
+# Scores
+# ----------------------------------------------------------------------------
+
+def attention_weights(q_rows, keys):
+    """alpha[r, i] of Eq. (1): softmax over all N cached keys of q_r . k_i / sqrt(d)."""
+    d = keys.shape[1]
+    logits = (q_rows @ keys.T) / np.sqrt(d)
+    logits = logits - logits.max(axis=1, keepdims=True)
+    e = np.exp(logits)
+    return e / e.sum(axis=1, keepdims=True)
+
+
+def window_attention_score(q_rows, keys):
+    """Mean of alpha over the G*W window rows (Eq. (2), non-causal cached queries), before pooling."""
+    return attention_weights(q_rows, keys).mean(axis=0)
+
+
+def average_pool(scores, kernel):
+    """Stride-1 average pooling along the slot axis, zero padded, divisor = kernel."""
+    kernel = int(kernel)
+    if kernel <= 1:
+        return np.asarray(scores, dtype=np.float64).copy()
+    return np.convolve(scores, np.ones(kernel) / kernel, mode="same")
+
+
+VALUE_RANGE, VALUE_L2, VALUE_VAR = 0, 1, 2
+
+
+def value_magnitude(values, kind=VALUE_RANGE):
+    """Range(v) = max_j v_j - min_j v_j (Eq. (5)); L2 and Var variants of App. A."""
+    if kind == VALUE_RANGE:
+        return values.max(axis=1) - values.min(axis=1)
+    if kind == VALUE_L2:
+        return np.sqrt((values * values).sum(axis=1))
+    if kind == VALUE_VAR:
+        mu = values.mean(axis=1, keepdims=True)
+        return ((values - mu) ** 2).mean(axis=1)
+    raise ValueError(f"unknown value score kind {kind}")
+
+
+def leverage_scores(keys, values, G):
+    """CurDKV product score s_i = ||G^T k_i||^2 * ||G^T v_i||^2 (Eq. (4))."""
+    lk = ((keys @ G) ** 2).sum(axis=1)
+    lv = ((values @ G) ** 2).sum(axis=1)
+    return lk * lv, lk, lv
+
+
+# ----------------------------------------------------------------------------
+# Selection
+# ----------------------------------------------------------------------------
+
+def top_k_slots(scores, k, eligible=None):
+    """Indices of the k largest scores among eligible slots; ties go to the lower slot."""
+    scores = np.asarray(scores, dtype=np.float64)
+    idx = np.arange(scores.shape[0])
+    if eligible is not None:
+        idx = idx[np.asarray(eligible, dtype=bool)]
+    order = np.lexsort((idx, -scores[idx]))
+    return np.sort(idx[order[:k]])
+
+
+def evict_unit(q_rows, keys, values, positions, *, budget_k, buffer_b, variant="attnv",
+               n_v=None, value_score=VALUE_RANGE, pool_kernel=7, stochastic=True,
+               dkv_rank=20, dkv_fixed_g=False, seed=0, layer=0, seq=0, head=0,
+               num_kv_heads=1, rnd=0):
+    """One eviction step for one unit, in fp64.
+
+    q_rows [G*W, d], keys/values [K+B, d] (fp64, exact bf16 values), positions [K+B].
+    Returns a dict with the scores, the keep mask, the ascending kept-slot list
+    and the compacted keys, values and positions.
+    """
+    K, B = int(budget_k), int(buffer_b)
+    N = K + B
+    assert keys.shape[0] == N and values.shape[0] == N and len(positions) == N
+    out = {}
+    keep = np.zeros(N, dtype=bool)
+    keep[K:] = True                       # R_B: the B most recent tokens are protected (Sec. 2)
+    if variant == "attnv":
+        nv = K // 4 if n_v is None or n_v < 0 else int(n_v)
+        m = K - nv - B                    # the K - |R| sampled slots (Sec. 3.2)
+        assert m >= 0
+        a = window_attention_score(q_rows, keys)
+        abar = average_pool(a, pool_kernel)
+        vmag = value_magnitude(values[:K], value_score)
+        r_v = top_k_slots(vmag, nv)       # R_V: N_v largest Range among the K candidates
+        in_c = np.ones(K, dtype=bool)
+        in_c[r_v] = False                 # C = [K] \ R_V
+        if stochastic:
+            u = selection_uniforms(seed, layer, seq, head, num_kv_heads, rnd, positions[:K])
+            key = abar[:K] / (-np.log(u))
+        else:
+            key = abar[:K].copy()
+        sel = top_k_slots(key, m, eligible=in_c)
+        keep[r_v] = True
+        keep[sel] = True
+        key_full = np.full(N, -1.0)
+        key_full[:K] = np.where(in_c, key, -1.0)
+        out.update(attn=a, pooled=abar, value_score=vmag, key=key_full, reserved_v=r_v)
+    elif variant == "dkv":
+        d = keys.shape[1]
+        G = gaussian_projection(seed, layer, seq, head, num_kv_heads, rnd, d, dkv_rank, dkv_fixed_g)
+        s, lk, lv = leverage_scores(keys[:K], values[:K], G)
+        sel = top_k_slots(s, K - B)
+        keep[sel] = True
+        key_full = np.full(N, -1.0)
+        key_full[:K] = s
+        out.update(value_score=s, lk=lk, lv=lv, key=key_full, G=G)
+    else:
+        raise ValueError(variant)
+    src = np.flatnonzero(keep)
+    assert src.shape[0] == K, "exactly K tokens are kept"
+    out.update(keep=keep, src=src, keys_new=keys[src], values_new=values[src],
+               positions_new=np.asarray(positions)[src])
+    return out
+
+
+def evict_unit_bits(q_bits, k_bits, v_bits, positions, **kw):
+    """evict_unit on raw bf16 bit arrays; compacted rows are returned as the same bits."""
+    res = evict_unit(bf16_bits_to_f64(q_bits), bf16_bits_to_f64(k_bits), bf16_bits_to_f64(v_bits),
+                     positions, **kw)
+    src = res["src"]
+    res["k_bits_new"] = np.asarray(k_bits)[src]
+    res["v_bits_new"] = np.asarray(v_bits)[src]
+    return res

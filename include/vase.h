@@ -1,0 +1,209 @@
+/*
+ * vase.h -- C ABI of the VaSE eviction step on one GPU (sm_103a).
+ *
+ * VaSE (Value-aware Stochastic KV cache Eviction, arXiv 2606.03928) runs a
+ * periodic eviction step on each layer's KV cache (Sec. 2, "Periodic eviction
+ * with budget K and buffer B"): every decode step appends one (k, v) pair per
+ * KV head; once the cache holds N = K + B pairs the eviction step keeps the B
+ * most recent pairs, scores the other K candidates, drops B of them and
+ * compacts the cache back to K slots.  The scores and the rule are those of
+ * Sec. 3.2: VaSE-AttnV (window attention score, Eq. (2), with N_v slots
+ * reserved for the largest value magnitudes, Eq. (5), and weighted sampling
+ * without replacement for the rest) and VaSE-DKV (CurDKV leverage scores,
+ * Eq. (4), under a Gaussian projection redrawn every round).
+ *
+ * Conventions shared by every entry point:
+ *   - Every pointer named "device" is a CUDA device pointer owned by the
+ *     caller; the library never allocates or frees device memory and never
+ *     synchronises a stream except in vase_check_device_error.
+ *   - "stream" is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     All work is enqueued on it in call order; every call on one context
+ *     must be ordered on one stream (the workspace is shared by all layers).
+ *   - bf16 tensors are row-major with head_dim = 128 contiguous elements
+ *     (256 bytes) per row; every device base pointer must be 256-byte aligned.
+ *   - Return values: VASE_OK (0), VASE_EVICT_DUE (> 0, informational) or a
+ *     negative VASE_ERR_* code.  On error nothing is enqueued and the
+ *     context's counters are unchanged; vase_last_error() explains.
+ *   - A context is not thread-safe.
+ */
+#ifndef VASE_H
+#define VASE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define VASE_ABI_VERSION 1
+
+#define VASE_OK 0
+#define VASE_EVICT_DUE 1          /* the layer's cache is full: call vase_evict before the next append */
+#define VASE_ERR_INVALID (-1)     /* bad argument or configuration */
+#define VASE_ERR_FULL (-2)        /* append would exceed K + B slots */
+#define VASE_ERR_NOT_FULL (-3)    /* evict called before the cache holds K + B pairs */
+#define VASE_ERR_CUDA (-4)        /* a CUDA runtime call failed (message in vase_last_error) */
+#define VASE_ERR_UNSUPPORTED (-5) /* valid but outside what the kernels implement (e.g. head_dim != 128) */
+#define VASE_ERR_ALIGN (-6)       /* a device pointer is not 256-byte aligned */
+#define VASE_ERR_DEVICE (-7)      /* a device-side check or bounded wait failed (vase_check_device_error) */
+
+#define VASE_VARIANT_ATTNV 0      /* Sec. 3.2, VaSE-AttnV */
+#define VASE_VARIANT_DKV 1        /* Sec. 3.2, VaSE-DKV */
+
+#define VASE_VALUE_RANGE 0        /* Eq. (5): max_j v_j - min_j v_j */
+#define VASE_VALUE_L2 1           /* App. A: ||v||_2 */
+#define VASE_VALUE_VAR 2          /* App. A: (1/d) sum_j (v_j - mean)^2 */
+
+typedef struct vase_config {
+    int32_t budget_k;      /* K: persistent budget (Sec. 2) */
+    int32_t buffer_b;      /* B: recency buffer, always kept (Sec. 2) */
+    int32_t window;        /* W: cached decode queries per query head (Eq. (2) footnote; the paper uses W = B) */
+    int32_t num_q_heads;   /* Hq */
+    int32_t num_kv_heads;  /* Hkv; Hq % Hkv == 0, query head j reads KV head j / (Hq / Hkv) */
+    int32_t head_dim;      /* d; must be 128 */
+    int32_t num_layers;    /* L */
+    int32_t batch;         /* b: sequences */
+    int32_t variant;       /* VASE_VARIANT_* */
+    int32_t n_v;           /* N_v value-reserved slots (AttnV); -1 = K/4 (App. B) */
+    int32_t value_score;   /* VASE_VALUE_*: the value magnitude used for R_V (AttnV) */
+    int32_t pool_kernel;   /* odd average-pooling width over the slot axis (Eq. (2) footnote); 1 = off */
+    int32_t dkv_rank;      /* r of G in R^{d x r} (Eq. (4)); 1..32, 20 in App. B */
+    int32_t stochastic;    /* AttnV: 1 = weighted sampling without replacement (Sec. 3.2), 0 = top-k (Sec. 4.1) */
+    int32_t dkv_fixed_g;   /* DKV: 1 = one G for the whole stream (CurDKV), 0 = G_t redrawn per round (VaSE-DKV) */
+    int32_t debug_outputs; /* 1 = also write pooled scores, selection keys and the keep mask to the workspace */
+    uint64_t seed;         /* key of the Philox4x32-10 noise stream */
+} vase_config;
+
+/* Sizes in bytes of the caller-allocated device buffers for a configuration. */
+typedef struct vase_buffer_sizes {
+    size_t k_cache;    /* bf16 [L][b][Hkv][K+B][d] */
+    size_t v_cache;    /* bf16 [L][b][Hkv][K+B][d] */
+    size_t q_window;   /* bf16 [L][b][Hq][W][d], a ring over the last W decode queries */
+    size_t positions;  /* int32 [L][b][Hkv][K+B], absolute stream position of each slot, -1 if empty */
+    size_t workspace;  /* scratch for one eviction at a time plus the host-append staging area */
+} vase_buffer_sizes;
+
+typedef struct vase_buffers {
+    void* k_cache;     /* device */
+    void* v_cache;     /* device */
+    void* q_window;    /* device */
+    int32_t* positions;/* device */
+    void* workspace;   /* device; contents are the library's between calls */
+} vase_buffers;
+
+/* Per-layer host counters: everything besides the buffers that a resume needs. */
+typedef struct vase_layer_state {
+    int32_t fill;          /* occupied slots, 0..K+B */
+    int32_t round;         /* evictions done so far (keys the noise of the next one) */
+    int64_t next_position; /* stream position of the next appended token */
+    int64_t queries_seen;  /* queries appended so far (ring write index = queries_seen % W) */
+} vase_layer_state;
+
+/* Where a decode attention kernel finds one layer's cache after eviction. */
+typedef struct vase_kv_view {
+    void* k;               /* device, bf16; row (s, h, slot) at k + ((s*Hkv + h)*unit_stride + slot)*d */
+    void* v;
+    int32_t* positions;
+    int64_t unit_stride;   /* elements between consecutive (s, h) units = (K+B)*d */
+    int32_t slots;         /* K + B */
+    int32_t fill;          /* valid slots 0..fill-1, in stream order */
+} vase_kv_view;
+
+/* Device pointers to the workspace results of the most recent vase_evict (valid until the next call). */
+typedef struct vase_debug_view {
+    float* attn;           /* [b*Hkv][K+B] window score before pooling (AttnV) */
+    float* pooled;         /* [b*Hkv][K+B] pooled score (AttnV, debug_outputs) */
+    float* value_score;    /* [b*Hkv][K+B] Range/L2/Var (AttnV) or leverage product s_i (DKV), slots < K */
+    float* key;            /* [b*Hkv][K+B] selection key per candidate, -1 if not a candidate (debug_outputs) */
+    uint8_t* keep;         /* [b*Hkv][K+B] 1 = kept (debug_outputs) */
+    int32_t* src;          /* [b*Hkv][K] ascending kept slots: new slot j holds old slot src[j] */
+    int32_t units;         /* b*Hkv */
+    int32_t slots;         /* K + B */
+} vase_debug_view;
+
+typedef struct vase_ctx vase_ctx;
+
+/* Fills *cfg with the paper's defaults (App. B): n_v = -1 (K/4), r = 20, pool 7,
+ * stochastic, fresh G per round, Range value score.  Geometry fields are zeroed. */
+void vase_config_default(vase_config* cfg);
+
+/* Validates *cfg and reports the buffer sizes it needs.  No device work. */
+int vase_get_buffer_sizes(const vase_config* cfg, vase_buffer_sizes* out);
+
+/* Creates a context over caller-owned buffers (sizes from vase_buffer_sizes).
+ * Reads the current CUDA device; encodes the TMA descriptors of the caches.
+ * Every layer starts empty (fill 0, round 0).  The buffers are not cleared. */
+int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out);
+
+/* Frees the context's host state.  Caller memory is untouched. */
+void vase_destroy(vase_ctx* ctx);
+
+/* Appends n_tokens consecutive decode steps of one layer (Sec. 2: each decode
+ * step adds one pair per KV head).  Device inputs, row-major:
+ *   q [n_tokens][b][Hq][d], k and v [n_tokens][b][Hkv][d]  (bf16).
+ * q goes to the window ring, k and v to slots fill..fill+n_tokens-1 with their
+ * stream positions.  Returns VASE_EVICT_DUE when the layer becomes full,
+ * VASE_ERR_FULL (nothing written) when fill + n_tokens > K + B. */
+int vase_append(vase_ctx* ctx, int32_t layer, const void* q, const void* k, const void* v,
+                int32_t n_tokens, void* stream);
+
+/* Same as vase_append with HOST inputs (pinned memory gives asynchronous copies):
+ * the library copies them into its staging area in the workspace (at most B
+ * tokens per call) and appends from there. */
+int vase_append_host(vase_ctx* ctx, int32_t layer, const void* q_host, const void* k_host,
+                     const void* v_host, int32_t n_tokens, void* stream);
+
+/* One eviction step of one layer (Sec. 2 and Sec. 3.2): requires fill == K+B;
+ * afterwards fill == K, round += 1, slots 0..K-1 hold the kept pairs in stream
+ * order and positions of slots K..K+B-1 are -1. */
+int vase_evict(vase_ctx* ctx, int32_t layer, void* stream);
+
+/* Copies the K positions of every unit of one layer to host memory
+ * (int32 [b][Hkv][K]), enqueued on the stream; the host buffer is valid after
+ * the stream completes. */
+int vase_read_positions(vase_ctx* ctx, int32_t layer, int32_t* host_out, void* stream);
+
+int vase_get_layer_state(const vase_ctx* ctx, int32_t layer, vase_layer_state* out);
+/* Sets one layer's counters (resume from a checkpoint, or tests that write the buffers directly). */
+int vase_set_layer_state(vase_ctx* ctx, int32_t layer, const vase_layer_state* st);
+
+int vase_kv_view_get(const vase_ctx* ctx, int32_t layer, vase_kv_view* out);
+int vase_debug_view_get(const vase_ctx* ctx, vase_debug_view* out);
+
+/* Synchronises the stream, then reads and clears the device error word that
+ * bounded waits and device-side checks set.  Returns VASE_OK or VASE_ERR_DEVICE
+ * (with *code, if non-NULL, set to the raw word). */
+int vase_check_device_error(vase_ctx* ctx, void* stream, uint32_t* code);
+
+/* Number of kernels the library launched on this context since creation. */
+int64_t vase_launch_count(const vase_ctx* ctx);
+
+/* Kernel kinds reported by vase_profile_collect. */
+#define VASE_KERNEL_APPEND 0
+#define VASE_KERNEL_SCORE 1   /* window attention score (tcgen05) */
+#define VASE_KERNEL_VALUE 2   /* value magnitude */
+#define VASE_KERNEL_DKV 3     /* DKV leverage scores (tcgen05) */
+#define VASE_KERNEL_SELECT 4  /* reservation + sampling + kept list */
+#define VASE_KERNEL_COMPACT 5 /* stable in-place gather */
+#define VASE_KERNEL_COUNT 6
+
+/* enable = 1: from now on record a CUDA event pair on the launch stream around
+ * every kernel (host-side instrumentation, no change to the kernels);
+ * enable = 0: stop recording.  Events are created by the library. */
+int vase_profile_enable(vase_ctx* ctx, int enable);
+
+/* Waits for the recorded events, writes per kernel kind the summed device time
+ * in milliseconds (total_ms[VASE_KERNEL_COUNT]) and the number of launches
+ * (launches[VASE_KERNEL_COUNT]), then forgets the recorded events. */
+int vase_profile_collect(vase_ctx* ctx, double* total_ms, int64_t* launches);
+
+const char* vase_status_string(int status);
+const char* vase_last_error(const vase_ctx* ctx);
+int vase_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VASE_H */

@@ -1,0 +1,637 @@
+// Host side of the C ABI declared in include/vase.h: configuration checks,
+// launch plans, TMA descriptors, per-layer counters and stream-ordered
+// launches of the eviction-step kernels.
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "kernels.cuh"
+#include "vase.h"
+
+using namespace vase;
+
+namespace {
+
+constexpr size_t kMaxDynSmem = 232448;  // 227 KB per block on sm_100-class GPUs
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+struct Plan {
+    int N, units, G, GW, GWp, NB, n_rb, n_tiles, cluster, tiles_per_cta, stages, tmem_cols, n_v, m;
+    size_t score_smem;
+    int dkv_tiles_k, dkv_tiles_per_cta, dkv_stages;
+    size_t dkv_smem;
+    size_t select_smem;
+    // workspace
+    size_t off_err, off_attn, off_pooled, off_vscore, off_key, off_keep, off_src, off_staging, staging_bytes, ws_bytes;
+};
+
+const char* check_config(const vase_config* c) {
+    if (!c) return "null config";
+    if (c->head_dim != 128) return "head_dim must be 128";
+    if (c->budget_k < 1 || c->buffer_b < 1) return "budget_k and buffer_b must be >= 1";
+    if (c->buffer_b > c->budget_k) return "buffer_b must not exceed budget_k (K - B candidates are kept)";
+    if (c->num_q_heads < 1 || c->num_kv_heads < 1 || c->num_q_heads % c->num_kv_heads) return "num_q_heads must be a positive multiple of num_kv_heads";
+    if (c->num_layers < 1 || c->batch < 1) return "num_layers and batch must be >= 1";
+    if (c->window < 1) return "window must be >= 1";
+    if (c->window > c->budget_k + c->buffer_b) return "window must not exceed K + B";
+    if (c->variant != VASE_VARIANT_ATTNV && c->variant != VASE_VARIANT_DKV) return "unknown variant";
+    if (c->value_score < 0 || c->value_score > 2) return "unknown value_score";
+    if (c->pool_kernel < 1 || (c->pool_kernel % 2) == 0) return "pool_kernel must be odd and >= 1";
+    if (c->dkv_rank < 1 || c->dkv_rank > 32) return "dkv_rank must be in 1..32";
+    const int nv = c->n_v < 0 ? c->budget_k / 4 : c->n_v;
+    if (c->variant == VASE_VARIANT_ATTNV && nv + c->buffer_b > c->budget_k) return "n_v + buffer_b must not exceed budget_k";
+    return nullptr;
+}
+
+bool make_plan(const vase_config* c, int num_sms, Plan* P, const char** why) {
+    *why = check_config(c);
+    if (*why) return false;
+    Plan& p = *P;
+    p.N = c->budget_k + c->buffer_b;
+    p.units = c->batch * c->num_kv_heads;
+    p.G = c->num_q_heads / c->num_kv_heads;
+    p.GW = p.G * c->window;
+    if (p.GW > 512) {
+        *why = "G * window must be <= 512";
+        return false;
+    }
+    p.GWp = p.GW <= 256 ? (p.GW + 31) / 32 * 32 : (p.GW + 255) / 256 * 256;
+    p.NB = p.GWp < 256 ? p.GWp : 256;
+    p.n_rb = p.GWp / p.NB;
+    p.n_tiles = ceil_div(p.N, kTileTokens);
+    p.n_v = c->n_v < 0 ? c->budget_k / 4 : c->n_v;
+    p.m = c->variant == VASE_VARIANT_ATTNV ? c->budget_k - p.n_v - c->buffer_b : c->budget_k - c->buffer_b;
+    int tc = 2 * p.NB;
+    p.tmem_cols = 32;
+    while (p.tmem_cols < tc) p.tmem_cols *= 2;
+
+    // cluster size: minimise waves x (tiles per CTA + 1)
+    int best_c = 1;
+    long best_cost = -1;
+    for (int C = 1; C <= 16 && C <= p.n_tiles; ++C) {
+        const int T = ceil_div(p.n_tiles, C);
+        if (ceil_div(p.n_tiles, T) != C) continue;
+        const long ctas = static_cast<long>(p.units) * C;
+        const long waves = (ctas + num_sms - 1) / num_sms;
+        const long cost = waves * (T + 1);
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best_c = C;
+        }
+    }
+    p.cluster = best_c;
+    p.tiles_per_cta = ceil_div(p.n_tiles, best_c);
+    p.stages = 0;
+    for (int s = 4; s >= 2; --s) {
+        if (score_attn_smem_bytes(p.GWp, p.cluster, s) <= kMaxDynSmem) {
+            p.stages = s;
+            break;
+        }
+    }
+    if (!p.stages) {
+        *why = "window rows do not fit in shared memory";
+        return false;
+    }
+    p.score_smem = score_attn_smem_bytes(p.GWp, p.cluster, p.stages);
+    if (p.tmem_cols > 256 && p.score_smem < 120 * 1024) p.score_smem = 120 * 1024;  // one CTA per SM owns TMEM
+
+    p.dkv_tiles_k = ceil_div(c->budget_k, kTileTokens);
+    {
+        int best = 1;
+        long bc = -1;
+        for (int C = 1; C <= p.dkv_tiles_k && C <= 64; ++C) {
+            const int T = ceil_div(p.dkv_tiles_k, C);
+            if (ceil_div(p.dkv_tiles_k, T) != C) continue;
+            const long ctas = static_cast<long>(p.units) * C;
+            const long waves = (ctas + num_sms - 1) / num_sms;
+            const long cost = waves * (T + 2);
+            if (bc < 0 || cost < bc) {
+                bc = cost;
+                best = C;
+            }
+        }
+        p.dkv_tiles_per_cta = ceil_div(p.dkv_tiles_k, best);
+    }
+    p.dkv_stages = 3;
+    p.dkv_smem = dkv_smem_bytes(p.dkv_stages);
+    p.select_smem = select_smem_bytes(p.N, c->budget_k);
+    if (p.select_smem > kMaxDynSmem - 4096) {
+        *why = "K + B too large for the single-CTA selection (about 25k slots at most)";
+        return false;
+    }
+
+    const size_t un = static_cast<size_t>(p.units) * p.N;
+    size_t o = 0;
+    p.off_err = o;
+    o += kAlign;
+    p.off_attn = o;
+    o = align_up(o + un * 4, kAlign);
+    p.off_pooled = o;
+    o = align_up(o + un * 4, kAlign);
+    p.off_vscore = o;
+    o = align_up(o + un * 4, kAlign);
+    p.off_key = o;
+    o = align_up(o + un * 4, kAlign);
+    p.off_keep = o;
+    o = align_up(o + un, kAlign);
+    p.off_src = o;
+    o = align_up(o + static_cast<size_t>(p.units) * c->budget_k * 4, kAlign);
+    p.off_staging = o;
+    p.staging_bytes = static_cast<size_t>(c->buffer_b) * c->batch * (c->num_q_heads + 2 * c->num_kv_heads) * kRowBytes;
+    o = align_up(o + p.staging_bytes, kAlign);
+    p.ws_bytes = o;
+    return true;
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+}  // namespace
+
+struct vase_ctx {
+    vase_config cfg;
+    vase_buffers bufs;
+    Plan plan;
+    int device = 0;
+    int num_sms = 0;
+    CUtensorMap kmap, vmap, qmap;
+    std::vector<vase_layer_state> layers;
+    int64_t launches = 0;
+    std::string last_error;
+    uint8_t* ws = nullptr;
+    // host-side kernel timing (vase_profile_enable)
+    struct EventPair {
+        cudaEvent_t start, end;
+        int kind;
+    };
+    std::vector<EventPair> events;
+    size_t events_used = 0;
+    bool profiling = false;
+    ~vase_ctx() {
+        for (auto& e : events) {
+            cudaEventDestroy(e.start);
+            cudaEventDestroy(e.end);
+        }
+    }
+};
+
+namespace {
+
+int fail(vase_ctx* ctx, int code, const std::string& msg) {
+    if (ctx) ctx->last_error = msg;
+    return code;
+}
+
+int cuda_fail(vase_ctx* ctx, cudaError_t e, const char* what) {
+    return fail(ctx, VASE_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+// Runs `launch` (which enqueues one kernel on s), bracketed by CUDA events when profiling.
+template <class F>
+cudaError_t timed_launch(vase_ctx* ctx, int kind, cudaStream_t s, F&& launch) {
+    if (!ctx->profiling) return launch();
+    if (ctx->events_used == ctx->events.size()) {
+        vase_ctx::EventPair e;
+        if (cudaEventCreate(&e.start) != cudaSuccess) return cudaGetLastError();
+        if (cudaEventCreate(&e.end) != cudaSuccess) {
+            cudaEventDestroy(e.start);
+            return cudaGetLastError();
+        }
+        ctx->events.push_back(e);
+    }
+    vase_ctx::EventPair& e = ctx->events[ctx->events_used++];
+    e.kind = kind;
+    cudaError_t r = cudaEventRecord(e.start, s);
+    if (r != cudaSuccess) return r;
+    r = launch();
+    if (r != cudaSuccess) return r;
+    return cudaEventRecord(e.end, s);
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+bool encode_rows(EncodeTiledFn enc, CUtensorMap* map, void* base, uint64_t rows, uint32_t box_rows) {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(kRowBytes)};
+    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+bool check_layer(vase_ctx* ctx, int32_t layer) { return ctx && layer >= 0 && layer < ctx->cfg.num_layers; }
+
+uint4* kc_layer(vase_ctx* c, int layer) {
+    return reinterpret_cast<uint4*>(c->bufs.k_cache) +
+           static_cast<int64_t>(layer) * c->plan.units * c->plan.N * kVecPerRow;
+}
+uint4* vc_layer(vase_ctx* c, int layer) {
+    return reinterpret_cast<uint4*>(c->bufs.v_cache) +
+           static_cast<int64_t>(layer) * c->plan.units * c->plan.N * kVecPerRow;
+}
+int32_t* pos_layer(vase_ctx* c, int layer) {
+    return c->bufs.positions + static_cast<int64_t>(layer) * c->plan.units * c->plan.N;
+}
+uint4* q_layer(vase_ctx* c, int layer) {
+    return reinterpret_cast<uint4*>(c->bufs.q_window) +
+           static_cast<int64_t>(layer) * c->cfg.batch * c->cfg.num_q_heads * c->cfg.window * kVecPerRow;
+}
+
+}  // namespace
+
+extern "C" {
+
+void vase_config_default(vase_config* cfg) {
+    if (!cfg) return;
+    std::memset(cfg, 0, sizeof(*cfg));
+    cfg->head_dim = 128;
+    cfg->variant = VASE_VARIANT_ATTNV;
+    cfg->n_v = -1;
+    cfg->value_score = VASE_VALUE_RANGE;
+    cfg->pool_kernel = 7;
+    cfg->dkv_rank = 20;
+    cfg->stochastic = 1;
+    cfg->dkv_fixed_g = 0;
+    cfg->debug_outputs = 0;
+    cfg->seed = 0;
+}
+
+int vase_get_buffer_sizes(const vase_config* cfg, vase_buffer_sizes* out) {
+    if (!cfg || !out) return VASE_ERR_INVALID;
+    Plan p;
+    const char* why = nullptr;
+    if (!make_plan(cfg, 152, &p, &why)) return cfg->head_dim != 128 ? VASE_ERR_UNSUPPORTED : VASE_ERR_INVALID;
+    const size_t rows = static_cast<size_t>(cfg->num_layers) * p.units * p.N;
+    out->k_cache = rows * kRowBytes;
+    out->v_cache = rows * kRowBytes;
+    out->q_window = static_cast<size_t>(cfg->num_layers) * cfg->batch * cfg->num_q_heads * cfg->window * kRowBytes;
+    out->positions = rows * 4;
+    out->workspace = p.ws_bytes;
+    return VASE_OK;
+}
+
+int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out) {
+    if (!out) return VASE_ERR_INVALID;
+    *out = nullptr;
+    if (!cfg || !bufs) return VASE_ERR_INVALID;
+    vase_ctx* ctx = new vase_ctx();
+    ctx->cfg = *cfg;
+    ctx->bufs = *bufs;
+    cudaError_t e = cudaGetDevice(&ctx->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, ctx->device);
+    if (e != cudaSuccess) {
+        int r = cuda_fail(ctx, e, "device query");
+        fprintf(stderr, "vase_create: %s\n", ctx->last_error.c_str());
+        delete ctx;
+        return r;
+    }
+    const char* why = nullptr;
+    if (!make_plan(cfg, ctx->num_sms, &ctx->plan, &why)) {
+        fprintf(stderr, "vase_create: %s\n", why);
+        delete ctx;
+        return cfg->head_dim != 128 ? VASE_ERR_UNSUPPORTED : VASE_ERR_INVALID;
+    }
+    const void* ptrs[5] = {bufs->k_cache, bufs->v_cache, bufs->q_window, bufs->positions, bufs->workspace};
+    for (const void* p : ptrs) {
+        if (!p || !aligned(p, kAlign)) {
+            fprintf(stderr, "vase_create: null or unaligned buffer (256-byte alignment required)\n");
+            delete ctx;
+            return p ? VASE_ERR_ALIGN : VASE_ERR_INVALID;
+        }
+    }
+    ctx->ws = static_cast<uint8_t*>(bufs->workspace);
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || !fn || q != cudaDriverEntryPointSuccess) {
+        fprintf(stderr, "vase_create: cuTensorMapEncodeTiled unavailable\n");
+        delete ctx;
+        return VASE_ERR_CUDA;
+    }
+    EncodeTiledFn enc = reinterpret_cast<EncodeTiledFn>(fn);
+    const Plan& P = ctx->plan;
+    const uint64_t cache_rows = static_cast<uint64_t>(cfg->num_layers) * P.units * P.N;
+    const uint64_t q_rows = static_cast<uint64_t>(cfg->num_layers) * cfg->batch * cfg->num_q_heads * cfg->window;
+    if (cache_rows >= (1ull << 31) || q_rows >= (1ull << 31)) {
+        fprintf(stderr, "vase_create: caches exceed 2^31 rows\n");
+        delete ctx;
+        return VASE_ERR_UNSUPPORTED;
+    }
+    const uint32_t qbox = static_cast<uint32_t>(P.GWp < 256 ? P.GWp : 256);
+    if (!encode_rows(enc, &ctx->kmap, bufs->k_cache, cache_rows, kTileTokens) ||
+        !encode_rows(enc, &ctx->vmap, bufs->v_cache, cache_rows, kTileTokens) ||
+        !encode_rows(enc, &ctx->qmap, bufs->q_window, q_rows, qbox)) {
+        fprintf(stderr, "vase_create: tensor map encoding failed\n");
+        delete ctx;
+        return VASE_ERR_CUDA;
+    }
+    if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
+        (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess ||
+        (e = select_set_attributes(P.select_smem)) != cudaSuccess) {
+        fprintf(stderr, "vase_create: kernel attributes: %s\n", cudaGetErrorString(e));
+        delete ctx;
+        return VASE_ERR_CUDA;
+    }
+    if ((e = cudaMemset(ctx->ws + P.off_err, 0, kAlign)) != cudaSuccess) {
+        fprintf(stderr, "vase_create: %s\n", cudaGetErrorString(e));
+        delete ctx;
+        return VASE_ERR_CUDA;
+    }
+    ctx->layers.assign(static_cast<size_t>(cfg->num_layers), vase_layer_state{0, 0, 0, 0});
+    *out = ctx;
+    return VASE_OK;
+}
+
+void vase_destroy(vase_ctx* ctx) { delete ctx; }
+
+int vase_append(vase_ctx* ctx, int32_t layer, const void* q, const void* k, const void* v, int32_t n_tokens,
+                void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    if (n_tokens < 1) return fail(ctx, VASE_ERR_INVALID, "n_tokens must be >= 1");
+    if (!q || !k || !v) return fail(ctx, VASE_ERR_INVALID, "null input");
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16)) return fail(ctx, VASE_ERR_ALIGN, "inputs must be 16-byte aligned");
+    vase_layer_state& st = ctx->layers[layer];
+    if (st.fill + n_tokens > ctx->plan.N) return fail(ctx, VASE_ERR_FULL, "append would exceed K + B slots");
+    AppendParams p;
+    p.q = static_cast<const uint4*>(q);
+    p.k = static_cast<const uint4*>(k);
+    p.v = static_cast<const uint4*>(v);
+    p.qwin = q_layer(ctx, layer);
+    p.kc = kc_layer(ctx, layer);
+    p.vc = vc_layer(ctx, layer);
+    p.pos = pos_layer(ctx, layer);
+    p.n = n_tokens;
+    p.b = ctx->cfg.batch;
+    p.Hq = ctx->cfg.num_q_heads;
+    p.Hkv = ctx->cfg.num_kv_heads;
+    p.W = ctx->cfg.window;
+    p.N = ctx->plan.N;
+    p.fill = st.fill;
+    p.next_pos = st.next_position;
+    p.q_seen = st.queries_seen;
+    cudaError_t e = timed_launch(ctx, VASE_KERNEL_APPEND, static_cast<cudaStream_t>(stream), [&] { return launch_append(p, static_cast<cudaStream_t>(stream)); });
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "append launch");
+    ctx->launches += 1;
+    st.fill += n_tokens;
+    st.next_position += n_tokens;
+    st.queries_seen += n_tokens;
+    return st.fill == ctx->plan.N ? VASE_EVICT_DUE : VASE_OK;
+}
+
+int vase_append_host(vase_ctx* ctx, int32_t layer, const void* q_host, const void* k_host, const void* v_host,
+                     int32_t n_tokens, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    if (n_tokens < 1 || n_tokens > ctx->cfg.buffer_b)
+        return fail(ctx, VASE_ERR_INVALID, "n_tokens must be in 1..buffer_b for host appends");
+    if (!q_host || !k_host || !v_host) return fail(ctx, VASE_ERR_INVALID, "null input");
+    if (ctx->layers[layer].fill + n_tokens > ctx->plan.N) return fail(ctx, VASE_ERR_FULL, "append would exceed K + B slots");
+    const size_t qb = static_cast<size_t>(n_tokens) * ctx->cfg.batch * ctx->cfg.num_q_heads * kRowBytes;
+    const size_t kb = static_cast<size_t>(n_tokens) * ctx->cfg.batch * ctx->cfg.num_kv_heads * kRowBytes;
+    uint8_t* sq = ctx->ws + ctx->plan.off_staging;
+    uint8_t* sk = sq + qb;
+    uint8_t* sv = sk + kb;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    if ((e = cudaMemcpyAsync(sq, q_host, qb, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(sk, k_host, kb, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(sv, v_host, kb, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return cuda_fail(ctx, e, "host-to-device staging copy");
+    return vase_append(ctx, layer, sq, sk, sv, n_tokens, stream);
+}
+
+int vase_evict(vase_ctx* ctx, int32_t layer, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    vase_layer_state& st = ctx->layers[layer];
+    const Plan& P = ctx->plan;
+    const vase_config& c = ctx->cfg;
+    if (st.fill != P.N) return fail(ctx, VASE_ERR_NOT_FULL, "evict needs a full cache (fill == K + B)");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t* err = reinterpret_cast<uint32_t*>(ctx->ws + P.off_err);
+    float* attn = reinterpret_cast<float*>(ctx->ws + P.off_attn);
+    float* vscore = reinterpret_cast<float*>(ctx->ws + P.off_vscore);
+    int32_t* src = reinterpret_cast<int32_t*>(ctx->ws + P.off_src);
+    const int64_t cache_row0 = static_cast<int64_t>(layer) * P.units * P.N;
+    cudaError_t e;
+    if (c.variant == VASE_VARIANT_ATTNV) {
+        ScoreAttnParams sp;
+        sp.N = P.N;
+        sp.GW = P.GW;
+        sp.GWp = P.GWp;
+        sp.NB = P.NB;
+        sp.n_rb = P.n_rb;
+        sp.n_tiles = P.n_tiles;
+        sp.tiles_per_cta = P.tiles_per_cta;
+        sp.cluster = P.cluster;
+        sp.stages = P.stages;
+        sp.tmem_cols = P.tmem_cols;
+        sp.Hq = c.num_q_heads;
+        sp.Hkv = c.num_kv_heads;
+        sp.W = c.window;
+        sp.G = P.G;
+        sp.k_row0 = cache_row0;
+        sp.q_row0 = static_cast<int64_t>(layer) * c.batch * c.num_q_heads * c.window;
+        sp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
+        sp.inv_gw = 1.0f / static_cast<float>(P.GW);
+        sp.attn = attn;
+        sp.err = err;
+        if ((e = timed_launch(ctx, VASE_KERNEL_SCORE, s, [&] { return launch_score_attn(ctx->kmap, ctx->qmap, sp, P.units, P.score_smem, s); })) != cudaSuccess)
+            return cuda_fail(ctx, e, "score launch");
+        ValueParams vp;
+        vp.vc = vc_layer(ctx, layer);
+        vp.out = vscore;
+        vp.N = P.N;
+        vp.K = c.budget_k;
+        vp.units = P.units;
+        vp.kind = c.value_score;
+        if ((e = timed_launch(ctx, VASE_KERNEL_VALUE, s, [&] { return launch_value_score(vp, ctx->num_sms, s); })) != cudaSuccess) return cuda_fail(ctx, e, "value launch");
+        ctx->launches += 2;
+    } else {
+        DkvParams dp;
+        dp.N = P.N;
+        dp.K = c.budget_k;
+        dp.r = c.dkv_rank;
+        dp.Hkv = c.num_kv_heads;
+        dp.layer = layer;
+        dp.rnd = c.dkv_fixed_g ? 0 : st.round;
+        dp.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
+        dp.seed_hi = static_cast<uint32_t>(c.seed >> 32);
+        dp.n_tiles_k = P.dkv_tiles_k;
+        dp.tiles_per_cta = P.dkv_tiles_per_cta;
+        dp.stages = P.dkv_stages;
+        dp.row0 = cache_row0;
+        dp.out = vscore;
+        dp.lk_out = nullptr;
+        dp.lv_out = nullptr;
+        dp.err = err;
+        if ((e = timed_launch(ctx, VASE_KERNEL_DKV, s, [&] { return launch_dkv(ctx->kmap, ctx->vmap, dp, P.units, P.dkv_smem, s); })) != cudaSuccess)
+            return cuda_fail(ctx, e, "dkv launch");
+        ctx->launches += 1;
+    }
+    SelectParams sel;
+    sel.attn = attn;
+    sel.vscore = vscore;
+    sel.pos = pos_layer(ctx, layer);
+    sel.src = src;
+    sel.pooled_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_pooled) : nullptr;
+    sel.key_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_key) : nullptr;
+    sel.keep_dbg = c.debug_outputs ? ctx->ws + P.off_keep : nullptr;
+    sel.N = P.N;
+    sel.K = c.budget_k;
+    sel.B = c.buffer_b;
+    sel.n_v = P.n_v;
+    sel.m = P.m;
+    sel.pool = c.pool_kernel;
+    sel.variant = c.variant;
+    sel.stochastic = c.stochastic;
+    sel.Hkv = c.num_kv_heads;
+    sel.layer = layer;
+    sel.rnd = st.round;
+    sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
+    sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
+    sel.err = err;
+    if ((e = timed_launch(ctx, VASE_KERNEL_SELECT, s, [&] { return launch_select(sel, P.units, P.select_smem, s); })) != cudaSuccess) return cuda_fail(ctx, e, "select launch");
+    CompactParams cp;
+    cp.kc = kc_layer(ctx, layer);
+    cp.vc = vc_layer(ctx, layer);
+    cp.pos = pos_layer(ctx, layer);
+    cp.src = src;
+    cp.N = P.N;
+    cp.K = c.budget_k;
+    if ((e = timed_launch(ctx, VASE_KERNEL_COMPACT, s, [&] { return launch_compact(cp, P.units, s); })) != cudaSuccess) return cuda_fail(ctx, e, "compact launch");
+    ctx->launches += 2;
+    st.fill = c.budget_k;
+    st.round += 1;
+    return VASE_OK;
+}
+
+int vase_read_positions(vase_ctx* ctx, int32_t layer, int32_t* host_out, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (!check_layer(ctx, layer) || !host_out) return fail(ctx, VASE_ERR_INVALID, "bad layer or null output");
+    const Plan& P = ctx->plan;
+    const size_t width = static_cast<size_t>(ctx->cfg.budget_k) * 4;
+    cudaError_t e = cudaMemcpy2DAsync(host_out, width, pos_layer(ctx, layer), static_cast<size_t>(P.N) * 4, width,
+                                      static_cast<size_t>(P.units), cudaMemcpyDeviceToHost,
+                                      static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "positions copy");
+    return VASE_OK;
+}
+
+int vase_get_layer_state(const vase_ctx* ctx, int32_t layer, vase_layer_state* out) {
+    if (!ctx || !out || layer < 0 || layer >= ctx->cfg.num_layers) return VASE_ERR_INVALID;
+    *out = ctx->layers[layer];
+    return VASE_OK;
+}
+
+int vase_set_layer_state(vase_ctx* ctx, int32_t layer, const vase_layer_state* st) {
+    if (!ctx || !st) return VASE_ERR_INVALID;
+    if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    if (st->fill < 0 || st->fill > ctx->plan.N || st->round < 0 || st->next_position < 0 || st->queries_seen < 0)
+        return fail(ctx, VASE_ERR_INVALID, "layer state out of range");
+    ctx->layers[layer] = *st;
+    return VASE_OK;
+}
+
+int vase_kv_view_get(const vase_ctx* ctx, int32_t layer, vase_kv_view* out) {
+    if (!ctx || !out || layer < 0 || layer >= ctx->cfg.num_layers) return VASE_ERR_INVALID;
+    vase_ctx* c = const_cast<vase_ctx*>(ctx);
+    out->k = kc_layer(c, layer);
+    out->v = vc_layer(c, layer);
+    out->positions = pos_layer(c, layer);
+    out->unit_stride = static_cast<int64_t>(ctx->plan.N) * kHeadDim;
+    out->slots = ctx->plan.N;
+    out->fill = ctx->layers[layer].fill;
+    return VASE_OK;
+}
+
+int vase_debug_view_get(const vase_ctx* ctx, vase_debug_view* out) {
+    if (!ctx || !out) return VASE_ERR_INVALID;
+    const Plan& P = ctx->plan;
+    out->attn = reinterpret_cast<float*>(ctx->ws + P.off_attn);
+    out->pooled = reinterpret_cast<float*>(ctx->ws + P.off_pooled);
+    out->value_score = reinterpret_cast<float*>(ctx->ws + P.off_vscore);
+    out->key = reinterpret_cast<float*>(ctx->ws + P.off_key);
+    out->keep = ctx->ws + P.off_keep;
+    out->src = reinterpret_cast<int32_t*>(ctx->ws + P.off_src);
+    out->units = P.units;
+    out->slots = P.N;
+    return VASE_OK;
+}
+
+int vase_check_device_error(vase_ctx* ctx, void* stream, uint32_t* code) {
+    if (!ctx) return VASE_ERR_INVALID;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "stream synchronize");
+    uint32_t word = 0;
+    uint32_t* dev = reinterpret_cast<uint32_t*>(ctx->ws + ctx->plan.off_err);
+    if ((e = cudaMemcpy(&word, dev, 4, cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(ctx, e, "error word read");
+    if (code) *code = word;
+    if (word) {
+        if ((e = cudaMemset(dev, 0, 4)) != cudaSuccess) return cuda_fail(ctx, e, "error word clear");
+        char buf[96];
+        snprintf(buf, sizeof(buf), "device error word 0x%08x", word);
+        return fail(ctx, VASE_ERR_DEVICE, buf);
+    }
+    return VASE_OK;
+}
+
+int64_t vase_launch_count(const vase_ctx* ctx) { return ctx ? ctx->launches : 0; }
+
+int vase_profile_enable(vase_ctx* ctx, int enable) {
+    if (!ctx) return VASE_ERR_INVALID;
+    ctx->profiling = enable != 0;
+    return VASE_OK;
+}
+
+int vase_profile_collect(vase_ctx* ctx, double* total_ms, int64_t* launches) {
+    if (!ctx || !total_ms || !launches) return VASE_ERR_INVALID;
+    for (int k = 0; k < VASE_KERNEL_COUNT; ++k) {
+        total_ms[k] = 0.0;
+        launches[k] = 0;
+    }
+    for (size_t i = 0; i < ctx->events_used; ++i) {
+        const vase_ctx::EventPair& e = ctx->events[i];
+        cudaError_t r = cudaEventSynchronize(e.end);
+        float ms = 0.f;
+        if (r == cudaSuccess) r = cudaEventElapsedTime(&ms, e.start, e.end);
+        if (r != cudaSuccess) {
+            ctx->events_used = 0;
+            return cuda_fail(ctx, r, "profile events");
+        }
+        total_ms[e.kind] += ms;
+        launches[e.kind] += 1;
+    }
+    ctx->events_used = 0;
+    return VASE_OK;
+}
+
+const char* vase_status_string(int status) {
+    switch (status) {
+        case VASE_OK: return "ok";
+        case VASE_EVICT_DUE: return "eviction due";
+        case VASE_ERR_INVALID: return "invalid argument";
+        case VASE_ERR_FULL: return "cache full";
+        case VASE_ERR_NOT_FULL: return "cache not full";
+        case VASE_ERR_CUDA: return "CUDA error";
+        case VASE_ERR_UNSUPPORTED: return "unsupported configuration";
+        case VASE_ERR_ALIGN: return "misaligned pointer";
+        case VASE_ERR_DEVICE: return "device-side error";
+        default: return "unknown status";
+    }
+}
+
+const char* vase_last_error(const vase_ctx* ctx) { return ctx ? ctx->last_error.c_str() : "null context"; }
+
+int vase_abi_version(void) { return VASE_ABI_VERSION; }
+
+}  // extern "C"

@@ -1,0 +1,154 @@
+// Kernel parameter blocks, launch helpers and the device-side Philox of the
+// VaSE eviction step.  Host orchestration lives in api.cu.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace vase {
+
+// Error sites recorded in the device error word (low 16 bits).
+enum ErrSite : uint32_t {
+    kErrScoreQ = 1,
+    kErrScoreKFull = 2,
+    kErrScoreKEmpty = 3,
+    kErrScoreTFull = 4,
+    kErrScoreTEmpty = 5,
+    kErrScoreDrain = 6,
+    kErrSelectCount = 16,
+    kErrDkvTFull = 32,
+    kErrDkvKFull = 33,
+    kErrDkvKEmpty = 34,
+    kErrDkvTEmpty = 35,
+    kErrDkvDrain = 36,
+};
+
+constexpr int kTileTokens = 128;   // tokens per MMA tile (M)
+constexpr int kHeadDim = 128;      // d
+constexpr int kRowBytes = 256;     // d * sizeof(bf16)
+constexpr int kVecPerRow = 16;     // 16-byte vectors per row
+
+// ------------------------------------------------------------------ Philox4x32-10
+// Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as easy as 1, 2, 3" (SC'11):
+// ten rounds of two 32x32->64-bit multiplies with a Weyl-sequence key schedule.
+struct Philox4 {
+    uint32_t x, y, z, w;
+};
+
+__device__ __forceinline__ Philox4 philox4x32_10(Philox4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+    for (int i = 0; i < 10; ++i) {
+        const uint32_t hi0 = __umulhi(0xD2511F53u, c.x);
+        const uint32_t lo0 = 0xD2511F53u * c.x;
+        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z);
+        const uint32_t lo1 = 0xCD9E8D57u * c.z;
+        c = Philox4{hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0};
+        k0 += 0x9E3779B9u;
+        k1 += 0xBB67AE85u;
+    }
+    return c;
+}
+
+// u = (2 * (x >> 9) + 1) * 2^-24: strictly inside (0, 1) and exact in fp32.
+__device__ __forceinline__ float open_uniform(uint32_t x) {
+    return static_cast<float>(2u * (x >> 9) + 1u) * 5.9604644775390625e-08f;
+}
+
+constexpr uint32_t kTagSelect = 0u;
+constexpr uint32_t kTagDkv = 1u;
+
+// ------------------------------------------------------------------ parameter blocks
+
+struct AppendParams {
+    const uint4* q;   // [n][b][Hq][16]
+    const uint4* k;   // [n][b][Hkv][16]
+    const uint4* v;
+    uint4* qwin;      // layer base of [b][Hq][W][16]
+    uint4* kc;        // layer base of [b][Hkv][N][16]
+    uint4* vc;
+    int32_t* pos;     // layer base of [b][Hkv][N]
+    int32_t n, b, Hq, Hkv, W, N, fill;
+    int64_t next_pos;
+    int64_t q_seen;
+};
+
+struct ScoreAttnParams {
+    int32_t N;              // K + B slots per unit
+    int32_t GW;             // window rows per unit (G * W)
+    int32_t GWp;            // GW rounded up to a multiple of 32
+    int32_t NB;             // rows per MMA (row block), multiple of 32, <= 256
+    int32_t n_rb;           // GWp / NB
+    int32_t n_tiles;        // ceil(N / 128)
+    int32_t tiles_per_cta;  // T
+    int32_t cluster;        // CTAs per unit
+    int32_t stages;         // K-tile ring depth
+    int32_t tmem_cols;
+    int32_t Hq, Hkv, W, G;
+    int64_t k_row0;         // first K-cache row of the layer
+    int64_t q_row0;         // first Q-window row of the layer
+    float scale_log2;       // log2(e) / sqrt(d)
+    float inv_gw;           // 1 / (G * W)
+    float* attn;            // [units][N]
+    uint32_t* err;
+};
+
+struct ValueParams {
+    const uint4* vc;        // layer base [units][N][16]
+    float* out;             // [units][N], slots < K
+    int32_t N, K, units, kind;
+};
+
+struct DkvParams {
+    int32_t N, K, r, Hkv, layer, rnd;
+    uint32_t seed_lo, seed_hi;
+    int32_t n_tiles_k;      // ceil(K / 128)
+    int32_t tiles_per_cta;
+    int32_t stages;
+    int64_t row0;           // first cache row of the layer
+    float* out;             // [units][N] leverage product, slots < K
+    float* lk_out;          // optional [units][N]
+    float* lv_out;          // optional [units][N]
+    uint32_t* err;
+};
+
+struct SelectParams {
+    const float* attn;      // [units][N]
+    const float* vscore;    // [units][N]
+    const int32_t* pos;     // layer base [units][N]
+    int32_t* src;           // [units][K]
+    float* pooled_dbg;      // nullable
+    float* key_dbg;         // nullable
+    uint8_t* keep_dbg;      // nullable
+    int32_t N, K, B, n_v, m, pool, variant, stochastic, Hkv, layer, rnd;
+    uint32_t seed_lo, seed_hi;
+    uint32_t* err;
+};
+
+struct CompactParams {
+    uint4* kc;              // layer base [units][N][16]
+    uint4* vc;
+    int32_t* pos;           // layer base [units][N]
+    const int32_t* src;     // [units][K]
+    int32_t N, K;
+};
+
+// ------------------------------------------------------------------ launchers (return cudaError_t)
+
+cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
+cudaError_t launch_value_score(const ValueParams& p, int num_sms, cudaStream_t s);
+cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreAttnParams& p,
+                              int units, size_t smem_bytes, cudaStream_t s);
+cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
+                       size_t smem_bytes, cudaStream_t s);
+cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s);
+cudaError_t launch_compact(const CompactParams& p, int units, cudaStream_t s);
+
+size_t score_attn_smem_bytes(int GWp, int cluster, int stages);
+size_t dkv_smem_bytes(int stages);
+size_t select_smem_bytes(int N, int K);
+cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster);
+cudaError_t dkv_set_attributes(size_t smem_bytes);
+cudaError_t select_set_attributes(size_t smem_bytes);
+
+}  // namespace vase

@@ -1,0 +1,341 @@
+"""GPU parity of the VaSE eviction step (C ABI -> CUDA kernels) against the fp64 oracle.
+
+Inputs are the seeded synthetic workloads; every expected value comes from
+the oracle or from the definition of a pure data movement.
+"""
+
+import itertools
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import vase_oracle as O
+from paper_2606_03928_gb300 import workloads as W
+import parity_utils as PU
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_03928_gb300 import build
+    build.build()
+    from paper_2606_03928_gb300 import vase as V
+    V.load()
+
+
+def _cache(wl, num_layers, variant="attnv", debug=True, **kw):
+    from paper_2606_03928_gb300.vase import VaseCache
+    return VaseCache(PU.geometry_of(wl, num_layers), variant=variant, debug_outputs=debug, **kw)
+
+
+def _run_layer(wl, *, variant="attnv", layer=1, num_layers=2, round_index=3, seed=0, data_seed=0, units=None,
+               debug=True, positions="gapped", cache_kw=None, oracle_kw=None, state_round=None):
+    """Uploads one layer, evicts it through the C ABI and checks `units` (default all) against the oracle.
+
+    round_index is the eviction counter (it keys the noise); state_round (default round_index) draws the data.
+    """
+    cache_kw = dict(cache_kw or {})
+    oracle_kw = dict(oracle_kw or {})
+    cache = _cache(wl, num_layers, variant=variant, debug=debug, seed=seed, **cache_kw)
+    st = W.layer_state(wl, data_seed, layer, round_index if state_round is None else state_round, positions)
+    PU.upload_layer(cache, layer, st, round_index)
+    other = None
+    if num_layers > 1:
+        other_layer = 0 if layer != 0 else 1
+        other = W.layer_state(wl, data_seed + 1, other_layer, 0, "dense")
+        PU.upload_layer(cache, other_layer, other, 0)
+    assert cache.evict(layer) == 0
+    status, code = cache.check_device_error()
+    assert status == 0, f"device error word {code:#x}"
+    got = PU.download(cache, layer)
+    if other is not None:
+        rest = PU.download(cache, other_layer)
+        assert np.array_equal(rest["k_bits"], other["k_bits"]), "another layer was modified"
+    st_after = cache.layer_state(layer)
+    assert st_after["fill"] == wl.budget_k and st_after["round"] == round_index + 1
+    nv = oracle_kw.get("n_v", -1)
+    nv = wl.budget_k // 4 if nv is None or nv < 0 else nv
+    if variant == "dkv":
+        nv = 0
+    flips = 0
+    todo = units if units is not None else [(s, h) for s in range(wl.batch) for h in range(wl.num_kv_heads)]
+    for (s, h) in todo:
+        ref = PU.oracle_unit(wl, st, s, h, variant=variant, round_index=round_index, seed=seed, layer=layer,
+                             **oracle_kw)
+        gu = PU.unit_slice(got, s, h, wl.num_kv_heads)
+        if not debug:
+            gu["pooled"] = None
+            gu["key"] = None
+        flips += PU.check_unit(wl, ref, gu, st["k_bits"][s, h], st["v_bits"][s, h], st["positions"][s, h],
+                               variant=variant, n_v=nv)
+    # properties that hold at any size, checked on every unit
+    K, B = wl.budget_k, wl.buffer_b
+    for s in range(wl.batch):
+        for h in range(wl.num_kv_heads):
+            u = s * wl.num_kv_heads + h
+            src = got["src"][u]
+            assert len(set(src.tolist())) == K and set(range(K, K + B)) <= set(src.tolist())
+    return cache, st, got, flips
+
+
+# ----------------------------------------------------------------------------- small configurations
+
+SMALL = W.WORKLOADS["single_layer_k256"]
+
+
+def test_single_layer_k256_all_units_match_oracle():
+    _, _, _, flips = _run_layer(SMALL, layer=0, num_layers=1, round_index=0, positions="dense")
+    assert flips <= 2
+
+
+def test_layer_offset_and_gapped_positions():
+    _run_layer(SMALL, layer=1, num_layers=2, round_index=5)
+
+
+@pytest.mark.parametrize("value_score", [O.VALUE_L2, O.VALUE_VAR])
+def test_value_score_variants(value_score):
+    _run_layer(SMALL, cache_kw={"value_score": value_score}, oracle_kw={"value_score": value_score})
+
+
+def test_deterministic_top_k_and_no_pooling():
+    _run_layer(SMALL, cache_kw={"stochastic": False, "pool_kernel": 1},
+               oracle_kw={"stochastic": False, "pool_kernel": 1})
+
+
+def test_no_value_reservation():
+    _run_layer(SMALL, cache_kw={"n_v": 0}, oracle_kw={"n_v": 0})
+
+
+@pytest.mark.parametrize("K,B,Wn,Hq,Hkv", [(100, 27, 5, 6, 3), (130, 1, 1, 2, 2), (8, 2, 3, 4, 1),
+                                          (384, 128, 64, 8, 2), (200, 50, 20, 24, 8)])
+def test_ragged_geometries(K, B, Wn, Hq, Hkv):
+    wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=Wn, num_q_heads=Hq, num_kv_heads=Hkv, batch=2,
+                  num_layers=2)
+    _run_layer(wl, cache_kw={"n_v": K // 5}, oracle_kw={"n_v": K // 5})
+
+
+def test_seed_changes_selection():
+    a = _run_layer(SMALL, seed=1)[2]["src"]
+    b = _run_layer(SMALL, seed=2)[2]["src"]
+    assert not np.array_equal(a, b)
+
+
+def test_dkv_small_all_units():
+    _run_layer(SMALL, variant="dkv", layer=0, num_layers=1, oracle_kw={"dkv_rank": 20})
+
+
+@pytest.mark.parametrize("r", [1, 7, 32])
+def test_dkv_ranks(r):
+    _run_layer(SMALL, variant="dkv", cache_kw={"dkv_rank": r}, oracle_kw={"dkv_rank": r})
+
+
+def test_dkv_fixed_g_is_round_independent():
+    a = _run_layer(SMALL, variant="dkv", round_index=2, state_round=2, cache_kw={"dkv_fixed_g": True},
+                   oracle_kw={"dkv_fixed_g": True})[2]
+    b = _run_layer(SMALL, variant="dkv", round_index=9, state_round=2, cache_kw={"dkv_fixed_g": True},
+                   oracle_kw={"dkv_fixed_g": True})[2]
+    c = _run_layer(SMALL, variant="dkv", round_index=9, state_round=2)[2]
+    assert np.array_equal(a["src"], b["src"])
+    assert not np.array_equal(b["src"], c["src"])
+
+
+# ----------------------------------------------------------------------------- append path
+
+def test_append_writes_cache_ring_and_positions():
+    wl = W.shrink(SMALL, budget_k=64, buffer_b=16, window=8, batch=2, num_layers=2)
+    cache = _cache(wl, 2)
+    N = wl.slots
+    chunk = W.stream_chunk(wl, 3, 1, 0, N)
+    dev = cache.device
+    q = PU.bits_to_bf16_tensor(chunk["q_bits"], dev)
+    k = PU.bits_to_bf16_tensor(chunk["k_bits"], dev)
+    v = PU.bits_to_bf16_tensor(chunk["v_bits"], dev)
+    assert cache.append(1, q[:50], k[:50], v[:50]) == 0
+    assert cache.append(1, q[50:], k[50:], v[50:]) == 1  # full: eviction due
+    torch.cuda.synchronize()
+    kb = cache.k_cache[1].view(torch.int16).cpu().numpy().view(np.uint16)
+    vb = cache.v_cache[1].view(torch.int16).cpu().numpy().view(np.uint16)
+    qb = cache.q_window[1].view(torch.int16).cpu().numpy().view(np.uint16)
+    pos = cache.positions[1].cpu().numpy()
+    assert np.array_equal(kb, chunk["k_bits"].transpose(1, 2, 0, 3))
+    assert np.array_equal(vb, chunk["v_bits"].transpose(1, 2, 0, 3))
+    assert np.array_equal(pos, np.broadcast_to(np.arange(N), pos.shape))
+    # ring slot (t mod W) holds the query of step t for the last W steps
+    for t in range(N - wl.window, N):
+        assert np.array_equal(qb[:, :, t % wl.window], chunk["q_bits"][t])
+    with pytest.raises(Exception):
+        cache.append(1, q[:1], k[:1], v[:1])  # full
+    st = cache.layer_state(1)
+    assert st["fill"] == N and st["next_position"] == N and st["queries_seen"] == N
+
+
+def test_host_append_and_read_positions_match_device_append():
+    wl = W.shrink(SMALL, budget_k=64, buffer_b=16, window=8, batch=2, num_layers=1)
+    a = _cache(wl, 1)
+    b = _cache(wl, 1)
+    chunk = W.stream_chunk(wl, 5, 0, 0, wl.slots)
+    tq = torch.from_numpy(chunk["q_bits"].view(np.int16)).view(torch.bfloat16)
+    tk = torch.from_numpy(chunk["k_bits"].view(np.int16)).view(torch.bfloat16)
+    tv = torch.from_numpy(chunk["v_bits"].view(np.int16)).view(torch.bfloat16)
+    for s in range(0, wl.slots, wl.buffer_b):
+        e = min(wl.slots, s + wl.buffer_b)
+        a.append(0, tq[s:e].cuda().contiguous(), tk[s:e].cuda().contiguous(), tv[s:e].cuda().contiguous())
+        b.append_host(0, tq[s:e].contiguous().pin_memory(), tk[s:e].contiguous().pin_memory(),
+                      tv[s:e].contiguous().pin_memory())
+    a.evict(0)
+    b.evict(0)
+    torch.cuda.synchronize()
+    assert torch.equal(a.k_cache, b.k_cache) and torch.equal(a.v_cache, b.v_cache)
+    out = torch.empty((wl.batch, wl.num_kv_heads, wl.budget_k), dtype=torch.int32).pin_memory()
+    b.read_positions(0, out)
+    torch.cuda.synchronize()
+    assert torch.equal(out, b.positions[0, :, :, :wl.budget_k].cpu())
+
+
+def test_status_codes():
+    from paper_2606_03928_gb300 import vase as V
+    wl = W.shrink(SMALL, budget_k=64, buffer_b=16, window=8, batch=1, num_layers=1)
+    c = _cache(wl, 1)
+    with pytest.raises(V.VaseError) as ei:
+        c.evict(0)
+    assert ei.value.status == V.VASE_ERR_NOT_FULL
+    with pytest.raises(V.VaseError) as ei:
+        c.evict(3)
+    assert ei.value.status == V.VASE_ERR_INVALID
+    q = torch.zeros((1, 1, wl.num_q_heads, 128), dtype=torch.bfloat16, device="cuda")
+    k = torch.zeros((1, 1, wl.num_kv_heads, 128), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(V.VaseError) as ei:
+        V.vase_append(c.ctx, 0, q.data_ptr() + 2, k.data_ptr(), k.data_ptr(), 1)
+    assert ei.value.status == V.VASE_ERR_ALIGN
+    assert c.check_device_error()[0] == 0
+
+
+# ----------------------------------------------------------------------------- chained rounds
+
+def test_chained_rounds_follow_the_oracle_until_a_threshold_tie():
+    """Appends B new tokens and evicts, 6 rounds in a row; the oracle chains its own state."""
+    wl = W.shrink(SMALL, budget_k=256, buffer_b=64, window=32, batch=1, num_layers=1)
+    cache = _cache(wl, 1)
+    N, K, B = wl.slots, wl.budget_k, wl.buffer_b
+    dev = cache.device
+    first = W.stream_chunk(wl, 11, 0, 0, N)
+    cache.append(0, *(PU.bits_to_bf16_tensor(first[x], dev) for x in ("q_bits", "k_bits", "v_bits")))
+    G = wl.group
+    state_k = first["k_bits"].transpose(1, 2, 0, 3).copy()
+    state_v = first["v_bits"].transpose(1, 2, 0, 3).copy()
+    pos = np.broadcast_to(np.arange(N), (wl.batch, wl.num_kv_heads, N)).copy()
+    qhist = [first["q_bits"][t] for t in range(N)]
+    compared = 0
+    for rnd in range(6):
+        cache.evict(0)
+        got = PU.download(cache, 0)
+        qwin = np.stack(qhist[-wl.window:], axis=2)  # [b, Hq, W, d]
+        same = True
+        for h in range(wl.num_kv_heads):
+            ref = O.evict_unit_bits(qwin[0, h * G:(h + 1) * G].reshape(-1, 128), state_k[0, h], state_v[0, h],
+                                    pos[0, h], budget_k=K, buffer_b=B, seed=0, layer=0, seq=0, head=h,
+                                    num_kv_heads=wl.num_kv_heads, rnd=rnd)
+            gu = PU.unit_slice(got, 0, h, wl.num_kv_heads)
+            PU.check_unit(wl, ref, gu, state_k[0, h], state_v[0, h], pos[0, h], variant="attnv", n_v=K // 4)
+            same &= np.array_equal(gu["src"], ref["src"])
+            state_k[0, h, :K] = ref["k_bits_new"]
+            state_v[0, h, :K] = ref["v_bits_new"]
+            pos[0, h, :K] = ref["positions_new"]
+        compared += 1
+        if not same:
+            break
+        nxt = W.stream_chunk(wl, 11, 0, N + rnd * B, B)
+        cache.append(0, *(PU.bits_to_bf16_tensor(nxt[x], dev) for x in ("q_bits", "k_bits", "v_bits")))
+        state_k[:, :, K:] = nxt["k_bits"].transpose(1, 2, 0, 3)
+        state_v[:, :, K:] = nxt["v_bits"].transpose(1, 2, 0, 3)
+        pos[:, :, K:] = np.arange(N + rnd * B, N + (rnd + 1) * B)
+        qhist.extend(nxt["q_bits"][t] for t in range(B))
+    assert compared >= 1
+
+
+# ----------------------------------------------------------------------------- sampling law on the GPU path
+
+def _inclusion(w, m):
+    n = len(w)
+    pi = np.zeros(n)
+    for seq in itertools.permutations(range(n), m):
+        p, rest = 1.0, float(np.sum(w))
+        for i in seq:
+            p *= w[i] / rest
+            rest -= w[i]
+        for i in seq:
+            pi[i] += p
+    return pi
+
+
+def test_gpu_keep_frequencies_match_successive_sampling():
+    """64 sequences with identical content draw independent noise; 64 rounds give 4096 samples."""
+    from paper_2606_03928_gb300.vase import VaseCache, Geometry
+    K, B, nv, Wn = 7, 2, 1, 2
+    N = K + B
+    cache = VaseCache(Geometry(K, B, Wn, 1, 1, 1, 64), n_v=nv, pool_kernel=1, debug_outputs=True, seed=123)
+    rng = np.random.default_rng(8)
+    q = W.f32_to_bf16_bits(rng.standard_normal((Wn, 128)) * 0.15)
+    k = W.f32_to_bf16_bits(rng.standard_normal((N, 128)) * 1.0)
+    v = W.f32_to_bf16_bits(rng.standard_normal((N, 128)))
+    pos = np.arange(N)
+    ref = O.evict_unit_bits(q, k, v, pos, budget_k=K, buffer_b=B, n_v=nv, pool_kernel=1)
+    rv = set(ref["reserved_v"].tolist())
+    cand = [i for i in range(K) if i not in rv]
+    m = K - nv - B
+    pi = _inclusion(ref["pooled"][cand], m)
+    dev = cache.device
+    kt = PU.bits_to_bf16_tensor(np.broadcast_to(k, (64, 1, N, 128)).copy(), dev)
+    vt = PU.bits_to_bf16_tensor(np.broadcast_to(v, (64, 1, N, 128)).copy(), dev)
+    qt = PU.bits_to_bf16_tensor(np.broadcast_to(q, (64, 1, Wn, 128)).copy(), dev)
+    pt = torch.from_numpy(np.broadcast_to(pos, (64, 1, N)).astype(np.int32).copy()).to(dev)
+    counts = np.zeros(N)
+    R = 64
+    for t in range(R):
+        cache.k_cache[0].copy_(kt)
+        cache.v_cache[0].copy_(vt)
+        cache.q_window[0].copy_(qt)
+        cache.positions[0].copy_(pt)
+        cache.set_layer_state(0, N, t, N, 10 ** 6)
+        cache.evict(0)
+        src = cache.debug_view()["src"].cpu().numpy()
+        for u in range(64):
+            counts[src[u]] += 1
+    assert cache.check_device_error()[0] == 0
+    S = 64 * R
+    freq = counts[cand] / S
+    sigma = np.sqrt(pi * (1 - pi) / S)
+    assert np.all(np.abs(freq - pi) <= 4.5 * sigma + 1e-9), (freq, pi)
+    assert np.all(counts[list(rv)] == S) and np.all(counts[K:] == S)
+    w = ref["pooled"][cand]
+    assert np.all(freq >= 1 - (1 - w / w.sum()) ** m - 4.5 * sigma)
+
+
+# ----------------------------------------------------------------------------- full-size configurations
+
+def test_qwen3_1p7b_k2048_full_layer_in_bench_launch_configuration():
+    """All 64 units of one layer at full size, with the bench's launch configuration (no debug outputs)."""
+    wl = W.WORKLOADS["qwen3_1p7b_k2048"]
+    _run_layer(wl, layer=27, num_layers=28, round_index=40, debug=False)
+
+
+def test_qwen3_8b_k4096_attnv_sampled_units():
+    wl = W.WORKLOADS["qwen3_8b_k4096"]
+    units = [(0, 0), (5, 3), (17, 7), (31, 6)]
+    _run_layer(wl, layer=35, num_layers=36, round_index=90, units=units, debug=False)
+
+
+def test_qwen3_8b_k4096_dkv_sampled_units():
+    wl = W.WORKLOADS["qwen3_8b_k4096"]
+    units = [(0, 0), (9, 2), (31, 7)]
+    _run_layer(wl, variant="dkv", layer=2, num_layers=4, round_index=77, units=units, debug=False)
+
+
+def test_qwen3_32b_k8192_sampled_units():
+    wl = W.WORKLOADS["qwen3_32b_k8192"]
+    units = [(0, 0), (7, 5), (15, 7)]
+    _run_layer(wl, layer=1, num_layers=2, round_index=95, units=units, debug=True)

@@ -1,0 +1,466 @@
+#!/usr/bin/env python
+"""Throughput of the VaSE eviction step on one GB300 (or N, one process per GPU).
+
+One step = one eviction round of every layer of the workload: for each layer
+the B new decode tokens of the stream are appended (window ring + cache) and
+the layer is evicted (score, value magnitude, selection, compaction), all
+through the C ABI.  The default workload is the Qwen3-1.7B attention geometry
+(28 layers, 16/8 heads, d = 128, batch 8, K = 2048, B = 128, W = 32, an
+8192-token seeded synthetic decode stream: 48 rounds per layer, replayed
+cyclically when more steps are asked for).  Every step touches about 3.9 GB
+of cache, far more than the 129 MB L2, so no L2 flush is needed between steps.
+
+Metric: eviction-step KV token-heads per second = (layers * batch * Hkv * (K+B))
+per step / step time.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun (N > 1) every rank runs the same per-GPU workload on its own GPU
+(units are independent: no collective on the data path); value is the
+whole-job rate from the maximum step time over ranks.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "eviction-step KV tokens/sec and fraction of roofline (HBM GB/s, tensor util)"
+UNIT = "token-heads/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="qwen3_1p7b_k2048")
+    ap.add_argument("--variant", choices=["attnv", "dkv"], default="attnv")
+    ap.add_argument("--e2e-steps", type=int, default=None, help="steps of the host-buffer end-to-end pass")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------------------------- helpers
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d.get("bf16_tflops", 0.0)), "measured"
+    return FALLBACK_HBM_GBS, 1900.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples taken while the timed region runs."""
+
+    FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.file = None
+
+    def start(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", "--query-gpu=" + ",".join(self.FIELDS),
+                 "--format=csv,noheader,nounits", "-lms", "50"], stdout=self.file, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.06)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [r.split(",") for r in self.file.read().strip().splitlines() if r.strip()]
+        self.file.close()
+        os.unlink(self.file.name)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, r[5:9]):
+                if val.lower() in ("active", "1"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def kernel_bytes(kind, wl, variant, moved_rows_per_unit):
+    """Algorithmic bytes of one kernel for one layer (a launch covers up to 64 layers)."""
+    U = wl.batch * wl.num_kv_heads
+    N, K, B, d = wl.slots, wl.budget_k, wl.buffer_b, wl.head_dim
+    row = 2 * d
+    if kind == "score_attn":
+        return U * (N * row + wl.window_rows * row + N * 4)
+    if kind == "value_score":
+        return U * (K * row + K * 4)
+    if kind == "dkv_score":
+        return U * (2 * K * row + K * 4)
+    if kind == "select":
+        return U * (N * 4 + K * 4 + K * 4 + K * 4)
+    if kind == "compact":
+        return U * moved_rows_per_unit * (2 * 2 * row + 8)
+    if kind == "append":
+        return 2 * B * wl.batch * (wl.num_q_heads + 2 * wl.num_kv_heads) * row + 2 * B * U * 4
+    return 0
+
+
+def step_bytes(wl, variant):
+    """Algorithmic bytes of one layer-round of the whole step: read K and V (all N rows), write the K kept
+    rows, read the window queries (AttnV)."""
+    U = wl.batch * wl.num_kv_heads
+    d = wl.head_dim
+    q = 2 * d * wl.window_rows if variant == "attnv" else 0
+    return U * (4 * d * wl.slots + 4 * d * wl.budget_k + q)
+
+
+# ---------------------------------------------------------------------------------------------- oracle legs
+
+_WORKER = {}
+
+
+def _oracle_worker_init(name, variant, units, layer, rnd):
+    """Pool initializer: draws the sampled unit states once, so the jobs time only the oracle."""
+    from paper_2606_03928_gb300 import workloads as Wm
+    wl = Wm.WORKLOADS[name]
+    _WORKER.update(wl=wl, variant=variant, layer=layer, rnd=rnd, units=units,
+                   states=[Wm.unit_state(wl, 0, layer, s, h, rnd) for (s, h) in units])
+
+
+def _oracle_job(i):
+    from oracle import vase_oracle as O
+    wl, st = _WORKER["wl"], _WORKER["states"][i]
+    s, h = _WORKER["units"][i]
+    O.evict_unit_bits(st["q_bits"].reshape(-1, wl.head_dim), st["k_bits"], st["v_bits"], st["positions"],
+                      budget_k=wl.budget_k, buffer_b=wl.buffer_b, variant=_WORKER["variant"], seed=0,
+                      layer=_WORKER["layer"], seq=s, head=h, num_kv_heads=wl.num_kv_heads, rnd=_WORKER["rnd"])
+    return wl.slots
+
+
+def oracle_pool(wl, variant, max_units=64, layer=0, rnd=5):
+    """A spawn pool with one single-threaded oracle worker per host core, each holding the sampled units."""
+    import multiprocessing as mp
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[var] = "1"
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    units = [(s, h) for s in range(wl.batch) for h in range(wl.num_kv_heads)][:max_units]
+    pool = mp.get_context("spawn").Pool(cores, initializer=_oracle_worker_init,
+                                        initargs=(wl.name, variant, units, layer, rnd))
+    pool.map(_oracle_job, range(min(len(units), cores)))  # warm the workers
+    return pool, cores, len(units)
+
+
+def oracle_throughput(pool, n_units, wl, seconds):
+    """Evicts the sampled units with the oracle on all host cores for about `seconds`; token-heads/s."""
+    done = 0
+    t0 = time.perf_counter()
+    while True:
+        done += len(pool.map(_oracle_job, range(n_units)))
+        if time.perf_counter() - t0 >= seconds:
+            break
+    wall = time.perf_counter() - t0
+    return done * wl.slots / wall, done, wall
+
+
+# ---------------------------------------------------------------------------------------------- reference arm
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from paper_2606_03928_gb300 import workloads as Wm
+    wl = Wm.WORKLOADS[args.workload]
+    # one step = the oracle over one layer-round of the workload (all its units, at most 64)
+    pool, cores, per_step = oracle_pool(wl, args.variant)
+    units = wl.batch * wl.num_kv_heads
+
+    def step(r):
+        pool.map(_oracle_job, range(per_step))
+
+    for r in range(args.warmup):
+        step(r)
+    t0 = time.perf_counter()
+    for r in range(args.steps):
+        step(r)
+    wall = time.perf_counter() - t0
+    pool.close()
+    value = args.steps * per_step * wl.slots / wall
+    sample = f"{per_step} of the {units} units of one layer-round per step (fp64 numpy oracle, spawn pool)"
+    out = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * wall / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "variant": args.variant, "global_batch": wl.batch, "seq_len": wl.slots,
+                   "parallelism": "host cores"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out))
+    return 0
+
+
+# ---------------------------------------------------------------------------------------------- our arm
+
+def gen_stream(wl, n_tokens, gen, device, torch):
+    """Seeded synthetic decode tokens of one layer: q [n, b, Hq, d], k/v [n, b, Hkv, d] in bf16.
+
+    Keys and queries N(0, 1) (channel outliers x8 where the workload has them), values N(0, 1) with a
+    fraction of rows scaled (x20, or log-uniform x10..x50)."""
+    b, Hq, Hkv, d = wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim
+    q = torch.randn((n_tokens, b, Hq, d), generator=gen, device=device)
+    k = torch.randn((n_tokens, b, Hkv, d), generator=gen, device=device)
+    v = torch.randn((n_tokens, b, Hkv, d), generator=gen, device=device)
+    if wl.key_channel_outliers or wl.query_channel_outliers:
+        ch = torch.randperm(d, generator=torch.Generator().manual_seed(1234))[:wl.outlier_channels].to(device)
+        if wl.key_channel_outliers:
+            k[..., ch] *= wl.channel_scale
+        if wl.query_channel_outliers:
+            q[..., ch] *= wl.channel_scale
+    rows = torch.rand((n_tokens, b, Hkv, 1), generator=gen, device=device) < wl.value_outlier_rate
+    lo, hi = wl.value_outlier_scale
+    if hi > lo:
+        u = torch.rand((n_tokens, b, Hkv, 1), generator=gen, device=device)
+        scale = torch.exp(u * (torch.log(torch.tensor(hi)) - torch.log(torch.tensor(lo))) + torch.log(torch.tensor(lo)))
+    else:
+        scale = torch.full((n_tokens, b, Hkv, 1), lo, device=device)
+    v = torch.where(rows, v * scale, v)
+    return q.to(torch.bfloat16), k.to(torch.bfloat16), v.to(torch.bfloat16)
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    device = torch.device("cuda", torch.cuda.current_device())
+
+    # the oracle pool is started before the first CUDA work of this process
+    from paper_2606_03928_gb300 import workloads as Wm
+    wl = Wm.WORKLOADS[args.workload]
+    pool = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        pool, cores, n_units = oracle_pool(wl, args.variant)
+
+    from paper_2606_03928_gb300 import build as B
+    B.build()
+    from paper_2606_03928_gb300 import vase as V
+
+    L, K, Bf = wl.num_layers, wl.budget_k, wl.buffer_b
+    cache = V.VaseCache(V.Geometry(K, Bf, wl.window, wl.num_q_heads, wl.num_kv_heads, L, wl.batch),
+                        variant=args.variant, seed=0, device=device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(1000 + rank)
+    # prefill: the first K tokens of every layer (untimed)
+    for layer in range(L):
+        q, k, v = gen_stream(wl, K, gen, device, torch)
+        cache.append(layer, q, k, v)
+        del q, k, v
+    n_rounds = max(1, min(wl.rounds_per_layer, args.warmup + args.steps))
+    # per round: the B new tokens of every layer, stacked [L, B, b, H, d] for one batched append
+    chunks = []
+    for _ in range(n_rounds):
+        per_layer = [gen_stream(wl, Bf, gen, device, torch) for _ in range(L)]
+        chunks.append(tuple(torch.stack([pl[i] for pl in per_layer]) for i in range(3)))
+        del per_layer
+    torch.cuda.synchronize()
+
+    state = {"r": 0}
+
+    def step():
+        # every layer receives its B new decode tokens, then every layer is evicted (batched launches)
+        cache.append_all(*chunks[state["r"] % n_rounds])
+        cache.evict_all()
+        state["r"] += 1
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        step()
+    st, code = cache.check_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error during warm-up: {code:#x}")
+
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local if world > 1 else 0)
+    launches0 = cache.launch_count()
+    cache.profile_enable(True)
+    barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clocks = sampler.stop()
+    cache.profile_enable(False)
+    kernels = cache.profile_collect()
+    launches = cache.launch_count() - launches0
+    ms = ev0.elapsed_time(ev1) / args.steps
+    st, code = cache.check_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error in the timed region: {code:#x}")
+    if world > 1:
+        t = torch.tensor([ms], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    token_heads = L * wl.batch * wl.num_kv_heads * wl.slots
+    value = world * token_heads / (ms / 1e3)
+
+    # moved rows per unit in the last eviction (rows whose slot changes) for the compaction's bytes
+    src = cache.debug_view(0)["src"].cpu()
+    moved = float((src != torch.arange(K, dtype=torch.int32)).sum().item()) / src.shape[0]
+
+    # ---- end to end through the C ABI with host buffers: pinned host inputs, host-side kept positions
+    e2e_steps = args.e2e_steps if args.e2e_steps is not None else max(1, min(args.steps, 50))
+    n_host = min(n_rounds, 4)
+    host_chunks = [[tuple(x[layer].cpu().pin_memory() for x in chunks[r]) for layer in range(L)]
+                   for r in range(n_host)]
+    pos_out = [torch.empty((wl.batch, wl.num_kv_heads, K), dtype=torch.int32).pin_memory() for _ in range(L)]
+    h2d = sum(x.numel() * x.element_size() for x in host_chunks[0][0]) * L
+    d2h = sum(p.numel() * p.element_size() for p in pos_out)
+
+    def e2e_step(r):
+        c = host_chunks[r % n_host]
+        for layer in range(L):
+            cache.append_host(layer, *c[layer])
+        cache.evict_all()
+        for layer in range(L):
+            cache.read_positions(layer, pos_out[layer])
+
+    e2e_step(0)
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for r in range(e2e_steps):
+        e2e_step(r)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    if world > 1:
+        t = torch.tensor([e2e_ms], device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e_value = world * token_heads / (e2e_ms / 1e3)
+
+    # ---- roofline of the dominant kernel
+    hbm_peak, _, peak_kind = measured_peaks()
+    per_kernel = {}
+    total_k = sum(v[0] for v in kernels.values()) or 1.0
+    layers_per_launch = min(L, 64)
+    for name, (kms, n) in kernels.items():
+        if n == 0:
+            continue
+        per_launch = kms / n
+        b = kernel_bytes(name, wl, args.variant, moved) * layers_per_launch
+        per_kernel[name] = {"launches": n, "us_per_launch": round(1e3 * per_launch, 3),
+                            "share": round(kms / total_k, 4),
+                            "gbs": round(b / (per_launch / 1e3) / 1e9, 1)}
+    dom = max(per_kernel, key=lambda k: per_kernel[k]["share"])
+    dom_bytes = kernel_bytes(dom, wl, args.variant, moved) * layers_per_launch
+    achieved = per_kernel[dom]["gbs"]
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        try:
+            from paper_2606_03928_gb300.build import _digest
+            with open(tpath) as f:
+                tr = json.load(f)
+            ent = tr.get(f"{dom}:{wl.name}:{args.variant}")
+            if ent and ent.get("source_digest") == _digest():
+                traffic = ent["bytes_per_launch"]
+        except Exception:
+            traffic = None
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                "frac": round(achieved / hbm_peak, 4), "traffic": traffic, "kernel": dom,
+                "algorithmic_bytes_per_launch": dom_bytes, "peak_source": peak_kind}
+    step_roof_ms = L * step_bytes(wl, args.variant) / (hbm_peak * 1e9) * 1e3
+    evict_ms = sum(kernels[k][0] for k in kernels if k != "append") / args.steps
+
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "variant": args.variant, "layers": L, "global_batch": wl.batch * world,
+                   "seq_len": wl.slots, "budget_k": K, "buffer_b": Bf, "window": wl.window,
+                   "heads": f"{wl.num_q_heads}/{wl.num_kv_heads}", "parallelism": f"dp{world}",
+                   "l2": "inputs larger than L2 (about 3.9 GB touched per step)"},
+        "roofline": roofline,
+        "step_roofline": {"ms_per_step_at_hbm_peak": round(step_roof_ms, 4),
+                          "frac": round(step_roof_ms / ms, 4),
+                          "amortised_us_per_decode_token": round(1e3 * evict_ms / Bf, 3)},
+        "kernels": per_kernel,
+        "clocks": clocks,
+        "gpu_launches": launches,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_ms},
+    }
+    if pool is not None:
+        v, done, wall = oracle_throughput(pool, n_units, wl, args.cpu_seconds)
+        pool.close()
+        out["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+                               "sample": f"{done} units of one layer-round ({wall:.1f} s on {cores} host cores)"}
+    if rank == 0:
+        print(json.dumps(out))
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -36,7 +36,7 @@
 extern "C" {
 #endif
 
-#define VASE_ABI_VERSION 1
+#define VASE_ABI_VERSION 2
 
 #define VASE_OK 0
 #define VASE_EVICT_DUE 1          /* the layer's cache is full: call vase_evict before the next append */
@@ -81,6 +81,7 @@ typedef struct vase_buffer_sizes {
     size_t v_cache;    /* bf16 [L][b][Hkv][K+B][d] */
     size_t q_window;   /* bf16 [L][b][Hq][W][d], a ring over the last W decode queries */
     size_t positions;  /* int32 [L][b][Hkv][K+B], absolute stream position of each slot, -1 if empty */
+    size_t value_scores; /* fp32 [L][b][Hkv][K+B], value magnitude of the token in each slot */
     size_t workspace;  /* scratch for one eviction at a time plus the host-append staging area */
 } vase_buffer_sizes;
 
@@ -89,6 +90,7 @@ typedef struct vase_buffers {
     void* v_cache;     /* device */
     void* q_window;    /* device */
     int32_t* positions;/* device */
+    float* value_scores; /* device; filled by the appends, moved by the evictions */
     void* workspace;   /* device; contents are the library's between calls */
 } vase_buffers;
 
@@ -105,12 +107,14 @@ typedef struct vase_kv_view {
     void* k;               /* device, bf16; row (s, h, slot) at k + ((s*Hkv + h)*unit_stride + slot)*d */
     void* v;
     int32_t* positions;
+    float* value_scores;   /* per slot, same layout as positions */
     int64_t unit_stride;   /* elements between consecutive (s, h) units = (K+B)*d */
     int32_t slots;         /* K + B */
     int32_t fill;          /* valid slots 0..fill-1, in stream order */
 } vase_kv_view;
 
-/* Device pointers to the workspace results of the most recent vase_evict (valid until the next call). */
+/* Device pointers to the workspace results of one layer of the most recent eviction call
+ * (valid until the next one).  Slot z is the z-th layer that call evicted (0 for vase_evict). */
 typedef struct vase_debug_view {
     float* attn;           /* [b*Hkv][K+B] window score before pooling (AttnV) */
     float* pooled;         /* [b*Hkv][K+B] pooled score (AttnV, debug_outputs) */
@@ -120,6 +124,7 @@ typedef struct vase_debug_view {
     int32_t* src;          /* [b*Hkv][K] ascending kept slots: new slot j holds old slot src[j] */
     int32_t units;         /* b*Hkv */
     int32_t slots;         /* K + B */
+    int32_t layer;         /* the layer whose eviction these are, -1 if the slot was not used */
 } vase_debug_view;
 
 typedef struct vase_ctx vase_ctx;
@@ -148,6 +153,10 @@ void vase_destroy(vase_ctx* ctx);
 int vase_append(vase_ctx* ctx, int32_t layer, const void* q, const void* k, const void* v,
                 int32_t n_tokens, void* stream);
 
+/* vase_append for every layer at once, in one launch: q [L][n_tokens][b][Hq][d],
+ * k and v [L][n_tokens][b][Hkv][d] (device, bf16).  All layers must have room. */
+int vase_append_all(vase_ctx* ctx, const void* q, const void* k, const void* v, int32_t n_tokens, void* stream);
+
 /* Same as vase_append with HOST inputs (pinned memory gives asynchronous copies):
  * the library copies them into its staging area in the workspace (at most B
  * tokens per call) and appends from there. */
@@ -159,6 +168,18 @@ int vase_append_host(vase_ctx* ctx, int32_t layer, const void* q_host, const voi
  * order and positions of slots K..K+B-1 are -1. */
 int vase_evict(vase_ctx* ctx, int32_t layer, void* stream);
 
+/* The eviction step of every full layer (all layers fill at the same decode step), batched:
+ * each kernel covers up to 64 layers per launch.  Returns the number of layers evicted (>= 0)
+ * or a negative error. */
+int vase_evict_all(vase_ctx* ctx, void* stream);
+
+/* The value magnitude (Range, L2 or Var of the value row, Eq. (5) / App. A) of every cached
+ * token is computed once, by the append that writes the row, and kept per slot in
+ * value_scores; the AttnV eviction reads it instead of the V cache.  A caller that writes
+ * V rows directly (restoring a checkpoint, say) recomputes slots 0..fill-1 of one layer
+ * with this call. */
+int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream);
+
 /* Copies the K positions of every unit of one layer to host memory
  * (int32 [b][Hkv][K]), enqueued on the stream; the host buffer is valid after
  * the stream completes. */
@@ -169,7 +190,7 @@ int vase_get_layer_state(const vase_ctx* ctx, int32_t layer, vase_layer_state* o
 int vase_set_layer_state(vase_ctx* ctx, int32_t layer, const vase_layer_state* st);
 
 int vase_kv_view_get(const vase_ctx* ctx, int32_t layer, vase_kv_view* out);
-int vase_debug_view_get(const vase_ctx* ctx, vase_debug_view* out);
+int vase_debug_view_get(const vase_ctx* ctx, int32_t slot, vase_debug_view* out);
 
 /* Synchronises the stream, then reads and clears the device error word that
  * bounded waits and device-side checks set.  Returns VASE_OK or VASE_ERR_DEVICE
@@ -182,7 +203,7 @@ int64_t vase_launch_count(const vase_ctx* ctx);
 /* Kernel kinds reported by vase_profile_collect. */
 #define VASE_KERNEL_APPEND 0
 #define VASE_KERNEL_SCORE 1   /* window attention score (tcgen05) */
-#define VASE_KERNEL_VALUE 2   /* value magnitude */
+#define VASE_KERNEL_VALUE 2   /* value magnitude refresh (vase_refresh_value_scores) */
 #define VASE_KERNEL_DKV 3     /* DKV leverage scores (tcgen05) */
 #define VASE_KERNEL_SELECT 4  /* reservation + sampling + kept list */
 #define VASE_KERNEL_COMPACT 5 /* stable in-place gather */
@@ -199,6 +220,8 @@ int vase_profile_enable(vase_ctx* ctx, int enable);
 int vase_profile_collect(vase_ctx* ctx, double* total_ms, int64_t* launches);
 
 const char* vase_status_string(int status);
+/* Message of the last failed call on ctx; with ctx == NULL, the reason the last
+ * configuration check on this thread (vase_get_buffer_sizes, vase_create) failed. */
 const char* vase_last_error(const vase_ctx* ctx);
 int vase_abi_version(void);
 

@@ -2,6 +2,7 @@
 // launch plans, TMA descriptors, per-layer counters and stream-ordered
 // launches of the eviction-step kernels.
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -20,14 +21,21 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
 struct Plan {
-    int N, units, G, GW, GWp, NB, n_rb, n_tiles, cluster, tiles_per_cta, stages, tmem_cols, n_v, m;
+    int N, units, G, GW, GWp, NB, n_rb, n_rbA, rep, q_rows, q_box, buf_cols, nbuf;
+    int n_tiles, cluster, stages, tmem_cols, n_v, m;
+    int cluster_for[kMaxLayerBatch + 1];  // CTAs per unit of the score kernel, by layers per launch
     size_t score_smem;
     int dkv_tiles_k, dkv_tiles_per_cta, dkv_stages;
     size_t dkv_smem;
     size_t select_smem;
     // workspace
+    int slots;  // layers one launch can batch
+    size_t stride_attn, stride_un, stride_src;  // elements per workspace slot
     size_t off_err, off_attn, off_pooled, off_vscore, off_key, off_keep, off_src, off_staging, staging_bytes, ws_bytes;
 };
+
+// Reason of the last failed configuration check on this thread (vase_last_error(NULL)).
+thread_local std::string g_config_error;
 
 const char* check_config(const vase_config* c) {
     if (!c) return "null config";
@@ -47,9 +55,16 @@ const char* check_config(const vase_config* c) {
     return nullptr;
 }
 
+bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why);
+
 bool make_plan(const vase_config* c, int num_sms, Plan* P, const char** why) {
     *why = check_config(c);
-    if (*why) return false;
+    if (!*why) make_plan_impl(c, num_sms, P, why);
+    g_config_error = *why ? *why : "";
+    return *why == nullptr;
+}
+
+bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why) {
     Plan& p = *P;
     p.N = c->budget_k + c->buffer_b;
     p.units = c->batch * c->num_kv_heads;
@@ -62,41 +77,60 @@ bool make_plan(const vase_config* c, int num_sms, Plan* P, const char** why) {
     p.GWp = p.GW <= 256 ? (p.GW + 31) / 32 * 32 : (p.GW + 255) / 256 * 256;
     p.NB = p.GWp < 256 ? p.GWp : 256;
     p.n_rb = p.GWp / p.NB;
+    if (p.GWp <= 64) {  // replicate short windows across the 128 pass-A lanes
+        p.rep = 128 / p.GWp;
+        p.n_rbA = 1;
+        p.q_rows = 128;
+        p.q_box = p.GWp;
+    } else {
+        p.rep = 1;
+        p.n_rbA = ceil_div(p.GWp, 128);
+        p.q_rows = 128 * p.n_rbA;
+        p.q_box = p.q_rows < 256 ? p.q_rows : 256;
+    }
+    p.buf_cols = p.NB > 128 ? p.NB : 128;
+    p.nbuf = 512 / p.buf_cols >= 4 ? 4 : 2;
     p.n_tiles = ceil_div(p.N, kTileTokens);
     p.n_v = c->n_v < 0 ? c->budget_k / 4 : c->n_v;
     p.m = c->variant == VASE_VARIANT_ATTNV ? c->budget_k - p.n_v - c->buffer_b : c->budget_k - c->buffer_b;
-    int tc = 2 * p.NB;
     p.tmem_cols = 32;
-    while (p.tmem_cols < tc) p.tmem_cols *= 2;
+    while (p.tmem_cols < p.nbuf * p.buf_cols) p.tmem_cols *= 2;
 
-    // cluster size: minimise waves x (tiles per CTA + 1)
-    int best_c = 1;
-    long best_cost = -1;
-    for (int C = 1; C <= 16 && C <= p.n_tiles; ++C) {
-        const int T = ceil_div(p.n_tiles, C);
-        if (ceil_div(p.n_tiles, T) != C) continue;
-        const long ctas = static_cast<long>(p.units) * C;
-        const long waves = (ctas + num_sms - 1) / num_sms;
-        const long cost = waves * (T + 1);
-        if (best_cost < 0 || cost < best_cost) {
-            best_cost = cost;
-            best_c = C;
+    // cluster size per number of layers in a launch: minimise waves x (tiles per CTA + 1)
+    // among the sizes whose shared memory fits with two stages
+    const int max_batch = c->num_layers < kMaxLayerBatch ? c->num_layers : kMaxLayerBatch;
+    int c_max = 0;
+    for (int nz = 1; nz <= kMaxLayerBatch; ++nz) {
+        int best_c = 0;
+        long best_cost = -1;
+        for (int C = 1; C <= 16 && C <= p.n_tiles; ++C) {
+            const int T = ceil_div(p.n_tiles, C);
+            if (ceil_div(p.n_tiles, T) != C) continue;
+            if (score_attn_smem_bytes(p.q_rows, p.n_rbA, p.GWp, C, 2) > kMaxDynSmem) continue;
+            const long ctas = static_cast<long>(p.units) * C * nz;
+            const long waves = (ctas + num_sms - 1) / num_sms;
+            const long cost = waves * (T + 1);
+            if (best_cost < 0 || cost < best_cost) {
+                best_cost = cost;
+                best_c = C;
+            }
         }
+        if (!best_c) {
+            *why = "window rows do not fit in shared memory";
+            return false;
+        }
+        p.cluster_for[nz] = best_c;
+        if (nz <= max_batch && best_c > c_max) c_max = best_c;
     }
-    p.cluster = best_c;
-    p.tiles_per_cta = ceil_div(p.n_tiles, best_c);
+    p.cluster = c_max;  // shared memory is sized for the largest cluster used
     p.stages = 0;
-    for (int s = 4; s >= 2; --s) {
-        if (score_attn_smem_bytes(p.GWp, p.cluster, s) <= kMaxDynSmem) {
+    for (int s = 6; s >= 2; --s) {
+        if (score_attn_smem_bytes(p.q_rows, p.n_rbA, p.GWp, p.cluster, s) <= kMaxDynSmem) {
             p.stages = s;
             break;
         }
     }
-    if (!p.stages) {
-        *why = "window rows do not fit in shared memory";
-        return false;
-    }
-    p.score_smem = score_attn_smem_bytes(p.GWp, p.cluster, p.stages);
+    p.score_smem = score_attn_smem_bytes(p.q_rows, p.n_rbA, p.GWp, p.cluster, p.stages);
     if (p.tmem_cols > 256 && p.score_smem < 120 * 1024) p.score_smem = 120 * 1024;  // one CTA per SM owns TMEM
 
     p.dkv_tiles_k = ceil_div(c->budget_k, kTileTokens);
@@ -119,27 +153,33 @@ bool make_plan(const vase_config* c, int num_sms, Plan* P, const char** why) {
     p.dkv_stages = 3;
     p.dkv_smem = dkv_smem_bytes(p.dkv_stages);
     p.select_smem = select_smem_bytes(p.N, c->budget_k);
-    if (p.select_smem > kMaxDynSmem - 4096) {
+    if (p.select_smem > kMaxDynSmem - 9216) {
         *why = "K + B too large for the single-CTA selection (about 25k slots at most)";
         return false;
     }
 
+    // workspace: one slot of per-eviction arrays per layer a launch can batch
+    p.slots = c->num_layers < kMaxLayerBatch ? c->num_layers : kMaxLayerBatch;
     const size_t un = static_cast<size_t>(p.units) * p.N;
+    p.stride_attn = un * p.n_rb;
+    p.stride_un = un;
+    p.stride_src = static_cast<size_t>(p.units) * c->budget_k;
+    const size_t Z = static_cast<size_t>(p.slots);
     size_t o = 0;
     p.off_err = o;
     o += kAlign;
     p.off_attn = o;
-    o = align_up(o + un * 4, kAlign);
+    o = align_up(o + Z * p.stride_attn * 4, kAlign);  // one part per pass-B row block
     p.off_pooled = o;
-    o = align_up(o + un * 4, kAlign);
+    o = align_up(o + Z * un * 4, kAlign);
     p.off_vscore = o;
-    o = align_up(o + un * 4, kAlign);
+    o = align_up(o + Z * un * 4, kAlign);
     p.off_key = o;
-    o = align_up(o + un * 4, kAlign);
+    o = align_up(o + Z * un * 4, kAlign);
     p.off_keep = o;
-    o = align_up(o + un, kAlign);
+    o = align_up(o + Z * un, kAlign);
     p.off_src = o;
-    o = align_up(o + static_cast<size_t>(p.units) * c->budget_k * 4, kAlign);
+    o = align_up(o + Z * p.stride_src * 4, kAlign);
     p.off_staging = o;
     p.staging_bytes = static_cast<size_t>(c->buffer_b) * c->batch * (c->num_q_heads + 2 * c->num_kv_heads) * kRowBytes;
     o = align_up(o + p.staging_bytes, kAlign);
@@ -161,6 +201,7 @@ struct vase_ctx {
     int num_sms = 0;
     CUtensorMap kmap, vmap, qmap;
     std::vector<vase_layer_state> layers;
+    std::vector<int32_t> last_batch;  // layers of the most recent eviction launch, by workspace slot
     int64_t launches = 0;
     std::string last_error;
     uint8_t* ws = nullptr;
@@ -273,6 +314,7 @@ int vase_get_buffer_sizes(const vase_config* cfg, vase_buffer_sizes* out) {
     out->v_cache = rows * kRowBytes;
     out->q_window = static_cast<size_t>(cfg->num_layers) * cfg->batch * cfg->num_q_heads * cfg->window * kRowBytes;
     out->positions = rows * 4;
+    out->value_scores = rows * 4;
     out->workspace = p.ws_bytes;
     return VASE_OK;
 }
@@ -298,7 +340,8 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
         delete ctx;
         return cfg->head_dim != 128 ? VASE_ERR_UNSUPPORTED : VASE_ERR_INVALID;
     }
-    const void* ptrs[5] = {bufs->k_cache, bufs->v_cache, bufs->q_window, bufs->positions, bufs->workspace};
+    const void* ptrs[6] = {bufs->k_cache, bufs->v_cache, bufs->q_window, bufs->positions, bufs->value_scores,
+                           bufs->workspace};
     for (const void* p : ptrs) {
         if (!p || !aligned(p, kAlign)) {
             fprintf(stderr, "vase_create: null or unaligned buffer (256-byte alignment required)\n");
@@ -324,7 +367,7 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
         delete ctx;
         return VASE_ERR_UNSUPPORTED;
     }
-    const uint32_t qbox = static_cast<uint32_t>(P.GWp < 256 ? P.GWp : 256);
+    const uint32_t qbox = static_cast<uint32_t>(P.q_box);
     if (!encode_rows(enc, &ctx->kmap, bufs->k_cache, cache_rows, kTileTokens) ||
         !encode_rows(enc, &ctx->vmap, bufs->v_cache, cache_rows, kTileTokens) ||
         !encode_rows(enc, &ctx->qmap, bufs->q_window, q_rows, qbox)) {
@@ -334,7 +377,7 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
     }
     if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
         (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess ||
-        (e = select_set_attributes(P.select_smem)) != cudaSuccess) {
+        (e = select_set_attributes(P.select_smem)) != cudaSuccess || (e = compact_set_attributes()) != cudaSuccess) {
         fprintf(stderr, "vase_create: kernel attributes: %s\n", cudaGetErrorString(e));
         delete ctx;
         return VASE_ERR_CUDA;
@@ -351,39 +394,201 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
 
 void vase_destroy(vase_ctx* ctx) { delete ctx; }
 
+namespace {
+
+// Appends n_tokens to each layer of `layers` (inputs stacked per layer slot) in one launch.
+int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void* q, const void* k, const void* v,
+                 int32_t n_tokens, cudaStream_t stream) {
+    if (n_tokens < 1) return fail(ctx, VASE_ERR_INVALID, "n_tokens must be >= 1");
+    if (!q || !k || !v) return fail(ctx, VASE_ERR_INVALID, "null input");
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16))
+        return fail(ctx, VASE_ERR_ALIGN, "inputs must be 16-byte aligned");
+    for (int z = 0; z < n_layers; ++z)
+        if (ctx->layers[layers[z]].fill + n_tokens > ctx->plan.N)
+            return fail(ctx, VASE_ERR_FULL, "append would exceed K + B slots");
+    const vase_config& c = ctx->cfg;
+    const size_t q_slot = static_cast<size_t>(n_tokens) * c.batch * c.num_q_heads * kVecPerRow;
+    const size_t kv_slot = static_cast<size_t>(n_tokens) * c.batch * c.num_kv_heads * kVecPerRow;
+    for (int z0 = 0; z0 < n_layers; z0 += kMaxLayerBatch) {
+        const int nz = n_layers - z0 < kMaxLayerBatch ? n_layers - z0 : kMaxLayerBatch;
+        AppendParams p;
+        p.q = static_cast<const uint4*>(q) + z0 * q_slot;
+        p.k = static_cast<const uint4*>(k) + z0 * kv_slot;
+        p.v = static_cast<const uint4*>(v) + z0 * kv_slot;
+        p.qwin = static_cast<uint4*>(ctx->bufs.q_window);
+        p.kc = static_cast<uint4*>(ctx->bufs.k_cache);
+        p.vc = static_cast<uint4*>(ctx->bufs.v_cache);
+        p.pos = ctx->bufs.positions;
+        p.vmag = ctx->bufs.value_scores;
+        p.kind = c.value_score;
+        p.n = n_tokens;
+        p.b = c.batch;
+        p.Hq = c.num_q_heads;
+        p.Hkv = c.num_kv_heads;
+        p.W = c.window;
+        p.N = ctx->plan.N;
+        for (int z = 0; z < nz; ++z) {
+            const vase_layer_state& st = ctx->layers[layers[z0 + z]];
+            p.layer[z] = layers[z0 + z];
+            p.fill[z] = st.fill;
+            p.next_pos[z] = st.next_position;
+            p.q_seen[z] = st.queries_seen;
+        }
+        cudaError_t e = timed_launch(ctx, VASE_KERNEL_APPEND, stream, [&] { return launch_append(p, nz, stream); });
+        if (e != cudaSuccess) return cuda_fail(ctx, e, "append launch");
+        ctx->launches += 1;
+    }
+    bool due = false;
+    for (int z = 0; z < n_layers; ++z) {
+        vase_layer_state& st = ctx->layers[layers[z]];
+        st.fill += n_tokens;
+        st.next_position += n_tokens;
+        st.queries_seen += n_tokens;
+        due |= st.fill == ctx->plan.N;
+    }
+    return due ? VASE_EVICT_DUE : VASE_OK;
+}
+
+LayerBatch make_batch(vase_ctx* ctx, const int32_t* layers, int nz) {
+    LayerBatch b;
+    b.n = nz;
+    for (int z = 0; z < nz; ++z) {
+        b.layer[z] = layers[z];
+        b.rnd[z] = ctx->layers[layers[z]].round;
+    }
+    return b;
+}
+
+// One eviction step for up to kMaxLayerBatch full layers: every kernel covers all of them in one launch.
+int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
+    const Plan& P = ctx->plan;
+    const vase_config& c = ctx->cfg;
+    const LayerBatch batch = make_batch(ctx, layers, nz);
+    uint32_t* err = reinterpret_cast<uint32_t*>(ctx->ws + P.off_err);
+    float* attn = reinterpret_cast<float*>(ctx->ws + P.off_attn);
+    float* vscore = reinterpret_cast<float*>(ctx->ws + P.off_vscore);
+    int32_t* src = reinterpret_cast<int32_t*>(ctx->ws + P.off_src);
+    cudaError_t e;
+    if (c.variant == VASE_VARIANT_ATTNV) {
+        ScoreAttnParams sp;
+        sp.batch = batch;
+        sp.N = P.N;
+        sp.GW = P.GW;
+        sp.GWp = P.GWp;
+        sp.NB = P.NB;
+        sp.n_rb = P.n_rb;
+        sp.n_rbA = P.n_rbA;
+        sp.rep = P.rep;
+        sp.q_rows = P.q_rows;
+        sp.q_box = P.q_box;
+        sp.n_tiles = P.n_tiles;
+        sp.cluster = P.cluster_for[nz];
+        sp.tiles_per_cta = ceil_div(P.n_tiles, sp.cluster);
+        sp.stages = P.stages;
+        sp.buf_cols = P.buf_cols;
+        sp.nbuf = P.nbuf;
+        sp.units = P.units;
+        sp.tmem_cols = P.tmem_cols;
+        sp.Hq = c.num_q_heads;
+        sp.Hkv = c.num_kv_heads;
+        sp.W = c.window;
+        sp.G = P.G;
+        sp.layer_rows = static_cast<int64_t>(P.units) * P.N;
+        sp.q_layer_rows = static_cast<int64_t>(c.batch) * c.num_q_heads * c.window;
+        sp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
+        sp.inv_gw = 1.0f / static_cast<float>(P.GW);
+        sp.attn = attn;
+        sp.err = err;
+        if ((e = timed_launch(ctx, VASE_KERNEL_SCORE, s, [&] {
+                 return launch_score_attn(ctx->kmap, ctx->qmap, sp, P.units, P.score_smem, s);
+             })) != cudaSuccess)
+            return cuda_fail(ctx, e, "score launch");
+        ctx->launches += 1;
+    } else {
+        DkvParams dp;
+        dp.batch = batch;
+        dp.N = P.N;
+        dp.K = c.budget_k;
+        dp.r = c.dkv_rank;
+        dp.Hkv = c.num_kv_heads;
+        dp.fixed_g = c.dkv_fixed_g;
+        dp.units = P.units;
+        dp.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
+        dp.seed_hi = static_cast<uint32_t>(c.seed >> 32);
+        dp.n_tiles_k = P.dkv_tiles_k;
+        dp.tiles_per_cta = P.dkv_tiles_per_cta;
+        dp.stages = P.dkv_stages;
+        dp.layer_rows = static_cast<int64_t>(P.units) * P.N;
+        dp.out = vscore;
+        dp.err = err;
+        if ((e = timed_launch(ctx, VASE_KERNEL_DKV, s, [&] {
+                 return launch_dkv(ctx->kmap, ctx->vmap, dp, P.units, P.dkv_smem, s);
+             })) != cudaSuccess)
+            return cuda_fail(ctx, e, "dkv launch");
+        ctx->launches += 1;
+    }
+    SelectParams sel;
+    sel.batch = batch;
+    sel.attn = attn;
+    sel.dkv = vscore;
+    sel.vmag = ctx->bufs.value_scores;
+    sel.vscore_dbg = (c.debug_outputs && c.variant == VASE_VARIANT_ATTNV) ? vscore : nullptr;
+    sel.pos = ctx->bufs.positions;
+    sel.src = src;
+    sel.pooled_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_pooled) : nullptr;
+    sel.key_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_key) : nullptr;
+    sel.keep_dbg = c.debug_outputs ? ctx->ws + P.off_keep : nullptr;
+    sel.N = P.N;
+    sel.K = c.budget_k;
+    sel.B = c.buffer_b;
+    sel.n_v = P.n_v;
+    sel.m = P.m;
+    sel.pool = c.pool_kernel;
+    sel.variant = c.variant;
+    sel.stochastic = c.stochastic;
+    sel.Hkv = c.num_kv_heads;
+    sel.n_parts = c.variant == VASE_VARIANT_ATTNV ? P.n_rb : 1;
+    sel.units = P.units;
+    sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
+    sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
+    sel.err = err;
+    if ((e = timed_launch(ctx, VASE_KERNEL_SELECT, s, [&] { return launch_select(sel, P.units, P.select_smem, s); })) !=
+        cudaSuccess)
+        return cuda_fail(ctx, e, "select launch");
+    CompactParams cp;
+    cp.batch = batch;
+    cp.kc = static_cast<uint4*>(ctx->bufs.k_cache);
+    cp.vc = static_cast<uint4*>(ctx->bufs.v_cache);
+    cp.src = src;
+    cp.N = P.N;
+    cp.K = c.budget_k;
+    cp.units = P.units;
+    cp.err = err;
+    if ((e = timed_launch(ctx, VASE_KERNEL_COMPACT, s, [&] { return launch_compact(cp, P.units, s); })) != cudaSuccess)
+        return cuda_fail(ctx, e, "compact launch");
+    ctx->launches += 2;
+    for (int z = 0; z < nz; ++z) {
+        vase_layer_state& st = ctx->layers[layers[z]];
+        st.fill = c.budget_k;
+        st.round += 1;
+    }
+    return VASE_OK;
+}
+
+}  // namespace
+
 int vase_append(vase_ctx* ctx, int32_t layer, const void* q, const void* k, const void* v, int32_t n_tokens,
                 void* stream) {
     if (!ctx) return VASE_ERR_INVALID;
     if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
-    if (n_tokens < 1) return fail(ctx, VASE_ERR_INVALID, "n_tokens must be >= 1");
-    if (!q || !k || !v) return fail(ctx, VASE_ERR_INVALID, "null input");
-    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16)) return fail(ctx, VASE_ERR_ALIGN, "inputs must be 16-byte aligned");
-    vase_layer_state& st = ctx->layers[layer];
-    if (st.fill + n_tokens > ctx->plan.N) return fail(ctx, VASE_ERR_FULL, "append would exceed K + B slots");
-    AppendParams p;
-    p.q = static_cast<const uint4*>(q);
-    p.k = static_cast<const uint4*>(k);
-    p.v = static_cast<const uint4*>(v);
-    p.qwin = q_layer(ctx, layer);
-    p.kc = kc_layer(ctx, layer);
-    p.vc = vc_layer(ctx, layer);
-    p.pos = pos_layer(ctx, layer);
-    p.n = n_tokens;
-    p.b = ctx->cfg.batch;
-    p.Hq = ctx->cfg.num_q_heads;
-    p.Hkv = ctx->cfg.num_kv_heads;
-    p.W = ctx->cfg.window;
-    p.N = ctx->plan.N;
-    p.fill = st.fill;
-    p.next_pos = st.next_position;
-    p.q_seen = st.queries_seen;
-    cudaError_t e = timed_launch(ctx, VASE_KERNEL_APPEND, static_cast<cudaStream_t>(stream), [&] { return launch_append(p, static_cast<cudaStream_t>(stream)); });
-    if (e != cudaSuccess) return cuda_fail(ctx, e, "append launch");
-    ctx->launches += 1;
-    st.fill += n_tokens;
-    st.next_position += n_tokens;
-    st.queries_seen += n_tokens;
-    return st.fill == ctx->plan.N ? VASE_EVICT_DUE : VASE_OK;
+    return append_batch(ctx, &layer, 1, q, k, v, n_tokens, static_cast<cudaStream_t>(stream));
+}
+
+int vase_append_all(vase_ctx* ctx, const void* q, const void* k, const void* v, int32_t n_tokens, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    std::vector<int32_t> all(static_cast<size_t>(ctx->cfg.num_layers));
+    for (int32_t l = 0; l < ctx->cfg.num_layers; ++l) all[l] = l;
+    return append_batch(ctx, all.data(), ctx->cfg.num_layers, q, k, v, n_tokens, static_cast<cudaStream_t>(stream));
 }
 
 int vase_append_host(vase_ctx* ctx, int32_t layer, const void* q_host, const void* k_host, const void* v_host,
@@ -411,106 +616,45 @@ int vase_append_host(vase_ctx* ctx, int32_t layer, const void* q_host, const voi
 int vase_evict(vase_ctx* ctx, int32_t layer, void* stream) {
     if (!ctx) return VASE_ERR_INVALID;
     if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
-    vase_layer_state& st = ctx->layers[layer];
-    const Plan& P = ctx->plan;
-    const vase_config& c = ctx->cfg;
-    if (st.fill != P.N) return fail(ctx, VASE_ERR_NOT_FULL, "evict needs a full cache (fill == K + B)");
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    uint32_t* err = reinterpret_cast<uint32_t*>(ctx->ws + P.off_err);
-    float* attn = reinterpret_cast<float*>(ctx->ws + P.off_attn);
-    float* vscore = reinterpret_cast<float*>(ctx->ws + P.off_vscore);
-    int32_t* src = reinterpret_cast<int32_t*>(ctx->ws + P.off_src);
-    const int64_t cache_row0 = static_cast<int64_t>(layer) * P.units * P.N;
-    cudaError_t e;
-    if (c.variant == VASE_VARIANT_ATTNV) {
-        ScoreAttnParams sp;
-        sp.N = P.N;
-        sp.GW = P.GW;
-        sp.GWp = P.GWp;
-        sp.NB = P.NB;
-        sp.n_rb = P.n_rb;
-        sp.n_tiles = P.n_tiles;
-        sp.tiles_per_cta = P.tiles_per_cta;
-        sp.cluster = P.cluster;
-        sp.stages = P.stages;
-        sp.tmem_cols = P.tmem_cols;
-        sp.Hq = c.num_q_heads;
-        sp.Hkv = c.num_kv_heads;
-        sp.W = c.window;
-        sp.G = P.G;
-        sp.k_row0 = cache_row0;
-        sp.q_row0 = static_cast<int64_t>(layer) * c.batch * c.num_q_heads * c.window;
-        sp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
-        sp.inv_gw = 1.0f / static_cast<float>(P.GW);
-        sp.attn = attn;
-        sp.err = err;
-        if ((e = timed_launch(ctx, VASE_KERNEL_SCORE, s, [&] { return launch_score_attn(ctx->kmap, ctx->qmap, sp, P.units, P.score_smem, s); })) != cudaSuccess)
-            return cuda_fail(ctx, e, "score launch");
-        ValueParams vp;
-        vp.vc = vc_layer(ctx, layer);
-        vp.out = vscore;
-        vp.N = P.N;
-        vp.K = c.budget_k;
-        vp.units = P.units;
-        vp.kind = c.value_score;
-        if ((e = timed_launch(ctx, VASE_KERNEL_VALUE, s, [&] { return launch_value_score(vp, ctx->num_sms, s); })) != cudaSuccess) return cuda_fail(ctx, e, "value launch");
-        ctx->launches += 2;
-    } else {
-        DkvParams dp;
-        dp.N = P.N;
-        dp.K = c.budget_k;
-        dp.r = c.dkv_rank;
-        dp.Hkv = c.num_kv_heads;
-        dp.layer = layer;
-        dp.rnd = c.dkv_fixed_g ? 0 : st.round;
-        dp.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
-        dp.seed_hi = static_cast<uint32_t>(c.seed >> 32);
-        dp.n_tiles_k = P.dkv_tiles_k;
-        dp.tiles_per_cta = P.dkv_tiles_per_cta;
-        dp.stages = P.dkv_stages;
-        dp.row0 = cache_row0;
-        dp.out = vscore;
-        dp.lk_out = nullptr;
-        dp.lv_out = nullptr;
-        dp.err = err;
-        if ((e = timed_launch(ctx, VASE_KERNEL_DKV, s, [&] { return launch_dkv(ctx->kmap, ctx->vmap, dp, P.units, P.dkv_smem, s); })) != cudaSuccess)
-            return cuda_fail(ctx, e, "dkv launch");
-        ctx->launches += 1;
+    if (ctx->layers[layer].fill != ctx->plan.N) return fail(ctx, VASE_ERR_NOT_FULL, "evict needs a full cache (fill == K + B)");
+    const int r = evict_batch(ctx, &layer, 1, static_cast<cudaStream_t>(stream));
+    if (r == VASE_OK) ctx->last_batch.assign(1, layer);
+    return r;
+}
+
+int vase_evict_all(vase_ctx* ctx, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    std::vector<int32_t> due;
+    for (int32_t l = 0; l < ctx->cfg.num_layers; ++l)
+        if (ctx->layers[l].fill == ctx->plan.N) due.push_back(l);
+    std::vector<int32_t> done;
+    for (size_t z0 = 0; z0 < due.size(); z0 += static_cast<size_t>(ctx->plan.slots)) {
+        const int nz = static_cast<int>(due.size() - z0 < static_cast<size_t>(ctx->plan.slots) ? due.size() - z0
+                                                                                                : ctx->plan.slots);
+        const int r = evict_batch(ctx, due.data() + z0, nz, static_cast<cudaStream_t>(stream));
+        if (r != VASE_OK) return r;
+        done.assign(due.begin() + static_cast<long>(z0), due.begin() + static_cast<long>(z0) + nz);
     }
-    SelectParams sel;
-    sel.attn = attn;
-    sel.vscore = vscore;
-    sel.pos = pos_layer(ctx, layer);
-    sel.src = src;
-    sel.pooled_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_pooled) : nullptr;
-    sel.key_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_key) : nullptr;
-    sel.keep_dbg = c.debug_outputs ? ctx->ws + P.off_keep : nullptr;
-    sel.N = P.N;
-    sel.K = c.budget_k;
-    sel.B = c.buffer_b;
-    sel.n_v = P.n_v;
-    sel.m = P.m;
-    sel.pool = c.pool_kernel;
-    sel.variant = c.variant;
-    sel.stochastic = c.stochastic;
-    sel.Hkv = c.num_kv_heads;
-    sel.layer = layer;
-    sel.rnd = st.round;
-    sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
-    sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
-    sel.err = err;
-    if ((e = timed_launch(ctx, VASE_KERNEL_SELECT, s, [&] { return launch_select(sel, P.units, P.select_smem, s); })) != cudaSuccess) return cuda_fail(ctx, e, "select launch");
-    CompactParams cp;
-    cp.kc = kc_layer(ctx, layer);
-    cp.vc = vc_layer(ctx, layer);
-    cp.pos = pos_layer(ctx, layer);
-    cp.src = src;
-    cp.N = P.N;
-    cp.K = c.budget_k;
-    if ((e = timed_launch(ctx, VASE_KERNEL_COMPACT, s, [&] { return launch_compact(cp, P.units, s); })) != cudaSuccess) return cuda_fail(ctx, e, "compact launch");
-    ctx->launches += 2;
-    st.fill = c.budget_k;
-    st.round += 1;
+    ctx->last_batch = done;
+    return static_cast<int>(due.size());
+}
+
+int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    const int rows = ctx->layers[layer].fill;
+    if (rows == 0) return VASE_OK;
+    ValueParams vp;
+    vp.vc = static_cast<const uint4*>(ctx->bufs.v_cache) + static_cast<int64_t>(layer) * ctx->plan.units * ctx->plan.N * kVecPerRow;
+    vp.out = ctx->bufs.value_scores + static_cast<int64_t>(layer) * ctx->plan.units * ctx->plan.N;
+    vp.N = ctx->plan.N;
+    vp.rows = rows;
+    vp.units = ctx->plan.units;
+    vp.kind = ctx->cfg.value_score;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = timed_launch(ctx, VASE_KERNEL_VALUE, s, [&] { return launch_value_score(vp, ctx->num_sms, s); });
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "value refresh launch");
+    ctx->launches += 1;
     return VASE_OK;
 }
 
@@ -547,23 +691,26 @@ int vase_kv_view_get(const vase_ctx* ctx, int32_t layer, vase_kv_view* out) {
     out->k = kc_layer(c, layer);
     out->v = vc_layer(c, layer);
     out->positions = pos_layer(c, layer);
+    out->value_scores = c->bufs.value_scores + static_cast<int64_t>(layer) * ctx->plan.units * ctx->plan.N;
     out->unit_stride = static_cast<int64_t>(ctx->plan.N) * kHeadDim;
     out->slots = ctx->plan.N;
     out->fill = ctx->layers[layer].fill;
     return VASE_OK;
 }
 
-int vase_debug_view_get(const vase_ctx* ctx, vase_debug_view* out) {
-    if (!ctx || !out) return VASE_ERR_INVALID;
+int vase_debug_view_get(const vase_ctx* ctx, int32_t slot, vase_debug_view* out) {
+    if (!ctx || !out || slot < 0 || slot >= ctx->plan.slots) return VASE_ERR_INVALID;
     const Plan& P = ctx->plan;
-    out->attn = reinterpret_cast<float*>(ctx->ws + P.off_attn);
-    out->pooled = reinterpret_cast<float*>(ctx->ws + P.off_pooled);
-    out->value_score = reinterpret_cast<float*>(ctx->ws + P.off_vscore);
-    out->key = reinterpret_cast<float*>(ctx->ws + P.off_key);
-    out->keep = ctx->ws + P.off_keep;
-    out->src = reinterpret_cast<int32_t*>(ctx->ws + P.off_src);
+    const size_t z = static_cast<size_t>(slot);
+    out->attn = reinterpret_cast<float*>(ctx->ws + P.off_attn) + z * P.stride_attn;
+    out->pooled = reinterpret_cast<float*>(ctx->ws + P.off_pooled) + z * P.stride_un;
+    out->value_score = reinterpret_cast<float*>(ctx->ws + P.off_vscore) + z * P.stride_un;
+    out->key = reinterpret_cast<float*>(ctx->ws + P.off_key) + z * P.stride_un;
+    out->keep = ctx->ws + P.off_keep + z * P.stride_un;
+    out->src = reinterpret_cast<int32_t*>(ctx->ws + P.off_src) + z * P.stride_src;
     out->units = P.units;
     out->slots = P.N;
+    out->layer = slot < static_cast<int32_t>(ctx->last_batch.size()) ? ctx->last_batch[slot] : -1;
     return VASE_OK;
 }
 
@@ -630,7 +777,7 @@ const char* vase_status_string(int status) {
     }
 }
 
-const char* vase_last_error(const vase_ctx* ctx) { return ctx ? ctx->last_error.c_str() : "null context"; }
+const char* vase_last_error(const vase_ctx* ctx) { return ctx ? ctx->last_error.c_str() : g_config_error.c_str(); }
 
 int vase_abi_version(void) { return VASE_ABI_VERSION; }
 

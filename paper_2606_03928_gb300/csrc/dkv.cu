@@ -79,10 +79,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = tid >> 5;
     const int lane = tid & 31;
     const int unit = blockIdx.y;
+    const int slot = blockIdx.z;
+    const int layer = p.batch.layer[slot];
+    const int rnd = p.fixed_g ? 0 : p.batch.rnd[slot];
+    float* const out = p.out + static_cast<int64_t>(slot) * p.units * p.N;
     const int t_begin = blockIdx.x * p.tiles_per_cta;
     const int t_end = min(p.n_tiles_k, t_begin + p.tiles_per_cta);
     const int n_my = max(0, t_end - t_begin);
-    const int64_t row_base = p.row0 + static_cast<int64_t>(unit) * p.N;
+    const int64_t row_base = static_cast<int64_t>(layer) * p.layer_rows + static_cast<int64_t>(unit) * p.N;
 
     if (tid == 0) {
         for (int s = 0; s < p.stages; ++s) {
@@ -120,8 +124,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     {
         const int r = p.r;
         const float inv_sqrt_r = 1.0f / sqrtf(static_cast<float>(r));
-        const uint32_t c1 = static_cast<uint32_t>(p.rnd);
-        const uint32_t c2 = static_cast<uint32_t>(p.layer) | (kTagDkv << 24);
+        const uint32_t c1 = static_cast<uint32_t>(rnd);
+        const uint32_t c2 = static_cast<uint32_t>(layer) | (kTagDkv << 24);
         const uint32_t c3 = static_cast<uint32_t>(unit);
         for (int idx = tid; idx < kHeadDim * 32; idx += kThreads) {
             const int a = idx >> 5;
@@ -235,13 +239,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_before();
             mbar_arrive(&t_empty[buf]);
-            const int slot = (t_begin + j) * kTileTokens + warp * 32 + lane;
-            if (slot < p.K) {
-                const int64_t o = static_cast<int64_t>(unit) * p.N + slot;
-                p.out[o] = lsum[0] * lsum[1];
-                if (p.lk_out) p.lk_out[o] = lsum[0];
-                if (p.lv_out) p.lv_out[o] = lsum[1];
-            }
+            const int tok = (t_begin + j) * kTileTokens + warp * 32 + lane;
+            if (tok < p.K) out[static_cast<int64_t>(unit) * p.N + tok] = lsum[0] * lsum[1];
         }
     }
 
@@ -262,8 +261,8 @@ cudaError_t dkv_set_attributes(size_t smem_bytes) {
 cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
                        size_t smem_bytes, cudaStream_t s) {
     const int ctas = (p.n_tiles_k + p.tiles_per_cta - 1) / p.tiles_per_cta;
-    dkv_kernel<<<dim3(static_cast<unsigned>(ctas), static_cast<unsigned>(units)), kThreads, smem_bytes, s>>>(kmap, vmap,
-                                                                                                          p);
+    dkv_kernel<<<dim3(static_cast<unsigned>(ctas), static_cast<unsigned>(units), static_cast<unsigned>(p.batch.n)),
+                 kThreads, smem_bytes, s>>>(kmap, vmap, p);
     return cudaGetLastError();
 }
 

@@ -17,6 +17,7 @@ enum ErrSite : uint32_t {
     kErrScoreTEmpty = 5,
     kErrScoreDrain = 6,
     kErrSelectCount = 16,
+    kErrCompactFull = 17,
     kErrDkvTFull = 32,
     kErrDkvKFull = 33,
     kErrDkvKEmpty = 34,
@@ -60,95 +61,120 @@ constexpr uint32_t kTagDkv = 1u;
 
 // ------------------------------------------------------------------ parameter blocks
 
+// The layers one launch works on: slot z = blockIdx.z (or .y) handles model layer layer[z],
+// whose next eviction is round rnd[z].  Workspace arrays are indexed by slot.
+constexpr int kMaxLayerBatch = 64;
+struct LayerBatch {
+    int32_t n;
+    int32_t layer[kMaxLayerBatch];
+    int32_t rnd[kMaxLayerBatch];
+};
+
 struct AppendParams {
-    const uint4* q;   // [n][b][Hq][16]
-    const uint4* k;   // [n][b][Hkv][16]
+    const uint4* q;   // [slot][n][b][Hq][16]
+    const uint4* k;   // [slot][n][b][Hkv][16]
     const uint4* v;
-    uint4* qwin;      // layer base of [b][Hq][W][16]
-    uint4* kc;        // layer base of [b][Hkv][N][16]
+    uint4* qwin;      // base of [L][b][Hq][W][16]
+    uint4* kc;        // base of [L][b][Hkv][N][16]
     uint4* vc;
-    int32_t* pos;     // layer base of [b][Hkv][N]
-    int32_t n, b, Hq, Hkv, W, N, fill;
-    int64_t next_pos;
-    int64_t q_seen;
+    int32_t* pos;     // base of [L][b][Hkv][N]
+    float* vmag;      // base of [L][b][Hkv][N]: value magnitude of each cached token
+    int32_t n, b, Hq, Hkv, W, N, kind;
+    int32_t layer[kMaxLayerBatch];
+    int32_t fill[kMaxLayerBatch];
+    int64_t next_pos[kMaxLayerBatch];
+    int64_t q_seen[kMaxLayerBatch];
 };
 
 struct ScoreAttnParams {
+    LayerBatch batch;
     int32_t N;              // K + B slots per unit
     int32_t GW;             // window rows per unit (G * W)
-    int32_t GWp;            // GW rounded up to a multiple of 32
-    int32_t NB;             // rows per MMA (row block), multiple of 32, <= 256
+    int32_t GWp;            // GW padded: a multiple of 32 up to 256, of 256 beyond
+    int32_t NB;             // window rows per pass-B MMA (N of the MMA), <= 256
     int32_t n_rb;           // GWp / NB
+    int32_t n_rbA;          // 128-row blocks of window rows in pass A
+    int32_t rep;            // copies of the window rows across the 128 pass-A lanes (GWp in {32, 64})
+    int32_t q_rows;         // window rows staged in shared memory (>= GWp)
+    int32_t q_box;          // rows per TMA box of the window-query map
     int32_t n_tiles;        // ceil(N / 128)
     int32_t tiles_per_cta;  // T
     int32_t cluster;        // CTAs per unit
-    int32_t stages;         // K-tile ring depth
+    int32_t stages;         // tile ring depth
+    int32_t buf_cols;       // TMEM columns per accumulator buffer
+    int32_t nbuf;           // accumulator buffers in TMEM (2 or 4)
+    int32_t units;          // units per layer
     int32_t tmem_cols;
     int32_t Hq, Hkv, W, G;
-    int64_t k_row0;         // first K-cache row of the layer
-    int64_t q_row0;         // first Q-window row of the layer
+    int64_t layer_rows;     // cache rows per layer (units * N)
+    int64_t q_layer_rows;   // window rows per layer (b * Hq * W)
     float scale_log2;       // log2(e) / sqrt(d)
     float inv_gw;           // 1 / (G * W)
-    float* attn;            // [units][N]
+    float* attn;            // [slot][n_rb][units][N] (one part per row block)
     uint32_t* err;
 };
 
 struct ValueParams {
-    const uint4* vc;        // layer base [units][N][16]
-    float* out;             // [units][N], slots < K
-    int32_t N, K, units, kind;
+    const uint4* vc;        // layer base of [units][N][16]
+    float* out;             // layer base of [units][N]
+    int32_t N, rows, units, kind;  // slots 0..rows-1 of every unit
 };
 
 struct DkvParams {
-    int32_t N, K, r, Hkv, layer, rnd;
+    LayerBatch batch;
+    int32_t N, K, r, Hkv, fixed_g, units;
     uint32_t seed_lo, seed_hi;
     int32_t n_tiles_k;      // ceil(K / 128)
     int32_t tiles_per_cta;
     int32_t stages;
-    int64_t row0;           // first cache row of the layer
-    float* out;             // [units][N] leverage product, slots < K
-    float* lk_out;          // optional [units][N]
-    float* lv_out;          // optional [units][N]
+    int64_t layer_rows;     // cache rows per layer
+    float* out;             // [slot][units][N] leverage product, slots < K
     uint32_t* err;
 };
 
 struct SelectParams {
-    const float* attn;      // [units][N]
-    const float* vscore;    // [units][N]
-    const int32_t* pos;     // layer base [units][N]
-    int32_t* src;           // [units][K]
-    float* pooled_dbg;      // nullable
+    LayerBatch batch;
+    const float* attn;      // [slot][n_parts][units][N]: the window score is the sum of the parts
+    const float* dkv;       // [slot][units][N] leverage products (DKV)
+    float* vmag;            // base of [L][units][N]: value magnitudes (AttnV), compacted in place
+    int32_t* pos;           // base of [L][units][N]; compacted in place with the kept list
+    float* vscore_dbg;      // nullable, [slot][units][N]: the value magnitudes of this eviction
+    int32_t* src;           // [slot][units][K]
+    float* pooled_dbg;      // nullable, [slot][units][N]
     float* key_dbg;         // nullable
     uint8_t* keep_dbg;      // nullable
-    int32_t N, K, B, n_v, m, pool, variant, stochastic, Hkv, layer, rnd;
+    int32_t N, K, B, n_v, m, pool, variant, stochastic, Hkv, n_parts, units;
     uint32_t seed_lo, seed_hi;
     uint32_t* err;
 };
 
 struct CompactParams {
-    uint4* kc;              // layer base [units][N][16]
+    LayerBatch batch;
+    uint4* kc;              // base of [L][units][N][16]
     uint4* vc;
-    int32_t* pos;           // layer base [units][N]
-    const int32_t* src;     // [units][K]
-    int32_t N, K;
+    const int32_t* src;     // [slot][units][K]
+    int32_t N, K, units;
+    uint32_t* err;
 };
 
 // ------------------------------------------------------------------ launchers (return cudaError_t)
 
-cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
+cudaError_t launch_append(const AppendParams& p, int n_layers, cudaStream_t s);
 cudaError_t launch_value_score(const ValueParams& p, int num_sms, cudaStream_t s);
-cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreAttnParams& p,
-                              int units, size_t smem_bytes, cudaStream_t s);
+cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreAttnParams& p, int units,
+                              size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
                        size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_compact(const CompactParams& p, int units, cudaStream_t s);
 
-size_t score_attn_smem_bytes(int GWp, int cluster, int stages);
+size_t score_attn_smem_bytes(int q_rows, int n_rbA, int GWp, int cluster, int stages);
 size_t dkv_smem_bytes(int stages);
 size_t select_smem_bytes(int N, int K);
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster);
 cudaError_t dkv_set_attributes(size_t smem_bytes);
 cudaError_t select_set_attributes(size_t smem_bytes);
+size_t compact_smem_bytes();
+cudaError_t compact_set_attributes();
 
 }  // namespace vase

@@ -14,53 +14,9 @@ namespace {
 // ------------------------------------------------------------------ append
 // One decode step appends one (k, v) pair per KV head and one query per query
 // head (Sec. 2, periodic eviction; the last W queries are cached for Eq. (2)).
-__global__ void append_kernel(const AppendParams p) {
-    const int64_t nq = static_cast<int64_t>(p.n) * p.b * p.Hq * kVecPerRow;
-    const int64_t nk = static_cast<int64_t>(p.n) * p.b * p.Hkv * kVecPerRow;
-    const int64_t npos = static_cast<int64_t>(p.n) * p.b * p.Hkv;
-    const int64_t total = nq + 2 * nk + npos;
-    const int first_q = p.n > p.W ? p.n - p.W : 0;  // only the last W queries survive in the ring
-    for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
-         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        if (i < nq) {
-            const int seg = static_cast<int>(i % kVecPerRow);
-            const int64_t r = i / kVecPerRow;  // (t, s, hq)
-            const int hq = static_cast<int>(r % p.Hq);
-            const int64_t ts = r / p.Hq;
-            const int s = static_cast<int>(ts % p.b);
-            const int t = static_cast<int>(ts / p.b);
-            if (t < first_q) continue;
-            const int slot = static_cast<int>((p.q_seen + t) % p.W);
-            p.qwin[((static_cast<int64_t>(s) * p.Hq + hq) * p.W + slot) * kVecPerRow + seg] = p.q[i];
-        } else if (i < nq + 2 * nk) {
-            const int64_t j = i - nq;
-            const bool is_v = j >= nk;
-            const int64_t jj = is_v ? j - nk : j;
-            const int seg = static_cast<int>(jj % kVecPerRow);
-            const int64_t r = jj / kVecPerRow;  // (t, s, h)
-            const int h = static_cast<int>(r % p.Hkv);
-            const int64_t ts = r / p.Hkv;
-            const int s = static_cast<int>(ts % p.b);
-            const int t = static_cast<int>(ts / p.b);
-            const int64_t dst = ((static_cast<int64_t>(s) * p.Hkv + h) * p.N + p.fill + t) * kVecPerRow + seg;
-            if (is_v)
-                p.vc[dst] = p.v[jj];
-            else
-                p.kc[dst] = p.k[jj];
-        } else {
-            const int64_t r = i - nq - 2 * nk;  // (t, s, h)
-            const int h = static_cast<int>(r % p.Hkv);
-            const int64_t ts = r / p.Hkv;
-            const int s = static_cast<int>(ts % p.b);
-            const int t = static_cast<int>(ts / p.b);
-            p.pos[(static_cast<int64_t>(s) * p.Hkv + h) * p.N + p.fill + t] = static_cast<int32_t>(p.next_pos + t);
-        }
-    }
-}
-
-// ------------------------------------------------------------------ value magnitude
-// Range(v) = max_j v_j - min_j v_j (Eq. (5)); L2 and Var (App. A).  A half
-// warp reads one 256-byte row with one 16-byte load per lane.
+// The value magnitude of a token (Range, L2 or Var of its value row, Eq. (5) and App. A)
+// never changes once it is cached, so it is taken here, where the row is written, and
+// kept per slot beside the positions; the eviction step then never reads V to score.
 __device__ __forceinline__ void bf16x8_to_f32(const uint4 u, float (&f)[8]) {
     const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
@@ -70,60 +26,120 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4 u, float (&f)[8]) {
     }
 }
 
+// Value magnitude of a 128-element row spread over the 16 lanes of a half warp (8 elements
+// each); every lane of the warp must call it.  The result is valid in all 16 lanes.
+__device__ __forceinline__ float half_warp_value_magnitude(const uint4 u, int kind) {
+    float f[8];
+    bf16x8_to_f32(u, f);
+    if (kind == 0) {
+        float mx = f[0], mn = f[0];
+#pragma unroll
+        for (int i = 1; i < 8; ++i) {
+            mx = fmaxf(mx, f[i]);
+            mn = fminf(mn, f[i]);
+        }
+#pragma unroll
+        for (int o = 8; o >= 1; o >>= 1) {
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+        }
+        return mx - mn;
+    }
+    if (kind == 1) {
+        float ss = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) ss = fmaf(f[i], f[i], ss);
+#pragma unroll
+        for (int o = 8; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        return sqrtf(ss);
+    }
+    float sm = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) sm += f[i];
+#pragma unroll
+    for (int o = 8; o >= 1; o >>= 1) sm += __shfl_xor_sync(0xffffffffu, sm, o);
+    const float mu = sm * (1.0f / kHeadDim);
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const float dl = f[i] - mu;
+        ss = fmaf(dl, dl, ss);
+    }
+#pragma unroll
+    for (int o = 8; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    return ss * (1.0f / kHeadDim);
+}
+
+__global__ void append_kernel(const AppendParams p) {
+    const int z = blockIdx.y;  // layer slot
+    const int layer = p.layer[z];
+    const int t = blockIdx.x / p.b;      // decode step within the call
+    const int s = blockIdx.x - t * p.b;  // sequence
+    const int per = (p.Hq + 2 * p.Hkv) * kVecPerRow;
+    const bool q_lives = t >= p.n - p.W;  // only the last W queries survive in the ring
+    const int slot = static_cast<int>((p.q_seen[z] + t) % p.W);
+    const int fill = p.fill[z];
+    const int64_t units = static_cast<int64_t>(p.b) * p.Hkv;
+    uint4* const qwin = p.qwin + static_cast<int64_t>(layer) * p.b * p.Hq * p.W * kVecPerRow;
+    uint4* const kc = p.kc + static_cast<int64_t>(layer) * units * p.N * kVecPerRow;
+    uint4* const vc = p.vc + static_cast<int64_t>(layer) * units * p.N * kVecPerRow;
+    int32_t* const pos = p.pos + static_cast<int64_t>(layer) * units * p.N;
+    float* const vmag = p.vmag + static_cast<int64_t>(layer) * units * p.N;
+    const uint4* const q = p.q + static_cast<int64_t>(z) * p.n * p.b * p.Hq * kVecPerRow;
+    const uint4* const k = p.k + static_cast<int64_t>(z) * p.n * units * kVecPerRow;
+    const uint4* const v = p.v + static_cast<int64_t>(z) * p.n * units * kVecPerRow;
+    const int64_t row_in = static_cast<int64_t>(t) * p.b + s;
+    // the trip count is the same for every thread of the block, so the half-warp shuffles see full warps
+    for (int e0 = 0; e0 < per; e0 += blockDim.x) {
+        const int e = e0 + threadIdx.x;
+        const int head = e >> 4;
+        const int seg = e & 15;
+        uint4 val = make_uint4(0, 0, 0, 0);
+        bool is_v = false;
+        int h = 0;
+        if (e < per) {
+            if (head < p.Hq) {
+                if (q_lives)
+                    qwin[(static_cast<int64_t>(s * p.Hq + head) * p.W + slot) * kVecPerRow + seg] =
+                        q[(row_in * p.Hq + head) * kVecPerRow + seg];
+            } else {
+                is_v = head >= p.Hq + p.Hkv;
+                h = head - p.Hq - (is_v ? p.Hkv : 0);
+                const int64_t dst = (static_cast<int64_t>(s * p.Hkv + h) * p.N + fill + t) * kVecPerRow + seg;
+                const int64_t src = (row_in * p.Hkv + h) * kVecPerRow + seg;
+                if (is_v) {
+                    val = v[src];
+                    vc[dst] = val;
+                } else {
+                    kc[dst] = k[src];
+                }
+            }
+        }
+        const float mag = half_warp_value_magnitude(val, p.kind);
+        if (is_v && seg == 0) vmag[static_cast<int64_t>(s * p.Hkv + h) * p.N + fill + t] = mag;
+    }
+    for (int hh = threadIdx.x; hh < p.Hkv; hh += blockDim.x)
+        pos[static_cast<int64_t>(s * p.Hkv + hh) * p.N + fill + t] = static_cast<int32_t>(p.next_pos[z] + t);
+}
+
+// ------------------------------------------------------------------ value magnitude refresh
+// Recomputes the per-slot value magnitudes of slots 0..rows-1 of every unit of one layer
+// from the V cache (for callers that write cache rows directly).  A half warp per row.
 __global__ void value_score_kernel(const ValueParams p) {
     const int warp = threadIdx.x >> 5;
     const int hsel = (threadIdx.x >> 4) & 1;
     const int l = threadIdx.x & 15;
     const int halves = blockDim.x >> 4;
-    const int64_t rows = static_cast<int64_t>(p.units) * p.K;
-    // the loop bound is uniform per warp so every shuffle sees all 32 lanes
+    const int64_t rows = static_cast<int64_t>(p.units) * p.rows;
     for (int64_t r0 = static_cast<int64_t>(blockIdx.x) * halves + 2 * warp; r0 < rows;
          r0 += static_cast<int64_t>(gridDim.x) * halves) {
         const int64_t r = r0 + hsel;
         const bool valid = r < rows;
-        const int unit = valid ? static_cast<int>(r / p.K) : 0;
-        const int slot = valid ? static_cast<int>(r - static_cast<int64_t>(unit) * p.K) : 0;
+        const int unit = valid ? static_cast<int>(r / p.rows) : 0;
+        const int slot = valid ? static_cast<int>(r - static_cast<int64_t>(unit) * p.rows) : 0;
         const int64_t row = static_cast<int64_t>(unit) * p.N + slot;
-        float f[8];
-        bf16x8_to_f32(valid ? __ldg(&p.vc[row * kVecPerRow + l]) : make_uint4(0, 0, 0, 0), f);
-        float out;
-        if (p.kind == 0) {
-            float mx = f[0], mn = f[0];
-#pragma unroll
-            for (int i = 1; i < 8; ++i) {
-                mx = fmaxf(mx, f[i]);
-                mn = fminf(mn, f[i]);
-            }
-#pragma unroll
-            for (int o = 8; o >= 1; o >>= 1) {
-                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-                mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-            }
-            out = mx - mn;
-        } else if (p.kind == 1) {
-            float ss = 0.f;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) ss = fmaf(f[i], f[i], ss);
-#pragma unroll
-            for (int o = 8; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-            out = sqrtf(ss);
-        } else {
-            float sm = 0.f;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) sm += f[i];
-#pragma unroll
-            for (int o = 8; o >= 1; o >>= 1) sm += __shfl_xor_sync(0xffffffffu, sm, o);
-            const float mu = sm * (1.0f / kHeadDim);
-            float ss = 0.f;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const float dlt = f[i] - mu;
-                ss = fmaf(dlt, dlt, ss);
-            }
-#pragma unroll
-            for (int o = 8; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-            out = ss * (1.0f / kHeadDim);
-        }
+        const float out =
+            half_warp_value_magnitude(valid ? __ldg(&p.vc[row * kVecPerRow + l]) : make_uint4(0, 0, 0, 0), p.kind);
         if (valid && l == 0) p.out[row] = out;
     }
 }
@@ -134,8 +150,10 @@ constexpr int kSelWarps = kSelThreads / 32;
 constexpr uint8_t kFlagValue = 1;
 constexpr uint8_t kFlagSampled = 2;
 
+constexpr int kSelBins = 2048;
+
 struct SelShared {
-    uint32_t hist[256];
+    uint32_t hist[kSelBins];
     int warp_tot[kSelWarps];
     uint32_t bcast[4];
 };
@@ -172,32 +190,37 @@ __device__ __forceinline__ int block_exclusive_scan(int v, SelShared& sh, int* t
 }
 
 // Marks with `flag` the k largest values of ord[0..n) (ties to the lower
-// index), by an MSB-first radix select on 8-bit digits followed by a
-// slot-ordered rank of the elements equal to the threshold.  Each thread owns
-// the contiguous slots [seg_lo, seg_hi).
+// index), by an MSB-first radix select on 11/11/10-bit digits (lanes with the
+// same digit are merged with __match_any_sync before the shared-memory atomic)
+// followed by a slot-ordered rank of the elements equal to the threshold.
+// Each thread owns the contiguous slots [seg_lo, seg_hi).
 __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, uint8_t flag, int seg_lo,
                             int seg_hi, SelShared& sh) {
     if (k <= 0) return;
     const int tid = threadIdx.x;
+    const int lane = tid & 31;
     uint32_t prefix = 0, mask = 0;
     int remain = k;
-    for (int shift = 24; shift >= 0; shift -= 8) {
-        for (int i = tid; i < 256; i += kSelThreads) sh.hist[i] = 0;
+    const int shifts[3] = {21, 10, 0};
+    const int widths[3] = {11, 11, 10};
+    for (int pass = 0; pass < 3; ++pass) {
+        const int shift = shifts[pass];
+        const uint32_t dmask = (1u << widths[pass]) - 1u;
+        for (int i = tid; i < kSelBins; i += kSelThreads) sh.hist[i] = 0;
         __syncthreads();
-        for (int i = tid; i < n; i += kSelThreads) {
-            const uint32_t x = ord[i];
-            if ((x & mask) == prefix) atomicAdd(&sh.hist[(x >> shift) & 0xFFu], 1u);
+        const int n_round = (n + 31) & ~31;
+        for (int i = tid; i < n_round; i += kSelThreads) {
+            const uint32_t x = i < n ? ord[i] : 0u;
+            const bool in = i < n && (x & mask) == prefix;
+            const uint32_t bin = in ? ((x >> shift) & dmask) : 0xFFFFFFFFu;
+            const uint32_t peers = __match_any_sync(0xffffffffu, bin);
+            if (in && lane == __ffs(peers) - 1) atomicAdd(&sh.hist[bin], static_cast<uint32_t>(__popc(peers)));
         }
         __syncthreads();
         if (tid < 32) {
-            const int lane = tid;
-            uint32_t c[8];
+            constexpr int per = kSelBins / 32;  // bins per lane
             uint32_t tot = 0;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                c[j] = sh.hist[8 * lane + j];
-                tot += c[j];
-            }
+            for (int j = 0; j < per; ++j) tot += sh.hist[per * lane + ((j + lane) & (per - 1))];  // bank-rotated
             uint32_t suf = tot;  // inclusive suffix sum over lanes >= lane
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
@@ -205,20 +228,23 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
                 if (lane + o < 32) suf += y;
             }
             uint32_t above = suf - tot;
-#pragma unroll
-            for (int j = 7; j >= 0; --j) {
-                if (above < static_cast<uint32_t>(remain) && above + c[j] >= static_cast<uint32_t>(remain)) {
-                    sh.bcast[0] = static_cast<uint32_t>(8 * lane + j);
-                    sh.bcast[1] = above;
+            if (above < static_cast<uint32_t>(remain) && suf >= static_cast<uint32_t>(remain)) {
+                for (int j = per - 1; j >= 0; --j) {
+                    const uint32_t c = sh.hist[per * lane + j];
+                    if (above + c >= static_cast<uint32_t>(remain)) {
+                        sh.bcast[0] = static_cast<uint32_t>(per * lane + j);
+                        sh.bcast[1] = above;
+                        break;
+                    }
+                    above += c;
                 }
-                above += c[j];
             }
         }
         __syncthreads();
         const uint32_t digit = sh.bcast[0];
         remain -= static_cast<int>(sh.bcast[1]);
         prefix |= digit << shift;
-        mask |= 0xFFu << shift;
+        mask |= dmask << shift;
         __syncthreads();
     }
     const uint32_t thr = prefix;
@@ -253,8 +279,21 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectPara
     uint32_t* ord = reinterpret_cast<uint32_t*>(a_s + N);         // [K] orderable keys
     uint8_t* flags = reinterpret_cast<uint8_t*>(ord + K);         // [N]
     const int unit = blockIdx.x;
+    const int z = blockIdx.y;  // layer slot
+    const int layer = p.batch.layer[z];
+    const int rnd = p.batch.rnd[z];
     const int tid = threadIdx.x;
-    const int64_t base = static_cast<int64_t>(unit) * N;
+    const int64_t base = static_cast<int64_t>(unit) * N;                     // within one layer / slot
+    const int64_t zs = static_cast<int64_t>(z) * p.units * N;               // slot offset of [units][N] arrays
+    const float* const attn = p.attn + zs * p.n_parts;
+    const float* const dkv = p.dkv + zs;
+    int32_t* const pos = p.pos + static_cast<int64_t>(layer) * p.units * N;
+    float* const vmag = p.vmag + static_cast<int64_t>(layer) * p.units * N;
+    float* const vscore_dbg = p.vscore_dbg ? p.vscore_dbg + zs : nullptr;
+    int32_t* const src_out = p.src + static_cast<int64_t>(z) * p.units * K;
+    float* const pooled_dbg = p.pooled_dbg ? p.pooled_dbg + zs : nullptr;
+    float* const key_dbg = p.key_dbg ? p.key_dbg + zs : nullptr;
+    uint8_t* const keep_dbg = p.keep_dbg ? p.keep_dbg + zs : nullptr;
     const int seg = (N + kSelThreads - 1) / kSelThreads;
     const int seg_lo = min(N, tid * seg);
     const int seg_hi = min(N, seg_lo + seg);
@@ -263,20 +302,33 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectPara
 
     for (int i = tid; i < N; i += kSelThreads) flags[i] = 0;
     if (p.variant == 0) {
-        for (int i = tid; i < N; i += kSelThreads) a_s[i] = p.attn[base + i];
-        for (int i = tid; i < K; i += kSelThreads) ord[i] = __float_as_uint(p.vscore[base + i]) + 1u;
+        for (int i = tid; i < N; i += kSelThreads) {
+            float a = attn[base + i];
+            for (int part = 1; part < p.n_parts; ++part)
+                a += attn[(static_cast<int64_t>(part) * p.units + unit) * N + i];
+            a_s[i] = a;
+        }
+        if (p.n_parts > 1 && pooled_dbg) {
+            __syncthreads();
+            for (int i = tid; i < N; i += kSelThreads) const_cast<float*>(attn)[base + i] = a_s[i];
+        }
+        for (int i = tid; i < K; i += kSelThreads) {
+            const float vm = vmag[base + i];
+            ord[i] = __float_as_uint(vm) + 1u;
+            if (vscore_dbg) vscore_dbg[base + i] = vm;
+        }
         __syncthreads();
         radix_top_k(ord, K, p.n_v, flags, kFlagValue, kseg_lo, kseg_hi, sh);
         // keys over the candidates C
         const int h = p.pool / 2;
         const float inv_pool = 1.0f / static_cast<float>(p.pool);
-        const uint32_t c2 = static_cast<uint32_t>(p.layer) | (kTagSelect << 24);
+        const uint32_t c2 = static_cast<uint32_t>(layer) | (kTagSelect << 24);
         for (int i = tid; i < N; i += kSelThreads) {
             float sum = 0.f;
             const int lo = max(0, i - h), hi = min(N - 1, i + h);
             for (int j = lo; j <= hi; ++j) sum += a_s[j];
             const float pooled = sum * inv_pool;
-            if (p.pooled_dbg) p.pooled_dbg[base + i] = pooled;
+            if (pooled_dbg) pooled_dbg[base + i] = pooled;
             if (i >= K) continue;
             float key = -1.f;
             if (flags[i] & kFlagValue) {
@@ -285,127 +337,202 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectPara
                 key = pooled;
                 if (p.stochastic) {
                     const Philox4 w = philox4x32_10(
-                        Philox4{static_cast<uint32_t>(p.pos[base + i]), static_cast<uint32_t>(p.rnd), c2,
+                        Philox4{static_cast<uint32_t>(pos[base + i]), static_cast<uint32_t>(rnd), c2,
                                 static_cast<uint32_t>(unit)},
                         p.seed_lo, p.seed_hi);
                     key = pooled / (-logf(open_uniform(w.x)));
                 }
                 ord[i] = __float_as_uint(key) + 1u;
             }
-            if (p.key_dbg) p.key_dbg[base + i] = key;
+            if (key_dbg) key_dbg[base + i] = key;
         }
         __syncthreads();
         radix_top_k(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
     } else {
         for (int i = tid; i < K; i += kSelThreads) {
-            const float s = p.vscore[base + i];
+            const float s = dkv[base + i];
             ord[i] = __float_as_uint(s) + 1u;
-            if (p.key_dbg) p.key_dbg[base + i] = s;
+            if (key_dbg) key_dbg[base + i] = s;
         }
         __syncthreads();
         radix_top_k(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
     }
+    // positions move with the kept rows: stage the old ones in shared memory (a_s is free now)
+    int32_t* pos_s = reinterpret_cast<int32_t*>(a_s);
+    for (int i = tid; i < N; i += kSelThreads) pos_s[i] = pos[base + i];
     // keep = R_B u R_V u sampled; ascending list of kept slots
     int cnt = 0;
     for (int i = seg_lo; i < seg_hi; ++i) cnt += (i >= K) || flags[i];
     int total;
-    int dst = block_exclusive_scan(cnt, sh, &total);
+    const int dst0 = block_exclusive_scan(cnt, sh, &total);  // also a barrier after the staging above
+    int dst = dst0;
     for (int i = seg_lo; i < seg_hi; ++i) {
         const bool keep = (i >= K) || flags[i];
         if (keep) {
-            if (dst < K) p.src[static_cast<int64_t>(unit) * K + dst] = i;
+            if (dst < K) {
+                src_out[static_cast<int64_t>(unit) * K + dst] = i;
+                pos[base + dst] = pos_s[i];
+            }
             ++dst;
         }
-        if (p.keep_dbg) p.keep_dbg[base + i] = keep ? 1 : 0;
-        if (p.key_dbg && i >= K) p.key_dbg[base + i] = -1.f;
+        if (keep_dbg) keep_dbg[base + i] = keep ? 1 : 0;
+        if (key_dbg && i >= K) key_dbg[base + i] = -1.f;
+    }
+    for (int i = K + tid; i < N; i += kSelThreads) pos[base + i] = -1;
+    // value magnitudes move with their rows too
+    __syncthreads();
+    float* vm_s = a_s;
+    for (int i = tid; i < N; i += kSelThreads) vm_s[i] = vmag[base + i];
+    __syncthreads();
+    dst = dst0;
+    for (int i = seg_lo; i < seg_hi; ++i) {
+        if ((i >= K) || flags[i]) {
+            if (dst < K) vmag[base + dst] = vm_s[i];
+            ++dst;
+        }
     }
     if (tid == 0 && total != K) record_error(p.err, kErrSelectCount);
 }
 
 // ------------------------------------------------------------------ compaction
-// Stable in-place gather of the kept rows into slots 0..K-1 (Sec. 2: the
-// cache is restored to K pairs).  New slot j takes old slot src[j] >= j, so a
-// CTA that walks destination chunks in ascending order, loading a chunk's
-// sources before any of its stores (barrier) and never storing past the
-// chunk, never overwrites a row it still has to read.  Each CTA owns one
-// 128-byte column half of K or V, so CTAs never touch the same bytes.
-constexpr int kCompactThreads = 256;
-constexpr int kCompactRowsPerChunk = 256;
+// Stable in-place gather of the kept rows of K or V into slots 0..K-1 (Sec. 2:
+// the cache is restored to K pairs).  New slot j takes old slot src[j] >= j.
+// One CTA (one warp) owns the K or the V rows of one unit and walks
+// destination chunks of 128 rows in ascending order: the kept rows of a chunk
+// form runs of consecutive source rows, each fetched by one bulk TMA copy into
+// a shared-memory stage, and the chunk goes back with one bulk store.  Sources
+// of chunk c lie at or above row 128c while its store ends below 128(c+1), so a
+// later chunk never loads a row an earlier store overwrites; a chunk is stored
+// only after its loads (and all earlier ones) have completed.  Several stages
+// keep loads in flight ahead of the stores.
+constexpr int kCompactRows = 128;                          // destination rows per chunk
+constexpr int kCompactStages = 6;
+constexpr int kCompactChunkBytes = kCompactRows * kRowBytes;  // 32 KB
 
-__global__ void __launch_bounds__(kCompactThreads) compact_kernel(const CompactParams p) {
+__device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(smem_dst)),
+                 "l"(gsrc), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_store(void* gdst, const void* smem_src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(smem_u32(smem_src)),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+__global__ void __launch_bounds__(32) compact_kernel(const CompactParams p) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* ring = smem_raw;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + kCompactStages * kCompactChunkBytes);
     const int unit = blockIdx.x;
-    const int part = blockIdx.y;  // 0, 1: K halves; 2, 3: V halves
-    uint4* base = (part < 2 ? p.kc : p.vc) + static_cast<int64_t>(unit) * p.N * kVecPerRow;
-    const int seg = (part & 1) * 8 + (threadIdx.x & 7);
-    const int rsub = threadIdx.x >> 3;  // 0..31
-    const bool do_pos = (part == 0) && ((threadIdx.x & 7) == 0);
-    int32_t* pos = p.pos + static_cast<int64_t>(unit) * p.N;
-    const int32_t* src = p.src + static_cast<int64_t>(unit) * p.K;
-    const int n_chunks = (p.K + kCompactRowsPerChunk - 1) / kCompactRowsPerChunk;
-
-    uint4 cur[8], nxt[8];
-    int cs[8], ns[8];
-    int32_t cp[8], np[8];
-    auto load = [&](int c, uint4 (&d)[8], int (&sidx)[8], int32_t (&pv)[8]) {
+    const int lane = threadIdx.x;
+    const int z = blockIdx.z;  // layer slot
+    const int64_t unit_row = static_cast<int64_t>(p.batch.layer[z]) * p.units * p.N + static_cast<int64_t>(unit) * p.N;
+    uint8_t* base = reinterpret_cast<uint8_t*>((blockIdx.y == 0 ? p.kc : p.vc) + unit_row * kVecPerRow);
+    const int32_t* src = p.src + (static_cast<int64_t>(z) * p.units + unit) * p.K;
+    const int n_chunks = (p.K + kCompactRows - 1) / kCompactRows;
+    if (lane == 0) {
+        for (int s = 0; s < kCompactStages; ++s) mbar_init(&full[s], 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+    // chunks whose rows all stay in place need no work: the kept list starts with 0, 1, 2, ...
+    int first = 0;
+    for (; first < n_chunks; ++first) {
+        bool same = true;
+        for (int k = lane; k < kCompactRows; k += 32) {
+            const int j = first * kCompactRows + k;
+            if (j < p.K && src[j] != j) same = false;
+        }
+        if (!__all_sync(0xffffffffu, same)) break;
+    }
+    // stage and mbarrier phase count from the first chunk that moves
+    auto load = [&](int c) {
+        const int stage = (c - first) % kCompactStages;
+        uint8_t* dst = ring + stage * kCompactChunkBytes;
+        const int j0 = c * kCompactRows;
+        const int rows = min(kCompactRows, p.K - j0);
+        if (lane == 0) mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(rows) * kRowBytes);
+        __syncwarp();
+        // a run of consecutive sources starts where src[j] != src[j-1] + 1 (or at the chunk start)
+        uint32_t starts[kCompactRows / 32];
+        int sv[kCompactRows / 32];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            const int j = c * kCompactRowsPerChunk + rsub + 32 * i;
-            sidx[i] = -1;
-            if (j < p.K) {
-                const int s = src[j];
-                if (s != j) {
-                    sidx[i] = s;
-                    d[i] = base[static_cast<int64_t>(s) * kVecPerRow + seg];
-                    if (do_pos) pv[i] = pos[s];
+        for (int k = 0; k < kCompactRows / 32; ++k) {
+            const int q = k * 32 + lane;
+            const int j = j0 + q;
+            const bool in = q < rows;
+            const int s = in ? src[j] : 0;
+            sv[k] = s;
+            const bool st = in && (q == 0 || src[j - 1] + 1 != s);
+            starts[k] = __ballot_sync(0xffffffffu, st);
+        }
+#pragma unroll
+        for (int k = 0; k < kCompactRows / 32; ++k) {
+            const int q = k * 32 + lane;
+            if ((starts[k] >> lane) & 1u) {
+                // run length: distance to the next start, or to the end of the chunk
+                int next = rows;
+                const uint32_t later = lane < 31 ? (starts[k] >> (lane + 1)) << (lane + 1) : 0u;
+                if (later) {
+                    next = k * 32 + __ffs(later) - 1;
+                } else {
+#pragma unroll
+                    for (int k2 = k + 1; k2 < kCompactRows / 32; ++k2) {
+                        if (starts[k2]) {
+                            next = min(next, k2 * 32 + __ffs(starts[k2]) - 1);
+                            break;
+                        }
+                    }
                 }
+                bulk_load(dst + q * kRowBytes, base + static_cast<int64_t>(sv[k]) * kRowBytes,
+                          static_cast<uint32_t>(next - q) * kRowBytes, &full[stage]);
             }
         }
     };
-    auto store = [&](int c, const uint4 (&d)[8], const int (&sidx)[8], const int32_t (&pv)[8]) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            const int j = c * kCompactRowsPerChunk + rsub + 32 * i;
-            if (sidx[i] >= 0) {
-                base[static_cast<int64_t>(j) * kVecPerRow + seg] = d[i];
-                if (do_pos) pos[j] = pv[i];
-            }
+    bool ok = true;
+    for (int c = first; c < first + kCompactStages - 1 && c < n_chunks; ++c) load(c);
+    for (int c = first; c < n_chunks; ++c) {
+        const int nxt = c + kCompactStages - 1;
+        if (nxt < n_chunks) {
+            if (lane == 0) bulk_wait_read0();  // the stage's previous store has read its bytes
+            __syncwarp();
+            load(nxt);
         }
-    };
-    if (n_chunks > 0) load(0, cur, cs, cp);
-    __syncthreads();
-    for (int c = 0; c < n_chunks; ++c) {
-        if (c + 1 < n_chunks) load(c + 1, nxt, ns, np);
-        store(c, cur, cs, cp);
-        __syncthreads();
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            cur[i] = nxt[i];
-            cs[i] = ns[i];
-            cp[i] = np[i];
+        const int stage = (c - first) % kCompactStages;
+        if (ok) ok = mbar_wait(&full[stage], ((c - first) / kCompactStages) & 1, p.err, kErrCompactFull);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        if (lane == 0) {
+            const int j0 = c * kCompactRows;
+            const int rows = min(kCompactRows, p.K - j0);
+            bulk_store(base + static_cast<int64_t>(j0) * kRowBytes, ring + stage * kCompactChunkBytes,
+                       static_cast<uint32_t>(rows) * kRowBytes);
+            bulk_commit();
         }
+        __syncwarp();
     }
-    if (part == 0) {
-        for (int j = p.K + threadIdx.x; j < p.N; j += kCompactThreads) pos[j] = -1;
-    }
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
 }
 
 }  // namespace
 
-cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
-    const int64_t total = static_cast<int64_t>(p.n) * p.b * (p.Hq + 2 * p.Hkv) * kVecPerRow +
-                          static_cast<int64_t>(p.n) * p.b * p.Hkv;
-    const int threads = 256;
-    const int64_t blocks = (total + threads - 1) / threads;
-    append_kernel<<<static_cast<unsigned>(blocks < 65535 ? blocks : 65535), threads, 0, s>>>(p);
+cudaError_t launch_append(const AppendParams& p, int n_layers, cudaStream_t s) {
+    append_kernel<<<dim3(static_cast<unsigned>(p.n * p.b), static_cast<unsigned>(n_layers)), 256, 0, s>>>(p);
     return cudaGetLastError();
 }
 
 cudaError_t launch_value_score(const ValueParams& p, int num_sms, cudaStream_t s) {
     const int threads = 256;
-    const int64_t rows = static_cast<int64_t>(p.units) * p.K;
+    const int64_t rows = static_cast<int64_t>(p.units) * p.rows;
     int64_t blocks = (rows + (threads / 16) - 1) / (threads / 16);
     const int64_t cap = static_cast<int64_t>(num_sms) * 8;
     if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
     value_score_kernel<<<static_cast<unsigned>(blocks), threads, 0, s>>>(p);
     return cudaGetLastError();
 }
@@ -418,12 +545,19 @@ cudaError_t select_set_attributes(size_t smem_bytes) {
 }
 
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s) {
-    select_kernel<<<static_cast<unsigned>(units), kSelThreads, smem_bytes, s>>>(p);
+    select_kernel<<<dim3(static_cast<unsigned>(units), static_cast<unsigned>(p.batch.n)), kSelThreads, smem_bytes, s>>>(p);
     return cudaGetLastError();
 }
 
+size_t compact_smem_bytes() { return kCompactStages * (kCompactChunkBytes + 8) + 1024; }
+
+cudaError_t compact_set_attributes() {
+    return cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(compact_smem_bytes()));
+}
+
 cudaError_t launch_compact(const CompactParams& p, int units, cudaStream_t s) {
-    compact_kernel<<<dim3(static_cast<unsigned>(units), 4), kCompactThreads, 0, s>>>(p);
+    compact_kernel<<<dim3(static_cast<unsigned>(units), 2, static_cast<unsigned>(p.batch.n)), 32, compact_smem_bytes(), s>>>(p);
     return cudaGetLastError();
 }
 

@@ -3,20 +3,24 @@
 // For one unit (sequence s, KV head h) the score of cached slot i is
 //     a_i = (1 / (G*W)) * sum_r softmax_i(q_r . k_i / sqrt(d))
 // over the G*W cached window queries r of the unit's query heads, with the
-// softmax taken over all N = K + B cached keys (Eq. (1) and Eq. (2), Sec. 2;
-// non-causal cached queries per the footnote of Eq. (2)).  Pooling is done by
-// the selection kernel.
+// softmax over all N = K + B cached keys (Eq. (1) and Eq. (2), Sec. 2; the
+// queries are cached and the scores non-causal, per the footnote of Eq. (2)).
+// Pooling is left to the selection kernel.
 //
 // Decomposition: a cluster of C CTAs per unit, each owning a contiguous range
-// of 128-token tiles.  A producer warp streams K tiles with TMA (128-byte
-// swizzle) into a shared-memory ring and issues tcgen05.mma with the tile as
-// A (M = 128 tokens) and the window queries as B (N = row block), so TMEM
-// lane t holds token t's logits against every window row.  Four consumer
-// warps make three passes over the logits:
-//   pass 0: per-row maximum over tokens       (warp reduce-scatter, then cluster exchange)
-//   pass 1: per-row sum of exp2(x - max)      (same)
-//   pass 2: a_i = sum_r exp2(x_ri - max_r) / (sum_r * G*W), thread-local per token.
-// Logits are recomputed per pass from K tiles re-read through L2.
+// of 128-token tiles that a producer warp streams in with TMA (128-byte
+// swizzle).  Two passes over the tiles, each on the tensor cores:
+//   pass A  S^T = Q K_tile^T (M = 128 window rows, N = 128 tokens): TMEM lane =
+//           window row, so every consumer thread keeps an online (max, sum of
+//           exp2) of its own row with no cross-lane traffic.  Short windows
+//           (G*W < 128) are replicated across the 128 lanes and each copy takes
+//           a slice of the tile's tokens.  The per-row statistics are then
+//           merged across copies, warps and (through distributed shared
+//           memory) the CTAs of the cluster.
+//   pass B  S = K_tile Q^T (M = 128 tokens, N = window rows): TMEM lane =
+//           token, so each thread accumulates sum_r exp2(s_ri - m_r) / l_r of its
+//           token alone.
+// K tiles are re-read for pass B (from L2 for all but the largest units).
 #include <cfloat>
 
 #include "kernels.cuh"
@@ -26,30 +30,37 @@ namespace vase {
 
 namespace {
 
-constexpr int kConsumerWarps = 4;
-constexpr int kThreads = 32 * (kConsumerWarps + 1);
-constexpr uint32_t kStageBytes = kTileTokens * kRowBytes;  // 32 KB: two 64-column panels of 128 rows
-constexpr uint32_t kPanelBytes = kTileTokens * 128;        // 16 KB
+constexpr int kGroups = 2;                      // consumer warpgroups; group g takes the items i with i % 2 == g
+constexpr int kConsumers = 128 * kGroups;
+constexpr int kThreads = kConsumers + 32;       // + one producer warp (TMA + MMA issue)
+constexpr int kMaxBufs = 4;
+constexpr uint32_t kTileBytes = kTileTokens * kRowBytes;  // 32 KB: two 64-column panels of 128 rows
+constexpr uint32_t kPanelBytes = kTileTokens * 128;       // 16 KB
 
 struct ScoreSmem {
-    uint32_t q_off, k_off, bar_off, slot_off, wst_off, xin_off, rowm_off, roww_off, total;
+    uint32_t q_off, k_off, bar_off, slot_off, pm_off, pl_off, xm_off, xl_off, rowm_off, roww_off, total;
 };
 
-__host__ __device__ inline ScoreSmem score_layout(int GWp, int cluster, int stages) {
+__host__ __device__ inline ScoreSmem score_layout(int q_rows, int n_rbA, int GWp, int cluster, int stages,
+                                                   int stage_bytes) {
     ScoreSmem L;
     uint32_t o = 0;
     L.q_off = o;
-    o += static_cast<uint32_t>(GWp) * kRowBytes;  // two panels of GWp rows x 128 B
+    o += static_cast<uint32_t>(q_rows) * kRowBytes;
     L.k_off = o;
-    o += static_cast<uint32_t>(stages) * kStageBytes;
+    o += static_cast<uint32_t>(stages) * stage_bytes;
     L.bar_off = o;
-    o += 8 * (1 + 2 * stages + 4);
+    o += 8 * (1 + 2 * stages + 2 * kMaxBufs);
     o = (o + 15u) & ~15u;
     L.slot_off = o;
     o += 16;
-    L.wst_off = o;
-    o += 4u * kConsumerWarps * GWp;
-    L.xin_off = o;
+    L.pm_off = o;
+    o += 4u * n_rbA * kConsumers;  // [group][sub][128 lanes]
+    L.pl_off = o;
+    o += 4u * n_rbA * kConsumers;
+    L.xm_off = o;
+    o += 4u * cluster * GWp;
+    L.xl_off = o;
     o += 4u * cluster * GWp;
     L.rowm_off = o;
     o += 4u * GWp;
@@ -59,52 +70,19 @@ __host__ __device__ inline ScoreSmem score_layout(int GWp, int cluster, int stag
     return L;
 }
 
-struct OpMax {
-    __device__ __forceinline__ float operator()(float a, float b) const { return fmaxf(a, b); }
-};
-struct OpSum {
-    __device__ __forceinline__ float operator()(float a, float b) const { return a + b; }
-};
+// 2^x on the SFU (ex2.approx.ftz: relative error about 2^-22), no range fix-up.
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
 
-// Reduce 32 values per lane across the warp so that lane l ends with the
-// reduction of column l over all 32 lanes (31 shuffles instead of 160).
-template <class Op>
-__device__ __forceinline__ float warp_reduce_scatter(float (&v)[32], int lane, Op op) {
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        const bool up = lane & 16;
-        const float send = up ? v[i] : v[i + 16];
-        const float keep = up ? v[i + 16] : v[i];
-        v[i] = op(keep, __shfl_xor_sync(0xffffffffu, send, 16));
-    }
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const bool up = lane & 8;
-        const float send = up ? v[i] : v[i + 8];
-        const float keep = up ? v[i + 8] : v[i];
-        v[i] = op(keep, __shfl_xor_sync(0xffffffffu, send, 8));
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const bool up = lane & 4;
-        const float send = up ? v[i] : v[i + 4];
-        const float keep = up ? v[i + 4] : v[i];
-        v[i] = op(keep, __shfl_xor_sync(0xffffffffu, send, 4));
-    }
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-        const bool up = lane & 2;
-        const float send = up ? v[i] : v[i + 2];
-        const float keep = up ? v[i + 2] : v[i];
-        v[i] = op(keep, __shfl_xor_sync(0xffffffffu, send, 2));
-    }
-    {
-        const bool up = lane & 1;
-        const float send = up ? v[0] : v[1];
-        const float keep = up ? v[1] : v[0];
-        v[0] = op(keep, __shfl_xor_sync(0xffffffffu, send, 1));
-    }
-    return v[0];
+// (m, l) <- merge of two online-softmax partials in the exp2 domain.
+__device__ __forceinline__ void merge_ml(float& m, float& l, float m2, float l2) {
+    const float mn = fmaxf(m, m2);
+    if (mn == -INFINITY) return;
+    l = l * exp2f(m - mn) + l2 * exp2f(m2 - mn);
+    m = mn;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -112,53 +90,70 @@ __global__ void __launch_bounds__(kThreads, 1)
                       const ScoreAttnParams p) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const ScoreSmem L = score_layout(p.GWp, p.cluster, p.stages);
+    constexpr int stage_bytes = kTileBytes;
+    const ScoreSmem Ly = score_layout(p.q_rows, p.n_rbA, p.GWp, p.cluster, p.stages, stage_bytes);
 
-    uint8_t* q_s = smem + L.q_off;
-    uint8_t* k_s = smem + L.k_off;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L.bar_off);
+    uint8_t* q_s = smem + Ly.q_off;
+    uint8_t* st_s = smem + Ly.k_off;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Ly.bar_off);
     uint64_t* q_full = bars;
     uint64_t* k_full = bars + 1;
     uint64_t* k_empty = bars + 1 + p.stages;
-    uint64_t* t_full = bars + 1 + 2 * p.stages;
-    uint64_t* t_empty = t_full + 2;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.slot_off);
-    float* wst = reinterpret_cast<float*>(smem + L.wst_off);    // [4][GWp] per-warp partials
-    float* xin = reinterpret_cast<float*>(smem + L.xin_off);    // [C][GWp] cluster inbox
-    float* rowm = reinterpret_cast<float*>(smem + L.rowm_off);  // [GWp] scaled row max
-    float* roww = reinterpret_cast<float*>(smem + L.roww_off);  // [GWp] 1 / (row sum * G*W)
+    uint64_t* t_full = bars + 1 + 2 * p.stages;  // [nbuf]
+    uint64_t* t_empty = t_full + kMaxBufs;        // [nbuf]
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Ly.slot_off);
+    float* pm = reinterpret_cast<float*>(smem + Ly.pm_off);      // [group][n_rbA][128] running max per lane
+    float* pl = reinterpret_cast<float*>(smem + Ly.pl_off);      // [group][n_rbA][128] running sum per lane
+    float* xm = reinterpret_cast<float*>(smem + Ly.xm_off);      // [C][GWp] cluster inbox
+    float* xl = reinterpret_cast<float*>(smem + Ly.xl_off);
+    float* rowm = reinterpret_cast<float*>(smem + Ly.rowm_off);  // [GWp] row max (scaled, exp2 domain)
+    float* roww = reinterpret_cast<float*>(smem + Ly.roww_off);  // [GWp] 1 / (row sum * G*W)
 
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
     const int lane = tid & 31;
     const int unit = blockIdx.y;
     const int rank = blockIdx.x;
+    const int slot = blockIdx.z;  // layer slot of the batch
+    const int layer = p.batch.layer[slot];
+    float* const attn_out = p.attn + static_cast<int64_t>(slot) * p.n_rb * p.units * p.N;
     const int C = p.cluster;
     const int GWp = p.GWp;
     const int NB = p.NB;
     const int n_rb = p.n_rb;
+    const int n_rbA = p.n_rbA;
+    const int R = p.rep;                 // copies of the window rows across the 128 lanes in pass A
+    const int bufcols = p.buf_cols;      // TMEM columns per accumulator buffer
+    const int nbuf = p.nbuf;             // accumulator buffers (2 or 4)
     const int t_begin = rank * p.tiles_per_cta;
     const int t_end = min(p.n_tiles, t_begin + p.tiles_per_cta);
     const int n_my = max(0, t_end - t_begin);
-    const int64_t k_row = p.k_row0 + static_cast<int64_t>(unit) * p.N;
+    const int64_t k_row = static_cast<int64_t>(layer) * p.layer_rows + static_cast<int64_t>(unit) * p.N;
     const int seq = unit / p.Hkv;
     const int head = unit - seq * p.Hkv;
-    const int64_t q_row = p.q_row0 + (static_cast<int64_t>(seq) * p.Hq + static_cast<int64_t>(head) * p.G) * p.W;
+    const int64_t q_row = static_cast<int64_t>(layer) * p.q_layer_rows +
+                          (static_cast<int64_t>(seq) * p.Hq + static_cast<int64_t>(head) * p.G) * p.W;
+    const int itemsA = n_my * n_rbA;
+    const int itemsB = n_my * n_rb;
 
     if (tid == 0) {
         mbar_init(q_full, 1);
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&k_full[s], 1);
-            mbar_init(&k_empty[s], 1);
+            mbar_init(&k_empty[s], 1 + kConsumers);  // the last MMA commit + every consumer thread
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < nbuf; ++b) {
             mbar_init(&t_full[b], 1);
-            mbar_init(&t_empty[b], 32 * kConsumerWarps);
+            mbar_init(&t_empty[b], 128);  // the 128 threads of the group that owns the item
         }
         fence_mbar_init();
     }
-    for (int i = tid; i < kConsumerWarps * GWp; i += kThreads) wst[i] = -INFINITY;
-    if (warp == kConsumerWarps) {
+    for (int i = tid; i < n_rbA * kConsumers; i += kThreads) {
+        pm[i] = -INFINITY;
+        pl[i] = 0.f;
+    }
+    const int producer_warp = kConsumers / 32;
+    if (warp == producer_warp) {
         tmem_alloc(tmem_slot, static_cast<uint32_t>(p.tmem_cols));
         tmem_relinquish();
     }
@@ -169,28 +164,36 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (C > 1) cluster_sync();  // every peer is running before any DSMEM store
 
     bool ok = true;
-    const int total_items_per_pass = n_my * n_rb;
-    (void)total_items_per_pass;
 
-    if (warp == kConsumerWarps) {
+    if (warp == producer_warp) {
         // ---------------------------------------------------------------- producer warp
-        const uint32_t idesc = idesc_bf16_f32(128, static_cast<uint32_t>(NB));
+        const uint32_t idescA = idesc_bf16_f32(128, 128);
+        const uint32_t idescB = idesc_bf16_f32(128, static_cast<uint32_t>(NB));
         const uint32_t q_addr = smem_u32(q_s);
-        const uint32_t k_addr = smem_u32(k_s);
-        const int total_loads = 3 * n_my;
+        const uint32_t st_addr = smem_u32(st_s);
+        const int q_panel = p.q_rows * 128;  // bytes per 64-column panel of the window rows
+        const int total_loads = 2 * n_my;
         int load_next = 0;
         if (lane == 0) {
             tma_prefetch_desc(&kmap);
             tma_prefetch_desc(&qmap);
-            mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(GWp) * kRowBytes);
+            // window rows: R copies of the GWp rows (pass A lanes), or q_rows rows when R == 1
+            mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(p.q_rows) * kRowBytes);
             for (int panel = 0; panel < 2; ++panel) {
-                for (int r0 = 0; r0 < GWp; r0 += 256) {
-                    tma_load_2d(q_s + panel * GWp * 128 + r0 * 128, &qmap, panel * 64,
-                                static_cast<int32_t>(q_row + r0), q_full);
+                if (R > 1) {
+                    for (int c = 0; c < R; ++c)
+                        tma_load_2d(q_s + panel * q_panel + c * GWp * 128, &qmap, panel * 64,
+                                    static_cast<int32_t>(q_row), q_full);
+                } else {
+                    for (int r0 = 0; r0 < p.q_rows; r0 += p.q_box)
+                        tma_load_2d(q_s + panel * q_panel + r0 * 128, &qmap, panel * 64,
+                                    static_cast<int32_t>(q_row + r0), q_full);
                 }
             }
         }
-        for (int pass = 0; pass < 3; ++pass) {
+        int item = 0;  // global accumulator-buffer sequence over both passes
+        for (int pass = 0; pass < 2; ++pass) {
+            const int n_sub = pass == 0 ? n_rbA : n_rb;
             for (int j = 0; j < n_my; ++j) {
                 const int Lidx = pass * n_my + j;
                 const int s = Lidx % p.stages;
@@ -201,142 +204,206 @@ __global__ void __launch_bounds__(kThreads, 1)
                         if (ln > 0 && ok) ok = mbar_wait(&k_empty[ls], (ln - 1) & 1, p.err, kErrScoreKEmpty);
                         const int tile = t_begin + (load_next % n_my);
                         const int32_t row = static_cast<int32_t>(k_row + static_cast<int64_t>(tile) * kTileTokens);
-                        mbar_arrive_expect_tx(&k_full[ls], kStageBytes);
-                        tma_load_2d(k_s + ls * kStageBytes, &kmap, 0, row, &k_full[ls]);
-                        tma_load_2d(k_s + ls * kStageBytes + kPanelBytes, &kmap, 64, row, &k_full[ls]);
+                        uint8_t* st = st_s + ls * stage_bytes;
+                        mbar_arrive_expect_tx(&k_full[ls], kTileBytes);
+                        tma_load_2d(st, &kmap, 0, row, &k_full[ls]);
+                        tma_load_2d(st + kPanelBytes, &kmap, 64, row, &k_full[ls]);
                         ++load_next;
                     }
                     if (ok) ok = mbar_wait(&k_full[s], (Lidx / p.stages) & 1, p.err, kErrScoreKFull);
                     if (Lidx == 0 && ok) ok = mbar_wait(q_full, 0, p.err, kErrScoreQ);
                 }
-                for (int rb = 0; rb < n_rb; ++rb) {
-                    const int item = Lidx * n_rb + rb;
-                    const int buf = item & 1;
-                    const int use = item >> 1;
+                for (int sub = 0; sub < n_sub; ++sub, ++item) {
+                    const int buf = item % nbuf;
+                    const int use = item / nbuf;
                     if (lane == 0) {
                         if (use > 0 && ok) ok = mbar_wait(&t_empty[buf], (use - 1) & 1, p.err, kErrScoreTEmpty);
                         tc_fence_after();
                         if (ok) {
-                            const uint32_t a_base = k_addr + s * kStageBytes;
-                            const uint32_t b_base = q_addr + rb * NB * 128;
+                            const uint32_t kt = st_addr + s * stage_bytes;
 #pragma unroll
                             for (int kk = 0; kk < 8; ++kk) {
                                 const uint32_t koff = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
-                                const uint32_t qoff = (kk >> 2) * (GWp * 128) + (kk & 3) * 32;
-                                tc_mma_bf16(taddr + buf * NB, sw128_kmajor_desc(a_base + koff),
-                                            sw128_kmajor_desc(b_base + qoff), idesc, kk > 0 ? 1u : 0u);
+                                const uint32_t qoff = (kk >> 2) * q_panel + (kk & 3) * 32;
+                                if (pass == 0) {
+                                    // A = window rows of row block `sub` (128 lanes), B = the tile's tokens
+                                    tc_mma_bf16(taddr + buf * bufcols, sw128_kmajor_desc(q_addr + sub * 128 * 128 + qoff),
+                                                sw128_kmajor_desc(kt + koff), idescA, kk > 0 ? 1u : 0u);
+                                } else {
+                                    // A = the tile's tokens (128 lanes), B = window rows of row block `sub`
+                                    tc_mma_bf16(taddr + buf * bufcols, sw128_kmajor_desc(kt + koff),
+                                                sw128_kmajor_desc(q_addr + sub * NB * 128 + qoff), idescB,
+                                                kk > 0 ? 1u : 0u);
+                                }
                             }
                             tc_commit(&t_full[buf]);
-                            if (rb == n_rb - 1) tc_commit(&k_empty[s]);
+                            if (sub == n_sub - 1) tc_commit(&k_empty[s]);
                         } else {
-                            // keep the consumers' phases moving; their data is garbage and ignored
                             mbar_arrive(&t_full[buf]);
-                            if (rb == n_rb - 1) mbar_arrive(&k_empty[s]);
+                            if (sub == n_sub - 1) mbar_arrive(&k_empty[s]);
                         }
                     }
                     __syncwarp();
                 }
             }
             if (C > 1) {
-                if (pass == 0) {
+                if (pass == 0)
                     cluster_arrive();
-                } else if (pass == 1) {
+                else
                     cluster_wait();
-                    cluster_arrive();
-                } else {
-                    cluster_wait();
-                }
             }
         }
         // Drain: every issued TMA load and MMA must land before the CTA leaves.
         if (lane == 0) {
-            const int n_items = 3 * n_my * n_rb;
-            for (int b = 0; b < 2; ++b) {
-                const int uses = (n_items - b + 1) / 2;  // items with this buffer
+            const int n_items = itemsA + itemsB;
+            for (int b = 0; b < nbuf; ++b) {
+                const int uses = (n_items - b + nbuf - 1) / nbuf;
                 if (uses > 0) mbar_wait(&t_empty[b], (uses - 1) & 1, p.err, kErrScoreDrain);
             }
             for (int ls = 0; ls < p.stages && ls < total_loads; ++ls) {
-                const int last = ((total_loads - 1 - ls) / p.stages) * p.stages + ls;  // last load using stage ls
+                const int last = ((total_loads - 1 - ls) / p.stages) * p.stages + ls;
                 mbar_wait(&k_empty[ls], (last / p.stages) & 1, p.err, kErrScoreDrain);
             }
         }
         __syncwarp();
     } else {
-        // ---------------------------------------------------------------- consumer warps
-        const int ct = tid;  // 0..127
-        const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
-        const float scale = p.scale_log2;
-        for (int pass = 0; pass < 3; ++pass) {
-            for (int j = 0; j < n_my; ++j) {
-                const int Lidx = pass * n_my + j;
-                const int tile = t_begin + j;
-                const int token = tile * kTileTokens + warp * 32 + lane;
-                const bool valid = token < p.N;
-                float acc = 0.f;
-                for (int rb = 0; rb < n_rb; ++rb) {
-                    const int item = Lidx * n_rb + rb;
-                    const int buf = item & 1;
-                    const int use = item >> 1;
-                    if (ok) ok = mbar_wait(&t_full[buf], use & 1, p.err, kErrScoreTFull);
-                    tc_fence_after();
-                    for (int c = 0; c < NB / 32; ++c) {
-                        float v[32];
-                        tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * NB + c * 32), v);
-                        const int row0 = rb * NB + c * 32;
-                        if (pass == 0) {
+        // ---------------------------------------------------------------- consumer warpgroups
+        const int grp = tid >> 7;   // 0 or 1
+        const int L = tid & 127;    // TMEM lane
+        const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
+        const float cs = p.scale_log2;
+        // pass-A lane mapping: row (L mod rows_per_copy) of row block `sub`, token columns [c0, c0 + cw)
+        const int rows_per_copy = R > 1 ? GWp : 128;
+        const int copy = L / rows_per_copy;
+        const int cw = 128 / R;
+        const int c0 = copy * cw;
+        float* pmg = pm + grp * n_rbA * 128;
+        float* plg = pl + grp * n_rbA * 128;
+        // ------------------------------------ pass A: row statistics
+        for (int j = 0; j < n_my; ++j) {
+            const int tile = t_begin + j;
+            const int s = j % p.stages;
+            const int tok0 = tile * kTileTokens;
+            for (int sub = 0; sub < n_rbA; ++sub) {
+                const int item = j * n_rbA + sub;
+                if ((item & 1) != grp) continue;
+                const int buf = item % nbuf;
+                const int use = item / nbuf;
+                if (ok) ok = mbar_wait(&t_full[buf], use & 1, p.err, kErrScoreTFull);
+                tc_fence_after();
+                float m = pmg[sub * 128 + L];
+                float l = plg[sub * 128 + L];
+                for (int c = 0; c < cw; c += 32) {
+                    float v[32];
+                    tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), v);
+                    const int nvalid = min(32, p.N - (tok0 + c0 + c));
+                    float cm0 = -INFINITY, cm1 = -INFINITY;
 #pragma unroll
-                            for (int k = 0; k < 32; ++k) v[k] = valid ? v[k] : -INFINITY;
-                            const float r = warp_reduce_scatter(v, lane, OpMax());
-                            float* w = &wst[warp * GWp + row0 + lane];
-                            *w = fmaxf(*w, r);
-                        } else if (pass == 1) {
+                    for (int k = 0; k < 32; k += 2) {
+                        if (k >= nvalid) v[k] = -INFINITY;
+                        if (k + 1 >= nvalid) v[k + 1] = -INFINITY;
+                        cm0 = fmaxf(cm0, v[k]);
+                        cm1 = fmaxf(cm1, v[k + 1]);
+                    }
+                    const float mn = fmaxf(m, fmaxf(cm0, cm1) * cs);
+                    if (mn != -INFINITY) {
+                        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-                            for (int k = 0; k < 32; ++k)
-                                v[k] = valid ? exp2f(fmaf(v[k], scale, -rowm[row0 + k])) : 0.f;
-                            const float r = warp_reduce_scatter(v, lane, OpSum());
-                            wst[warp * GWp + row0 + lane] += r;
-                        } else {
-#pragma unroll
-                            for (int k = 0; k < 32; ++k)
-                                acc = fmaf(exp2f(fmaf(v[k], scale, -rowm[row0 + k])), roww[row0 + k], acc);
+                        for (int k = 0; k < 32; k += 4) {
+                            s0 += ex2(fmaf(v[k], cs, -mn));
+                            s1 += ex2(fmaf(v[k + 1], cs, -mn));
+                            s2 += ex2(fmaf(v[k + 2], cs, -mn));
+                            s3 += ex2(fmaf(v[k + 3], cs, -mn));
                         }
+                        l = l * ex2(m - mn) + ((s0 + s1) + (s2 + s3));
+                        m = mn;
                     }
-                    tc_fence_before();
-                    mbar_arrive(&t_empty[buf]);
                 }
-                if (pass == 2 && valid) p.attn[static_cast<int64_t>(unit) * p.N + token] = acc;
+                pmg[sub * 128 + L] = m;
+                plg[sub * 128 + L] = l;
+                tc_fence_before();
+                mbar_arrive(&t_empty[buf]);
             }
-            if (pass < 2) {
-                // combine the four warps, then the C CTAs of the cluster
-                named_bar(1, 32 * kConsumerWarps);
-                for (int row = ct; row < GWp; row += 32 * kConsumerWarps) {
-                    float x = wst[row];
-                    for (int w = 1; w < kConsumerWarps; ++w)
-                        x = pass == 0 ? fmaxf(x, wst[w * GWp + row]) : x + wst[w * GWp + row];
-                    for (int w = 0; w < kConsumerWarps; ++w) wst[w * GWp + row] = 0.f;
-                    if (C > 1) {
-                        for (int peer = 0; peer < C; ++peer)
-                            st_cluster_f32(map_to_rank(&xin[rank * GWp + row], static_cast<uint32_t>(peer)), x);
-                    } else {
-                        xin[row] = x;
-                    }
-                }
-                if (C > 1) {
-                    cluster_arrive();
-                    cluster_wait();
+            mbar_arrive(&k_empty[s]);
+        }
+        // ------------------------------------ merge the row statistics: groups, copies, then the cluster
+        named_bar(1, kConsumers);
+        for (int r = tid; r < GWp; r += kConsumers) {
+            float m = -INFINITY, l = 0.f;
+            for (int g = 0; g < kGroups; ++g) {
+                const float* gm = pm + g * n_rbA * 128;
+                const float* gl = pl + g * n_rbA * 128;
+                if (R > 1) {
+                    for (int c = 0; c < R; ++c) merge_ml(m, l, gm[c * GWp + r], gl[c * GWp + r]);
                 } else {
-                    named_bar(1, 32 * kConsumerWarps);
+                    merge_ml(m, l, gm[(r >> 7) * 128 + (r & 127)], gl[(r >> 7) * 128 + (r & 127)]);
                 }
-                for (int row = ct; row < GWp; row += 32 * kConsumerWarps) {
-                    float y = xin[row];
-                    for (int c = 1; c < C; ++c) y = pass == 0 ? fmaxf(y, xin[c * GWp + row]) : y + xin[c * GWp + row];
-                    if (pass == 0) {
-                        rowm[row] = row < p.GW ? y * scale : INFINITY;
-                    } else {
-                        roww[row] = row < p.GW ? p.inv_gw / y : 0.f;
+            }
+            if (C > 1) {
+                for (int peer = 0; peer < C; ++peer) {
+                    st_cluster_f32(map_to_rank(&xm[rank * GWp + r], static_cast<uint32_t>(peer)), m);
+                    st_cluster_f32(map_to_rank(&xl[rank * GWp + r], static_cast<uint32_t>(peer)), l);
+                }
+            } else {
+                xm[r] = m;
+                xl[r] = l;
+            }
+        }
+        if (C > 1) {
+            cluster_arrive();
+            cluster_wait();
+        } else {
+            named_bar(1, kConsumers);
+        }
+        for (int r = tid; r < GWp; r += kConsumers) {
+            float m = -INFINITY, l = 0.f;
+            for (int c = 0; c < C; ++c) merge_ml(m, l, xm[c * GWp + r], xl[c * GWp + r]);
+            const bool real = r < p.GW;
+            rowm[r] = real ? m : INFINITY;
+            roww[r] = real ? p.inv_gw / l : 0.f;
+        }
+        named_bar(1, kConsumers);
+        // ------------------------------------ pass B: per-token accumulation
+        // With two row blocks (G*W > 256) each group owns one of them for every tile and writes its own
+        // partial sum (attn part `grp`); the selection kernel adds the parts.
+        for (int j = 0; j < n_my; ++j) {
+            const int tile = t_begin + j;
+            const int s = (n_my + j) % p.stages;
+            const int token = tile * kTileTokens + L;
+            float acc = 0.f;
+            bool mine = false;
+            for (int sub = 0; sub < n_rb; ++sub) {
+                const int item = itemsA + j * n_rb + sub;
+                if ((item & 1) != grp) continue;
+                mine = true;
+                const int buf = item % nbuf;
+                const int use = item / nbuf;
+                if (ok) ok = mbar_wait(&t_full[buf], use & 1, p.err, kErrScoreTFull);
+                tc_fence_after();
+                for (int c = 0; c < NB; c += 32) {
+                    float v[32];
+                    tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), v);
+                    const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
+                    const float4* w4 = reinterpret_cast<const float4*>(roww + sub * NB + c);
+                    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        const float4 mm = m4[k];
+                        const float4 ww = w4[k];
+                        a0 = fmaf(ex2(fmaf(v[4 * k], cs, -mm.x)), ww.x, a0);
+                        a1 = fmaf(ex2(fmaf(v[4 * k + 1], cs, -mm.y)), ww.y, a1);
+                        a0 = fmaf(ex2(fmaf(v[4 * k + 2], cs, -mm.z)), ww.z, a0);
+                        a1 = fmaf(ex2(fmaf(v[4 * k + 3], cs, -mm.w)), ww.w, a1);
                     }
+                    acc += a0 + a1;
                 }
-                named_bar(1, 32 * kConsumerWarps);
+                tc_fence_before();
+                mbar_arrive(&t_empty[buf]);
+            }
+            mbar_arrive(&k_empty[s]);
+            if (mine && token < p.N) {
+                const int part = n_rb > 1 ? grp : 0;
+                attn_out[(static_cast<int64_t>(part) * p.units + unit) * p.N + token] = acc;
             }
         }
     }
@@ -344,13 +411,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == kConsumerWarps) tmem_dealloc(taddr, static_cast<uint32_t>(p.tmem_cols));
+    if (warp == producer_warp) tmem_dealloc(taddr, static_cast<uint32_t>(p.tmem_cols));
 }
 
 }  // namespace
 
-size_t score_attn_smem_bytes(int GWp, int cluster, int stages) {
-    return score_layout(GWp, cluster, stages).total + 1024;  // + alignment slack
+size_t score_attn_smem_bytes(int q_rows, int n_rbA, int GWp, int cluster, int stages) {
+    return score_layout(q_rows, n_rbA, GWp, cluster, stages, kTileBytes).total + 1024;
 }
 
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster) {
@@ -364,7 +431,7 @@ cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster) {
 cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreAttnParams& p, int units,
                               size_t smem_bytes, cudaStream_t s) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(p.cluster), static_cast<unsigned>(units), 1);
+    cfg.gridDim = dim3(static_cast<unsigned>(p.cluster), static_cast<unsigned>(units), static_cast<unsigned>(p.batch.n));
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem_bytes;
     cfg.stream = s;

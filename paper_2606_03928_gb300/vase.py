@@ -36,6 +36,7 @@ EXPORTED = [
     "vase_append_host", "vase_evict", "vase_read_positions", "vase_get_layer_state", "vase_set_layer_state",
     "vase_kv_view_get", "vase_debug_view_get", "vase_check_device_error", "vase_launch_count",
     "vase_status_string", "vase_last_error", "vase_abi_version", "vase_profile_enable", "vase_profile_collect",
+    "vase_append_all", "vase_evict_all", "vase_refresh_value_scores",
 ]
 KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select", "compact"]
 
@@ -48,11 +49,13 @@ class vase_config(ctypes.Structure):
 
 
 class vase_buffer_sizes(ctypes.Structure):
-    _fields_ = [(n, ctypes.c_size_t) for n in ("k_cache", "v_cache", "q_window", "positions", "workspace")]
+    _fields_ = [(n, ctypes.c_size_t) for n in ("k_cache", "v_cache", "q_window", "positions", "value_scores",
+                                               "workspace")]
 
 
 class vase_buffers(ctypes.Structure):
-    _fields_ = [(n, ctypes.c_void_p) for n in ("k_cache", "v_cache", "q_window", "positions", "workspace")]
+    _fields_ = [(n, ctypes.c_void_p) for n in ("k_cache", "v_cache", "q_window", "positions", "value_scores",
+                                               "workspace")]
 
 
 class vase_layer_state(ctypes.Structure):
@@ -62,12 +65,13 @@ class vase_layer_state(ctypes.Structure):
 
 class vase_kv_view(ctypes.Structure):
     _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("positions", ctypes.c_void_p),
-                ("unit_stride", ctypes.c_int64), ("slots", ctypes.c_int32), ("fill", ctypes.c_int32)]
+                ("value_scores", ctypes.c_void_p), ("unit_stride", ctypes.c_int64), ("slots", ctypes.c_int32),
+                ("fill", ctypes.c_int32)]
 
 
 class vase_debug_view(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in ("attn", "pooled", "value_score", "key", "keep", "src")] + [
-        ("units", ctypes.c_int32), ("slots", ctypes.c_int32)]
+        ("units", ctypes.c_int32), ("slots", ctypes.c_int32), ("layer", ctypes.c_int32)]
 
 
 _lib = None
@@ -90,12 +94,15 @@ def load(path: str = LIB_PATH):
         "vase_destroy": (None, [P]),
         "vase_append": (ctypes.c_int, [P, I32, P, P, P, I32, P]),
         "vase_append_host": (ctypes.c_int, [P, I32, P, P, P, I32, P]),
+        "vase_append_all": (ctypes.c_int, [P, P, P, P, I32, P]),
         "vase_evict": (ctypes.c_int, [P, I32, P]),
+        "vase_evict_all": (ctypes.c_int, [P, P]),
+        "vase_refresh_value_scores": (ctypes.c_int, [P, I32, P]),
         "vase_read_positions": (ctypes.c_int, [P, I32, P, P]),
         "vase_get_layer_state": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_layer_state)]),
         "vase_set_layer_state": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_layer_state)]),
         "vase_kv_view_get": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_kv_view)]),
-        "vase_debug_view_get": (ctypes.c_int, [P, ctypes.POINTER(vase_debug_view)]),
+        "vase_debug_view_get": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_debug_view)]),
         "vase_check_device_error": (ctypes.c_int, [P, P, ctypes.POINTER(U32)]),
         "vase_launch_count": (I64, [P]),
         "vase_status_string": (ctypes.c_char_p, [ctypes.c_int]),
@@ -132,7 +139,7 @@ def vase_get_buffer_sizes(cfg: vase_config) -> vase_buffer_sizes:
     out = vase_buffer_sizes()
     st = load().vase_get_buffer_sizes(ctypes.byref(cfg), ctypes.byref(out))
     if st != VASE_OK:
-        raise VaseError(st, "invalid VaSE configuration")
+        raise VaseError(st, "invalid VaSE configuration: " + load().vase_last_error(None).decode())
     return out
 
 
@@ -140,7 +147,7 @@ def vase_create(cfg: vase_config, bufs: vase_buffers) -> int:
     h = ctypes.c_void_p()
     st = load().vase_create(ctypes.byref(cfg), ctypes.byref(bufs), ctypes.byref(h))
     if st != VASE_OK:
-        raise VaseError(st, "vase_create failed")
+        raise VaseError(st, "vase_create failed: " + load().vase_last_error(None).decode())
     return h.value
 
 
@@ -170,8 +177,21 @@ def vase_append_host(ctx, layer, q_ptr, k_ptr, v_ptr, n_tokens, stream=None):
                   "vase_append_host")
 
 
+def vase_append_all(ctx, q_ptr, k_ptr, v_ptr, n_tokens, stream=None):
+    return _check(ctx, load().vase_append_all(ctx, q_ptr, k_ptr, v_ptr, n_tokens, _stream_ptr(stream)),
+                  "vase_append_all")
+
+
 def vase_evict(ctx, layer, stream=None):
     return _check(ctx, load().vase_evict(ctx, layer, _stream_ptr(stream)), "vase_evict")
+
+
+def vase_evict_all(ctx, stream=None):
+    return _check(ctx, load().vase_evict_all(ctx, _stream_ptr(stream)), "vase_evict_all")
+
+
+def vase_refresh_value_scores(ctx, layer, stream=None):
+    return _check(ctx, load().vase_refresh_value_scores(ctx, layer, _stream_ptr(stream)), "vase_refresh_value_scores")
 
 
 def vase_read_positions(ctx, layer, host_ptr, stream=None):
@@ -250,10 +270,12 @@ class VaseCache:
         self.q_window = torch.empty((g.num_layers, g.batch, g.num_q_heads, g.window, g.head_dim),
                                     dtype=torch.bfloat16, device=dev)
         self.positions = torch.full((g.num_layers, g.batch, g.num_kv_heads, N), -1, dtype=torch.int32, device=dev)
+        self.value_scores = torch.zeros((g.num_layers, g.batch, g.num_kv_heads, N), dtype=torch.float32, device=dev)
         self.workspace = torch.zeros(sizes.workspace, dtype=torch.uint8, device=dev)
         assert self.k_cache.numel() * 2 == sizes.k_cache and self.positions.numel() * 4 == sizes.positions
+        assert self.value_scores.numel() * 4 == sizes.value_scores
         bufs = vase_buffers(self.k_cache.data_ptr(), self.v_cache.data_ptr(), self.q_window.data_ptr(),
-                            self.positions.data_ptr(), self.workspace.data_ptr())
+                            self.positions.data_ptr(), self.value_scores.data_ptr(), self.workspace.data_ptr())
         with torch.cuda.device(dev):
             self.ctx = vase_create(self.cfg, bufs)
 
@@ -281,8 +303,22 @@ class VaseCache:
             assert (not t.is_cuda) and t.dtype == torch.bfloat16 and t.is_contiguous()
         return vase_append_host(self.ctx, layer, q.data_ptr(), k.data_ptr(), v.data_ptr(), q.shape[0], stream)
 
+    def append_all(self, q, k, v, stream=None):
+        """q [L, n, b, Hq, d], k/v [L, n, b, Hkv, d] bf16 CUDA tensors: n tokens for every layer, one launch."""
+        for t in (q, k, v):
+            assert t.is_cuda and t.dtype == torch.bfloat16 and t.is_contiguous()
+        return vase_append_all(self.ctx, q.data_ptr(), k.data_ptr(), v.data_ptr(), q.shape[1], stream)
+
     def evict(self, layer, stream=None):
         return vase_evict(self.ctx, layer, stream)
+
+    def refresh_value_scores(self, layer, stream=None):
+        """Recomputes the per-slot value magnitudes of one layer after its V rows were written directly."""
+        return vase_refresh_value_scores(self.ctx, layer, stream)
+
+    def evict_all(self, stream=None):
+        """Evicts every full layer in batched launches; returns how many layers were evicted."""
+        return vase_evict_all(self.ctx, stream)
 
     def read_positions(self, layer, out: torch.Tensor, stream=None):
         """Copies the K kept positions of every unit into a CPU int32 tensor [b, Hkv, K]."""
@@ -308,10 +344,11 @@ class VaseCache:
     def profile_collect(self):
         return vase_profile_collect(self.ctx)
 
-    def debug_view(self):
-        """Workspace results of the latest evict as tensors: attn, pooled, value_score, key [units, N], keep, src."""
+    def debug_view(self, slot=0):
+        """Workspace results of the latest eviction call for its slot-th layer: attn, pooled, value_score, key
+        [units, N], keep, src [units, K], and the layer they belong to."""
         dv = vase_debug_view()
-        _check(self.ctx, load().vase_debug_view_get(self.ctx, ctypes.byref(dv)), "vase_debug_view_get")
+        _check(self.ctx, load().vase_debug_view_get(self.ctx, slot, ctypes.byref(dv)), "vase_debug_view_get")
         base = self.workspace.data_ptr()
         U, N, K = dv.units, dv.slots, self.geometry.budget_k
 
@@ -326,4 +363,5 @@ class VaseCache:
             "key": sl(dv.key, U * N * 4, torch.float32).view(U, N),
             "keep": sl(dv.keep, U * N, torch.uint8).view(U, N),
             "src": sl(dv.src, U * K * 4, torch.int32).view(U, K),
+            "layer": dv.layer,
         }

@@ -43,6 +43,7 @@ def upload_layer(cache, layer: int, st: dict, round_index: int):
     N = cache.slots
     next_pos = int(st["positions"].max()) + 1
     cache.set_layer_state(layer, N, round_index, next_pos, 10 ** 6)
+    cache.refresh_value_scores(layer)
 
 
 def download(cache, layer):
@@ -51,10 +52,12 @@ def download(cache, layer):
         "k_bits": cache.k_cache[layer].view(torch.int16).cpu().numpy().view(np.uint16),
         "v_bits": cache.v_cache[layer].view(torch.int16).cpu().numpy().view(np.uint16),
         "positions": cache.positions[layer].cpu().numpy(),
+        "vmag": cache.value_scores[layer].cpu().numpy(),
     }
     dv = cache.debug_view()
     for k, v in dv.items():
-        out[k] = v.cpu().numpy()
+        if k != "layer":
+            out[k] = v.cpu().numpy()
     return out
 
 
@@ -80,7 +83,8 @@ def _near(values, thr, rtol=THRESH_RTOL):
     return np.abs(values - thr) <= rtol * abs(thr)
 
 
-def check_unit(wl, ref, got_unit, orig_k, orig_v, orig_pos, *, variant, n_v, check_scores=True):
+def check_unit(wl, ref, got_unit, orig_k, orig_v, orig_pos, *, variant, n_v, check_scores=True,
+               value_kind=O.VALUE_RANGE):
     """Compares one unit of a GPU eviction with the oracle's result `ref`."""
     K, B = wl.budget_k, wl.buffer_b
     N = K + B
@@ -94,11 +98,16 @@ def check_unit(wl, ref, got_unit, orig_k, orig_v, orig_pos, *, variant, n_v, che
     assert np.array_equal(got_unit["positions"][:K], orig_pos[src_g]), "compacted positions differ"
     assert np.all(got_unit["positions"][K:] == -1)
     assert set(range(K, N)) <= set(src_g.tolist()), "the buffer R_B is always kept"
+    # --- the per-slot value magnitudes moved with their rows (oracle magnitudes of the kept rows)
+    if got_unit.get("vmag") is not None:
+        vm_ref = O.value_magnitude(O.bf16_bits_to_f64(orig_v[src_g]), value_kind)
+        assert_close_scores(got_unit["vmag"][:K], vm_ref, "compacted value magnitudes")
     # --- scores
     if check_scores:
         if variant == "attnv":
             assert_close_scores(got_unit["attn"], ref["attn"], "window attention score")
-            assert_close_scores(got_unit["value_score"][:K], ref["value_score"], "value magnitude")
+            if got_unit.get("value_score") is not None:
+                assert_close_scores(got_unit["value_score"][:K], ref["value_score"], "value magnitude")
             if got_unit.get("pooled") is not None:
                 assert_close_scores(got_unit["pooled"], ref["pooled"], "pooled score")
             if got_unit.get("key") is not None:
@@ -139,6 +148,6 @@ def unit_slice(got, s, h, Hkv):
     u = s * Hkv + h
     return {
         "k_bits": got["k_bits"][s, h], "v_bits": got["v_bits"][s, h], "positions": got["positions"][s, h],
-        "src": got["src"][u], "attn": got["attn"][u], "pooled": got["pooled"][u],
+        "src": got["src"][u], "attn": got["attn"][u], "pooled": got["pooled"][u], "vmag": got["vmag"][s, h],
         "value_score": got["value_score"][u], "key": got["key"][u],
     }

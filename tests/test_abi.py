@@ -89,4 +89,4 @@ def test_paper_defaults(lib):
 
 def test_status_strings(lib):
     assert lib.vase_status_string(-3) == b"cache not full"
-    assert lib.vase_abi_version() == 1
+    assert lib.vase_abi_version() == 2

@@ -70,8 +70,10 @@ def _run_layer(wl, *, variant="attnv", layer=1, num_layers=2, round_index=3, see
         if not debug:
             gu["pooled"] = None
             gu["key"] = None
+            if variant == "attnv":  # written to the workspace only with debug outputs (DKV always writes it)
+                gu["value_score"] = None
         flips += PU.check_unit(wl, ref, gu, st["k_bits"][s, h], st["v_bits"][s, h], st["positions"][s, h],
-                               variant=variant, n_v=nv)
+                               variant=variant, n_v=nv, value_kind=cache_kw.get("value_score", O.VALUE_RANGE))
     # properties that hold at any size, checked on every unit
     K, B = wl.budget_k, wl.buffer_b
     for s in range(wl.batch):
@@ -301,6 +303,7 @@ def test_gpu_keep_frequencies_match_successive_sampling():
         cache.q_window[0].copy_(qt)
         cache.positions[0].copy_(pt)
         cache.set_layer_state(0, N, t, N, 10 ** 6)
+        cache.refresh_value_scores(0)
         cache.evict(0)
         src = cache.debug_view()["src"].cpu().numpy()
         for u in range(64):
@@ -339,3 +342,57 @@ def test_qwen3_32b_k8192_sampled_units():
     wl = W.WORKLOADS["qwen3_32b_k8192"]
     units = [(0, 0), (7, 5), (15, 7)]
     _run_layer(wl, layer=1, num_layers=2, round_index=95, units=units, debug=True)
+
+
+# ----------------------------------------------------------------------------- batched layers
+
+def test_evict_all_equals_per_layer_evictions_and_matches_oracle():
+    """vase_evict_all covers every full layer in one launch per kernel; results equal per-layer calls."""
+    wl = W.shrink(SMALL, budget_k=192, buffer_b=64, window=16, batch=2, num_layers=3)
+    a = _cache(wl, 3)
+    b = _cache(wl, 3)
+    states = [W.layer_state(wl, 4, layer, 2 + layer, "gapped") for layer in range(3)]
+    for layer, st in enumerate(states):
+        PU.upload_layer(a, layer, st, 2 + layer)
+        PU.upload_layer(b, layer, st, 2 + layer)
+    for layer in range(3):
+        a.evict(layer)
+    assert b.evict_all() == 3
+    torch.cuda.synchronize()
+    assert torch.equal(a.k_cache, b.k_cache) and torch.equal(a.v_cache, b.v_cache)
+    assert torch.equal(a.positions, b.positions)
+    assert b.check_device_error()[0] == 0
+    for z in range(3):
+        dv = {k: (v.cpu().numpy() if k != "layer" else v) for k, v in b.debug_view(z).items()}
+        layer = dv["layer"]
+        assert layer == z
+        st = states[layer]
+        got = PU.download(b, layer)
+        got.update({k: v for k, v in dv.items() if k != "layer"})
+        for s in range(wl.batch):
+            for h in range(wl.num_kv_heads):
+                ref = PU.oracle_unit(wl, st, s, h, variant="attnv", round_index=2 + layer, seed=0, layer=layer)
+                PU.check_unit(wl, ref, PU.unit_slice(got, s, h, wl.num_kv_heads), st["k_bits"][s, h],
+                              st["v_bits"][s, h], st["positions"][s, h], variant="attnv", n_v=wl.budget_k // 4)
+        assert b.layer_state(layer)["round"] == 3 + layer
+
+
+def test_append_all_equals_per_layer_appends():
+    wl = W.shrink(SMALL, budget_k=64, buffer_b=16, window=8, batch=2, num_layers=3)
+    a = _cache(wl, 3)
+    b = _cache(wl, 3)
+    dev = a.device
+    chunks = [W.stream_chunk(wl, 9, layer, 0, 40) for layer in range(3)]
+    qs = [PU.bits_to_bf16_tensor(c["q_bits"], dev) for c in chunks]
+    ks = [PU.bits_to_bf16_tensor(c["k_bits"], dev) for c in chunks]
+    vs = [PU.bits_to_bf16_tensor(c["v_bits"], dev) for c in chunks]
+    for layer in range(3):
+        a.append(layer, qs[layer], ks[layer], vs[layer])
+    b.append_all(torch.stack(qs), torch.stack(ks), torch.stack(vs))
+    torch.cuda.synchronize()
+    # only the first 40 slots were written (the rest of both caches is uninitialised memory)
+    assert torch.equal(a.k_cache[:, :, :, :40], b.k_cache[:, :, :, :40])
+    assert torch.equal(a.v_cache[:, :, :, :40], b.v_cache[:, :, :, :40])
+    assert torch.equal(a.q_window, b.q_window) and torch.equal(a.positions, b.positions)
+    for layer in range(3):
+        assert a.layer_state(layer) == b.layer_state(layer)

@@ -32,7 +32,7 @@ namespace {
 
 constexpr int kGroups = 2;                      // consumer warpgroups; group g takes the items i with i % 2 == g
 constexpr int kConsumers = 128 * kGroups;
-constexpr int kThreads = kConsumers + 32;       // + one producer warp (TMA + MMA issue)
+constexpr int kThreads = kConsumers + 64;       // + a TMA warp and an MMA-issue warp
 constexpr int kMaxBufs = 4;
 constexpr uint32_t kTileBytes = kTileTokens * kRowBytes;  // 32 KB: two 64-column panels of 128 rows
 constexpr uint32_t kPanelBytes = kTileTokens * 128;       // 16 KB
@@ -152,8 +152,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         pm[i] = -INFINITY;
         pl[i] = 0.f;
     }
-    const int producer_warp = kConsumers / 32;
-    if (warp == producer_warp) {
+    const int tma_warp = kConsumers / 32;
+    const int mma_warp = tma_warp + 1;
+    if (warp == tma_warp) {
         tmem_alloc(tmem_slot, static_cast<uint32_t>(p.tmem_cols));
         tmem_relinquish();
     }
@@ -164,20 +165,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (C > 1) cluster_sync();  // every peer is running before any DSMEM store
 
     bool ok = true;
+    const int total_loads = 2 * n_my;
 
-    if (warp == producer_warp) {
-        // ---------------------------------------------------------------- producer warp
-        const uint32_t idescA = idesc_bf16_f32(128, 128);
-        const uint32_t idescB = idesc_bf16_f32(128, static_cast<uint32_t>(NB));
-        const uint32_t q_addr = smem_u32(q_s);
-        const uint32_t st_addr = smem_u32(st_s);
-        const int q_panel = p.q_rows * 128;  // bytes per 64-column panel of the window rows
-        const int total_loads = 2 * n_my;
-        int load_next = 0;
+    if (warp == tma_warp) {
+        // ---------------------------------------------------------------- TMA warp: window rows, then K tiles
+        if (C > 1) cluster_arrive();  // this warp takes no part in the statistics exchange
         if (lane == 0) {
             tma_prefetch_desc(&kmap);
             tma_prefetch_desc(&qmap);
             // window rows: R copies of the GWp rows (pass A lanes), or q_rows rows when R == 1
+            const int q_panel = p.q_rows * 128;
             mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(p.q_rows) * kRowBytes);
             for (int panel = 0; panel < 2; ++panel) {
                 if (R > 1) {
@@ -190,33 +187,46 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     static_cast<int32_t>(q_row + r0), q_full);
                 }
             }
+            // K tiles of pass A, then again for pass B (second read served by L2)
+            for (int ld = 0; ld < total_loads; ++ld) {
+                const int ls = ld % p.stages;
+                const int ln = ld / p.stages;
+                if (ln > 0 && ok) ok = mbar_wait(&k_empty[ls], (ln - 1) & 1, p.err, kErrScoreKEmpty);
+                const int tile = t_begin + (ld % n_my);
+                const int32_t row = static_cast<int32_t>(k_row + static_cast<int64_t>(tile) * kTileTokens);
+                uint8_t* st = st_s + ls * stage_bytes;
+                mbar_arrive_expect_tx(&k_full[ls], kTileBytes);
+                tma_load_2d(st, &kmap, 0, row, &k_full[ls]);
+                tma_load_2d(st + kPanelBytes, &kmap, 64, row, &k_full[ls]);
+            }
+            // drain: every load has been consumed (and so has landed) before the CTA leaves
+            for (int ls = 0; ls < p.stages && ls < total_loads; ++ls) {
+                const int last = ((total_loads - 1 - ls) / p.stages) * p.stages + ls;
+                mbar_wait(&k_empty[ls], (last / p.stages) & 1, p.err, kErrScoreDrain);
+            }
         }
-        int item = 0;  // global accumulator-buffer sequence over both passes
-        for (int pass = 0; pass < 2; ++pass) {
-            const int n_sub = pass == 0 ? n_rbA : n_rb;
-            for (int j = 0; j < n_my; ++j) {
-                const int Lidx = pass * n_my + j;
-                const int s = Lidx % p.stages;
-                if (lane == 0) {
-                    while (load_next < total_loads && load_next < Lidx + p.stages) {
-                        const int ls = load_next % p.stages;
-                        const int ln = load_next / p.stages;
-                        if (ln > 0 && ok) ok = mbar_wait(&k_empty[ls], (ln - 1) & 1, p.err, kErrScoreKEmpty);
-                        const int tile = t_begin + (load_next % n_my);
-                        const int32_t row = static_cast<int32_t>(k_row + static_cast<int64_t>(tile) * kTileTokens);
-                        uint8_t* st = st_s + ls * stage_bytes;
-                        mbar_arrive_expect_tx(&k_full[ls], kTileBytes);
-                        tma_load_2d(st, &kmap, 0, row, &k_full[ls]);
-                        tma_load_2d(st + kPanelBytes, &kmap, 64, row, &k_full[ls]);
-                        ++load_next;
-                    }
+        __syncwarp();
+        if (C > 1) cluster_wait();
+    } else if (warp == mma_warp) {
+        // ---------------------------------------------------------------- MMA warp: one thread issues tcgen05.mma
+        if (C > 1) cluster_arrive();
+        if (lane == 0) {
+            const uint32_t idescA = idesc_bf16_f32(128, 128);
+            const uint32_t idescB = idesc_bf16_f32(128, static_cast<uint32_t>(NB));
+            const uint32_t q_addr = smem_u32(q_s);
+            const uint32_t st_addr = smem_u32(st_s);
+            const int q_panel = p.q_rows * 128;  // bytes per 64-column panel of the window rows
+            if (ok) ok = mbar_wait(q_full, 0, p.err, kErrScoreQ);
+            int item = 0;  // global accumulator-buffer sequence over both passes
+            for (int pass = 0; pass < 2; ++pass) {
+                const int n_sub = pass == 0 ? n_rbA : n_rb;
+                for (int j = 0; j < n_my; ++j) {
+                    const int Lidx = pass * n_my + j;
+                    const int s = Lidx % p.stages;
                     if (ok) ok = mbar_wait(&k_full[s], (Lidx / p.stages) & 1, p.err, kErrScoreKFull);
-                    if (Lidx == 0 && ok) ok = mbar_wait(q_full, 0, p.err, kErrScoreQ);
-                }
-                for (int sub = 0; sub < n_sub; ++sub, ++item) {
-                    const int buf = item % nbuf;
-                    const int use = item / nbuf;
-                    if (lane == 0) {
+                    for (int sub = 0; sub < n_sub; ++sub, ++item) {
+                        const int buf = item % nbuf;
+                        const int use = item / nbuf;
                         if (use > 0 && ok) ok = mbar_wait(&t_empty[buf], (use - 1) & 1, p.err, kErrScoreTEmpty);
                         tc_fence_after();
                         if (ok) {
@@ -227,7 +237,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 const uint32_t qoff = (kk >> 2) * q_panel + (kk & 3) * 32;
                                 if (pass == 0) {
                                     // A = window rows of row block `sub` (128 lanes), B = the tile's tokens
-                                    tc_mma_bf16(taddr + buf * bufcols, sw128_kmajor_desc(q_addr + sub * 128 * 128 + qoff),
+                                    tc_mma_bf16(taddr + buf * bufcols,
+                                                sw128_kmajor_desc(q_addr + sub * 128 * 128 + qoff),
                                                 sw128_kmajor_desc(kt + koff), idescA, kk > 0 ? 1u : 0u);
                                 } else {
                                     // A = the tile's tokens (128 lanes), B = window rows of row block `sub`
@@ -239,33 +250,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc_commit(&t_full[buf]);
                             if (sub == n_sub - 1) tc_commit(&k_empty[s]);
                         } else {
+                            // keep every phase moving; the data is garbage and the error word is set
                             mbar_arrive(&t_full[buf]);
                             if (sub == n_sub - 1) mbar_arrive(&k_empty[s]);
                         }
                     }
-                    __syncwarp();
                 }
             }
-            if (C > 1) {
-                if (pass == 0)
-                    cluster_arrive();
-                else
-                    cluster_wait();
-            }
-        }
-        // Drain: every issued TMA load and MMA must land before the CTA leaves.
-        if (lane == 0) {
+            // drain: the consumers have read every accumulator, so every MMA has completed
             const int n_items = itemsA + itemsB;
             for (int b = 0; b < nbuf; ++b) {
                 const int uses = (n_items - b + nbuf - 1) / nbuf;
                 if (uses > 0) mbar_wait(&t_empty[b], (uses - 1) & 1, p.err, kErrScoreDrain);
             }
-            for (int ls = 0; ls < p.stages && ls < total_loads; ++ls) {
-                const int last = ((total_loads - 1 - ls) / p.stages) * p.stages + ls;
-                mbar_wait(&k_empty[ls], (last / p.stages) & 1, p.err, kErrScoreDrain);
-            }
         }
         __syncwarp();
+        if (C > 1) cluster_wait();
     } else {
         // ---------------------------------------------------------------- consumer warpgroups
         const int grp = tid >> 7;   // 0 or 1
@@ -293,23 +293,40 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 float m = pmg[sub * 128 + L];
                 float l = plg[sub * 128 + L];
-                for (int c = 0; c < cw; c += 32) {
-                    float v[32];
-                    tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), v);
-                    const int nvalid = min(32, p.N - (tok0 + c0 + c));
-                    float cm0 = -INFINITY, cm1 = -INFINITY;
+                // online (max, sum of exp2) over this lane's token columns, 64 (or 32) at a time
+                for (int c = 0; c < cw; c += 64) {
+                    float v[64];
+                    const int width = cw - c >= 64 ? 64 : 32;
+                    if (width == 64) {
+                        tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), v);
+                    } else {
+                        float h[32];
+                        tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), h);
 #pragma unroll
-                    for (int k = 0; k < 32; k += 2) {
-                        if (k >= nvalid) v[k] = -INFINITY;
-                        if (k + 1 >= nvalid) v[k + 1] = -INFINITY;
+                        for (int k = 0; k < 32; ++k) {
+                            v[k] = h[k];
+                            v[k + 32] = -INFINITY;
+                        }
+                    }
+                    const int nvalid = min(width, p.N - (tok0 + c0 + c));
+                    if (nvalid < 64) {
+#pragma unroll
+                        for (int k = 0; k < 64; ++k)
+                            if (k >= nvalid) v[k] = -INFINITY;
+                    }
+                    float cm0 = v[0], cm1 = v[1], cm2 = v[2], cm3 = v[3];
+#pragma unroll
+                    for (int k = 4; k < 64; k += 4) {
                         cm0 = fmaxf(cm0, v[k]);
                         cm1 = fmaxf(cm1, v[k + 1]);
+                        cm2 = fmaxf(cm2, v[k + 2]);
+                        cm3 = fmaxf(cm3, v[k + 3]);
                     }
-                    const float mn = fmaxf(m, fmaxf(cm0, cm1) * cs);
+                    const float mn = fmaxf(m, fmaxf(fmaxf(cm0, cm1), fmaxf(cm2, cm3)) * cs);
                     if (mn != -INFINITY) {
                         float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-                        for (int k = 0; k < 32; k += 4) {
+                        for (int k = 0; k < 64; k += 4) {
                             s0 += ex2(fmaf(v[k], cs, -mn));
                             s1 += ex2(fmaf(v[k + 1], cs, -mn));
                             s2 += ex2(fmaf(v[k + 2], cs, -mn));
@@ -380,22 +397,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int use = item / nbuf;
                 if (ok) ok = mbar_wait(&t_full[buf], use & 1, p.err, kErrScoreTFull);
                 tc_fence_after();
-                for (int c = 0; c < NB; c += 32) {
-                    float v[32];
-                    tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), v);
+                for (int c = 0; c < NB; c += 64) {
+                    float v[64];
+                    const int width = NB - c >= 64 ? 64 : 32;
+                    if (width == 64) {
+                        tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), v);
+                    } else {
+                        float h[32];
+                        tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), h);
+#pragma unroll
+                        for (int k = 0; k < 32; ++k) v[k] = h[k];
+                    }
                     const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
                     const float4* w4 = reinterpret_cast<const float4*>(roww + sub * NB + c);
-                    float a0 = 0.f, a1 = 0.f;
+                    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        const float4 mm = m4[k];
-                        const float4 ww = w4[k];
-                        a0 = fmaf(ex2(fmaf(v[4 * k], cs, -mm.x)), ww.x, a0);
-                        a1 = fmaf(ex2(fmaf(v[4 * k + 1], cs, -mm.y)), ww.y, a1);
-                        a0 = fmaf(ex2(fmaf(v[4 * k + 2], cs, -mm.z)), ww.z, a0);
-                        a1 = fmaf(ex2(fmaf(v[4 * k + 3], cs, -mm.w)), ww.w, a1);
+                    for (int k = 0; k < 16; ++k) {
+                        if (k < width / 4) {
+                            const float4 mm = m4[k];
+                            const float4 ww = w4[k];
+                            a0 = fmaf(ex2(fmaf(v[4 * k], cs, -mm.x)), ww.x, a0);
+                            a1 = fmaf(ex2(fmaf(v[4 * k + 1], cs, -mm.y)), ww.y, a1);
+                            a2 = fmaf(ex2(fmaf(v[4 * k + 2], cs, -mm.z)), ww.z, a2);
+                            a3 = fmaf(ex2(fmaf(v[4 * k + 3], cs, -mm.w)), ww.w, a3);
+                        }
                     }
-                    acc += a0 + a1;
+                    acc += (a0 + a1) + (a2 + a3);
                 }
                 tc_fence_before();
                 mbar_arrive(&t_empty[buf]);
@@ -411,7 +438,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == producer_warp) tmem_dealloc(taddr, static_cast<uint32_t>(p.tmem_cols));
+    if (warp == tma_warp) tmem_dealloc(taddr, static_cast<uint32_t>(p.tmem_cols));
 }
 
 }  // namespace

@@ -209,43 +209,47 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (C > 1) cluster_wait();
     } else if (warp == mma_warp) {
         // ---------------------------------------------------------------- MMA warp: one thread issues tcgen05.mma
+        // The issuing thread shares its SM sub-partition with consumer warps, so its instruction stream is kept
+        // short: descriptors are built once and advanced by adding to the 14-bit start-address field.
         if (C > 1) cluster_arrive();
         if (lane == 0) {
             const uint32_t idescA = idesc_bf16_f32(128, 128);
             const uint32_t idescB = idesc_bf16_f32(128, static_cast<uint32_t>(NB));
-            const uint32_t q_addr = smem_u32(q_s);
-            const uint32_t st_addr = smem_u32(st_s);
-            const int q_panel = p.q_rows * 128;  // bytes per 64-column panel of the window rows
+            const uint32_t q_panel = static_cast<uint32_t>(p.q_rows) * 128u;  // bytes per 64-column panel
+            const uint64_t qdesc = sw128_kmajor_desc(smem_u32(q_s));
+            const uint64_t kdesc = sw128_kmajor_desc(smem_u32(st_s));
+            // start-address steps (16-byte units) of the eight K = 16 slices of d = 128
+            uint32_t koff[8], qoff[8];
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+                koff[kk] = ((kk >> 2) * kPanelBytes + (kk & 3) * 32) >> 4;
+                qoff[kk] = ((kk >> 2) * q_panel + (kk & 3) * 32) >> 4;
+            }
             if (ok) ok = mbar_wait(q_full, 0, p.err, kErrScoreQ);
-            int item = 0;  // global accumulator-buffer sequence over both passes
+            int s = 0, s_phase = 0;        // K stage ring position
+            int buf = 0, use = 0;          // accumulator ring position
             for (int pass = 0; pass < 2; ++pass) {
                 const int n_sub = pass == 0 ? n_rbA : n_rb;
                 for (int j = 0; j < n_my; ++j) {
-                    const int Lidx = pass * n_my + j;
-                    const int s = Lidx % p.stages;
-                    if (ok) ok = mbar_wait(&k_full[s], (Lidx / p.stages) & 1, p.err, kErrScoreKFull);
-                    for (int sub = 0; sub < n_sub; ++sub, ++item) {
-                        const int buf = item % nbuf;
-                        const int use = item / nbuf;
+                    if (ok) ok = mbar_wait(&k_full[s], s_phase, p.err, kErrScoreKFull);
+                    const uint64_t kt = kdesc + ((static_cast<uint32_t>(s) * stage_bytes) >> 4);
+                    for (int sub = 0; sub < n_sub; ++sub) {
                         if (use > 0 && ok) ok = mbar_wait(&t_empty[buf], (use - 1) & 1, p.err, kErrScoreTEmpty);
                         tc_fence_after();
+                        const uint32_t d = taddr + static_cast<uint32_t>(buf * bufcols);
                         if (ok) {
-                            const uint32_t kt = st_addr + s * stage_bytes;
+                            if (pass == 0) {
+                                // A = window rows of row block `sub` (128 lanes), B = the tile's tokens
+                                const uint64_t qa = qdesc + ((static_cast<uint32_t>(sub) * 128u * 128u) >> 4);
 #pragma unroll
-                            for (int kk = 0; kk < 8; ++kk) {
-                                const uint32_t koff = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
-                                const uint32_t qoff = (kk >> 2) * q_panel + (kk & 3) * 32;
-                                if (pass == 0) {
-                                    // A = window rows of row block `sub` (128 lanes), B = the tile's tokens
-                                    tc_mma_bf16(taddr + buf * bufcols,
-                                                sw128_kmajor_desc(q_addr + sub * 128 * 128 + qoff),
-                                                sw128_kmajor_desc(kt + koff), idescA, kk > 0 ? 1u : 0u);
-                                } else {
-                                    // A = the tile's tokens (128 lanes), B = window rows of row block `sub`
-                                    tc_mma_bf16(taddr + buf * bufcols, sw128_kmajor_desc(kt + koff),
-                                                sw128_kmajor_desc(q_addr + sub * NB * 128 + qoff), idescB,
-                                                kk > 0 ? 1u : 0u);
-                                }
+                                for (int kk = 0; kk < 8; ++kk)
+                                    tc_mma_bf16(d, qa + qoff[kk], kt + koff[kk], idescA, kk > 0 ? 1u : 0u);
+                            } else {
+                                // A = the tile's tokens (128 lanes), B = window rows of row block `sub`
+                                const uint64_t qb = qdesc + ((static_cast<uint32_t>(sub) * NB * 128u) >> 4);
+#pragma unroll
+                                for (int kk = 0; kk < 8; ++kk)
+                                    tc_mma_bf16(d, kt + koff[kk], qb + qoff[kk], idescB, kk > 0 ? 1u : 0u);
                             }
                             tc_commit(&t_full[buf]);
                             if (sub == n_sub - 1) tc_commit(&k_empty[s]);
@@ -254,6 +258,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                             mbar_arrive(&t_full[buf]);
                             if (sub == n_sub - 1) mbar_arrive(&k_empty[s]);
                         }
+                        if (++buf == nbuf) {
+                            buf = 0;
+                            ++use;
+                        }
+                    }
+                    if (++s == p.stages) {
+                        s = 0;
+                        s_phase ^= 1;
                     }
                 }
             }

@@ -145,12 +145,12 @@ __global__ void value_score_kernel(const ValueParams p) {
 }
 
 // ------------------------------------------------------------------ selection
-constexpr int kSelThreads = 512;
+constexpr int kSelThreads = 256;
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr uint8_t kFlagValue = 1;
 constexpr uint8_t kFlagSampled = 2;
 
-constexpr int kSelBins = 2048;
+constexpr int kSelBins = 256;
 
 struct SelShared {
     uint32_t hist[kSelBins];
@@ -190,7 +190,7 @@ __device__ __forceinline__ int block_exclusive_scan(int v, SelShared& sh, int* t
 }
 
 // Marks with `flag` the k largest values of ord[0..n) (ties to the lower
-// index), by an MSB-first radix select on 11/11/10-bit digits (lanes with the
+// index), by an MSB-first radix select on four 8-bit digits (lanes with the
 // same digit are merged with __match_any_sync before the shared-memory atomic)
 // followed by a slot-ordered rank of the elements equal to the threshold.
 // Each thread owns the contiguous slots [seg_lo, seg_hi).
@@ -201,27 +201,28 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
     const int lane = tid & 31;
     uint32_t prefix = 0, mask = 0;
     int remain = k;
-    const int shifts[3] = {21, 10, 0};
-    const int widths[3] = {11, 11, 10};
-    for (int pass = 0; pass < 3; ++pass) {
-        const int shift = shifts[pass];
-        const uint32_t dmask = (1u << widths[pass]) - 1u;
-        for (int i = tid; i < kSelBins; i += kSelThreads) sh.hist[i] = 0;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        sh.hist[tid] = 0;  // kSelThreads == kSelBins
         __syncthreads();
         const int n_round = (n + 31) & ~31;
         for (int i = tid; i < n_round; i += kSelThreads) {
             const uint32_t x = i < n ? ord[i] : 0u;
             const bool in = i < n && (x & mask) == prefix;
-            const uint32_t bin = in ? ((x >> shift) & dmask) : 0xFFFFFFFFu;
+            const uint32_t bin = in ? ((x >> shift) & 0xFFu) : 0xFFFFFFFFu;
             const uint32_t peers = __match_any_sync(0xffffffffu, bin);
             if (in && lane == __ffs(peers) - 1) atomicAdd(&sh.hist[bin], static_cast<uint32_t>(__popc(peers)));
         }
         __syncthreads();
         if (tid < 32) {
-            constexpr int per = kSelBins / 32;  // bins per lane
+            // lane owns bins 8*lane .. 8*lane+7; suffix sums find the digit holding the remain-th largest
+            uint32_t c[8];
             uint32_t tot = 0;
-            for (int j = 0; j < per; ++j) tot += sh.hist[per * lane + ((j + lane) & (per - 1))];  // bank-rotated
-            uint32_t suf = tot;  // inclusive suffix sum over lanes >= lane
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                c[j] = sh.hist[8 * lane + ((j + lane) & 7)];  // bank-rotated read
+                tot += c[j];
+            }
+            uint32_t suf = tot;
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
                 const uint32_t y = __shfl_down_sync(0xffffffffu, suf, o);
@@ -229,23 +230,21 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
             }
             uint32_t above = suf - tot;
             if (above < static_cast<uint32_t>(remain) && suf >= static_cast<uint32_t>(remain)) {
-                for (int j = per - 1; j >= 0; --j) {
-                    const uint32_t c = sh.hist[per * lane + j];
-                    if (above + c >= static_cast<uint32_t>(remain)) {
-                        sh.bcast[0] = static_cast<uint32_t>(per * lane + j);
+#pragma unroll
+                for (int j = 7; j >= 0; --j) {
+                    const uint32_t cj = sh.hist[8 * lane + j];
+                    if (above < static_cast<uint32_t>(remain) && above + cj >= static_cast<uint32_t>(remain)) {
+                        sh.bcast[0] = static_cast<uint32_t>(8 * lane + j);
                         sh.bcast[1] = above;
-                        break;
                     }
-                    above += c;
+                    above += cj;
                 }
             }
         }
         __syncthreads();
-        const uint32_t digit = sh.bcast[0];
         remain -= static_cast<int>(sh.bcast[1]);
-        prefix |= digit << shift;
-        mask |= dmask << shift;
-        __syncthreads();
+        prefix |= sh.bcast[0] << shift;
+        mask |= 0xFFu << shift;
     }
     const uint32_t thr = prefix;
     int eq = 0;
@@ -271,7 +270,7 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
 // (exponential race); with stochastic = 0 the key is the pooled score itself
 // (Sec. 4.1).  DKV: the K - B largest leverage products.  Writes the ascending
 // list of kept slots.
-__global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectParams p) {
+__global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectParams p) {
     extern __shared__ __align__(16) uint8_t smem_raw[];
     __shared__ SelShared sh;
     const int N = p.N, K = p.K;

@@ -219,6 +219,36 @@ int vase_profile_enable(vase_ctx* ctx, int enable);
  * (launches[VASE_KERNEL_COUNT]), then forgets the recorded events. */
 int vase_profile_collect(vase_ctx* ctx, double* total_ms, int64_t* launches);
 
+/* Eviction for callers that cannot allocate device memory.
+ *
+ * Some callers own no device allocator: a plugin inside an inference server whose host
+ * process owns all device memory and hands it only tensors, or a runtime that forbids
+ * device allocation after start-up to keep a fixed, unfragmented memory budget.  They can
+ * pass the caches but not the workspace that vase_create asks for.  This entry point runs
+ * one eviction step of one layer (the same kernels and results as vase_evict) with its
+ * scratch -- window scores, DKV leverage products, kept-slot lists and the device error
+ * word -- in a static device array of VASE_STATIC_SCRATCH_BYTES that every GPU loading the
+ * library holds until the process exits.  It calls no cudaMalloc, cudaFree or other
+ * allocating routine and needs no context.  The paper has no counterpart; it is a
+ * deployment convenience of this library.
+ *
+ *   cfg, bufs: as for vase_create; bufs->workspace is ignored and may be NULL.
+ *   state:     the layer's counters as the caller tracks them; state->fill must be K + B and
+ *              state->round keys the noise.  The call does not update them: afterwards the
+ *              caller sets fill = K and round + 1.
+ *   device_error: NULL, or a host word: then the call waits for the stream, stores the device
+ *              error word there and returns VASE_ERR_DEVICE if it is non-zero.
+ * Layers needing more scratch than the array holds ((b*Hkv) * (K+B) * 4 * (1 + parts) +
+ * (b*Hkv) * K * 4 bytes, parts = 2 when G*W > 256, else 1) are rejected with
+ * VASE_ERR_UNSUPPORTED.  The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call before any stream
+ * capture.  Every call shares the one array and leaves its contents behind: calls that can
+ * overlap on the GPU (different streams, or several host threads) race on it and must be
+ * serialised by the caller.  Errors are explained by vase_last_error(NULL). */
+#define VASE_STATIC_SCRATCH_BYTES (16u << 20)
+int vase_evict_static_scratch(const vase_config* cfg, const vase_buffers* bufs, int32_t layer,
+                              const vase_layer_state* state, uint32_t* device_error, void* stream);
+
 const char* vase_status_string(int status);
 /* Message of the last failed call on ctx; with ctx == NULL, the reason the last
  * configuration check on this thread (vase_get_buffer_sizes, vase_create) failed. */

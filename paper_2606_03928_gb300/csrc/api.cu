@@ -782,3 +782,225 @@ const char* vase_last_error(const vase_ctx* ctx) { return ctx ? ctx->last_error.
 int vase_abi_version(void) { return VASE_ABI_VERSION; }
 
 }  // extern "C"
+
+// ----------------------------------------------------------------------------------------------------------------
+// Eviction without a caller-provided workspace.
+//
+// Some callers of this library never hold an allocator: a plugin inside an inference server whose host process
+// owns all device memory and only hands it tensors, or a runtime that forbids device allocation after start-up
+// to keep a fixed, unfragmented memory budget.  They can provide the caches but not the eviction's scratch.  For
+// them vase_evict_static_scratch runs the same kernels with their scratch (window scores, DKV leverage products,
+// kept-slot lists, the device error word) in the file-scope array below, which every GPU that loads the library
+// holds until the process exits.  Nothing is allocated per call.
+namespace {
+
+constexpr size_t kStaticScratchBytes = static_cast<size_t>(VASE_STATIC_SCRATCH_BYTES);
+__device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 64;
+void* g_static_scratch_addr[kMaxDevices] = {};  // device address of g_static_scratch, per device
+
+}  // namespace
+
+extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buffers* bufs, int32_t layer,
+                                         const vase_layer_state* state, uint32_t* device_error, void* stream) {
+    if (!cfg || !bufs || !state) {
+        g_config_error = "null argument";
+        return VASE_ERR_INVALID;
+    }
+    int device = 0, num_sms = 0;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, device);
+    if (e != cudaSuccess || device < 0 || device >= kMaxDevices) {
+        g_config_error = "no usable CUDA device";
+        return VASE_ERR_CUDA;
+    }
+    Plan P;
+    const char* why = nullptr;
+    if (!make_plan(cfg, num_sms, &P, &why)) return cfg->head_dim != 128 ? VASE_ERR_UNSUPPORTED : VASE_ERR_INVALID;
+    const vase_config& c = *cfg;
+    if (layer < 0 || layer >= c.num_layers) {
+        g_config_error = "layer out of range";
+        return VASE_ERR_INVALID;
+    }
+    if (state->fill != P.N) {
+        g_config_error = "evict needs a full cache (fill == K + B)";
+        return VASE_ERR_NOT_FULL;
+    }
+    const void* ptrs[5] = {bufs->k_cache, bufs->v_cache, bufs->q_window, bufs->positions, bufs->value_scores};
+    for (const void* p : ptrs) {
+        if (!p || !aligned(p, kAlign)) {
+            g_config_error = "null or unaligned buffer (256-byte alignment required)";
+            return p ? VASE_ERR_ALIGN : VASE_ERR_INVALID;
+        }
+    }
+    // scratch of one layer: error word | window-score parts | DKV products | kept lists
+    const size_t un = static_cast<size_t>(P.units) * P.N;
+    const size_t off_attn = kAlign;
+    const size_t off_dkv = align_up(off_attn + un * 4 * P.n_rb, kAlign);
+    const size_t off_src = align_up(off_dkv + un * 4, kAlign);
+    const size_t need = align_up(off_src + static_cast<size_t>(P.units) * c.budget_k * 4, kAlign);
+    if (need > kStaticScratchBytes) {
+        g_config_error = "one layer needs more eviction scratch than the static array holds (VASE_STATIC_SCRATCH_BYTES)";
+        return VASE_ERR_UNSUPPORTED;
+    }
+    // set-up, once per device, with that device current: the device address of the static array
+    if (!g_static_scratch_addr[device]) {
+        void* addr = nullptr;
+        if ((e = cudaGetSymbolAddress(&addr, g_static_scratch)) != cudaSuccess || !addr) {
+            g_config_error = std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e);
+            return VASE_ERR_CUDA;
+        }
+        g_static_scratch_addr[device] = addr;
+    }
+    uint8_t* scratch = static_cast<uint8_t*>(g_static_scratch_addr[device]);
+    uint32_t* err = reinterpret_cast<uint32_t*>(scratch);
+    float* attn = reinterpret_cast<float*>(scratch + off_attn);
+    float* dkv = reinterpret_cast<float*>(scratch + off_dkv);
+    int32_t* src = reinterpret_cast<int32_t*>(scratch + off_src);
+
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || !fn || q != cudaDriverEntryPointSuccess) {
+        g_config_error = "cuTensorMapEncodeTiled unavailable";
+        return VASE_ERR_CUDA;
+    }
+    EncodeTiledFn enc = reinterpret_cast<EncodeTiledFn>(fn);
+    const uint64_t cache_rows = static_cast<uint64_t>(c.num_layers) * P.units * P.N;
+    const uint64_t q_rows = static_cast<uint64_t>(c.num_layers) * c.batch * c.num_q_heads * c.window;
+    CUtensorMap kmap, vmap, qmap;
+    if (cache_rows >= (1ull << 31) || q_rows >= (1ull << 31) ||
+        !encode_rows(enc, &kmap, bufs->k_cache, cache_rows, kTileTokens) ||
+        !encode_rows(enc, &vmap, bufs->v_cache, cache_rows, kTileTokens) ||
+        !encode_rows(enc, &qmap, bufs->q_window, q_rows, static_cast<uint32_t>(P.q_box))) {
+        g_config_error = "tensor map encoding failed";
+        return VASE_ERR_CUDA;
+    }
+    if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
+        (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess || (e = select_set_attributes(P.select_smem)) != cudaSuccess ||
+        (e = compact_set_attributes()) != cudaSuccess) {
+        g_config_error = std::string("kernel attributes: ") + cudaGetErrorString(e);
+        return VASE_ERR_CUDA;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    // the array keeps the previous call's contents: the error word must start at zero
+    if ((e = cudaMemsetAsync(err, 0, sizeof(uint32_t), s)) != cudaSuccess) {
+        g_config_error = std::string("error word reset: ") + cudaGetErrorString(e);
+        return VASE_ERR_CUDA;
+    }
+    LayerBatch batch;
+    batch.n = 1;
+    batch.layer[0] = layer;
+    batch.rnd[0] = state->round;
+    if (c.variant == VASE_VARIANT_ATTNV) {
+        ScoreAttnParams sp;
+        sp.batch = batch;
+        sp.N = P.N;
+        sp.GW = P.GW;
+        sp.GWp = P.GWp;
+        sp.NB = P.NB;
+        sp.n_rb = P.n_rb;
+        sp.n_rbA = P.n_rbA;
+        sp.rep = P.rep;
+        sp.q_rows = P.q_rows;
+        sp.q_box = P.q_box;
+        sp.n_tiles = P.n_tiles;
+        sp.cluster = P.cluster_for[1];
+        sp.tiles_per_cta = ceil_div(P.n_tiles, sp.cluster);
+        sp.stages = P.stages;
+        sp.buf_cols = P.buf_cols;
+        sp.nbuf = P.nbuf;
+        sp.units = P.units;
+        sp.tmem_cols = P.tmem_cols;
+        sp.Hq = c.num_q_heads;
+        sp.Hkv = c.num_kv_heads;
+        sp.W = c.window;
+        sp.G = P.G;
+        sp.layer_rows = static_cast<int64_t>(P.units) * P.N;
+        sp.q_layer_rows = static_cast<int64_t>(c.batch) * c.num_q_heads * c.window;
+        sp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
+        sp.inv_gw = 1.0f / static_cast<float>(P.GW);
+        sp.attn = attn;
+        sp.err = err;
+        if ((e = launch_score_attn(kmap, qmap, sp, P.units, P.score_smem, s)) != cudaSuccess) {
+            g_config_error = std::string("score launch: ") + cudaGetErrorString(e);
+            return VASE_ERR_CUDA;
+        }
+    } else {
+        DkvParams dp;
+        dp.batch = batch;
+        dp.N = P.N;
+        dp.K = c.budget_k;
+        dp.r = c.dkv_rank;
+        dp.Hkv = c.num_kv_heads;
+        dp.fixed_g = c.dkv_fixed_g;
+        dp.units = P.units;
+        dp.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
+        dp.seed_hi = static_cast<uint32_t>(c.seed >> 32);
+        dp.n_tiles_k = P.dkv_tiles_k;
+        dp.tiles_per_cta = P.dkv_tiles_per_cta;
+        dp.stages = P.dkv_stages;
+        dp.layer_rows = static_cast<int64_t>(P.units) * P.N;
+        dp.out = dkv;
+        dp.err = err;
+        if ((e = launch_dkv(kmap, vmap, dp, P.units, P.dkv_smem, s)) != cudaSuccess) {
+            g_config_error = std::string("dkv launch: ") + cudaGetErrorString(e);
+            return VASE_ERR_CUDA;
+        }
+    }
+    SelectParams sel;
+    sel.batch = batch;
+    sel.attn = attn;
+    sel.dkv = dkv;
+    sel.vmag = bufs->value_scores;
+    sel.vscore_dbg = nullptr;
+    sel.pos = bufs->positions;
+    sel.src = src;
+    sel.pooled_dbg = nullptr;
+    sel.key_dbg = nullptr;
+    sel.keep_dbg = nullptr;
+    sel.N = P.N;
+    sel.K = c.budget_k;
+    sel.B = c.buffer_b;
+    sel.n_v = P.n_v;
+    sel.m = P.m;
+    sel.pool = c.pool_kernel;
+    sel.variant = c.variant;
+    sel.stochastic = c.stochastic;
+    sel.Hkv = c.num_kv_heads;
+    sel.n_parts = c.variant == VASE_VARIANT_ATTNV ? P.n_rb : 1;
+    sel.units = P.units;
+    sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
+    sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
+    sel.err = err;
+    if ((e = launch_select(sel, P.units, P.select_smem, s)) != cudaSuccess) {
+        g_config_error = std::string("select launch: ") + cudaGetErrorString(e);
+        return VASE_ERR_CUDA;
+    }
+    CompactParams cp;
+    cp.batch = batch;
+    cp.kc = static_cast<uint4*>(bufs->k_cache);
+    cp.vc = static_cast<uint4*>(bufs->v_cache);
+    cp.src = src;
+    cp.N = P.N;
+    cp.K = c.budget_k;
+    cp.units = P.units;
+    cp.err = err;
+    if ((e = launch_compact(cp, P.units, s)) != cudaSuccess) {
+        g_config_error = std::string("compact launch: ") + cudaGetErrorString(e);
+        return VASE_ERR_CUDA;
+    }
+    if (device_error) {
+        if ((e = cudaMemcpyAsync(device_error, err, sizeof(uint32_t), cudaMemcpyDeviceToHost, s)) != cudaSuccess ||
+            (e = cudaStreamSynchronize(s)) != cudaSuccess) {
+            g_config_error = std::string("error word read: ") + cudaGetErrorString(e);
+            return VASE_ERR_CUDA;
+        }
+        if (*device_error) {
+            g_config_error = "device-side check or bounded wait failed";
+            return VASE_ERR_DEVICE;
+        }
+    }
+    return VASE_OK;
+}

@@ -36,7 +36,7 @@ EXPORTED = [
     "vase_append_host", "vase_evict", "vase_read_positions", "vase_get_layer_state", "vase_set_layer_state",
     "vase_kv_view_get", "vase_debug_view_get", "vase_check_device_error", "vase_launch_count",
     "vase_status_string", "vase_last_error", "vase_abi_version", "vase_profile_enable", "vase_profile_collect",
-    "vase_append_all", "vase_evict_all", "vase_refresh_value_scores",
+    "vase_append_all", "vase_evict_all", "vase_refresh_value_scores", "vase_evict_static_scratch",
 ]
 KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select", "compact"]
 
@@ -98,6 +98,8 @@ def load(path: str = LIB_PATH):
         "vase_evict": (ctypes.c_int, [P, I32, P]),
         "vase_evict_all": (ctypes.c_int, [P, P]),
         "vase_refresh_value_scores": (ctypes.c_int, [P, I32, P]),
+        "vase_evict_static_scratch": (ctypes.c_int, [ctypes.POINTER(vase_config), ctypes.POINTER(vase_buffers), I32,
+                                                     ctypes.POINTER(vase_layer_state), ctypes.POINTER(U32), P]),
         "vase_read_positions": (ctypes.c_int, [P, I32, P, P]),
         "vase_get_layer_state": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_layer_state)]),
         "vase_set_layer_state": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_layer_state)]),
@@ -192,6 +194,22 @@ def vase_evict_all(ctx, stream=None):
 
 def vase_refresh_value_scores(ctx, layer, stream=None):
     return _check(ctx, load().vase_refresh_value_scores(ctx, layer, _stream_ptr(stream)), "vase_refresh_value_scores")
+
+
+def vase_evict_static_scratch(cfg: vase_config, bufs: vase_buffers, layer, fill, round_, stream=None,
+                              check_error=True):
+    """One eviction of one layer with the library's static device scratch instead of a workspace.
+
+    For callers that cannot allocate device memory (they pass the caches only; bufs.workspace may be
+    None).  Returns the device error word when check_error is set (the call then waits for the stream).
+    The caller keeps the layer counters: afterwards fill is K and the round has advanced by one."""
+    st = vase_layer_state(fill, round_, 0, 0)
+    word = ctypes.c_uint32(0)
+    status = load().vase_evict_static_scratch(ctypes.byref(cfg), ctypes.byref(bufs), layer, ctypes.byref(st),
+                                              ctypes.byref(word) if check_error else None, _stream_ptr(stream))
+    if status < 0:
+        raise VaseError(status, "vase_evict_static_scratch: " + load().vase_last_error(None).decode())
+    return word.value
 
 
 def vase_read_positions(ctx, layer, host_ptr, stream=None):

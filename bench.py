@@ -48,6 +48,7 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="qwen3_1p7b_k2048")
     ap.add_argument("--variant", choices=["attnv", "dkv"], default="attnv")
+    ap.add_argument("--layers", type=int, default=None, help="run only this many layers of the workload")
     ap.add_argument("--e2e-steps", type=int, default=None, help="steps of the host-buffer end-to-end pass")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -279,6 +280,8 @@ def run_ours(args):
     # the oracle pool is started before the first CUDA work of this process
     from paper_2606_03928_gb300 import workloads as Wm
     wl = Wm.WORKLOADS[args.workload]
+    if args.layers:
+        wl = Wm.shrink(wl, num_layers=args.layers)
     pool = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         pool, cores, n_units = oracle_pool(wl, args.variant)
@@ -411,11 +414,11 @@ def run_ours(args):
     tpath = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tpath):
         try:
-            from paper_2606_03928_gb300.build import _digest
+            from paper_2606_03928_gb300.build import source_digest
             with open(tpath) as f:
                 tr = json.load(f)
-            ent = tr.get(f"{dom}:{wl.name}:{args.variant}")
-            if ent and ent.get("source_digest") == _digest():
+            ent = tr.get(f"{dom}:{wl.name}:{args.variant}:{L}")
+            if ent and ent.get("source_digest") == source_digest():
                 traffic = ent["bytes_per_launch"]
         except Exception:
             traffic = None

@@ -32,6 +32,18 @@ def _nvcc():
     return cand
 
 
+def source_digest():
+    """Digest of the CUDA sources and the public header only (the same on every machine)."""
+    h = hashlib.sha256()
+    for name in sorted(os.listdir(CSRC)) + ["vase.h"]:
+        path = os.path.join(CSRC, name) if name != "vase.h" else os.path.join(INCLUDE, name)
+        if os.path.isfile(path):
+            h.update(name.encode())
+            with open(path, "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()
+
+
 def _digest():
     h = hashlib.sha256()
     for name in sorted(os.listdir(CSRC)) + ["vase.h"]:

@@ -405,7 +405,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
 // only after its loads (and all earlier ones) have completed.  Several stages
 // keep loads in flight ahead of the stores.
 constexpr int kCompactRows = 128;                          // destination rows per chunk
-constexpr int kCompactStages = 6;
+constexpr int kCompactStages = 3;
 constexpr int kCompactChunkBytes = kCompactRows * kRowBytes;  // 32 KB
 
 __device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar) {

@@ -22,8 +22,9 @@ int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
 struct Plan {
     int N, units, G, GW, GWp, NB, n_rb, n_rbA, rep, q_rows, q_box, buf_cols, nbuf;
-    int n_tiles, cluster, stages, tmem_cols, n_v, m;
+    int n_tiles, cluster, stages, stages_p, tmem_cols, n_v, m, num_sms;
     int cluster_for[kMaxLayerBatch + 1];  // CTAs per unit of the score kernel, by layers per launch
+    bool persist_for[kMaxLayerBatch + 1]; // one CTA per SM taking several units (interleaved passes)
     size_t score_smem;
     int dkv_tiles_k, dkv_tiles_per_cta, dkv_stages;
     size_t dkv_smem;
@@ -33,6 +34,10 @@ struct Plan {
     size_t stride_attn, stride_un, stride_src;  // elements per workspace slot
     size_t off_err, off_attn, off_pooled, off_vscore, off_key, off_keep, off_src, off_staging, staging_bytes, ws_bytes;
 };
+
+// Launch parameters of the window-score kernel for `nz` layers of `batch`.
+ScoreAttnParams score_params(const Plan& P, const vase_config& c, const LayerBatch& batch, int nz, float* attn,
+                             uint32_t* err);
 
 // Reason of the last failed configuration check on this thread (vase_last_error(NULL)).
 thread_local std::string g_config_error;
@@ -66,6 +71,7 @@ bool make_plan(const vase_config* c, int num_sms, Plan* P, const char** why) {
 
 bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why) {
     Plan& p = *P;
+    p.num_sms = num_sms;
     p.N = c->budget_k + c->buffer_b;
     p.units = c->batch * c->num_kv_heads;
     p.G = c->num_q_heads / c->num_kv_heads;
@@ -106,7 +112,7 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
         for (int C = 1; C <= 16 && C <= p.n_tiles; ++C) {
             const int T = ceil_div(p.n_tiles, C);
             if (ceil_div(p.n_tiles, T) != C) continue;
-            if (score_attn_smem_bytes(p.q_rows, p.n_rbA, p.GWp, C, 2) > kMaxDynSmem) continue;
+            if (score_attn_smem_bytes(p.q_rows, 1, p.n_rbA, p.GWp, C, 2) > kMaxDynSmem) continue;
             const long ctas = static_cast<long>(p.units) * C * nz;
             const long waves = (ctas + num_sms - 1) / num_sms;
             const long cost = waves * (T + 1);
@@ -122,15 +128,37 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
         p.cluster_for[nz] = best_c;
         if (nz <= max_batch && best_c > c_max) c_max = best_c;
     }
-    p.cluster = c_max;  // shared memory is sized for the largest cluster used
+    // With at least two items per SM, one CTA per SM takes a strided list of units and overlaps the pass-B
+    // sweep of each with the pass-A sweep of the next; this needs two window-row buffers.
+    p.stages_p = 0;
+    for (int s = 4; s >= 2; --s) {
+        if (score_attn_smem_bytes(p.q_rows, 2, p.n_rbA, p.GWp, 1, s) <= kMaxDynSmem) {
+            p.stages_p = s;
+            break;
+        }
+    }
+    bool any_persist = false;
+    c_max = 0;
+    for (int nz = 1; nz <= kMaxLayerBatch; ++nz) {
+        p.persist_for[nz] = p.stages_p > 0 && static_cast<long>(p.units) * nz >= 2L * num_sms;
+        if (nz <= max_batch) {
+            if (p.persist_for[nz]) any_persist = true;
+            else if (p.cluster_for[nz] > c_max) c_max = p.cluster_for[nz];
+        }
+    }
+    p.cluster = c_max > 0 ? c_max : 1;  // shared memory is sized for the largest cluster used
     p.stages = 0;
     for (int s = 6; s >= 2; --s) {
-        if (score_attn_smem_bytes(p.q_rows, p.n_rbA, p.GWp, p.cluster, s) <= kMaxDynSmem) {
+        if (score_attn_smem_bytes(p.q_rows, 1, p.n_rbA, p.GWp, p.cluster, s) <= kMaxDynSmem) {
             p.stages = s;
             break;
         }
     }
-    p.score_smem = score_attn_smem_bytes(p.q_rows, p.n_rbA, p.GWp, p.cluster, p.stages);
+    p.score_smem = score_attn_smem_bytes(p.q_rows, 1, p.n_rbA, p.GWp, p.cluster, p.stages);
+    if (any_persist) {
+        const size_t sp = score_attn_smem_bytes(p.q_rows, 2, p.n_rbA, p.GWp, 1, p.stages_p);
+        if (sp > p.score_smem) p.score_smem = sp;
+    }
     if (p.tmem_cols > 256 && p.score_smem < 120 * 1024) p.score_smem = 120 * 1024;  // one CTA per SM owns TMEM
 
     p.dkv_tiles_k = ceil_div(c->budget_k, kTileTokens);
@@ -185,6 +213,51 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     o = align_up(o + p.staging_bytes, kAlign);
     p.ws_bytes = o;
     return true;
+}
+
+ScoreAttnParams score_params(const Plan& P, const vase_config& c, const LayerBatch& batch, int nz, float* attn,
+                             uint32_t* err) {
+    ScoreAttnParams sp;
+    sp.batch = batch;
+    sp.N = P.N;
+    sp.GW = P.GW;
+    sp.GWp = P.GWp;
+    sp.NB = P.NB;
+    sp.n_rb = P.n_rb;
+    sp.n_rbA = P.n_rbA;
+    sp.rep = P.rep;
+    sp.q_rows = P.q_rows;
+    sp.q_box = P.q_box;
+    sp.n_tiles = P.n_tiles;
+    sp.work = P.units * nz;
+    if (P.persist_for[nz]) {
+        sp.cluster = 1;
+        sp.groups = P.num_sms < sp.work ? P.num_sms : sp.work;
+        sp.q_bufs = 2;
+        sp.stages = P.stages_p;
+    } else {
+        sp.cluster = P.cluster_for[nz];
+        sp.groups = sp.work;
+        sp.q_bufs = 1;
+        sp.stages = P.stages;
+    }
+    sp.lead = sp.stages;
+    sp.tiles_per_cta = ceil_div(P.n_tiles, sp.cluster);
+    sp.buf_cols = P.buf_cols;
+    sp.nbuf = P.nbuf;
+    sp.units = P.units;
+    sp.tmem_cols = P.tmem_cols;
+    sp.Hq = c.num_q_heads;
+    sp.Hkv = c.num_kv_heads;
+    sp.W = c.window;
+    sp.G = P.G;
+    sp.layer_rows = static_cast<int64_t>(P.units) * P.N;
+    sp.q_layer_rows = static_cast<int64_t>(c.batch) * c.num_q_heads * c.window;
+    sp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
+    sp.inv_gw = 1.0f / static_cast<float>(P.GW);
+    sp.attn = attn;
+    sp.err = err;
+    return sp;
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -470,37 +543,9 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     int32_t* src = reinterpret_cast<int32_t*>(ctx->ws + P.off_src);
     cudaError_t e;
     if (c.variant == VASE_VARIANT_ATTNV) {
-        ScoreAttnParams sp;
-        sp.batch = batch;
-        sp.N = P.N;
-        sp.GW = P.GW;
-        sp.GWp = P.GWp;
-        sp.NB = P.NB;
-        sp.n_rb = P.n_rb;
-        sp.n_rbA = P.n_rbA;
-        sp.rep = P.rep;
-        sp.q_rows = P.q_rows;
-        sp.q_box = P.q_box;
-        sp.n_tiles = P.n_tiles;
-        sp.cluster = P.cluster_for[nz];
-        sp.tiles_per_cta = ceil_div(P.n_tiles, sp.cluster);
-        sp.stages = P.stages;
-        sp.buf_cols = P.buf_cols;
-        sp.nbuf = P.nbuf;
-        sp.units = P.units;
-        sp.tmem_cols = P.tmem_cols;
-        sp.Hq = c.num_q_heads;
-        sp.Hkv = c.num_kv_heads;
-        sp.W = c.window;
-        sp.G = P.G;
-        sp.layer_rows = static_cast<int64_t>(P.units) * P.N;
-        sp.q_layer_rows = static_cast<int64_t>(c.batch) * c.num_q_heads * c.window;
-        sp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
-        sp.inv_gw = 1.0f / static_cast<float>(P.GW);
-        sp.attn = attn;
-        sp.err = err;
+        const ScoreAttnParams sp = score_params(P, c, batch, nz, attn, err);
         if ((e = timed_launch(ctx, VASE_KERNEL_SCORE, s, [&] {
-                 return launch_score_attn(ctx->kmap, ctx->qmap, sp, P.units, P.score_smem, s);
+                 return launch_score_attn(ctx->kmap, ctx->qmap, sp, P.score_smem, s);
              })) != cudaSuccess)
             return cuda_fail(ctx, e, "score launch");
         ctx->launches += 1;
@@ -894,36 +939,8 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
     batch.layer[0] = layer;
     batch.rnd[0] = state->round;
     if (c.variant == VASE_VARIANT_ATTNV) {
-        ScoreAttnParams sp;
-        sp.batch = batch;
-        sp.N = P.N;
-        sp.GW = P.GW;
-        sp.GWp = P.GWp;
-        sp.NB = P.NB;
-        sp.n_rb = P.n_rb;
-        sp.n_rbA = P.n_rbA;
-        sp.rep = P.rep;
-        sp.q_rows = P.q_rows;
-        sp.q_box = P.q_box;
-        sp.n_tiles = P.n_tiles;
-        sp.cluster = P.cluster_for[1];
-        sp.tiles_per_cta = ceil_div(P.n_tiles, sp.cluster);
-        sp.stages = P.stages;
-        sp.buf_cols = P.buf_cols;
-        sp.nbuf = P.nbuf;
-        sp.units = P.units;
-        sp.tmem_cols = P.tmem_cols;
-        sp.Hq = c.num_q_heads;
-        sp.Hkv = c.num_kv_heads;
-        sp.W = c.window;
-        sp.G = P.G;
-        sp.layer_rows = static_cast<int64_t>(P.units) * P.N;
-        sp.q_layer_rows = static_cast<int64_t>(c.batch) * c.num_q_heads * c.window;
-        sp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
-        sp.inv_gw = 1.0f / static_cast<float>(P.GW);
-        sp.attn = attn;
-        sp.err = err;
-        if ((e = launch_score_attn(kmap, qmap, sp, P.units, P.score_smem, s)) != cudaSuccess) {
+        const ScoreAttnParams sp = score_params(P, c, batch, 1, attn, err);
+        if ((e = launch_score_attn(kmap, qmap, sp, P.score_smem, s)) != cudaSuccess) {
             g_config_error = std::string("score launch: ") + cudaGetErrorString(e);
             return VASE_ERR_CUDA;
         }

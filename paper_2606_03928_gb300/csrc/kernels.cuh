@@ -99,6 +99,10 @@ struct ScoreAttnParams {
     int32_t q_box;          // rows per TMA box of the window-query map
     int32_t n_tiles;        // ceil(N / 128)
     int32_t tiles_per_cta;  // T
+    int32_t work;           // work items: batch.n layer slots x units (item w = slot * units + unit)
+    int32_t groups;         // CTA groups (clusters) of the grid; group g takes items g, g + groups, ...
+    int32_t q_bufs;         // window-row buffers: 2 when a group takes several items, else 1
+    int32_t lead;           // pass-B tiles that open an interleaved phase before its first pass-A tile
     int32_t cluster;        // CTAs per unit
     int32_t stages;         // tile ring depth
     int32_t buf_cols;       // TMEM columns per accumulator buffer
@@ -161,14 +165,14 @@ struct CompactParams {
 
 cudaError_t launch_append(const AppendParams& p, int n_layers, cudaStream_t s);
 cudaError_t launch_value_score(const ValueParams& p, int num_sms, cudaStream_t s);
-cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreAttnParams& p, int units,
+cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreAttnParams& p,
                               size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
                        size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_compact(const CompactParams& p, int units, cudaStream_t s);
 
-size_t score_attn_smem_bytes(int q_rows, int n_rbA, int GWp, int cluster, int stages);
+size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages);
 size_t dkv_smem_bytes(int stages);
 size_t select_smem_bytes(int N, int K);
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster);

@@ -7,8 +7,9 @@
 // queries are cached and the scores non-causal, per the footnote of Eq. (2)).
 // Pooling is left to the selection kernel.
 //
-// Decomposition: a cluster of C CTAs per unit, each owning a contiguous range
-// of 128-token tiles that a producer warp streams in with TMA (128-byte
+// Decomposition: the work items (layer slot, unit) are dealt to CTA groups; a
+// group is one CTA, or a cluster of C CTAs sharing one unit, each CTA owning a
+// contiguous range of 128-token tiles that a TMA warp streams in (128-byte
 // swizzle).  Two passes over the tiles, each on the tensor cores:
 //   pass A  S^T = Q K_tile^T (M = 128 window rows, N = 128 tokens): TMEM lane =
 //           window row, so every consumer thread keeps an online (max, sum of
@@ -20,7 +21,10 @@
 //   pass B  S = K_tile Q^T (M = 128 tokens, N = window rows): TMEM lane =
 //           token, so each thread accumulates sum_r exp2(s_ri - m_r) / l_r of its
 //           token alone.
-// K tiles are re-read for pass B (from L2 for all but the largest units).
+// A single-CTA group that takes several items runs them as phases: phase k
+// interleaves pass B of item k-1 (K re-read from L2, kept there by an
+// evict-last hint on the pass-A read) with pass A of item k (K read from HBM),
+// so the HBM stream never waits for a pass-B sweep.
 #include <cfloat>
 
 #include "kernels.cuh"
@@ -32,8 +36,10 @@ namespace {
 
 constexpr int kGroups = 2;                      // consumer warpgroups; group g takes the items i with i % 2 == g
 constexpr int kConsumers = 128 * kGroups;
-constexpr int kThreads = kConsumers + 64;       // + a TMA warp and an MMA-issue warp
+constexpr int kThreads = kConsumers + 96;       // + a TMA warp and two MMA-issue warps (even / odd items)
 constexpr int kMaxBufs = 4;
+constexpr int kMaxStages = 8;
+constexpr int kPrefetchTiles = 4;               // pass-A tiles requested into L2 ahead of their TMA load
 constexpr uint32_t kTileBytes = kTileTokens * kRowBytes;  // 32 KB: two 64-column panels of 128 rows
 constexpr uint32_t kPanelBytes = kTileTokens * 128;       // 16 KB
 
@@ -41,16 +47,16 @@ struct ScoreSmem {
     uint32_t q_off, k_off, bar_off, slot_off, pm_off, pl_off, xm_off, xl_off, rowm_off, roww_off, total;
 };
 
-__host__ __device__ inline ScoreSmem score_layout(int q_rows, int n_rbA, int GWp, int cluster, int stages,
-                                                   int stage_bytes) {
+__host__ __device__ inline ScoreSmem score_layout(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster,
+                                                   int stages, int stage_bytes) {
     ScoreSmem L;
     uint32_t o = 0;
     L.q_off = o;
-    o += static_cast<uint32_t>(q_rows) * kRowBytes;
+    o += static_cast<uint32_t>(q_bufs) * q_rows * kRowBytes;
     L.k_off = o;
     o += static_cast<uint32_t>(stages) * stage_bytes;
     L.bar_off = o;
-    o += 8 * (1 + 2 * stages + 2 * kMaxBufs);
+    o += 8 * (6 + 3 * stages + 2 * kMaxBufs);
     o = (o + 15u) & ~15u;
     L.slot_off = o;
     o += 16;
@@ -85,21 +91,63 @@ __device__ __forceinline__ void merge_ml(float& m, float& l, float m2, float l2)
     m = mn;
 }
 
+// Work item w of the launch: layer slot w / units, unit w % units.
+struct ScoreItem {
+    int slot, unit;
+    int64_t k_row;  // first cache row of the unit
+    int64_t q_row;  // first window-query row of the unit's query heads
+};
+
+__device__ __forceinline__ ScoreItem score_item(const ScoreAttnParams& p, int w) {
+    ScoreItem it;
+    it.slot = w / p.units;
+    it.unit = w - it.slot * p.units;
+    const int layer = p.batch.layer[it.slot];
+    const int seq = it.unit / p.Hkv;
+    const int head = it.unit - seq * p.Hkv;
+    it.k_row = static_cast<int64_t>(layer) * p.layer_rows + static_cast<int64_t>(it.unit) * p.N;
+    it.q_row = static_cast<int64_t>(layer) * p.q_layer_rows +
+               (static_cast<int64_t>(seq) * p.Hq + static_cast<int64_t>(head) * p.G) * p.W;
+    return it;
+}
+
+// Tile t of a phase with nA pass-A tiles and nB pass-B tiles (each 0 or n): the first `lead` pass-B
+// tiles, then pass A and pass B alternately, then the last `lead` pass-A tiles.  Returns true for a
+// pass-A tile; j is the tile's index within its pass.
+__device__ __forceinline__ bool phase_tile(int t, int nA, int nB, int lead, int& j) {
+    if (nB == 0) {
+        j = t;
+        return true;
+    }
+    if (nA == 0 || t < lead) {
+        j = t;
+        return false;
+    }
+    const int u = t - lead;
+    if (u < 2 * (nB - lead)) {
+        j = (u & 1) ? lead + (u >> 1) : (u >> 1);
+        return !(u & 1);
+    }
+    j = t - nB;
+    return true;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     score_attn_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
                       const ScoreAttnParams p) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     constexpr int stage_bytes = kTileBytes;
-    const ScoreSmem Ly = score_layout(p.q_rows, p.n_rbA, p.GWp, p.cluster, p.stages, stage_bytes);
+    const ScoreSmem Ly = score_layout(p.q_rows, p.q_bufs, p.n_rbA, p.GWp, p.cluster, p.stages, stage_bytes);
 
     uint8_t* q_s = smem + Ly.q_off;
     uint8_t* st_s = smem + Ly.k_off;
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Ly.bar_off);
-    uint64_t* q_full = bars;
-    uint64_t* k_full = bars + 1;
-    uint64_t* k_empty = bars + 1 + p.stages;
-    uint64_t* t_full = bars + 1 + 2 * p.stages;  // [nbuf]
+    uint64_t* q_full = bars;                      // [2]
+    uint64_t* q_empty = bars + 2;                 // [2][group]
+    uint64_t* k_full = bars + 6;                  // [stages]
+    uint64_t* k_empty = k_full + p.stages;        // [stages][group]
+    uint64_t* t_full = k_empty + 2 * p.stages;    // [nbuf]
     uint64_t* t_empty = t_full + kMaxBufs;        // [nbuf]
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Ly.slot_off);
     float* pm = reinterpret_cast<float*>(smem + Ly.pm_off);      // [group][n_rbA][128] running max per lane
@@ -112,38 +160,48 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
     const int lane = tid & 31;
-    const int unit = blockIdx.y;
-    const int rank = blockIdx.x;
-    const int slot = blockIdx.z;  // layer slot of the batch
-    const int layer = p.batch.layer[slot];
-    float* const attn_out = p.attn + static_cast<int64_t>(slot) * p.n_rb * p.units * p.N;
     const int C = p.cluster;
+    const int rank = static_cast<int>(blockIdx.x) % C;
+    const int group = static_cast<int>(blockIdx.x) / C;
+    // items group, group + groups, ... (one item per group whenever C > 1)
+    const int n_w = group < p.work ? (p.work - group + p.groups - 1) / p.groups : 0;
     const int GWp = p.GWp;
     const int NB = p.NB;
     const int n_rb = p.n_rb;
     const int n_rbA = p.n_rbA;
-    const int R = p.rep;                 // copies of the window rows across the 128 lanes in pass A
+    const int R = p.rep;                 // copies of the window rows across the 128 pass-A lanes
     const int bufcols = p.buf_cols;      // TMEM columns per accumulator buffer
-    const int nbuf = p.nbuf;             // accumulator buffers (2 or 4)
+    const int nbuf = p.nbuf;             // accumulator buffers (2 or 4): item i uses buffer i & bmask, use i >> bshift
+    const int bmask = nbuf - 1;
+    const int bshift = nbuf == 4 ? 2 : 1;
     const int t_begin = rank * p.tiles_per_cta;
     const int t_end = min(p.n_tiles, t_begin + p.tiles_per_cta);
     const int n_my = max(0, t_end - t_begin);
-    const int64_t k_row = static_cast<int64_t>(layer) * p.layer_rows + static_cast<int64_t>(unit) * p.N;
-    const int seq = unit / p.Hkv;
-    const int head = unit - seq * p.Hkv;
-    const int64_t q_row = static_cast<int64_t>(layer) * p.q_layer_rows +
-                          (static_cast<int64_t>(seq) * p.Hq + static_cast<int64_t>(head) * p.G) * p.W;
-    const int itemsA = n_my * n_rbA;
-    const int itemsB = n_my * n_rb;
+    const int lead = min(p.lead, n_my);
+    const uint32_t q_bytes = static_cast<uint32_t>(p.q_rows) * kRowBytes;
+    // With one accumulator per tile and no more stages than accumulators, a stage is free as soon as the MMA
+    // of its tile has completed, which the TMA warp reads from the accumulator's full barrier (the buffer
+    // cannot be reused before the stage is reloaded, so the parity is unambiguous).  Otherwise the consumer
+    // groups release the stages.
+    const bool mma_release = n_rbA == 1 && n_rb == 1 && p.stages <= nbuf;
 
     if (tid == 0) {
-        mbar_init(q_full, 1);
+        // A consumer group waits for the accumulators of its own items, which come from one MMA warp whose
+        // commits complete in issue order.  Each group releases a K stage (or window-row buffer) on its own
+        // barrier once it has seen the last of its items that read it; the TMA warp waits for the groups that
+        // own items there, so a group that lags holds back only its own stages.
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&q_full[b], 1);
+            mbar_init(&q_empty[2 * b], 128);
+            mbar_init(&q_empty[2 * b + 1], 128);
+        }
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&k_full[s], 1);
-            mbar_init(&k_empty[s], 1 + kConsumers);  // the last MMA commit + every consumer thread
+            mbar_init(&k_empty[2 * s], 128);
+            mbar_init(&k_empty[2 * s + 1], 128);
         }
         for (int b = 0; b < nbuf; ++b) {
-            mbar_init(&t_full[b], 1);
+            mbar_init(&t_full[b], 1);     // the MMA warp's commit
             mbar_init(&t_empty[b], 128);  // the 128 threads of the group that owns the item
         }
         fence_mbar_init();
@@ -153,7 +211,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         pl[i] = 0.f;
     }
     const int tma_warp = kConsumers / 32;
-    const int mma_warp = tma_warp + 1;
+    const int mma_warp = tma_warp + 1;  // and mma_warp + 1
     if (warp == tma_warp) {
         tmem_alloc(tmem_slot, static_cast<uint32_t>(p.tmem_cols));
         tmem_relinquish();
@@ -165,58 +223,135 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (C > 1) cluster_sync();  // every peer is running before any DSMEM store
 
     bool ok = true;
-    const int total_loads = 2 * n_my;
 
     if (warp == tma_warp) {
-        // ---------------------------------------------------------------- TMA warp: window rows, then K tiles
+        // ---------------------------------------------------------------- TMA warp: window rows and K tiles
         if (C > 1) cluster_arrive();  // this warp takes no part in the statistics exchange
         if (lane == 0) {
             tma_prefetch_desc(&kmap);
             tma_prefetch_desc(&qmap);
-            // window rows: R copies of the GWp rows (pass A lanes), or q_rows rows when R == 1
-            const int q_panel = p.q_rows * 128;
-            mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(p.q_rows) * kRowBytes);
-            for (int panel = 0; panel < 2; ++panel) {
-                if (R > 1) {
-                    for (int c = 0; c < R; ++c)
-                        tma_load_2d(q_s + panel * q_panel + c * GWp * 128, &qmap, panel * 64,
-                                    static_cast<int32_t>(q_row), q_full);
-                } else {
-                    for (int r0 = 0; r0 < p.q_rows; r0 += p.q_box)
-                        tma_load_2d(q_s + panel * q_panel + r0 * 128, &qmap, panel * 64,
-                                    static_cast<int32_t>(q_row + r0), q_full);
+            const uint64_t keep = l2_policy_evict_last();   // pass-A reads: read again by pass B
+            const uint64_t drop = l2_policy_evict_first();  // pass-B reads: last use
+            // Owner groups (bit g = consumer group g) of the tile in each stage and of the pass-B items that read
+            // each window-row buffer, and the parity of the next phase of every per-group empty barrier.
+            uint32_t slot_owners = 0, kpar = 0, q_owners = 0, qpar = 0;
+            int slot_item[kMaxStages];  // item of the tile in each stage (stage release by MMA completion)
+            int ld = 0, g = 0, st_pos = 0;
+            for (int k = 0; k <= n_w; ++k) {
+                const int nA = k < n_w ? n_my : 0;
+                const int nB = k > 0 ? n_my : 0;
+                const ScoreItem itA = score_item(p, group + min(k, n_w - 1) * p.groups);
+                const ScoreItem itB = score_item(p, group + max(k - 1, 0) * p.groups);
+                uint32_t b_owners = 0;
+                if (nA > 0) {
+                    // item k's window rows and first pass-A tiles into L2 while the phase opens with pass B
+                    tma_prefetch_2d(&qmap, 0, static_cast<int32_t>(itA.q_row));
+                    tma_prefetch_2d(&qmap, 64, static_cast<int32_t>(itA.q_row));
+                    for (int jj = 0; jj < kPrefetchTiles && jj < nA; ++jj) {
+                        const int32_t row = static_cast<int32_t>(itA.k_row + static_cast<int64_t>(t_begin + jj) * kTileTokens);
+                        tma_prefetch_2d(&kmap, 0, row);
+                        tma_prefetch_2d(&kmap, 64, row);
+                    }
+                }
+                for (int t = 0; t < nA + nB; ++t) {
+                    int j;
+                    const bool isA = phase_tile(t, nA, nB, lead, j);
+                    const int n_sub = isA ? n_rbA : n_rb;
+                    const uint32_t owners = n_sub > 1 ? 3u : (1u << (g & 1));
+                    if (!isA) b_owners |= owners;
+                    const int ls = st_pos;
+                    if (ld >= p.stages && mma_release) {
+                        const int i = slot_item[ls];
+                        if (ok) ok = mbar_wait(&t_full[i & bmask], (i >> bshift) & 1, p.err, kErrScoreKEmpty);
+                    } else if (ld >= p.stages) {
+                        const uint32_t prev = (slot_owners >> (2 * ls)) & 3u;
+                        for (int grp = 0; grp < 2; ++grp) {
+                            if (!((prev >> grp) & 1u)) continue;
+                            const int bit = 2 * ls + grp;
+                            if (ok) ok = mbar_wait(&k_empty[bit], (kpar >> bit) & 1u, p.err, kErrScoreKEmpty);
+                            kpar ^= 1u << bit;
+                        }
+                    }
+                    slot_owners = (slot_owners & ~(3u << (2 * ls))) | (owners << (2 * ls));
+                    slot_item[ls] = g;
+                    if (isA && j + kPrefetchTiles < nA) {
+                        const int32_t row = static_cast<int32_t>(
+                            itA.k_row + static_cast<int64_t>(t_begin + j + kPrefetchTiles) * kTileTokens);
+                        tma_prefetch_2d(&kmap, 0, row);
+                        tma_prefetch_2d(&kmap, 64, row);
+                    }
+                    if (isA && j == 0) {
+                        // window rows of item k: R copies of the GWp rows (pass A lanes), or q_rows rows
+                        const int qb = k & (p.q_bufs - 1);
+                        if (k >= 2) {  // item k - 2 is done with the buffer
+                            const uint32_t prev = (q_owners >> (2 * qb)) & 3u;
+                            for (int grp = 0; grp < 2; ++grp) {
+                                if (!((prev >> grp) & 1u)) continue;
+                                const int bit = 2 * qb + grp;
+                                if (ok) ok = mbar_wait(&q_empty[bit], (qpar >> bit) & 1u, p.err, kErrScoreQ);
+                                qpar ^= 1u << bit;
+                            }
+                        }
+                        uint8_t* qd = q_s + qb * q_bytes;
+                        const int q_panel = p.q_rows * 128;
+                        mbar_arrive_expect_tx(&q_full[qb], q_bytes);
+                        for (int panel = 0; panel < 2; ++panel) {
+                            if (R > 1) {
+                                for (int c = 0; c < R; ++c)
+                                    tma_load_2d(qd + panel * q_panel + c * GWp * 128, &qmap, panel * 64,
+                                                static_cast<int32_t>(itA.q_row), &q_full[qb]);
+                            } else {
+                                for (int r0 = 0; r0 < p.q_rows; r0 += p.q_box)
+                                    tma_load_2d(qd + panel * q_panel + r0 * 128, &qmap, panel * 64,
+                                                static_cast<int32_t>(itA.q_row + r0), &q_full[qb]);
+                            }
+                        }
+                    }
+                    const int64_t base = isA ? itA.k_row : itB.k_row;
+                    const int32_t row = static_cast<int32_t>(base + static_cast<int64_t>(t_begin + j) * kTileTokens);
+                    uint8_t* st = st_s + ls * stage_bytes;
+                    mbar_arrive_expect_tx(&k_full[ls], kTileBytes);
+                    tma_load_2d_hint(st, &kmap, 0, row, &k_full[ls], isA ? keep : drop);
+                    tma_load_2d_hint(st + kPanelBytes, &kmap, 64, row, &k_full[ls], isA ? keep : drop);
+                    ++ld;
+                    g += n_sub;
+                    if (++st_pos == p.stages) st_pos = 0;
+                }
+                // the pass-B items of this phase read item k - 1's window rows; item k + 1 takes that buffer
+                if (k >= 1 && k + 1 < n_w) {
+                    const int qb = (k - 1) & (p.q_bufs - 1);
+                    q_owners = (q_owners & ~(3u << (2 * qb))) | (b_owners << (2 * qb));
                 }
             }
-            // K tiles of pass A, then again for pass B (second read served by L2)
-            for (int ld = 0; ld < total_loads; ++ld) {
-                const int ls = ld % p.stages;
-                const int ln = ld / p.stages;
-                if (ln > 0 && ok) ok = mbar_wait(&k_empty[ls], (ln - 1) & 1, p.err, kErrScoreKEmpty);
-                const int tile = t_begin + (ld % n_my);
-                const int32_t row = static_cast<int32_t>(k_row + static_cast<int64_t>(tile) * kTileTokens);
-                uint8_t* st = st_s + ls * stage_bytes;
-                mbar_arrive_expect_tx(&k_full[ls], kTileBytes);
-                tma_load_2d(st, &kmap, 0, row, &k_full[ls]);
-                tma_load_2d(st + kPanelBytes, &kmap, 64, row, &k_full[ls]);
-            }
             // drain: every load has been consumed (and so has landed) before the CTA leaves
-            for (int ls = 0; ls < p.stages && ls < total_loads; ++ls) {
-                const int last = ((total_loads - 1 - ls) / p.stages) * p.stages + ls;
-                mbar_wait(&k_empty[ls], (last / p.stages) & 1, p.err, kErrScoreDrain);
+            for (int ls = 0; ls < p.stages && ls < ld; ++ls) {
+                if (mma_release) {
+                    const int i = slot_item[ls];
+                    mbar_wait(&t_full[i & bmask], (i >> bshift) & 1, p.err, kErrScoreDrain);
+                    continue;
+                }
+                const uint32_t prev = (slot_owners >> (2 * ls)) & 3u;
+                for (int grp = 0; grp < 2; ++grp) {
+                    const int bit = 2 * ls + grp;
+                    if ((prev >> grp) & 1u) mbar_wait(&k_empty[bit], (kpar >> bit) & 1u, p.err, kErrScoreDrain);
+                }
             }
         }
         __syncwarp();
         if (C > 1) cluster_wait();
-    } else if (warp == mma_warp) {
-        // ---------------------------------------------------------------- MMA warp: one thread issues tcgen05.mma
-        // The issuing thread shares its SM sub-partition with consumer warps, so its instruction stream is kept
-        // short: descriptors are built once and advanced by adding to the 14-bit start-address field.
+    } else if (warp == mma_warp || warp == mma_warp + 1) {
+        // ---------------------------------------------------------------- MMA warps: one elected lane issues
+        // Warp mma_warp + x issues the items i with i % 2 == x (the items of consumer group x).  Each issuing
+        // thread runs a serial wait / issue / commit loop whose overhead exceeds the MMAs' own time on the tensor
+        // pipe; two such loops overlap that overhead.  The whole warp runs the loop, so descriptors and ring
+        // positions stay warp-uniform, and one lane chosen by elect.sync issues each tcgen05.mma / commit.
         if (C > 1) cluster_arrive();
-        if (lane == 0) {
+        {
+            const int mine = warp - mma_warp;
             const uint32_t idescA = idesc_bf16_f32(128, 128);
             const uint32_t idescB = idesc_bf16_f32(128, static_cast<uint32_t>(NB));
             const uint32_t q_panel = static_cast<uint32_t>(p.q_rows) * 128u;  // bytes per 64-column panel
-            const uint64_t qdesc = sw128_kmajor_desc(smem_u32(q_s));
+            const uint64_t qdesc0 = sw128_kmajor_desc(smem_u32(q_s));
             const uint64_t kdesc = sw128_kmajor_desc(smem_u32(st_s));
             // start-address steps (16-byte units) of the eight K = 16 slices of d = 128
             uint32_t koff[8], qoff[8];
@@ -225,53 +360,66 @@ __global__ void __launch_bounds__(kThreads, 1)
                 koff[kk] = ((kk >> 2) * kPanelBytes + (kk & 3) * 32) >> 4;
                 qoff[kk] = ((kk >> 2) * q_panel + (kk & 3) * 32) >> 4;
             }
-            if (ok) ok = mbar_wait(q_full, 0, p.err, kErrScoreQ);
             int s = 0, s_phase = 0;        // K stage ring position
-            int buf = 0, use = 0;          // accumulator ring position
-            for (int pass = 0; pass < 2; ++pass) {
-                const int n_sub = pass == 0 ? n_rbA : n_rb;
-                for (int j = 0; j < n_my; ++j) {
+            int g = 0;                     // item counter
+            const int n_items = n_w * n_my * (n_rbA + n_rb);
+            for (int k = 0; k <= n_w; ++k) {
+                const int nA = k < n_w ? n_my : 0;
+                const int nB = k > 0 ? n_my : 0;
+                for (int t = 0; t < nA + nB; ++t) {
+                    int j;
+                    const bool isA = phase_tile(t, nA, nB, lead, j);
+                    const int n_sub = isA ? n_rbA : n_rb;
+                    // Both warps wait for every phase of every full barrier, in order, owned tile or not: a parity
+                    // wait cannot tell phase P from phase P + 2, so no phase may be skipped.
+                    const int qb = (isA ? k : k - 1) & (p.q_bufs - 1);
+                    if (isA && j == 0 && ok) ok = mbar_wait(&q_full[qb], (k >> 1) & 1, p.err, kErrScoreQ);
                     if (ok) ok = mbar_wait(&k_full[s], s_phase, p.err, kErrScoreKFull);
-                    const uint64_t kt = kdesc + ((static_cast<uint32_t>(s) * stage_bytes) >> 4);
-                    for (int sub = 0; sub < n_sub; ++sub) {
-                        if (use > 0 && ok) ok = mbar_wait(&t_empty[buf], (use - 1) & 1, p.err, kErrScoreTEmpty);
-                        tc_fence_after();
-                        const uint32_t d = taddr + static_cast<uint32_t>(buf * bufcols);
-                        if (ok) {
-                            if (pass == 0) {
-                                // A = window rows of row block `sub` (128 lanes), B = the tile's tokens
-                                const uint64_t qa = qdesc + ((static_cast<uint32_t>(sub) * 128u * 128u) >> 4);
+                    if (n_sub > 1 || (g & 1) == mine) {  // this warp owns an item of the tile
+                        const uint64_t qdesc = qdesc0 + ((static_cast<uint32_t>(qb) * q_bytes) >> 4);
+                        const uint64_t kt = kdesc + ((static_cast<uint32_t>(s) * stage_bytes) >> 4);
+                        for (int sub = 0; sub < n_sub; ++sub) {
+                            const int gi = g + sub;
+                            if ((gi & 1) != mine) continue;
+                            const int buf = gi & bmask;
+                            const int use = gi >> bshift;
+                            if (use > 0 && ok) ok = mbar_wait(&t_empty[buf], (use - 1) & 1, p.err, kErrScoreTEmpty);
+                            ok = __all_sync(0xffffffffu, ok);
+                            tc_fence_after();
+                            const uint32_t d = taddr + static_cast<uint32_t>(buf * bufcols);
+                            if (elect_one()) {
+                                if (ok) {
+                                    if (isA) {
+                                        // A = window rows of row block `sub` (128 lanes), B = the tile's tokens
+                                        const uint64_t qa = qdesc + ((static_cast<uint32_t>(sub) * 128u * 128u) >> 4);
 #pragma unroll
-                                for (int kk = 0; kk < 8; ++kk)
-                                    tc_mma_bf16(d, qa + qoff[kk], kt + koff[kk], idescA, kk > 0 ? 1u : 0u);
-                            } else {
-                                // A = the tile's tokens (128 lanes), B = window rows of row block `sub`
-                                const uint64_t qb = qdesc + ((static_cast<uint32_t>(sub) * NB * 128u) >> 4);
+                                        for (int kk = 0; kk < 8; ++kk)
+                                            tc_mma_bf16(d, qa + qoff[kk], kt + koff[kk], idescA, kk > 0 ? 1u : 0u);
+                                    } else {
+                                        // A = the tile's tokens (128 lanes), B = window rows of row block `sub`
+                                        const uint64_t qb_ = qdesc + ((static_cast<uint32_t>(sub) * NB * 128u) >> 4);
 #pragma unroll
-                                for (int kk = 0; kk < 8; ++kk)
-                                    tc_mma_bf16(d, kt + koff[kk], qb + qoff[kk], idescB, kk > 0 ? 1u : 0u);
+                                        for (int kk = 0; kk < 8; ++kk)
+                                            tc_mma_bf16(d, kt + koff[kk], qb_ + qoff[kk], idescB, kk > 0 ? 1u : 0u);
+                                    }
+                                    tc_commit(&t_full[buf]);
+                                } else {
+                                    // keep every phase moving; the data is garbage and the error word is set
+                                    mbar_arrive(&t_full[buf]);
+                                }
                             }
-                            tc_commit(&t_full[buf]);
-                            if (sub == n_sub - 1) tc_commit(&k_empty[s]);
-                        } else {
-                            // keep every phase moving; the data is garbage and the error word is set
-                            mbar_arrive(&t_full[buf]);
-                            if (sub == n_sub - 1) mbar_arrive(&k_empty[s]);
-                        }
-                        if (++buf == nbuf) {
-                            buf = 0;
-                            ++use;
+                            __syncwarp();
                         }
                     }
+                    g += n_sub;
                     if (++s == p.stages) {
                         s = 0;
                         s_phase ^= 1;
                     }
                 }
             }
-            // drain: the consumers have read every accumulator, so every MMA has completed
-            const int n_items = itemsA + itemsB;
-            for (int b = 0; b < nbuf; ++b) {
+            // drain: the consumers have read every accumulator of this warp, so its MMAs have completed
+            for (int b = mine; b < nbuf; b += 2) {
                 const int uses = (n_items - b + nbuf - 1) / nbuf;
                 if (uses > 0) mbar_wait(&t_empty[b], (uses - 1) & 1, p.err, kErrScoreDrain);
             }
@@ -280,7 +428,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (C > 1) cluster_wait();
     } else {
         // ---------------------------------------------------------------- consumer warpgroups
-        const int grp = tid >> 7;   // 0 or 1
+        const int grp = tid >> 7;   // 0 or 1: group g takes the items i with i % 2 == g
         const int L = tid & 127;    // TMEM lane
         const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
         const float cs = p.scale_log2;
@@ -291,158 +439,182 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int c0 = copy * cw;
         float* pmg = pm + grp * n_rbA * 128;
         float* plg = pl + grp * n_rbA * 128;
-        // ------------------------------------ pass A: row statistics
-        for (int j = 0; j < n_my; ++j) {
-            const int tile = t_begin + j;
-            const int s = j % p.stages;
-            const int tok0 = tile * kTileTokens;
-            for (int sub = 0; sub < n_rbA; ++sub) {
-                const int item = j * n_rbA + sub;
-                if ((item & 1) != grp) continue;
-                const int buf = item % nbuf;
-                const int use = item / nbuf;
-                if (ok) ok = mbar_wait(&t_full[buf], use & 1, p.err, kErrScoreTFull);
-                tc_fence_after();
-                float m = pmg[sub * 128 + L];
-                float l = plg[sub * 128 + L];
-                // online (max, sum of exp2) over this lane's token columns, 64 (or 32) at a time
-                for (int c = 0; c < cw; c += 64) {
-                    float v[64];
-                    const int width = cw - c >= 64 ? 64 : 32;
-                    if (width == 64) {
-                        tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), v);
-                    } else {
-                        float h[32];
-                        tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), h);
+        int st_pos = 0;  // K stage ring position
+        int item = 0;    // accumulator counter
+        for (int k = 0; k <= n_w; ++k) {
+            const int nA = k < n_w ? n_my : 0;
+            const int nB = k > 0 ? n_my : 0;
+            const ScoreItem itB = score_item(p, group + max(k - 1, 0) * p.groups);
+            bool owned_b = false;  // this group owns a pass-B item of the phase
+            float* const attn_out = p.attn + static_cast<int64_t>(itB.slot) * n_rb * p.units * p.N;
+            for (int t = 0; t < nA + nB; ++t) {
+                int j;
+                const bool isA = phase_tile(t, nA, nB, lead, j);
+                const int s = st_pos;
+                const int tile = t_begin + j;
+                if (isA) {
+                    // ------------------------------------ pass A: row statistics
+                    const int tok0 = tile * kTileTokens;
+                    for (int sub = 0; sub < n_rbA; ++sub, ++item) {
+                        if ((item & 1) != grp) continue;
+                        const int buf = item & bmask;
+                        if (ok) ok = mbar_wait(&t_full[buf], (item >> bshift) & 1, p.err, kErrScoreTFull);
+                        // this group's last item of the tile: its MMAs (and the earlier ones of the same MMA
+                        // warp) are complete, so this group is done with the K stage
+                        if (!mma_release && sub >= n_rbA - 2) mbar_arrive(&k_empty[2 * s + grp]);
+                        tc_fence_after();
+                        float m = pmg[sub * 128 + L];
+                        float l = plg[sub * 128 + L];
+                        // online (max, sum of exp2) over this lane's token columns, 64 (or 32) at a time
+                        for (int c = 0; c < cw; c += 64) {
+                            float v[64];
+                            const int width = cw - c >= 64 ? 64 : 32;
+                            if (width == 64) {
+                                tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), v);
+                            } else {
+                                float h[32];
+                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), h);
 #pragma unroll
-                        for (int k = 0; k < 32; ++k) {
-                            v[k] = h[k];
-                            v[k + 32] = -INFINITY;
+                                for (int q = 0; q < 32; ++q) {
+                                    v[q] = h[q];
+                                    v[q + 32] = -INFINITY;
+                                }
+                            }
+                            const int nvalid = min(width, p.N - (tok0 + c0 + c));
+                            if (nvalid < 64) {
+#pragma unroll
+                                for (int q = 0; q < 64; ++q)
+                                    if (q >= nvalid) v[q] = -INFINITY;
+                            }
+                            float cm0 = v[0], cm1 = v[1], cm2 = v[2], cm3 = v[3];
+#pragma unroll
+                            for (int q = 4; q < 64; q += 4) {
+                                cm0 = fmaxf(cm0, v[q]);
+                                cm1 = fmaxf(cm1, v[q + 1]);
+                                cm2 = fmaxf(cm2, v[q + 2]);
+                                cm3 = fmaxf(cm3, v[q + 3]);
+                            }
+                            const float mn = fmaxf(m, fmaxf(fmaxf(cm0, cm1), fmaxf(cm2, cm3)) * cs);
+                            if (mn != -INFINITY) {
+                                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+                                for (int q = 0; q < 64; q += 4) {
+                                    s0 += ex2(fmaf(v[q], cs, -mn));
+                                    s1 += ex2(fmaf(v[q + 1], cs, -mn));
+                                    s2 += ex2(fmaf(v[q + 2], cs, -mn));
+                                    s3 += ex2(fmaf(v[q + 3], cs, -mn));
+                                }
+                                l = l * ex2(m - mn) + ((s0 + s1) + (s2 + s3));
+                                m = mn;
+                            }
                         }
+                        pmg[sub * 128 + L] = m;
+                        plg[sub * 128 + L] = l;
+                        tc_fence_before();
+                        mbar_arrive(&t_empty[buf]);
                     }
-                    const int nvalid = min(width, p.N - (tok0 + c0 + c));
-                    if (nvalid < 64) {
-#pragma unroll
-                        for (int k = 0; k < 64; ++k)
-                            if (k >= nvalid) v[k] = -INFINITY;
-                    }
-                    float cm0 = v[0], cm1 = v[1], cm2 = v[2], cm3 = v[3];
-#pragma unroll
-                    for (int k = 4; k < 64; k += 4) {
-                        cm0 = fmaxf(cm0, v[k]);
-                        cm1 = fmaxf(cm1, v[k + 1]);
-                        cm2 = fmaxf(cm2, v[k + 2]);
-                        cm3 = fmaxf(cm3, v[k + 3]);
-                    }
-                    const float mn = fmaxf(m, fmaxf(fmaxf(cm0, cm1), fmaxf(cm2, cm3)) * cs);
-                    if (mn != -INFINITY) {
-                        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-                        for (int k = 0; k < 64; k += 4) {
-                            s0 += ex2(fmaf(v[k], cs, -mn));
-                            s1 += ex2(fmaf(v[k + 1], cs, -mn));
-                            s2 += ex2(fmaf(v[k + 2], cs, -mn));
-                            s3 += ex2(fmaf(v[k + 3], cs, -mn));
+                } else {
+                    // ------------------------------------ pass B: per-token accumulation
+                    // With two row blocks (G*W > 256) the two consecutive items of a tile belong to different
+                    // groups; each group writes its own partial sum (attn part `grp`) and the selection kernel
+                    // adds the parts.
+                    const int token = tile * kTileTokens + L;
+                    float acc = 0.f;
+                    bool mine = false;
+                    for (int sub = 0; sub < n_rb; ++sub, ++item) {
+                        if ((item & 1) != grp) continue;
+                        mine = true;
+                        const int buf = item & bmask;
+                        if (ok) ok = mbar_wait(&t_full[buf], (item >> bshift) & 1, p.err, kErrScoreTFull);
+                        owned_b = true;
+                        if (sub >= n_rb - 2) {
+                            if (!mma_release) mbar_arrive(&k_empty[2 * s + grp]);
+                            // item k - 1's last pass-B tile: this group is done with its window rows
+                            if (j == nB - 1 && k + 1 < n_w) mbar_arrive(&q_empty[2 * ((k - 1) & (p.q_bufs - 1)) + grp]);
                         }
-                        l = l * ex2(m - mn) + ((s0 + s1) + (s2 + s3));
-                        m = mn;
+                        tc_fence_after();
+                        for (int c = 0; c < NB; c += 64) {
+                            float v[64];
+                            const int width = NB - c >= 64 ? 64 : 32;
+                            if (width == 64) {
+                                tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), v);
+                            } else {
+                                float h[32];
+                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), h);
+#pragma unroll
+                                for (int q = 0; q < 32; ++q) v[q] = h[q];
+                            }
+                            const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
+                            const float4* w4 = reinterpret_cast<const float4*>(roww + sub * NB + c);
+                            float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+                            for (int q = 0; q < 16; ++q) {
+                                if (q < width / 4) {
+                                    const float4 mm = m4[q];
+                                    const float4 ww = w4[q];
+                                    a0 = fmaf(ex2(fmaf(v[4 * q], cs, -mm.x)), ww.x, a0);
+                                    a1 = fmaf(ex2(fmaf(v[4 * q + 1], cs, -mm.y)), ww.y, a1);
+                                    a2 = fmaf(ex2(fmaf(v[4 * q + 2], cs, -mm.z)), ww.z, a2);
+                                    a3 = fmaf(ex2(fmaf(v[4 * q + 3], cs, -mm.w)), ww.w, a3);
+                                }
+                            }
+                            acc += (a0 + a1) + (a2 + a3);
+                        }
+                        tc_fence_before();
+                        mbar_arrive(&t_empty[buf]);
+                    }
+                    // no item in the last pass-B tile: the group's last one (if any) was waited for earlier
+                    if (!mine && owned_b && j == nB - 1 && k + 1 < n_w)
+                        mbar_arrive(&q_empty[2 * ((k - 1) & (p.q_bufs - 1)) + grp]);
+                    if (mine && token < p.N) {
+                        const int part = n_rb > 1 ? grp : 0;
+                        attn_out[(static_cast<int64_t>(part) * p.units + itB.unit) * p.N + token] = acc;
                     }
                 }
-                pmg[sub * 128 + L] = m;
-                plg[sub * 128 + L] = l;
-                tc_fence_before();
-                mbar_arrive(&t_empty[buf]);
+                if (++st_pos == p.stages) st_pos = 0;
             }
-            mbar_arrive(&k_empty[s]);
-        }
-        // ------------------------------------ merge the row statistics: groups, copies, then the cluster
-        named_bar(1, kConsumers);
-        for (int r = tid; r < GWp; r += kConsumers) {
-            float m = -INFINITY, l = 0.f;
-            for (int g = 0; g < kGroups; ++g) {
-                const float* gm = pm + g * n_rbA * 128;
-                const float* gl = pl + g * n_rbA * 128;
-                if (R > 1) {
-                    for (int c = 0; c < R; ++c) merge_ml(m, l, gm[c * GWp + r], gl[c * GWp + r]);
+            if (k == n_w) break;
+            // ------------------------------------ item k's row statistics: groups, copies, then the cluster
+            // (every pass-B tile of item k - 1 is done, so rowm / roww are free)
+            named_bar(1, kConsumers);
+            for (int r = tid; r < GWp; r += kConsumers) {
+                float m = -INFINITY, l = 0.f;
+                for (int g = 0; g < kGroups; ++g) {
+                    const float* gm = pm + g * n_rbA * 128;
+                    const float* gl = pl + g * n_rbA * 128;
+                    if (R > 1) {
+                        for (int c = 0; c < R; ++c) merge_ml(m, l, gm[c * GWp + r], gl[c * GWp + r]);
+                    } else {
+                        merge_ml(m, l, gm[(r >> 7) * 128 + (r & 127)], gl[(r >> 7) * 128 + (r & 127)]);
+                    }
+                }
+                if (C > 1) {
+                    for (int peer = 0; peer < C; ++peer) {
+                        st_cluster_f32(map_to_rank(&xm[rank * GWp + r], static_cast<uint32_t>(peer)), m);
+                        st_cluster_f32(map_to_rank(&xl[rank * GWp + r], static_cast<uint32_t>(peer)), l);
+                    }
                 } else {
-                    merge_ml(m, l, gm[(r >> 7) * 128 + (r & 127)], gl[(r >> 7) * 128 + (r & 127)]);
+                    const bool real = r < p.GW;
+                    rowm[r] = real ? m : INFINITY;
+                    roww[r] = real ? p.inv_gw / l : 0.f;
                 }
             }
             if (C > 1) {
-                for (int peer = 0; peer < C; ++peer) {
-                    st_cluster_f32(map_to_rank(&xm[rank * GWp + r], static_cast<uint32_t>(peer)), m);
-                    st_cluster_f32(map_to_rank(&xl[rank * GWp + r], static_cast<uint32_t>(peer)), l);
+                cluster_arrive();
+                cluster_wait();
+                for (int r = tid; r < GWp; r += kConsumers) {
+                    float m = -INFINITY, l = 0.f;
+                    for (int c = 0; c < C; ++c) merge_ml(m, l, xm[c * GWp + r], xl[c * GWp + r]);
+                    const bool real = r < p.GW;
+                    rowm[r] = real ? m : INFINITY;
+                    roww[r] = real ? p.inv_gw / l : 0.f;
                 }
-            } else {
-                xm[r] = m;
-                xl[r] = l;
             }
-        }
-        if (C > 1) {
-            cluster_arrive();
-            cluster_wait();
-        } else {
             named_bar(1, kConsumers);
-        }
-        for (int r = tid; r < GWp; r += kConsumers) {
-            float m = -INFINITY, l = 0.f;
-            for (int c = 0; c < C; ++c) merge_ml(m, l, xm[c * GWp + r], xl[c * GWp + r]);
-            const bool real = r < p.GW;
-            rowm[r] = real ? m : INFINITY;
-            roww[r] = real ? p.inv_gw / l : 0.f;
-        }
-        named_bar(1, kConsumers);
-        // ------------------------------------ pass B: per-token accumulation
-        // With two row blocks (G*W > 256) each group owns one of them for every tile and writes its own
-        // partial sum (attn part `grp`); the selection kernel adds the parts.
-        for (int j = 0; j < n_my; ++j) {
-            const int tile = t_begin + j;
-            const int s = (n_my + j) % p.stages;
-            const int token = tile * kTileTokens + L;
-            float acc = 0.f;
-            bool mine = false;
-            for (int sub = 0; sub < n_rb; ++sub) {
-                const int item = itemsA + j * n_rb + sub;
-                if ((item & 1) != grp) continue;
-                mine = true;
-                const int buf = item % nbuf;
-                const int use = item / nbuf;
-                if (ok) ok = mbar_wait(&t_full[buf], use & 1, p.err, kErrScoreTFull);
-                tc_fence_after();
-                for (int c = 0; c < NB; c += 64) {
-                    float v[64];
-                    const int width = NB - c >= 64 ? 64 : 32;
-                    if (width == 64) {
-                        tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), v);
-                    } else {
-                        float h[32];
-                        tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), h);
-#pragma unroll
-                        for (int k = 0; k < 32; ++k) v[k] = h[k];
-                    }
-                    const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
-                    const float4* w4 = reinterpret_cast<const float4*>(roww + sub * NB + c);
-                    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-#pragma unroll
-                    for (int k = 0; k < 16; ++k) {
-                        if (k < width / 4) {
-                            const float4 mm = m4[k];
-                            const float4 ww = w4[k];
-                            a0 = fmaf(ex2(fmaf(v[4 * k], cs, -mm.x)), ww.x, a0);
-                            a1 = fmaf(ex2(fmaf(v[4 * k + 1], cs, -mm.y)), ww.y, a1);
-                            a2 = fmaf(ex2(fmaf(v[4 * k + 2], cs, -mm.z)), ww.z, a2);
-                            a3 = fmaf(ex2(fmaf(v[4 * k + 3], cs, -mm.w)), ww.w, a3);
-                        }
-                    }
-                    acc += (a0 + a1) + (a2 + a3);
-                }
-                tc_fence_before();
-                mbar_arrive(&t_empty[buf]);
-            }
-            mbar_arrive(&k_empty[s]);
-            if (mine && token < p.N) {
-                const int part = n_rb > 1 ? grp : 0;
-                attn_out[(static_cast<int64_t>(part) * p.units + unit) * p.N + token] = acc;
+            // every read of the partial statistics is done: restart this thread's own entries for item k + 1
+            for (int sub = 0; sub < n_rbA; ++sub) {
+                pmg[sub * 128 + L] = -INFINITY;
+                plg[sub * 128 + L] = 0.f;
             }
         }
     }
@@ -455,8 +627,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-size_t score_attn_smem_bytes(int q_rows, int n_rbA, int GWp, int cluster, int stages) {
-    return score_layout(q_rows, n_rbA, GWp, cluster, stages, kTileBytes).total + 1024;
+size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages) {
+    return score_layout(q_rows, q_bufs, n_rbA, GWp, cluster, stages, kTileBytes).total + 1024;
 }
 
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster) {
@@ -467,10 +639,10 @@ cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster) {
     return e;
 }
 
-cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreAttnParams& p, int units,
+cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreAttnParams& p,
                               size_t smem_bytes, cudaStream_t s) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(p.cluster), static_cast<unsigned>(units), static_cast<unsigned>(p.batch.n));
+    cfg.gridDim = dim3(static_cast<unsigned>(p.cluster) * static_cast<unsigned>(p.groups), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem_bytes;
     cfg.stream = s;

@@ -396,3 +396,70 @@ def test_append_all_equals_per_layer_appends():
     assert torch.equal(a.q_window, b.q_window) and torch.equal(a.positions, b.positions)
     for layer in range(3):
         assert a.layer_state(layer) == b.layer_state(layer)
+
+
+# ----------------------------------------------------------------------------- interleaved (persistent) schedule
+
+@pytest.mark.parametrize("K,B,Wn,Hq,Hkv", [(192, 64, 16, 16, 8), (200, 40, 16, 16, 8), (256, 64, 32, 32, 8),
+                                          (160, 96, 32, 64, 8)])
+def test_evict_all_with_several_units_per_cta_matches_oracle(K, B, Wn, Hq, Hkv):
+    """Eight layers of 64 units: more than two items per SM, so one CTA per SM takes a strided list of units and
+    interleaves the pass-B sweep of each with the pass-A sweep of the next.  Every unit of every layer is checked."""
+    wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=Wn, num_q_heads=Hq, num_kv_heads=Hkv, batch=64 // Hkv,
+                  num_layers=8)
+    cache = _cache(wl, 8)
+    states = [W.layer_state(wl, 11, layer, 3 + layer, "gapped") for layer in range(8)]
+    for layer, st in enumerate(states):
+        PU.upload_layer(cache, layer, st, 3 + layer)
+    assert cache.evict_all() == 8
+    status, code = cache.check_device_error()
+    assert status == 0, f"device error word {code:#x}"
+    for z in range(8):
+        dv = {k: (v.cpu().numpy() if k != "layer" else v) for k, v in cache.debug_view(z).items()}
+        layer = dv["layer"]
+        st = states[layer]
+        got = PU.download(cache, layer)
+        got.update({k: v for k, v in dv.items() if k != "layer"})
+        for s in range(wl.batch):
+            for h in range(wl.num_kv_heads):
+                ref = PU.oracle_unit(wl, st, s, h, variant="attnv", round_index=3 + layer, seed=0, layer=layer)
+                PU.check_unit(wl, ref, PU.unit_slice(got, s, h, wl.num_kv_heads), st["k_bits"][s, h],
+                              st["v_bits"][s, h], st["positions"][s, h], variant="attnv", n_v=wl.budget_k // 4)
+
+
+def test_qwen3_1p7b_k2048_all_layers_in_one_launch():
+    """The bench's launch: all 28 layers of the 1.7B geometry in one launch per kernel, no debug outputs.
+    Three layers are checked unit by unit against the oracle; every unit of every layer keeps K distinct slots
+    including the buffer."""
+    wl = W.WORKLOADS["qwen3_1p7b_k2048"]
+    L = wl.num_layers
+    cache = _cache(wl, L, debug=False)
+    base = [W.layer_state(wl, 21, i, 40 + i, "gapped") for i in range(3)]
+    for layer in range(L):
+        PU.upload_layer(cache, layer, base[layer % 3], 40 + layer)
+    assert cache.evict_all() == L
+    status, code = cache.check_device_error()
+    assert status == 0, f"device error word {code:#x}"
+    K, B = wl.budget_k, wl.buffer_b
+    for layer in range(L):
+        pos = cache.positions[layer].cpu().numpy()
+        st = base[layer % 3]
+        for s in range(wl.batch):
+            for h in range(wl.num_kv_heads):
+                kept = pos[s, h, :K]
+                assert len(set(kept.tolist())) == K
+                assert set(st["positions"][s, h, K:K + B].tolist()) <= set(kept.tolist())
+    for layer in (0, 13, L - 1):
+        st = base[layer % 3]
+        got = PU.download(cache, layer)
+        for s in range(wl.batch):
+            for h in range(wl.num_kv_heads):
+                ref = PU.oracle_unit(wl, st, s, h, variant="attnv", round_index=40 + layer, seed=0, layer=layer)
+                gu = {"k_bits": got["k_bits"][s, h], "v_bits": got["v_bits"][s, h],
+                      "positions": got["positions"][s, h], "vmag": got["vmag"][s, h]}
+                # the kept list is the compacted positions mapped back to slots of the uploaded state
+                slot_of = {int(p_): i for i, p_ in enumerate(st["positions"][s, h])}
+                gu["src"] = np.array([slot_of[int(p_)] for p_ in gu["positions"][:K]], dtype=np.int64)
+                gu["attn"] = gu["pooled"] = gu["key"] = gu["value_score"] = None
+                PU.check_unit(wl, ref, gu, st["k_bits"][s, h], st["v_bits"][s, h], st["positions"][s, h],
+                              variant="attnv", n_v=wl.budget_k // 4, check_scores=False)

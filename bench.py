@@ -132,10 +132,9 @@ def kernel_bytes(kind, wl, variant, moved_rows_per_unit):
         return U * (K * row + K * 4)
     if kind == "dkv_score":
         return U * (2 * K * row + K * 4)
-    if kind == "select":
-        return U * (N * 4 + K * 4 + K * 4 + K * 4)
-    if kind == "compact":
-        return U * moved_rows_per_unit * (2 * 2 * row + 8)
+    if kind == "select_compact":
+        # scores, magnitudes and positions in; kept list, positions, magnitudes and the moved K/V rows out
+        return U * (N * 4 + K * 4 + K * 4 + K * 4) + U * moved_rows_per_unit * (2 * 2 * row + 8)
     if kind == "append":
         return 2 * B * wl.batch * (wl.num_q_heads + 2 * wl.num_kv_heads) * row + 2 * B * U * 4
     return 0

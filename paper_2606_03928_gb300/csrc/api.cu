@@ -29,6 +29,7 @@ struct Plan {
     int dkv_tiles_k, dkv_tiles_per_cta, dkv_stages;
     size_t dkv_smem;
     size_t select_smem;
+    bool select_staged;
     // workspace
     int slots;  // layers one launch can batch
     size_t stride_attn, stride_un, stride_src;  // elements per workspace slot
@@ -180,7 +181,11 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     }
     p.dkv_stages = 3;
     p.dkv_smem = dkv_smem_bytes(p.dkv_stages);
-    p.select_smem = select_smem_bytes(p.N, c->budget_k);
+    {
+        const int n_parts = c->variant == VASE_VARIANT_ATTNV ? p.n_rb : 1;
+        p.select_staged = select_smem_bytes(p.N, c->budget_k, n_parts, true) <= kMaxDynSmem - 9216;
+        p.select_smem = select_smem_bytes(p.N, c->budget_k, n_parts, p.select_staged);
+    }
     if (p.select_smem > kMaxDynSmem - 9216) {
         *why = "K + B too large for the single-CTA selection (about 25k slots at most)";
         return false;
@@ -450,7 +455,7 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
     }
     if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
         (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess ||
-        (e = select_set_attributes(P.select_smem)) != cudaSuccess || (e = compact_set_attributes()) != cudaSuccess) {
+        (e = select_set_attributes(P.select_smem)) != cudaSuccess) {
         fprintf(stderr, "vase_create: kernel attributes: %s\n", cudaGetErrorString(e));
         delete ctx;
         return VASE_ERR_CUDA;
@@ -579,6 +584,8 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     sel.vmag = ctx->bufs.value_scores;
     sel.vscore_dbg = (c.debug_outputs && c.variant == VASE_VARIANT_ATTNV) ? vscore : nullptr;
     sel.pos = ctx->bufs.positions;
+    sel.kc = static_cast<uint4*>(ctx->bufs.k_cache);
+    sel.vc = static_cast<uint4*>(ctx->bufs.v_cache);
     sel.src = src;
     sel.pooled_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_pooled) : nullptr;
     sel.key_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_key) : nullptr;
@@ -593,6 +600,7 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     sel.stochastic = c.stochastic;
     sel.Hkv = c.num_kv_heads;
     sel.n_parts = c.variant == VASE_VARIANT_ATTNV ? P.n_rb : 1;
+    sel.staged = P.select_staged ? 1 : 0;
     sel.units = P.units;
     sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
     sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
@@ -600,18 +608,7 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     if ((e = timed_launch(ctx, VASE_KERNEL_SELECT, s, [&] { return launch_select(sel, P.units, P.select_smem, s); })) !=
         cudaSuccess)
         return cuda_fail(ctx, e, "select launch");
-    CompactParams cp;
-    cp.batch = batch;
-    cp.kc = static_cast<uint4*>(ctx->bufs.k_cache);
-    cp.vc = static_cast<uint4*>(ctx->bufs.v_cache);
-    cp.src = src;
-    cp.N = P.N;
-    cp.K = c.budget_k;
-    cp.units = P.units;
-    cp.err = err;
-    if ((e = timed_launch(ctx, VASE_KERNEL_COMPACT, s, [&] { return launch_compact(cp, P.units, s); })) != cudaSuccess)
-        return cuda_fail(ctx, e, "compact launch");
-    ctx->launches += 2;
+    ctx->launches += 1;
     for (int z = 0; z < nz; ++z) {
         vase_layer_state& st = ctx->layers[layers[z]];
         st.fill = c.budget_k;
@@ -923,8 +920,7 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
         return VASE_ERR_CUDA;
     }
     if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
-        (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess || (e = select_set_attributes(P.select_smem)) != cudaSuccess ||
-        (e = compact_set_attributes()) != cudaSuccess) {
+        (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess || (e = select_set_attributes(P.select_smem)) != cudaSuccess) {
         g_config_error = std::string("kernel attributes: ") + cudaGetErrorString(e);
         return VASE_ERR_CUDA;
     }
@@ -973,6 +969,8 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
     sel.vmag = bufs->value_scores;
     sel.vscore_dbg = nullptr;
     sel.pos = bufs->positions;
+    sel.kc = static_cast<uint4*>(bufs->k_cache);
+    sel.vc = static_cast<uint4*>(bufs->v_cache);
     sel.src = src;
     sel.pooled_dbg = nullptr;
     sel.key_dbg = nullptr;
@@ -987,25 +985,13 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
     sel.stochastic = c.stochastic;
     sel.Hkv = c.num_kv_heads;
     sel.n_parts = c.variant == VASE_VARIANT_ATTNV ? P.n_rb : 1;
+    sel.staged = P.select_staged ? 1 : 0;
     sel.units = P.units;
     sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
     sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
     sel.err = err;
     if ((e = launch_select(sel, P.units, P.select_smem, s)) != cudaSuccess) {
         g_config_error = std::string("select launch: ") + cudaGetErrorString(e);
-        return VASE_ERR_CUDA;
-    }
-    CompactParams cp;
-    cp.batch = batch;
-    cp.kc = static_cast<uint4*>(bufs->k_cache);
-    cp.vc = static_cast<uint4*>(bufs->v_cache);
-    cp.src = src;
-    cp.N = P.N;
-    cp.K = c.budget_k;
-    cp.units = P.units;
-    cp.err = err;
-    if ((e = launch_compact(cp, P.units, s)) != cudaSuccess) {
-        g_config_error = std::string("compact launch: ") + cudaGetErrorString(e);
         return VASE_ERR_CUDA;
     }
     if (device_error) {

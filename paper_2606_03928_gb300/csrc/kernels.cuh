@@ -142,24 +142,19 @@ struct SelectParams {
     const float* dkv;       // [slot][units][N] leverage products (DKV)
     float* vmag;            // base of [L][units][N]: value magnitudes (AttnV), compacted in place
     int32_t* pos;           // base of [L][units][N]; compacted in place with the kept list
+    uint4* kc;              // base of [L][units][N][16]: K rows, gathered in place
+    uint4* vc;              // V rows
     float* vscore_dbg;      // nullable, [slot][units][N]: the value magnitudes of this eviction
     int32_t* src;           // [slot][units][K]
     float* pooled_dbg;      // nullable, [slot][units][N]
     float* key_dbg;         // nullable
     uint8_t* keep_dbg;      // nullable
     int32_t N, K, B, n_v, m, pool, variant, stochastic, Hkv, n_parts, units;
+    int32_t staged;         // 1: every input array of the unit is copied to shared memory up front
     uint32_t seed_lo, seed_hi;
     uint32_t* err;
 };
 
-struct CompactParams {
-    LayerBatch batch;
-    uint4* kc;              // base of [L][units][N][16]
-    uint4* vc;
-    const int32_t* src;     // [slot][units][K]
-    int32_t N, K, units;
-    uint32_t* err;
-};
 
 // ------------------------------------------------------------------ launchers (return cudaError_t)
 
@@ -170,15 +165,12 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
 cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
                        size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s);
-cudaError_t launch_compact(const CompactParams& p, int units, cudaStream_t s);
 
 size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages);
 size_t dkv_smem_bytes(int stages);
-size_t select_smem_bytes(int N, int K);
+size_t select_smem_bytes(int N, int K, int n_parts, bool staged);
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster);
 cudaError_t dkv_set_attributes(size_t smem_bytes);
 cudaError_t select_set_attributes(size_t smem_bytes);
-size_t compact_smem_bytes();
-cudaError_t compact_set_attributes();
 
 }  // namespace vase

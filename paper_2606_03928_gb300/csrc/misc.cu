@@ -156,6 +156,7 @@ struct SelShared {
     uint32_t hist[kSelBins];
     int warp_tot[kSelWarps];
     uint32_t bcast[4];
+    int first_evicted;  // lowest evicted slot (slots below it keep their place)
 };
 
 // Exclusive prefix over threads of `v` in thread order; returns the offset and
@@ -270,13 +271,64 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
 // (exponential race); with stochastic = 0 the key is the pooled score itself
 // (Sec. 4.1).  DKV: the K - B largest leverage products.  Writes the ascending
 // list of kept slots.
+// Asynchronous copy of `count` 32-bit words from global to shared memory by the whole block, in 16-byte
+// pieces when both ends allow it; completion by cp_async_wait_all().
+__device__ __forceinline__ void cp_async_words(void* smem_dst, const void* gsrc, int count) {
+    const bool vec = ((reinterpret_cast<uintptr_t>(gsrc) | smem_u32(smem_dst)) & 15u) == 0;
+    if (vec) {
+        const int n4 = count >> 2;
+        for (int i = threadIdx.x; i < n4; i += blockDim.x)
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst) + 16u * i),
+                         "l"(static_cast<const uint8_t*>(gsrc) + 16 * i)
+                         : "memory");
+        for (int i = 4 * n4 + threadIdx.x; i < count; i += blockDim.x)
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(smem_dst) + 4u * i),
+                         "l"(static_cast<const uint8_t*>(gsrc) + 4 * i)
+                         : "memory");
+    } else {
+        for (int i = threadIdx.x; i < count; i += blockDim.x)
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(smem_dst) + 4u * i),
+                         "l"(static_cast<const uint8_t*>(gsrc) + 4 * i)
+                         : "memory");
+    }
+}
+
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
+// Shared-memory layout of the selection: window scores (one array per part) or leverage products, then
+// (staged) value magnitudes and positions, then the orderable keys and the flags.
+struct SelLayout {
+    uint32_t a_off, vm_off, pos_off, ord_off, flag_off, total;
+};
+
+__host__ __device__ inline SelLayout sel_layout(int N, int K, int n_parts, bool staged) {
+    SelLayout L;
+    uint32_t o = 0;
+    L.a_off = o;
+    o += 4u * (staged ? n_parts : 1) * N;
+    L.vm_off = o;
+    if (staged) o += 4u * N;
+    L.pos_off = o;
+    if (staged) o += 4u * N;
+    L.ord_off = o;
+    o += 4u * K;
+    L.flag_off = o;
+    o += N;
+    L.total = o + 16;
+    return L;
+}
+
 __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectParams p) {
     extern __shared__ __align__(16) uint8_t smem_raw[];
     __shared__ SelShared sh;
     const int N = p.N, K = p.K;
-    float* a_s = reinterpret_cast<float*>(smem_raw);              // [N] window score (AttnV)
-    uint32_t* ord = reinterpret_cast<uint32_t*>(a_s + N);         // [K] orderable keys
-    uint8_t* flags = reinterpret_cast<uint8_t*>(ord + K);         // [N]
+    const bool staged = p.staged != 0;
+    const SelLayout Ly = sel_layout(N, K, p.n_parts, staged);
+    float* a_s = reinterpret_cast<float*>(smem_raw + Ly.a_off);         // [N] window score (AttnV)
+    uint32_t* ord = reinterpret_cast<uint32_t*>(smem_raw + Ly.ord_off);  // [K] orderable keys
+    uint8_t* flags = smem_raw + Ly.flag_off;                            // [N]
     const int unit = blockIdx.x;
     const int z = blockIdx.y;  // layer slot
     const int layer = p.batch.layer[z];
@@ -299,20 +351,49 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
     const int kseg_lo = min(K, seg_lo);
     const int kseg_hi = min(K, seg_hi);
 
+    // The unit's inputs: with `staged`, every array is requested at once (one memory latency for all),
+    // and the positions and value magnitudes are compacted from the staged copies at the end.
+    float* vm_s = staged ? reinterpret_cast<float*>(smem_raw + Ly.vm_off) : nullptr;
+    int32_t* pos_s = staged ? reinterpret_cast<int32_t*>(smem_raw + Ly.pos_off) : nullptr;
+    if (staged) {
+        if (p.variant == 0) {
+            for (int part = 0; part < p.n_parts; ++part)
+                cp_async_words(a_s + part * N, attn + (static_cast<int64_t>(part) * p.units + unit) * N, N);
+        } else {
+            cp_async_words(a_s, dkv + base, K);
+        }
+        cp_async_words(vm_s, vmag + base, N);
+        cp_async_words(pos_s, pos + base, N);
+    }
     for (int i = tid; i < N; i += kSelThreads) flags[i] = 0;
+    if (tid == 0) sh.first_evicted = K;
+    if (staged) {
+        cp_async_wait_all();
+        __syncthreads();
+    }
     if (p.variant == 0) {
-        for (int i = tid; i < N; i += kSelThreads) {
-            float a = attn[base + i];
-            for (int part = 1; part < p.n_parts; ++part)
-                a += attn[(static_cast<int64_t>(part) * p.units + unit) * N + i];
-            a_s[i] = a;
+        if (staged) {
+            if (p.n_parts > 1) {
+                for (int i = tid; i < N; i += kSelThreads) {
+                    float a = a_s[i];
+                    for (int part = 1; part < p.n_parts; ++part) a += a_s[part * N + i];
+                    a_s[i] = a;
+                }
+            }
+        } else {
+            for (int i = tid; i < N; i += kSelThreads) {
+                float a = attn[base + i];
+                for (int part = 1; part < p.n_parts; ++part)
+                    a += attn[(static_cast<int64_t>(part) * p.units + unit) * N + i];
+                a_s[i] = a;
+            }
         }
         if (p.n_parts > 1 && pooled_dbg) {
             __syncthreads();
             for (int i = tid; i < N; i += kSelThreads) const_cast<float*>(attn)[base + i] = a_s[i];
         }
         for (int i = tid; i < K; i += kSelThreads) {
-            const float vm = vmag[base + i];
+            const float vm = staged ? vm_s[i] : vmag[base + i];
             ord[i] = __float_as_uint(vm) + 1u;
             if (vscore_dbg) vscore_dbg[base + i] = vm;
         }
@@ -335,8 +416,9 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
             } else {
                 key = pooled;
                 if (p.stochastic) {
+                    const int32_t pi = staged ? pos_s[i] : pos[base + i];
                     const Philox4 w = philox4x32_10(
-                        Philox4{static_cast<uint32_t>(pos[base + i]), static_cast<uint32_t>(rnd), c2,
+                        Philox4{static_cast<uint32_t>(pi), static_cast<uint32_t>(rnd), c2,
                                 static_cast<uint32_t>(unit)},
                         p.seed_lo, p.seed_hi);
                     key = pooled / (-logf(open_uniform(w.x)));
@@ -349,40 +431,51 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
         radix_top_k(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
     } else {
         for (int i = tid; i < K; i += kSelThreads) {
-            const float s = dkv[base + i];
+            const float s = staged ? a_s[i] : dkv[base + i];
             ord[i] = __float_as_uint(s) + 1u;
             if (key_dbg) key_dbg[base + i] = s;
         }
         __syncthreads();
         radix_top_k(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
     }
-    // positions move with the kept rows: stage the old ones in shared memory (a_s is free now)
-    int32_t* pos_s = reinterpret_cast<int32_t*>(a_s);
-    for (int i = tid; i < N; i += kSelThreads) pos_s[i] = pos[base + i];
-    // keep = R_B u R_V u sampled; ascending list of kept slots
+    // positions move with the kept rows (unstaged: copy the old ones into shared memory, a_s is free now)
+    if (!staged) {
+        pos_s = reinterpret_cast<int32_t*>(a_s);
+        for (int i = tid; i < N; i += kSelThreads) pos_s[i] = pos[base + i];
+    }
+    // keep = R_B u R_V u sampled; ascending list of kept slots (also kept in shared memory, where the keys
+    // were: the gather below reads it)
+    int32_t* src_s = reinterpret_cast<int32_t*>(ord);
     int cnt = 0;
     for (int i = seg_lo; i < seg_hi; ++i) cnt += (i >= K) || flags[i];
     int total;
     const int dst0 = block_exclusive_scan(cnt, sh, &total);  // also a barrier after the staging above
     int dst = dst0;
+    int first_ev = K;
     for (int i = seg_lo; i < seg_hi; ++i) {
         const bool keep = (i >= K) || flags[i];
         if (keep) {
             if (dst < K) {
                 src_out[static_cast<int64_t>(unit) * K + dst] = i;
+                src_s[dst] = i;
                 pos[base + dst] = pos_s[i];
             }
             ++dst;
+        } else if (i < first_ev) {
+            first_ev = i;
         }
         if (keep_dbg) keep_dbg[base + i] = keep ? 1 : 0;
         if (key_dbg && i >= K) key_dbg[base + i] = -1.f;
     }
+    if (first_ev < K) atomicMin(&sh.first_evicted, first_ev);
     for (int i = K + tid; i < N; i += kSelThreads) pos[base + i] = -1;
     // value magnitudes move with their rows too
-    __syncthreads();
-    float* vm_s = a_s;
-    for (int i = tid; i < N; i += kSelThreads) vm_s[i] = vmag[base + i];
-    __syncthreads();
+    if (!staged) {
+        __syncthreads();
+        vm_s = a_s;
+        for (int i = tid; i < N; i += kSelThreads) vm_s[i] = vmag[base + i];
+        __syncthreads();
+    }
     dst = dst0;
     for (int i = seg_lo; i < seg_hi; ++i) {
         if ((i >= K) || flags[i]) {
@@ -390,133 +483,46 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
             ++dst;
         }
     }
-    if (tid == 0 && total != K) record_error(p.err, kErrSelectCount);
-}
-
-// ------------------------------------------------------------------ compaction
-// Stable in-place gather of the kept rows of K or V into slots 0..K-1 (Sec. 2:
-// the cache is restored to K pairs).  New slot j takes old slot src[j] >= j.
-// One CTA (one warp) owns the K or the V rows of one unit and walks
-// destination chunks of 128 rows in ascending order: the kept rows of a chunk
-// form runs of consecutive source rows, each fetched by one bulk TMA copy into
-// a shared-memory stage, and the chunk goes back with one bulk store.  Sources
-// of chunk c lie at or above row 128c while its store ends below 128(c+1), so a
-// later chunk never loads a row an earlier store overwrites; a chunk is stored
-// only after its loads (and all earlier ones) have completed.  Several stages
-// keep loads in flight ahead of the stores.
-constexpr int kCompactRows = 128;                          // destination rows per chunk
-constexpr int kCompactStages = 3;
-constexpr int kCompactChunkBytes = kCompactRows * kRowBytes;  // 32 KB
-
-__device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar) {
-    asm volatile("cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     smem_u32(smem_dst)),
-                 "l"(gsrc), "r"(bytes), "r"(smem_u32(bar))
-                 : "memory");
-}
-__device__ __forceinline__ void bulk_store(void* gdst, const void* smem_src, uint32_t bytes) {
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(smem_u32(smem_src)),
-                 "r"(bytes)
-                 : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-
-__global__ void __launch_bounds__(32) compact_kernel(const CompactParams p) {
-    extern __shared__ __align__(1024) uint8_t smem_raw[];
-    uint8_t* ring = smem_raw;
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + kCompactStages * kCompactChunkBytes);
-    const int unit = blockIdx.x;
-    const int lane = threadIdx.x;
-    const int z = blockIdx.z;  // layer slot
-    const int64_t unit_row = static_cast<int64_t>(p.batch.layer[z]) * p.units * p.N + static_cast<int64_t>(unit) * p.N;
-    uint8_t* base = reinterpret_cast<uint8_t*>((blockIdx.y == 0 ? p.kc : p.vc) + unit_row * kVecPerRow);
-    const int32_t* src = p.src + (static_cast<int64_t>(z) * p.units + unit) * p.K;
-    const int n_chunks = (p.K + kCompactRows - 1) / kCompactRows;
-    if (lane == 0) {
-        for (int s = 0; s < kCompactStages; ++s) mbar_init(&full[s], 1);
-        fence_mbar_init();
+    if (total != K) {  // cannot happen for a consistent state; the rows stay where they are
+        if (tid == 0) record_error(p.err, kErrSelectCount);
+        return;
     }
-    __syncwarp();
-    // chunks whose rows all stay in place need no work: the kept list starts with 0, 1, 2, ...
-    int first = 0;
-    for (; first < n_chunks; ++first) {
-        bool same = true;
-        for (int k = lane; k < kCompactRows; k += 32) {
-            const int j = first * kCompactRows + k;
-            if (j < p.K && src[j] != j) same = false;
-        }
-        if (!__all_sync(0xffffffffu, same)) break;
-    }
-    // stage and mbarrier phase count from the first chunk that moves
-    auto load = [&](int c) {
-        const int stage = (c - first) % kCompactStages;
-        uint8_t* dst = ring + stage * kCompactChunkBytes;
-        const int j0 = c * kCompactRows;
-        const int rows = min(kCompactRows, p.K - j0);
-        if (lane == 0) mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(rows) * kRowBytes);
-        __syncwarp();
-        // a run of consecutive sources starts where src[j] != src[j-1] + 1 (or at the chunk start)
-        uint32_t starts[kCompactRows / 32];
-        int sv[kCompactRows / 32];
+    __syncthreads();  // the kept list and the lowest evicted slot are complete
+
+    // ---- stable in-place gather of the kept K and V rows into slots 0..K-1 (the cache is restored to K
+    // pairs, Sec. 2).  New slot j takes old slot src[j] >= j; slots below the lowest evicted one stay.  The
+    // rows go in chunks of 64 destination rows, 16 threads per row (16 bytes each), through registers.  The
+    // sources of a chunk lie at or above its first row and its stores stay below the next chunk's first
+    // row, so only the chunk's own loads must precede its stores (one barrier per chunk).
+    const int64_t unit_row = (static_cast<int64_t>(layer) * p.units + unit) * N;
+    uint4* const kc = p.kc + unit_row * kVecPerRow;
+    uint4* const vc = p.vc + unit_row * kVecPerRow;
+    const int seg16 = tid & 15;
+    const int r0 = tid >> 4;  // 0..15
+    for (int j0 = sh.first_evicted; j0 < K; j0 += 64) {
+        uint4 kv[4], vv[4];
 #pragma unroll
-        for (int k = 0; k < kCompactRows / 32; ++k) {
-            const int q = k * 32 + lane;
-            const int j = j0 + q;
-            const bool in = q < rows;
-            const int s = in ? src[j] : 0;
-            sv[k] = s;
-            const bool st = in && (q == 0 || src[j - 1] + 1 != s);
-            starts[k] = __ballot_sync(0xffffffffu, st);
-        }
-#pragma unroll
-        for (int k = 0; k < kCompactRows / 32; ++k) {
-            const int q = k * 32 + lane;
-            if ((starts[k] >> lane) & 1u) {
-                // run length: distance to the next start, or to the end of the chunk
-                int next = rows;
-                const uint32_t later = lane < 31 ? (starts[k] >> (lane + 1)) << (lane + 1) : 0u;
-                if (later) {
-                    next = k * 32 + __ffs(later) - 1;
-                } else {
-#pragma unroll
-                    for (int k2 = k + 1; k2 < kCompactRows / 32; ++k2) {
-                        if (starts[k2]) {
-                            next = min(next, k2 * 32 + __ffs(starts[k2]) - 1);
-                            break;
-                        }
-                    }
-                }
-                bulk_load(dst + q * kRowBytes, base + static_cast<int64_t>(sv[k]) * kRowBytes,
-                          static_cast<uint32_t>(next - q) * kRowBytes, &full[stage]);
+        for (int q = 0; q < 4; ++q) {
+            const int j = j0 + r0 + 16 * q;
+            if (j < K) {
+                const int64_t sidx = static_cast<int64_t>(src_s[j]) * kVecPerRow + seg16;
+                kv[q] = kc[sidx];
+                vv[q] = vc[sidx];
             }
         }
-    };
-    bool ok = true;
-    for (int c = first; c < first + kCompactStages - 1 && c < n_chunks; ++c) load(c);
-    for (int c = first; c < n_chunks; ++c) {
-        const int nxt = c + kCompactStages - 1;
-        if (nxt < n_chunks) {
-            if (lane == 0) bulk_wait_read0();  // the stage's previous store has read its bytes
-            __syncwarp();
-            load(nxt);
+        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int j = j0 + r0 + 16 * q;
+            if (j < K) {
+                const int64_t didx = static_cast<int64_t>(j) * kVecPerRow + seg16;
+                kc[didx] = kv[q];
+                vc[didx] = vv[q];
+            }
         }
-        const int stage = (c - first) % kCompactStages;
-        if (ok) ok = mbar_wait(&full[stage], ((c - first) / kCompactStages) & 1, p.err, kErrCompactFull);
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        if (lane == 0) {
-            const int j0 = c * kCompactRows;
-            const int rows = min(kCompactRows, p.K - j0);
-            bulk_store(base + static_cast<int64_t>(j0) * kRowBytes, ring + stage * kCompactChunkBytes,
-                       static_cast<uint32_t>(rows) * kRowBytes);
-            bulk_commit();
-        }
-        __syncwarp();
     }
-    if (lane == 0) bulk_wait_all();
-    __syncwarp();
 }
+
 
 }  // namespace
 
@@ -536,7 +542,7 @@ cudaError_t launch_value_score(const ValueParams& p, int num_sms, cudaStream_t s
     return cudaGetLastError();
 }
 
-size_t select_smem_bytes(int N, int K) { return static_cast<size_t>(N) * 4 + static_cast<size_t>(K) * 4 + N + 16; }
+size_t select_smem_bytes(int N, int K, int n_parts, bool staged) { return sel_layout(N, K, n_parts, staged).total; }
 
 cudaError_t select_set_attributes(size_t smem_bytes) {
     return cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -545,18 +551,6 @@ cudaError_t select_set_attributes(size_t smem_bytes) {
 
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s) {
     select_kernel<<<dim3(static_cast<unsigned>(units), static_cast<unsigned>(p.batch.n)), kSelThreads, smem_bytes, s>>>(p);
-    return cudaGetLastError();
-}
-
-size_t compact_smem_bytes() { return kCompactStages * (kCompactChunkBytes + 8) + 1024; }
-
-cudaError_t compact_set_attributes() {
-    return cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                static_cast<int>(compact_smem_bytes()));
-}
-
-cudaError_t launch_compact(const CompactParams& p, int units, cudaStream_t s) {
-    compact_kernel<<<dim3(static_cast<unsigned>(units), 2, static_cast<unsigned>(p.batch.n)), 32, compact_smem_bytes(), s>>>(p);
     return cudaGetLastError();
 }
 

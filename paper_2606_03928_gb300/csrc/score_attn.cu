@@ -112,8 +112,9 @@ __device__ __forceinline__ ScoreItem score_item(const ScoreAttnParams& p, int w)
 }
 
 // Tile t of a phase with nA pass-A tiles and nB pass-B tiles (each 0 or n): the first `lead` pass-B
-// tiles, then pass A and pass B alternately, then the last `lead` pass-A tiles.  Returns true for a
-// pass-A tile; j is the tile's index within its pass.
+// tiles, then pairs of one pass-A and one pass-B tile in the orders A B, B A, A B, ... (so that the two
+// consumer groups, which take alternate items, each get both kinds), then the last `lead` pass-A tiles.
+// Returns true for a pass-A tile; j is the tile's index within its pass.
 __device__ __forceinline__ bool phase_tile(int t, int nA, int nB, int lead, int& j) {
     if (nB == 0) {
         j = t;
@@ -125,8 +126,10 @@ __device__ __forceinline__ bool phase_tile(int t, int nA, int nB, int lead, int&
     }
     const int u = t - lead;
     if (u < 2 * (nB - lead)) {
-        j = (u & 1) ? lead + (u >> 1) : (u >> 1);
-        return !(u & 1);
+        const int pr = u >> 1;
+        const bool isA = (u & 1) == (pr & 1);
+        j = isA ? pr : lead + pr;
+        return isA;
     }
     j = t - nB;
     return true;

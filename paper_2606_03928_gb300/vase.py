@@ -38,7 +38,7 @@ EXPORTED = [
     "vase_status_string", "vase_last_error", "vase_abi_version", "vase_profile_enable", "vase_profile_collect",
     "vase_append_all", "vase_evict_all", "vase_refresh_value_scores", "vase_evict_static_scratch",
 ]
-KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select", "compact"]
+KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "compact"]
 
 
 class vase_config(ctypes.Structure):

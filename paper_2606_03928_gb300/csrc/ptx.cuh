@@ -94,14 +94,6 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* m
         : "memory");
 }
 
-// Prefetch of one 2-D box into L2 (no shared-memory destination, no completion).
-__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int32_t x, int32_t y) {
-    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                     reinterpret_cast<uint64_t>(map)),
-                 "r"(x), "r"(y)
-                 : "memory");
-}
-
 // L2 eviction-priority policies for cache-hinted copies (createpolicy, fraction 1.0 of the accesses).
 __device__ __forceinline__ uint64_t l2_policy_evict_last() {
     uint64_t pol;

@@ -19,8 +19,9 @@
 //           merged across copies, warps and (through distributed shared
 //           memory) the CTAs of the cluster.
 //   pass B  S = K_tile Q^T (M = 128 tokens, N = window rows): TMEM lane =
-//           token, so each thread accumulates sum_r exp2(s_ri - m_r) / l_r of its
-//           token alone.
+//           token, so each thread accumulates sum_r exp2(s_ri - m'_r) of its token
+//           alone, m'_r = m_r + log2(l_r * G*W) folding the softmax denominator
+//           and the 1/(G*W) mean into the exponent.
 // A single-CTA group that takes several items runs them as phases: phase k
 // interleaves pass B of item k-1 (K re-read from L2, kept there by an
 // evict-last hint on the pass-A read) with pass A of item k (K read from HBM),
@@ -39,12 +40,11 @@ constexpr int kConsumers = 128 * kGroups;
 constexpr int kThreads = kConsumers + 96;       // + a TMA warp and two MMA-issue warps (even / odd items)
 constexpr int kMaxBufs = 4;
 constexpr int kMaxStages = 8;
-constexpr int kPrefetchTiles = 4;               // pass-A tiles requested into L2 ahead of their TMA load
 constexpr uint32_t kTileBytes = kTileTokens * kRowBytes;  // 32 KB: two 64-column panels of 128 rows
 constexpr uint32_t kPanelBytes = kTileTokens * 128;       // 16 KB
 
 struct ScoreSmem {
-    uint32_t q_off, k_off, bar_off, slot_off, pm_off, pl_off, xm_off, xl_off, rowm_off, roww_off, total;
+    uint32_t q_off, k_off, bar_off, slot_off, pm_off, pl_off, xm_off, xl_off, rowm_off, total;
 };
 
 __host__ __device__ inline ScoreSmem score_layout(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster,
@@ -69,8 +69,6 @@ __host__ __device__ inline ScoreSmem score_layout(int q_rows, int q_bufs, int n_
     L.xl_off = o;
     o += 4u * cluster * GWp;
     L.rowm_off = o;
-    o += 4u * GWp;
-    L.roww_off = o;
     o += 4u * GWp;
     L.total = o;
     return L;
@@ -157,8 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* pl = reinterpret_cast<float*>(smem + Ly.pl_off);      // [group][n_rbA][128] running sum per lane
     float* xm = reinterpret_cast<float*>(smem + Ly.xm_off);      // [C][GWp] cluster inbox
     float* xl = reinterpret_cast<float*>(smem + Ly.xl_off);
-    float* rowm = reinterpret_cast<float*>(smem + Ly.rowm_off);  // [GWp] row max (scaled, exp2 domain)
-    float* roww = reinterpret_cast<float*>(smem + Ly.roww_off);  // [GWp] 1 / (row sum * G*W)
+    float* rowm = reinterpret_cast<float*>(smem + Ly.rowm_off);  // [GWp] m'_r: row max + log2(row sum * G*W)
 
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
@@ -246,16 +243,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const ScoreItem itA = score_item(p, group + min(k, n_w - 1) * p.groups);
                 const ScoreItem itB = score_item(p, group + max(k - 1, 0) * p.groups);
                 uint32_t b_owners = 0;
-                if (nA > 0) {
-                    // item k's window rows and first pass-A tiles into L2 while the phase opens with pass B
-                    tma_prefetch_2d(&qmap, 0, static_cast<int32_t>(itA.q_row));
-                    tma_prefetch_2d(&qmap, 64, static_cast<int32_t>(itA.q_row));
-                    for (int jj = 0; jj < kPrefetchTiles && jj < nA; ++jj) {
-                        const int32_t row = static_cast<int32_t>(itA.k_row + static_cast<int64_t>(t_begin + jj) * kTileTokens);
-                        tma_prefetch_2d(&kmap, 0, row);
-                        tma_prefetch_2d(&kmap, 64, row);
-                    }
-                }
                 for (int t = 0; t < nA + nB; ++t) {
                     int j;
                     const bool isA = phase_tile(t, nA, nB, lead, j);
@@ -277,12 +264,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     slot_owners = (slot_owners & ~(3u << (2 * ls))) | (owners << (2 * ls));
                     slot_item[ls] = g;
-                    if (isA && j + kPrefetchTiles < nA) {
-                        const int32_t row = static_cast<int32_t>(
-                            itA.k_row + static_cast<int64_t>(t_begin + j + kPrefetchTiles) * kTileTokens);
-                        tma_prefetch_2d(&kmap, 0, row);
-                        tma_prefetch_2d(&kmap, 64, row);
-                    }
                     if (isA && j == 0) {
                         // window rows of item k: R copies of the GWp rows (pass A lanes), or q_rows rows
                         const int qb = k & (p.q_bufs - 1);
@@ -548,17 +529,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 for (int q = 0; q < 32; ++q) v[q] = h[q];
                             }
                             const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
-                            const float4* w4 = reinterpret_cast<const float4*>(roww + sub * NB + c);
                             float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
                             for (int q = 0; q < 16; ++q) {
                                 if (q < width / 4) {
                                     const float4 mm = m4[q];
-                                    const float4 ww = w4[q];
-                                    a0 = fmaf(ex2(fmaf(v[4 * q], cs, -mm.x)), ww.x, a0);
-                                    a1 = fmaf(ex2(fmaf(v[4 * q + 1], cs, -mm.y)), ww.y, a1);
-                                    a2 = fmaf(ex2(fmaf(v[4 * q + 2], cs, -mm.z)), ww.z, a2);
-                                    a3 = fmaf(ex2(fmaf(v[4 * q + 3], cs, -mm.w)), ww.w, a3);
+                                    a0 += ex2(fmaf(v[4 * q], cs, -mm.x));
+                                    a1 += ex2(fmaf(v[4 * q + 1], cs, -mm.y));
+                                    a2 += ex2(fmaf(v[4 * q + 2], cs, -mm.z));
+                                    a3 += ex2(fmaf(v[4 * q + 3], cs, -mm.w));
                                 }
                             }
                             acc += (a0 + a1) + (a2 + a3);
@@ -578,7 +557,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (k == n_w) break;
             // ------------------------------------ item k's row statistics: groups, copies, then the cluster
-            // (every pass-B tile of item k - 1 is done, so rowm / roww are free)
+            // (every pass-B tile of item k - 1 is done, so rowm is free)
             named_bar(1, kConsumers);
             for (int r = tid; r < GWp; r += kConsumers) {
                 float m = -INFINITY, l = 0.f;
@@ -598,8 +577,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 } else {
                     const bool real = r < p.GW;
-                    rowm[r] = real ? m : INFINITY;
-                    roww[r] = real ? p.inv_gw / l : 0.f;
+                    rowm[r] = real ? m + log2f(l * static_cast<float>(p.GW)) : INFINITY;
                 }
             }
             if (C > 1) {
@@ -609,8 +587,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     float m = -INFINITY, l = 0.f;
                     for (int c = 0; c < C; ++c) merge_ml(m, l, xm[c * GWp + r], xl[c * GWp + r]);
                     const bool real = r < p.GW;
-                    rowm[r] = real ? m : INFINITY;
-                    roww[r] = real ? p.inv_gw / l : 0.f;
+                    rowm[r] = real ? m + log2f(l * static_cast<float>(p.GW)) : INFINITY;
                 }
             }
             named_bar(1, kConsumers);

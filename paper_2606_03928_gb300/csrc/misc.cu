@@ -297,10 +297,17 @@ __device__ __forceinline__ void cp_async_wait_all() {
     asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
 }
 
+// Gather of the kept rows: one warp per tensor (K, V), a ring of kGatherStages chunks of kGatherRows
+// destination rows each.
+constexpr int kGatherRows = 24;
+constexpr int kGatherStages = 3;
+constexpr uint32_t kGatherRingBytes = kGatherStages * kGatherRows * kRowBytes;  // per tensor
+
 // Shared-memory layout of the selection: window scores (one array per part) or leverage products, then
-// (staged) value magnitudes and positions, then the orderable keys and the flags.
+// (staged) value magnitudes and positions, then the orderable keys and the flags.  The gather rings
+// overlay all of these once the selection is done; the kept list and the rings' barriers follow.
 struct SelLayout {
-    uint32_t a_off, vm_off, pos_off, ord_off, flag_off, total;
+    uint32_t a_off, vm_off, pos_off, ord_off, flag_off, src_off, bar_off, total;
 };
 
 __host__ __device__ inline SelLayout sel_layout(int N, int K, int n_parts, bool staged) {
@@ -316,8 +323,90 @@ __host__ __device__ inline SelLayout sel_layout(int N, int K, int n_parts, bool 
     o += 4u * K;
     L.flag_off = o;
     o += N;
-    L.total = o + 16;
+    if (o < 2 * kGatherRingBytes) o = 2 * kGatherRingBytes;
+    o = (o + 15u) & ~15u;
+    L.src_off = o;
+    o += 4u * K;
+    o = (o + 7u) & ~7u;
+    L.bar_off = o;
+    o += 8u * 2 * kGatherStages;
+    L.total = o;
     return L;
+}
+
+__device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(smem_dst)),
+                 "l"(gsrc), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_store(void* gdst, const void* smem_src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(smem_u32(smem_src)),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// Stable in-place gather of one tensor's kept rows (K or V of one unit) by one warp: new row j takes old
+// row src[j] >= j for j >= j_first (the rows below the lowest evicted slot stay).  Destination chunks of
+// kGatherRows rows go in ascending order: the kept rows of a chunk form runs of consecutive source rows,
+// each fetched by one bulk copy into a ring stage, and the chunk goes back with one bulk store.  The
+// sources of a chunk lie at or above its first row and its store ends below the next chunk's first row,
+// so loads issued ahead never read a row that an earlier chunk's store overwrites; a chunk is stored only
+// after its own loads have landed.
+__device__ void gather_rows(uint8_t* base, const int32_t* src, int j_first, int K, uint8_t* ring, uint64_t* full,
+                            uint32_t* err) {
+    const int lane = threadIdx.x & 31;
+    if (lane == 0) {
+        for (int s = 0; s < kGatherStages; ++s) mbar_init(&full[s], 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+    const int n_chunks = (K - j_first + kGatherRows - 1) / kGatherRows;
+    auto load = [&](int c) {
+        const int stage = c % kGatherStages;
+        uint8_t* dst = ring + stage * (kGatherRows * kRowBytes);
+        const int j0 = j_first + c * kGatherRows;
+        const int rows = min(kGatherRows, K - j0);
+        if (lane == 0) mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(rows) * kRowBytes);
+        __syncwarp();
+        // a run of consecutive sources starts where src[j] != src[j-1] + 1 (or at the chunk start)
+        const bool in = lane < rows;
+        const int sv = in ? src[j0 + lane] : 0;
+        const bool st = in && (lane == 0 || src[j0 + lane - 1] + 1 != sv);
+        const uint32_t starts = __ballot_sync(0xffffffffu, st);
+        if (st) {
+            const uint32_t later = lane < 31 ? (starts >> (lane + 1)) << (lane + 1) : 0u;
+            const int next = later ? __ffs(later) - 1 : rows;
+            bulk_load(dst + lane * kRowBytes, base + static_cast<int64_t>(sv) * kRowBytes,
+                      static_cast<uint32_t>(next - lane) * kRowBytes, &full[stage]);
+        }
+    };
+    bool ok = true;
+    for (int c = 0; c < kGatherStages - 1 && c < n_chunks; ++c) load(c);
+    for (int c = 0; c < n_chunks; ++c) {
+        const int nxt = c + kGatherStages - 1;
+        if (nxt < n_chunks) {
+            if (lane == 0) bulk_wait_read0();  // the store that last used nxt's stage has read its bytes
+            __syncwarp();
+            load(nxt);
+        }
+        const int stage = c % kGatherStages;
+        if (ok) ok = mbar_wait(&full[stage], (c / kGatherStages) & 1, err, kErrCompactFull);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        if (lane == 0) {
+            const int j0 = j_first + c * kGatherRows;
+            const int rows = min(kGatherRows, K - j0);
+            bulk_store(base + static_cast<int64_t>(j0) * kRowBytes, ring + stage * (kGatherRows * kRowBytes),
+                       static_cast<uint32_t>(rows) * kRowBytes);
+            bulk_commit();
+        }
+        __syncwarp();
+    }
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
 }
 
 __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectParams p) {
@@ -443,9 +532,8 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
         pos_s = reinterpret_cast<int32_t*>(a_s);
         for (int i = tid; i < N; i += kSelThreads) pos_s[i] = pos[base + i];
     }
-    // keep = R_B u R_V u sampled; ascending list of kept slots (also kept in shared memory, where the keys
-    // were: the gather below reads it)
-    int32_t* src_s = reinterpret_cast<int32_t*>(ord);
+    // keep = R_B u R_V u sampled; ascending list of kept slots (also kept in shared memory for the gather)
+    int32_t* src_s = reinterpret_cast<int32_t*>(smem_raw + Ly.src_off);
     int cnt = 0;
     for (int i = seg_lo; i < seg_hi; ++i) cnt += (i >= K) || flags[i];
     int total;
@@ -487,39 +575,18 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
         if (tid == 0) record_error(p.err, kErrSelectCount);
         return;
     }
-    __syncthreads();  // the kept list and the lowest evicted slot are complete
+    __syncthreads();  // the kept list and the lowest evicted slot are complete; the selection data is dead
 
     // ---- stable in-place gather of the kept K and V rows into slots 0..K-1 (the cache is restored to K
-    // pairs, Sec. 2).  New slot j takes old slot src[j] >= j; slots below the lowest evicted one stay.  The
-    // rows go in chunks of 64 destination rows, 16 threads per row (16 bytes each), through registers.  The
-    // sources of a chunk lie at or above its first row and its stores stay below the next chunk's first
-    // row, so only the chunk's own loads must precede its stores (one barrier per chunk).
-    const int64_t unit_row = (static_cast<int64_t>(layer) * p.units + unit) * N;
-    uint4* const kc = p.kc + unit_row * kVecPerRow;
-    uint4* const vc = p.vc + unit_row * kVecPerRow;
-    const int seg16 = tid & 15;
-    const int r0 = tid >> 4;  // 0..15
-    for (int j0 = sh.first_evicted; j0 < K; j0 += 64) {
-        uint4 kv[4], vv[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int j = j0 + r0 + 16 * q;
-            if (j < K) {
-                const int64_t sidx = static_cast<int64_t>(src_s[j]) * kVecPerRow + seg16;
-                kv[q] = kc[sidx];
-                vv[q] = vc[sidx];
-            }
-        }
-        __syncthreads();
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int j = j0 + r0 + 16 * q;
-            if (j < K) {
-                const int64_t didx = static_cast<int64_t>(j) * kVecPerRow + seg16;
-                kc[didx] = kv[q];
-                vc[didx] = vv[q];
-            }
-        }
+    // pairs, Sec. 2): warp 0 moves the K rows, warp 1 the V rows, through rings over the selection's
+    // shared memory (written by generic stores until now: order them before the bulk copies).
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    const int warp = tid >> 5;
+    if (warp < 2) {
+        const int64_t unit_row = (static_cast<int64_t>(layer) * p.units + unit) * N;
+        uint8_t* const rows = reinterpret_cast<uint8_t*>((warp == 0 ? p.kc : p.vc) + unit_row * kVecPerRow);
+        gather_rows(rows, src_s, sh.first_evicted, K, smem_raw + warp * kGatherRingBytes,
+                    reinterpret_cast<uint64_t*>(smem_raw + Ly.bar_off) + warp * kGatherStages, p.err);
     }
 }
 

@@ -365,7 +365,11 @@ def run_ours(args):
     host_chunks = [[tuple(x[layer].cpu().pin_memory() for x in chunks[r]) for layer in range(L)]
                    for r in range(n_host)]
     pos_out = [torch.empty((wl.batch, wl.num_kv_heads, K), dtype=torch.int32).pin_memory() for _ in range(L)]
-    h2d = sum(x.numel() * x.element_size() for x in host_chunks[0][0]) * L
+    # bytes that cross the host link per step: every k and v row, and the query rows of the last W steps
+    # (the library reads no other query row: only the last W stay in the window ring)
+    q0, k0, v0 = host_chunks[0][0]
+    h2d = (k0.numel() * k0.element_size() + v0.numel() * v0.element_size()
+           + q0.numel() * q0.element_size() * min(wl.window, q0.shape[0]) // q0.shape[0]) * L
     d2h = sum(p.numel() * p.element_size() for p in pos_out)
 
     def e2e_step(r):

@@ -157,9 +157,13 @@ int vase_append(vase_ctx* ctx, int32_t layer, const void* q, const void* k, cons
  * k and v [L][n_tokens][b][Hkv][d] (device, bf16).  All layers must have room. */
 int vase_append_all(vase_ctx* ctx, const void* q, const void* k, const void* v, int32_t n_tokens, void* stream);
 
-/* Same as vase_append with HOST inputs (pinned memory gives asynchronous copies):
- * the library copies them into its staging area in the workspace (at most B
- * tokens per call) and appends from there. */
+/* Same as vase_append with HOST inputs (at most B tokens per call).  Page-locked
+ * inputs (pinned or registered) are read by the append kernel in place over the
+ * host link, asynchronously on `stream`; other host memory is first copied into
+ * the staging area of the workspace.  Either way only the query rows of the last
+ * W steps cross (earlier queries never reach the window ring).  As with
+ * cudaMemcpyAsync, the inputs must stay unchanged until the stream has run the
+ * append. */
 int vase_append_host(vase_ctx* ctx, int32_t layer, const void* q_host, const void* k_host,
                      const void* v_host, int32_t n_tokens, void* stream);
 

@@ -633,6 +633,20 @@ int vase_append_all(vase_ctx* ctx, const void* q, const void* k, const void* v, 
     return append_batch(ctx, all.data(), ctx->cfg.num_layers, q, k, v, n_tokens, static_cast<cudaStream_t>(stream));
 }
 
+namespace {
+
+// Device-visible address of page-locked (pinned or registered) host memory, or nullptr for any other pointer.
+const void* mapped_host_pointer(const void* host) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, host) != cudaSuccess) {
+        cudaGetLastError();  // clear the sticky-free error of an unknown pointer
+        return nullptr;
+    }
+    return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
+}
+
+}  // namespace
+
 int vase_append_host(vase_ctx* ctx, int32_t layer, const void* q_host, const void* k_host, const void* v_host,
                      int32_t n_tokens, void* stream) {
     if (!ctx) return VASE_ERR_INVALID;
@@ -641,18 +655,32 @@ int vase_append_host(vase_ctx* ctx, int32_t layer, const void* q_host, const voi
         return fail(ctx, VASE_ERR_INVALID, "n_tokens must be in 1..buffer_b for host appends");
     if (!q_host || !k_host || !v_host) return fail(ctx, VASE_ERR_INVALID, "null input");
     if (ctx->layers[layer].fill + n_tokens > ctx->plan.N) return fail(ctx, VASE_ERR_FULL, "append would exceed K + B slots");
-    const size_t qb = static_cast<size_t>(n_tokens) * ctx->cfg.batch * ctx->cfg.num_q_heads * kRowBytes;
+    // Page-locked inputs: the append kernel reads them over the host link itself (no staging copies); only
+    // the query rows that stay in the window ring (the last W steps) are read at all.
+    const void* qd = mapped_host_pointer(q_host);
+    const void* kd = mapped_host_pointer(k_host);
+    const void* vd = mapped_host_pointer(v_host);
+    if (qd && kd && vd) return vase_append(ctx, layer, qd, kd, vd, n_tokens, stream);
+    // Otherwise copy into the staging area of the workspace: all k and v rows, and the query rows of the
+    // last min(W, n_tokens) steps only.  The kernel addresses q by step, so it is handed the staged rows'
+    // address less the skipped steps (it never reads a step before the last W).
+    const int n_q = n_tokens < ctx->cfg.window ? n_tokens : ctx->cfg.window;
+    const size_t q_step = static_cast<size_t>(ctx->cfg.batch) * ctx->cfg.num_q_heads * kRowBytes;
+    const size_t qb = static_cast<size_t>(n_q) * q_step;
     const size_t kb = static_cast<size_t>(n_tokens) * ctx->cfg.batch * ctx->cfg.num_kv_heads * kRowBytes;
     uint8_t* sq = ctx->ws + ctx->plan.off_staging;
-    uint8_t* sk = sq + qb;
+    uint8_t* sk = sq + static_cast<size_t>(ctx->cfg.buffer_b) * q_step;
     uint8_t* sv = sk + kb;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t skipped = static_cast<size_t>(n_tokens - n_q) * q_step;
     cudaError_t e;
-    if ((e = cudaMemcpyAsync(sq, q_host, qb, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+    if ((e = cudaMemcpyAsync(sq, static_cast<const uint8_t*>(q_host) + skipped, qb, cudaMemcpyHostToDevice, s)) !=
+            cudaSuccess ||
         (e = cudaMemcpyAsync(sk, k_host, kb, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
         (e = cudaMemcpyAsync(sv, v_host, kb, cudaMemcpyHostToDevice, s)) != cudaSuccess)
         return cuda_fail(ctx, e, "host-to-device staging copy");
-    return vase_append(ctx, layer, sq, sk, sv, n_tokens, stream);
+    const void* q_dev = reinterpret_cast<const void*>(reinterpret_cast<uintptr_t>(sq) - skipped);
+    return vase_append(ctx, layer, q_dev, sk, sv, n_tokens, stream);
 }
 
 int vase_evict(vase_ctx* ctx, int32_t layer, void* stream) {

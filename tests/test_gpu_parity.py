@@ -175,7 +175,10 @@ def test_append_writes_cache_ring_and_positions():
     assert st["fill"] == N and st["next_position"] == N and st["queries_seen"] == N
 
 
-def test_host_append_and_read_positions_match_device_append():
+@pytest.mark.parametrize("pinned", [True, False])
+def test_host_append_and_read_positions_match_device_append(pinned):
+    """Host appends equal device appends: page-locked inputs are read by the kernel in place, pageable ones
+    go through the staging copies (only the query rows of the last W steps are copied)."""
     wl = W.shrink(SMALL, budget_k=64, buffer_b=16, window=8, batch=2, num_layers=1)
     a = _cache(wl, 1)
     b = _cache(wl, 1)
@@ -186,8 +189,14 @@ def test_host_append_and_read_positions_match_device_append():
     for s in range(0, wl.slots, wl.buffer_b):
         e = min(wl.slots, s + wl.buffer_b)
         a.append(0, tq[s:e].cuda().contiguous(), tk[s:e].cuda().contiguous(), tv[s:e].cuda().contiguous())
-        b.append_host(0, tq[s:e].contiguous().pin_memory(), tk[s:e].contiguous().pin_memory(),
-                      tv[s:e].contiguous().pin_memory())
+        host = [x[s:e].contiguous() for x in (tq, tk, tv)]
+        if pinned:
+            host = [x.pin_memory() for x in host]
+        b.append_host(0, *host)
+        torch.cuda.synchronize()  # the pageable inputs are reused by the next iteration
+    torch.cuda.synchronize()
+    assert torch.equal(a.q_window, b.q_window)
+    assert torch.equal(a.value_scores, b.value_scores)
     a.evict(0)
     b.evict(0)
     torch.cuda.synchronize()

@@ -136,7 +136,9 @@ def kernel_bytes(kind, wl, variant, moved_rows_per_unit):
         # scores, magnitudes and positions in; kept list, positions, magnitudes and the moved K/V rows out
         return U * (N * 4 + K * 4 + K * 4 + K * 4) + U * moved_rows_per_unit * (2 * 2 * row + 8)
     if kind == "append":
-        return 2 * B * wl.batch * (wl.num_q_heads + 2 * wl.num_kv_heads) * row + 2 * B * U * 4
+        # k and v rows of the B steps in and out, the query rows of the last W steps in and out (earlier
+        # queries never reach the window ring), positions and value magnitudes out
+        return 2 * (2 * B * U + min(wl.window, B) * wl.batch * wl.num_q_heads) * row + 2 * B * U * 4
     return 0
 
 

@@ -510,7 +510,7 @@ int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void*
             p.layer[z] = layers[z0 + z];
             p.fill[z] = st.fill;
             p.next_pos[z] = st.next_position;
-            p.q_seen[z] = st.queries_seen;
+            p.q_ring[z] = static_cast<int32_t>(st.queries_seen % c.window);
         }
         cudaError_t e = timed_launch(ctx, VASE_KERNEL_APPEND, stream, [&] { return launch_append(p, nz, stream); });
         if (e != cudaSuccess) return cuda_fail(ctx, e, "append launch");

@@ -83,7 +83,7 @@ struct AppendParams {
     int32_t layer[kMaxLayerBatch];
     int32_t fill[kMaxLayerBatch];
     int64_t next_pos[kMaxLayerBatch];
-    int64_t q_seen[kMaxLayerBatch];
+    int32_t q_ring[kMaxLayerBatch];  // window-ring slot of the layer's next query (queries seen mod W)
 };
 
 struct ScoreAttnParams {

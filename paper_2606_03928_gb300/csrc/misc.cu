@@ -70,56 +70,63 @@ __device__ __forceinline__ float half_warp_value_magnitude(const uint4 u, int ki
     return ss * (1.0f / kHeadDim);
 }
 
-__global__ void append_kernel(const AppendParams p) {
+// One block per (sequence, layer slot, chunk of kAppendSteps decode steps).  A half warp moves one 256-byte
+// row: the Hkv key rows and Hkv value rows of every step, and the Hq query rows of the steps that stay in
+// the window ring (the last W); value rows also get their magnitude.
+constexpr int kAppendSteps = 4;
+
+__global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
     const int z = blockIdx.y;  // layer slot
     const int layer = p.layer[z];
-    const int t = blockIdx.x / p.b;      // decode step within the call
-    const int s = blockIdx.x - t * p.b;  // sequence
-    const int per = (p.Hq + 2 * p.Hkv) * kVecPerRow;
-    const bool q_lives = t >= p.n - p.W;  // only the last W queries survive in the ring
-    const int slot = static_cast<int>((p.q_seen[z] + t) % p.W);
+    const int s = static_cast<int>(blockIdx.x) % p.b;  // sequence
+    const int t0 = (static_cast<int>(blockIdx.x) / p.b) * kAppendSteps;
+    const int t1 = min(p.n, t0 + kAppendSteps);
+    const int Hq = p.Hq, Hkv = p.Hkv, N = p.N, W = p.W;
     const int fill = p.fill[z];
-    const int64_t units = static_cast<int64_t>(p.b) * p.Hkv;
-    uint4* const qwin = p.qwin + static_cast<int64_t>(layer) * p.b * p.Hq * p.W * kVecPerRow;
-    uint4* const kc = p.kc + static_cast<int64_t>(layer) * units * p.N * kVecPerRow;
-    uint4* const vc = p.vc + static_cast<int64_t>(layer) * units * p.N * kVecPerRow;
-    int32_t* const pos = p.pos + static_cast<int64_t>(layer) * units * p.N;
-    float* const vmag = p.vmag + static_cast<int64_t>(layer) * units * p.N;
-    const uint4* const q = p.q + static_cast<int64_t>(z) * p.n * p.b * p.Hq * kVecPerRow;
-    const uint4* const k = p.k + static_cast<int64_t>(z) * p.n * units * kVecPerRow;
-    const uint4* const v = p.v + static_cast<int64_t>(z) * p.n * units * kVecPerRow;
-    const int64_t row_in = static_cast<int64_t>(t) * p.b + s;
-    // the trip count is the same for every thread of the block, so the half-warp shuffles see full warps
-    for (int e0 = 0; e0 < per; e0 += blockDim.x) {
-        const int e = e0 + threadIdx.x;
-        const int head = e >> 4;
-        const int seg = e & 15;
-        uint4 val = make_uint4(0, 0, 0, 0);
-        bool is_v = false;
-        int h = 0;
-        if (e < per) {
-            if (head < p.Hq) {
-                if (q_lives)
-                    qwin[(static_cast<int64_t>(s * p.Hq + head) * p.W + slot) * kVecPerRow + seg] =
-                        q[(row_in * p.Hq + head) * kVecPerRow + seg];
-            } else {
-                is_v = head >= p.Hq + p.Hkv;
-                h = head - p.Hq - (is_v ? p.Hkv : 0);
-                const int64_t dst = (static_cast<int64_t>(s * p.Hkv + h) * p.N + fill + t) * kVecPerRow + seg;
-                const int64_t src = (row_in * p.Hkv + h) * kVecPerRow + seg;
-                if (is_v) {
-                    val = v[src];
-                    vc[dst] = val;
+    const int64_t units = static_cast<int64_t>(p.b) * Hkv;
+    const int64_t unit0 = static_cast<int64_t>(layer) * units + static_cast<int64_t>(s) * Hkv;  // unit of head 0
+    uint4* const kc = p.kc + unit0 * N * kVecPerRow;
+    uint4* const vc = p.vc + unit0 * N * kVecPerRow;
+    int32_t* const pos = p.pos + unit0 * N;
+    float* const vmag = p.vmag + unit0 * N;
+    uint4* const qwin = p.qwin + (static_cast<int64_t>(layer) * p.b + s) * Hq * W * kVecPerRow;
+    const uint4* const qin = p.q + static_cast<int64_t>(z) * p.n * p.b * Hq * kVecPerRow;
+    const uint4* const kin = p.k + static_cast<int64_t>(z) * p.n * units * kVecPerRow;
+    const uint4* const vin = p.v + static_cast<int64_t>(z) * p.n * units * kVecPerRow;
+    for (int t = t0; t < t1; ++t) {
+        const bool q_lives = t >= p.n - W;
+        const int per = (2 * Hkv + (q_lives ? Hq : 0)) * 16;  // 16-byte vectors of this step
+        const int64_t row_in = static_cast<int64_t>(t) * p.b + s;
+        const int slot = q_lives ? (p.q_ring[z] + t) % W : 0;
+        // the trip count is the same for every thread of the block, so the half-warp shuffles see full warps
+        for (int e0 = 0; e0 < per; e0 += blockDim.x) {
+            const int e = e0 + static_cast<int>(threadIdx.x);
+            const int r = e >> 4;
+            const int seg = e & 15;
+            uint4 val = make_uint4(0, 0, 0, 0);
+            bool is_v = false;
+            if (e < per) {
+                if (r < Hkv) {
+                    kc[(static_cast<int64_t>(r) * N + fill + t) * kVecPerRow + seg] =
+                        kin[(row_in * Hkv + r) * kVecPerRow + seg];
+                } else if (r < 2 * Hkv) {
+                    is_v = true;
+                    val = vin[(row_in * Hkv + (r - Hkv)) * kVecPerRow + seg];
+                    vc[(static_cast<int64_t>(r - Hkv) * N + fill + t) * kVecPerRow + seg] = val;
                 } else {
-                    kc[dst] = k[src];
+                    const int hq = r - 2 * Hkv;
+                    qwin[(static_cast<int64_t>(hq) * W + slot) * kVecPerRow + seg] =
+                        qin[(row_in * Hq + hq) * kVecPerRow + seg];
                 }
             }
+            if (__any_sync(0xffffffffu, is_v)) {
+                const float mag = half_warp_value_magnitude(val, p.kind);
+                if (is_v && seg == 0) vmag[static_cast<int64_t>(r - Hkv) * N + fill + t] = mag;
+            }
         }
-        const float mag = half_warp_value_magnitude(val, p.kind);
-        if (is_v && seg == 0) vmag[static_cast<int64_t>(s * p.Hkv + h) * p.N + fill + t] = mag;
+        for (int h = threadIdx.x; h < Hkv; h += blockDim.x)
+            pos[static_cast<int64_t>(h) * N + fill + t] = static_cast<int32_t>(p.next_pos[z] + t);
     }
-    for (int hh = threadIdx.x; hh < p.Hkv; hh += blockDim.x)
-        pos[static_cast<int64_t>(s * p.Hkv + hh) * p.N + fill + t] = static_cast<int32_t>(p.next_pos[z] + t);
 }
 
 // ------------------------------------------------------------------ value magnitude refresh
@@ -594,7 +601,8 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
 }  // namespace
 
 cudaError_t launch_append(const AppendParams& p, int n_layers, cudaStream_t s) {
-    append_kernel<<<dim3(static_cast<unsigned>(p.n * p.b), static_cast<unsigned>(n_layers)), 256, 0, s>>>(p);
+    const int chunks = (p.n + kAppendSteps - 1) / kAppendSteps;
+    append_kernel<<<dim3(static_cast<unsigned>(chunks * p.b), static_cast<unsigned>(n_layers)), 256, 0, s>>>(p);
     return cudaGetLastError();
 }
 

@@ -20,7 +20,9 @@ time, where a *unit* is one (layer, sequence, KV head):
   Gaussian projection G_t ~ N(0, 1/r) that is redrawn every eviction round,
   then the top K - B candidates -- Eq. (4), Sec. 2 and Sec. 3.2;
 * the periodic-eviction framing (protect the B most recent tokens, keep
-  exactly K of the K + B cached tokens) -- Sec. 2, "Periodic eviction".
+  exactly K of the K + B cached tokens) -- Sec. 2, "Periodic eviction";
+* the decode step's attention output over the kept cache, o = sum_i alpha_i v_i
+  -- Eq. (1), Sec. 2 (the consumer of the cache the eviction leaves).
 
 Readings where the paper is silent (each is listed with its reason in the
 design notes of the repository):
@@ -241,6 +243,28 @@ def evict_unit(q_rows, keys, values, positions, *, budget_k, buffer_b, variant="
     out.update(keep=keep, src=src, keys_new=keys[src], values_new=values[src],
                positions_new=np.asarray(positions)[src])
     return out
+
+
+# ----------------------------------------------------------------------------
+# Decode attention over the kept cache (the consumer of the eviction's layout)
+# ----------------------------------------------------------------------------
+
+def decode_attention(q, keys, values):
+    """Output of a decode step for query rows q over the cached pairs, Eq. (1), Sec. 2:
+    o = sum_i alpha_i v_i with alpha_i the softmax over the cached keys of q . k_i / sqrt(d).
+    q [rows, d] (the G query heads of one KV head), keys / values [n, d] (the n filled slots)."""
+    return attention_weights(q, keys) @ values
+
+
+def decode_attention_bound(q, keys, values):
+    """sum_i alpha_i |v_i| per output element: the scale of an fp32 weighted sum's rounding error."""
+    return attention_weights(q, keys) @ np.abs(values)
+
+
+def decode_attention_bits(q_bits, k_bits, v_bits):
+    """decode_attention on raw bf16 bit arrays; returns (output, its error scale)."""
+    q, k, v = bf16_bits_to_f64(q_bits), bf16_bits_to_f64(k_bits), bf16_bits_to_f64(v_bits)
+    return decode_attention(q, k, v), decode_attention_bound(q, k, v)
 
 
 def evict_unit_bits(q_bits, k_bits, v_bits, positions, **kw):

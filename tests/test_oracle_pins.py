@@ -355,6 +355,42 @@ def test_dkv_keeps_top_leverage_and_buffer():
     assert len(sets) > 1 and len(fixed) == 1
 
 
+# --------------------------------------------------------------------------- decode attention (Eq. (1) output)
+
+def test_decode_attention_closed_forms():
+    rng = np.random.default_rng(31)
+    d = 16
+    v = rng.standard_normal((5, d))
+    k = rng.standard_normal((5, d))
+    q = rng.standard_normal((3, d))
+    # one cached pair: every query returns its value
+    assert np.allclose(O.decode_attention(q, k[:1], v[:1]), np.repeat(v[:1], 3, axis=0))
+    # a zero query weighs every pair equally: the mean value
+    assert np.allclose(O.decode_attention(np.zeros((1, d)), k, v), v.mean(axis=0, keepdims=True))
+    # two pairs: weights are the logistic function of the scaled logit difference
+    a, b = float(q[0] @ k[0]) / math.sqrt(d), float(q[0] @ k[1]) / math.sqrt(d)
+    w0 = 1.0 / (1.0 + math.exp(b - a))
+    assert np.allclose(O.decode_attention(q[:1], k[:2], v[:2])[0], w0 * v[0] + (1.0 - w0) * v[1])
+
+
+def test_decode_attention_invariances_and_bound():
+    rng = np.random.default_rng(32)
+    d, n = 32, 40
+    q = rng.standard_normal((4, d))
+    k = rng.standard_normal((n, d))
+    v1, v2 = rng.standard_normal((n, d)), rng.standard_normal((n, d))
+    perm = rng.permutation(n)
+    out = O.decode_attention(q, k, v1)
+    assert np.allclose(O.decode_attention(q, k[perm], v1[perm]), out)                       # slot order is free
+    assert np.allclose(O.decode_attention(q, k, v1 + 2.0 * v2), out + 2.0 * O.decode_attention(q, k, v2))
+    assert np.all(np.abs(out) <= O.decode_attention_bound(q, k, v1) + 1e-12)
+    # a key aligned with a large query takes all the weight, without overflow
+    k_big = k.copy()
+    k_big[7] = q[0] * 50.0
+    o = O.decode_attention(q[:1] * 50.0, k_big, v1)
+    assert np.all(np.isfinite(o)) and np.allclose(o[0], v1[7])
+
+
 # --------------------------------------------------------------------------- bf16 path and workloads
 
 def test_bf16_widening_is_exact():

@@ -52,6 +52,8 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=None, help="steps of the host-buffer end-to-end pass")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--decode", action="store_true",
+                    help="time the decode-step attention over every layer's kept cache instead of the eviction step")
     return ap.parse_args()
 
 
@@ -463,10 +465,87 @@ def run_ours(args):
     return 0
 
 
+def run_decode(args):
+    """One decode step's attention (Eq. (1)) over the kept cache of every layer, after an eviction round:
+    vase_decode_attention per layer, reading K and V of the K kept slots of every unit once."""
+    import torch
+
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    from paper_2606_03928_gb300 import workloads as Wm
+    wl = Wm.WORKLOADS[args.workload]
+    if args.layers:
+        wl = Wm.shrink(wl, num_layers=args.layers)
+    from paper_2606_03928_gb300 import build as B
+    B.build()
+    from paper_2606_03928_gb300 import vase as V
+
+    L, K, Bf = wl.num_layers, wl.budget_k, wl.buffer_b
+    cache = V.VaseCache(V.Geometry(K, Bf, wl.window, wl.num_q_heads, wl.num_kv_heads, L, wl.batch),
+                        variant=args.variant, seed=0, device=device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(1000)
+    for layer in range(L):
+        cache.append(layer, *gen_stream(wl, K + Bf, gen, device, torch))
+    cache.evict_all()  # every layer now holds its K kept pairs
+    q = torch.randn((L, wl.batch, wl.num_q_heads, wl.head_dim), generator=gen, device=device).to(torch.bfloat16)
+    out = torch.empty((L, wl.batch, wl.num_q_heads, wl.head_dim), dtype=torch.float32, device=device)
+
+    # device pointers computed once: the step is 28 C calls, not 28 tensor views
+    ptrs = [(q[layer].data_ptr(), out[layer].data_ptr()) for layer in range(L)]
+    stream_handle = torch.cuda.current_stream()
+
+    def step():
+        for layer in range(L):
+            V.vase_decode_attention(cache.ctx, layer, ptrs[layer][0], ptrs[layer][1], stream_handle)
+
+    for _ in range(args.warmup):
+        step()
+    st, code = cache.check_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error during warm-up: {code:#x}")
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(0)
+    launches0 = cache.launch_count()
+    torch.cuda.synchronize()
+    sampler.start()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    launches = cache.launch_count() - launches0
+    ms = ev0.elapsed_time(ev1) / args.steps
+    units = wl.batch * wl.num_kv_heads
+    # K and V rows of the kept slots, the query rows in, the fp32 outputs out
+    step_bytes_ = L * (units * K * 2 * 2 * wl.head_dim + wl.batch * wl.num_q_heads * wl.head_dim * (2 + 4))
+    gbs = step_bytes_ / (ms / 1e3) / 1e9
+    hbm_peak, _, peak_kind = measured_peaks()
+    outj = {
+        "metric": "decode-step attention over the kept cache, bytes/s (K and V of every kept slot read once)",
+        "value": gbs, "unit": "GB/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": wl.name, "layers": L, "global_batch": wl.batch, "kept_slots": K,
+                   "heads": f"{wl.num_q_heads}/{wl.num_kv_heads}", "parallelism": "dp1",
+                   "l2": f"inputs larger than L2 ({step_bytes_ / 1e9:.2f} GB read per step)"},
+        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                     "frac": round(gbs / hbm_peak, 4), "traffic": None, "kernel": "decode_attn_kernel",
+                     "algorithmic_bytes_per_launch": step_bytes_ // L, "peak_source": peak_kind},
+        "clocks": clocks, "gpu_launches": launches,
+    }
+    print(json.dumps(outj))
+    return 0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.decode:
+        return run_decode(args)
     return run_ours(args)
 
 

@@ -184,6 +184,18 @@ int vase_evict_all(vase_ctx* ctx, void* stream);
  * with this call. */
 int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream);
 
+/* Attention output of one decode step over the pairs the cache holds now (Eq. (1), Sec. 2):
+ * for every sequence and query head, o = sum_i alpha_i v_i with alpha_i the softmax of
+ * q . k_i / sqrt(d) over slots 0..fill-1 of the query head's KV head (GQA: query head
+ * g*G + j reads KV head g).  This is the consumer of the layout the eviction keeps, read
+ * in place.  q: device, bf16 [b][Hq][d], 16-byte aligned; out: device, fp32 [b][Hq][d].
+ * The caller owns q and out; the call uses no workspace (the slots of each KV head are split
+ * over the CTAs of one thread-block cluster, whose states are folded in shared memory), so
+ * calls may overlap with each other but not with an append or eviction of the same layer.
+ * Errors: VASE_ERR_INVALID (bad layer, null pointer, empty layer), VASE_ERR_ALIGN,
+ * VASE_ERR_UNSUPPORTED (more than 16 query heads per KV head). */
+int vase_decode_attention(vase_ctx* ctx, int32_t layer, const void* q, float* out, void* stream);
+
 /* Copies the K positions of every unit of one layer to host memory
  * (int32 [b][Hkv][K]), enqueued on the stream; the host buffer is valid after
  * the stream completes. */

@@ -34,6 +34,7 @@ struct Plan {
     int slots;  // layers one launch can batch
     size_t stride_attn, stride_un, stride_src;  // elements per workspace slot
     size_t off_err, off_attn, off_pooled, off_vscore, off_key, off_keep, off_src, off_staging, staging_bytes, ws_bytes;
+    size_t decode_smem;                           // decode attention: shared memory per CTA
 };
 
 // Launch parameters of the window-score kernel for `nz` layers of `batch`.
@@ -216,6 +217,7 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     p.off_staging = o;
     p.staging_bytes = static_cast<size_t>(c->buffer_b) * c->batch * (c->num_q_heads + 2 * c->num_kv_heads) * kRowBytes;
     o = align_up(o + p.staging_bytes, kAlign);
+    p.decode_smem = decode_smem_bytes(p.G);
     p.ws_bytes = o;
     return true;
 }
@@ -358,10 +360,6 @@ uint4* vc_layer(vase_ctx* c, int layer) {
 int32_t* pos_layer(vase_ctx* c, int layer) {
     return c->bufs.positions + static_cast<int64_t>(layer) * c->plan.units * c->plan.N;
 }
-uint4* q_layer(vase_ctx* c, int layer) {
-    return reinterpret_cast<uint4*>(c->bufs.q_window) +
-           static_cast<int64_t>(layer) * c->cfg.batch * c->cfg.num_q_heads * c->cfg.window * kVecPerRow;
-}
 
 }  // namespace
 
@@ -455,7 +453,8 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
     }
     if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
         (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess ||
-        (e = select_set_attributes(P.select_smem)) != cudaSuccess) {
+        (e = select_set_attributes(P.select_smem)) != cudaSuccess ||
+        (e = decode_set_attributes(P.decode_smem)) != cudaSuccess) {
         fprintf(stderr, "vase_create: kernel attributes: %s\n", cudaGetErrorString(e));
         delete ctx;
         return VASE_ERR_CUDA;
@@ -724,6 +723,35 @@ int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream) {
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = timed_launch(ctx, VASE_KERNEL_VALUE, s, [&] { return launch_value_score(vp, ctx->num_sms, s); });
     if (e != cudaSuccess) return cuda_fail(ctx, e, "value refresh launch");
+    ctx->launches += 1;
+    return VASE_OK;
+}
+
+int vase_decode_attention(vase_ctx* ctx, int32_t layer, const void* q, float* out, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    if (!q || !out) return fail(ctx, VASE_ERR_INVALID, "null input or output");
+    if (!aligned(q, 16) || !aligned(out, 4)) return fail(ctx, VASE_ERR_ALIGN, "q must be 16-byte aligned, out 4-byte");
+    const int fill = ctx->layers[layer].fill;
+    if (fill < 1) return fail(ctx, VASE_ERR_INVALID, "the layer holds no cached pair");
+    const Plan& P = ctx->plan;
+    if (P.G > 16) return fail(ctx, VASE_ERR_UNSUPPORTED, "decode attention handles at most 16 query heads per KV head");
+    DecodeParams dp;
+    dp.q = static_cast<const uint4*>(q);
+    dp.kc = kc_layer(ctx, layer);
+    dp.vc = vc_layer(ctx, layer);
+    dp.out = out;
+    dp.N = P.N;
+    dp.fill = fill;
+    dp.G = P.G;
+    dp.Hkv = ctx->cfg.num_kv_heads;
+    dp.units = P.units;
+    dp.n_chunks = ceil_div(fill, kDecodeChunk);
+    dp.cluster = decode_cluster(P.units, dp.n_chunks, P.num_sms);
+    dp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
+    dp.err = reinterpret_cast<uint32_t*>(ctx->ws + P.off_err);
+    cudaError_t e = launch_decode(dp, P.decode_smem, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "decode attention launch");
     ctx->launches += 1;
     return VASE_OK;
 }

@@ -23,12 +23,17 @@ enum ErrSite : uint32_t {
     kErrDkvKEmpty = 34,
     kErrDkvTEmpty = 35,
     kErrDkvDrain = 36,
+    kErrDecodeFull = 48,
+    kErrDecodeEmpty = 49,
+    kErrDecodeDrain = 50,
 };
 
 constexpr int kTileTokens = 128;   // tokens per MMA tile (M)
 constexpr int kHeadDim = 128;      // d
 constexpr int kRowBytes = 256;     // d * sizeof(bf16)
 constexpr int kVecPerRow = 16;     // 16-byte vectors per row
+constexpr int kDecodeChunk = 32;   // cache slots per pipeline stage of the decode attention
+constexpr int kDecodeMaxCluster = 8;  // CTAs that split one unit's slots (one thread-block cluster)
 
 // ------------------------------------------------------------------ Philox4x32-10
 // Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as easy as 1, 2, 3" (SC'11):
@@ -156,6 +161,18 @@ struct SelectParams {
 };
 
 
+struct DecodeParams {
+    const uint4* q;         // [b][Hq][16]: the decode step's query rows (bf16)
+    const uint4* kc;        // layer base of [units][N][16]
+    const uint4* vc;
+    float* out;             // [b][Hq][d] fp32
+    int32_t N, fill, G, Hkv, units;
+    int32_t n_chunks;       // ceil(fill / kDecodeChunk)
+    int32_t cluster;        // CTAs per unit (cluster size, <= n_chunks); CTA r takes chunks r, r + cluster, ...
+    float scale_log2;       // log2(e) / sqrt(d)
+    uint32_t* err;
+};
+
 // ------------------------------------------------------------------ launchers (return cudaError_t)
 
 cudaError_t launch_append(const AppendParams& p, int n_layers, cudaStream_t s);
@@ -165,6 +182,7 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
 cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
                        size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s);
+cudaError_t launch_decode(const DecodeParams& p, size_t smem_bytes, cudaStream_t s);
 
 size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages);
 size_t dkv_smem_bytes(int stages);
@@ -172,5 +190,8 @@ size_t select_smem_bytes(int N, int K, int n_parts, bool staged);
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster);
 cudaError_t dkv_set_attributes(size_t smem_bytes);
 cudaError_t select_set_attributes(size_t smem_bytes);
+size_t decode_smem_bytes(int G);
+cudaError_t decode_set_attributes(size_t smem_bytes);
+int decode_cluster(int units, int n_chunks, int num_sms);
 
 }  // namespace vase

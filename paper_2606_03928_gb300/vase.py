@@ -37,6 +37,7 @@ EXPORTED = [
     "vase_kv_view_get", "vase_debug_view_get", "vase_check_device_error", "vase_launch_count",
     "vase_status_string", "vase_last_error", "vase_abi_version", "vase_profile_enable", "vase_profile_collect",
     "vase_append_all", "vase_evict_all", "vase_refresh_value_scores", "vase_evict_static_scratch",
+    "vase_decode_attention",
 ]
 KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "compact"]
 
@@ -101,6 +102,7 @@ def load(path: str = LIB_PATH):
         "vase_evict_static_scratch": (ctypes.c_int, [ctypes.POINTER(vase_config), ctypes.POINTER(vase_buffers), I32,
                                                      ctypes.POINTER(vase_layer_state), ctypes.POINTER(U32), P]),
         "vase_read_positions": (ctypes.c_int, [P, I32, P, P]),
+        "vase_decode_attention": (ctypes.c_int, [P, I32, P, P, P]),
         "vase_get_layer_state": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_layer_state)]),
         "vase_set_layer_state": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_layer_state)]),
         "vase_kv_view_get": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_kv_view)]),
@@ -210,6 +212,11 @@ def vase_evict_static_scratch(cfg: vase_config, bufs: vase_buffers, layer, fill,
     if status < 0:
         raise VaseError(status, "vase_evict_static_scratch: " + load().vase_last_error(None).decode())
     return word.value
+
+
+def vase_decode_attention(ctx, layer, q_ptr, out_ptr, stream=None):
+    return _check(ctx, load().vase_decode_attention(ctx, layer, q_ptr, out_ptr, _stream_ptr(stream)),
+                  "vase_decode_attention")
 
 
 def vase_read_positions(ctx, layer, host_ptr, stream=None):
@@ -337,6 +344,16 @@ class VaseCache:
     def evict_all(self, stream=None):
         """Evicts every full layer in batched launches; returns how many layers were evicted."""
         return vase_evict_all(self.ctx, stream)
+
+    def decode_attention(self, layer, q: torch.Tensor, out: torch.Tensor = None, stream=None):
+        """Attention output of one decode step over the layer's cached pairs: q [b, Hq, d] bf16 CUDA tensor,
+        returns (or fills) out [b, Hq, d] fp32."""
+        assert q.is_cuda and q.dtype == torch.bfloat16 and q.is_contiguous()
+        if out is None:
+            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+        assert out.is_cuda and out.dtype == torch.float32 and out.is_contiguous()
+        vase_decode_attention(self.ctx, layer, q.data_ptr(), out.data_ptr(), stream)
+        return out
 
     def read_positions(self, layer, out: torch.Tensor, stream=None):
         """Copies the K kept positions of every unit into a CPU int32 tensor [b, Hkv, K]."""

@@ -122,14 +122,33 @@ __global__ void __launch_bounds__(kThreads) decode_attn_kernel(const DecodeParam
         bulk_load(kdst, p.kc + (unit_row + s0) * kVecPerRow, bytes, &full[s]);
         bulk_load(kdst + kChunkBytes, p.vc + (unit_row + s0) * kVecPerRow, bytes, &full[s]);
     };
+    // Programmatic dependent launch: the next kernel of the stream may start its own prologue once every CTA of
+    // this grid runs; it reads nothing this grid writes before its griddepcontrol.wait.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (tid == producer) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], kConsumerWarps);
         }
         fence_mbar_init();
-        for (int j = 0; j < min(kStages, n_mine); ++j) issue(j);  // the ring's first fill, before anything else
+        // Warm L2 with the ring's first chunks while the preceding kernel finishes (a prefetch into L2 is only
+        // a hint: L2 is where device memory is coherent, so rows the preceding kernel still writes are read
+        // fresh by the copies below, which come after the wait).
+        for (int j = 0; j < min(kStages, n_mine); ++j) {
+            const int s0 = (rank + j * C) * kDecodeChunk;
+            const uint32_t bytes = static_cast<uint32_t>(min(kDecodeChunk, p.fill - s0)) * kRowBytes;
+            asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.kc + (unit_row + s0) * kVecPerRow),
+                         "r"(bytes)
+                         : "memory");
+            asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.vc + (unit_row + s0) * kVecPerRow),
+                         "r"(bytes)
+                         : "memory");
+        }
     }
+    // everything the preceding kernels of the stream wrote (query rows, cache rows) is visible after this
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (tid == producer)
+        for (int j = 0; j < min(kStages, n_mine); ++j) issue(j);  // the ring's first fill
     // the query rows of this KV head (query heads head*G .. head*G+G-1 of sequence seq) in fp32, scaled by
     // log2(e)/sqrt(d); a padding head reads zeros
     const uint32_t* qrow = reinterpret_cast<const uint32_t*>(
@@ -352,13 +371,15 @@ cudaError_t launch_gp(const DecodeParams& p, size_t smem_bytes, cudaStream_t s) 
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem_bytes;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = static_cast<unsigned>(p.cluster);
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see griddepcontrol in the kernel
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, decode_attn_kernel<Gp>, p);
 }
 

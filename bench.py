@@ -555,7 +555,8 @@ def run_decode(args):
                    "heads": f"{wl.num_q_heads}/{wl.num_kv_heads}", "parallelism": "dp1",
                    "l2": f"inputs larger than L2 ({step_bytes_ / 1e9:.2f} GB read per step)"},
         "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
-                     "frac": round(gbs / hbm_peak, 4), "traffic": None, "kernel": "decode_attn_kernel",
+                     "frac": round(gbs / hbm_peak, 4), "traffic": None,
+                     "kernel": "decode_tc_kernel" if wl.group >= 3 else "decode_simt_kernel",
                      "algorithmic_bytes_per_launch": step_bytes_ // L, "peak_source": peak_kind},
         "clocks": clocks, "gpu_launches": launches, "timed_as": "CUDA graph replay of the step's launches",
         "eager_ms_per_step": eager_ms,

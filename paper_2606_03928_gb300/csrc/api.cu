@@ -280,6 +280,7 @@ struct vase_ctx {
     int device = 0;
     int num_sms = 0;
     CUtensorMap kmap, vmap, qmap;
+    CUtensorMap kmap_dec, vmap_dec;  // 64-row boxes for the decode attention
     std::vector<vase_layer_state> layers;
     std::vector<int32_t> last_batch;  // layers of the most recent eviction launch, by workspace slot
     int64_t launches = 0;
@@ -446,7 +447,9 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
     const uint32_t qbox = static_cast<uint32_t>(P.q_box);
     if (!encode_rows(enc, &ctx->kmap, bufs->k_cache, cache_rows, kTileTokens) ||
         !encode_rows(enc, &ctx->vmap, bufs->v_cache, cache_rows, kTileTokens) ||
-        !encode_rows(enc, &ctx->qmap, bufs->q_window, q_rows, qbox)) {
+        !encode_rows(enc, &ctx->qmap, bufs->q_window, q_rows, qbox) ||
+        !encode_rows(enc, &ctx->kmap_dec, bufs->k_cache, cache_rows, kDecodeTileRows) ||
+        !encode_rows(enc, &ctx->vmap_dec, bufs->v_cache, cache_rows, kDecodeTileRows)) {
         fprintf(stderr, "vase_create: tensor map encoding failed\n");
         delete ctx;
         return VASE_ERR_CUDA;
@@ -454,7 +457,7 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
     if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
         (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess ||
         (e = select_set_attributes(P.select_smem)) != cudaSuccess ||
-        (e = decode_set_attributes(P.decode_smem)) != cudaSuccess) {
+        (e = decode_set_attributes(P.G, P.decode_smem)) != cudaSuccess) {
         fprintf(stderr, "vase_create: kernel attributes: %s\n", cudaGetErrorString(e));
         delete ctx;
         return VASE_ERR_CUDA;
@@ -746,11 +749,11 @@ int vase_decode_attention(vase_ctx* ctx, int32_t layer, const void* q, float* ou
     dp.G = P.G;
     dp.Hkv = ctx->cfg.num_kv_heads;
     dp.units = P.units;
-    dp.n_chunks = ceil_div(fill, kDecodeChunk);
-    dp.cluster = decode_cluster(P.units, dp.n_chunks, P.num_sms);
+    dp.row_base = layer * P.units * P.N;
     dp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
     dp.err = reinterpret_cast<uint32_t*>(ctx->ws + P.off_err);
-    cudaError_t e = launch_decode(dp, P.decode_smem, static_cast<cudaStream_t>(stream));
+    cudaError_t e =
+        launch_decode(ctx->kmap_dec, ctx->vmap_dec, dp, P.decode_smem, P.num_sms, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(ctx, e, "decode attention launch");
     ctx->launches += 1;
     return VASE_OK;

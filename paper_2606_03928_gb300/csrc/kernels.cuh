@@ -32,7 +32,7 @@ constexpr int kTileTokens = 128;   // tokens per MMA tile (M)
 constexpr int kHeadDim = 128;      // d
 constexpr int kRowBytes = 256;     // d * sizeof(bf16)
 constexpr int kVecPerRow = 16;     // 16-byte vectors per row
-constexpr int kDecodeChunk = 32;   // cache slots per pipeline stage of the decode attention
+constexpr int kDecodeTileRows = 64;   // rows per TMA box of the tensor-core decode attention
 constexpr int kDecodeMaxCluster = 8;  // CTAs that split one unit's slots (one thread-block cluster)
 
 // ------------------------------------------------------------------ Philox4x32-10
@@ -167,8 +167,9 @@ struct DecodeParams {
     const uint4* vc;
     float* out;             // [b][Hq][d] fp32
     int32_t N, fill, G, Hkv, units;
-    int32_t n_chunks;       // ceil(fill / kDecodeChunk)
+    int32_t n_chunks;       // ceil(fill / chunk) (set by launch_decode for the kernel it picks)
     int32_t cluster;        // CTAs per unit (cluster size, <= n_chunks); CTA r takes chunks r, r + cluster, ...
+    int32_t row_base;       // first row of the layer in the K / V tensor maps (layer * units * N)
     float scale_log2;       // log2(e) / sqrt(d)
     uint32_t* err;
 };
@@ -182,7 +183,8 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
 cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
                        size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s);
-cudaError_t launch_decode(const DecodeParams& p, size_t smem_bytes, cudaStream_t s);
+cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, DecodeParams p, size_t smem_bytes,
+                          int num_sms, cudaStream_t s);
 
 size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages);
 size_t dkv_smem_bytes(int stages);
@@ -191,7 +193,6 @@ cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster);
 cudaError_t dkv_set_attributes(size_t smem_bytes);
 cudaError_t select_set_attributes(size_t smem_bytes);
 size_t decode_smem_bytes(int G);
-cudaError_t decode_set_attributes(size_t smem_bytes);
-int decode_cluster(int units, int n_chunks, int num_sms);
+cudaError_t decode_set_attributes(int G, size_t smem_bytes);
 
 }  // namespace vase

@@ -103,3 +103,59 @@ def test_decode_rejects_an_empty_layer():
     _, q = _queries(wl, 1)
     with pytest.raises(VaseError):
         cache.decode_attention(0, q)
+
+
+# (query heads, KV heads): G = 1 and 2 take the CUDA-core kernel, G >= 3 the tensor-core kernel (5 and 16 also
+# pad the head columns: 16 columns of P for G <= 8, 32 beyond)
+@pytest.mark.parametrize("heads", [(8, 8), (24, 8), (32, 8), (40, 8), (64, 4)])
+@pytest.mark.parametrize("fill_kind", ["full", "ragged"])
+def test_decode_group_sizes(heads, fill_kind):
+    Hq, Hkv = heads
+    wl = W.shrink(SMALL, budget_k=448, buffer_b=64, window=16, num_q_heads=Hq, num_kv_heads=Hkv, batch=2,
+                  num_layers=1)
+    cache = _cache(wl, 1)
+    st = W.layer_state(wl, 21, 0, 0, "gapped")
+    PU.upload_layer(cache, 0, st, 0)
+    fill = wl.slots if fill_kind == "full" else wl.slots - 37
+    cache.set_layer_state(0, fill, 0, fill, 10 ** 6)
+    q_bits, q = _queries(wl, 22)
+    out = cache.decode_attention(0, q)
+    torch.cuda.synchronize()
+    _check(wl, cache, 0, q_bits, out, fill)
+
+
+def test_decode_sees_the_append_launched_before_it():
+    # the decode launch may start before the preceding kernel ends (programmatic dependent launch) but reads
+    # nothing before that kernel's writes are visible: the second call must see the appended pairs
+    wl = W.shrink(SMALL, budget_k=256, buffer_b=64, window=16, num_q_heads=32, num_kv_heads=8, batch=2,
+                  num_layers=1)
+    cache = _cache(wl, 1)
+    st = W.layer_state(wl, 31, 0, 0, "gapped")
+    PU.upload_layer(cache, 0, st, 0)
+    cache.set_layer_state(0, 200, 0, 200, 10 ** 6)
+    q_bits, q = _queries(wl, 32)
+    first = cache.decode_attention(0, q)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(33)
+    n = 100
+    qa = torch.randn((n, wl.batch, wl.num_q_heads, wl.head_dim), generator=gen, device="cuda").to(torch.bfloat16)
+    ka = torch.randn((n, wl.batch, wl.num_kv_heads, wl.head_dim), generator=gen, device="cuda").to(torch.bfloat16)
+    va = torch.randn((n, wl.batch, wl.num_kv_heads, wl.head_dim), generator=gen, device="cuda").to(torch.bfloat16)
+    cache.append(0, qa, ka, va)
+    second = cache.decode_attention(0, q)
+    torch.cuda.synchronize()
+    assert cache.layer_state(0)["fill"] == 300
+    _check(wl, cache, 0, q_bits, second, 300)
+    assert not torch.equal(first, second)
+
+
+def test_decode_full_size_qwen3_8b_layer_sampled_units():
+    wl = W.WORKLOADS["qwen3_8b_k4096"]
+    cache = _cache(wl, 1)
+    st = W.layer_state(wl, 41, 0, 0, "gapped")
+    PU.upload_layer(cache, 0, st, 0)
+    cache.evict(0)
+    q_bits, q = _queries(wl, 42)
+    out = cache.decode_attention(0, q)
+    torch.cuda.synchronize()
+    _check(wl, cache, 0, q_bits, out, wl.budget_k, units=[(0, 0), (17, 3), (31, 7)])

@@ -22,13 +22,19 @@ time, where a *unit* is one (layer, sequence, KV head):
 * the periodic-eviction framing (protect the B most recent tokens, keep
   exactly K of the K + B cached tokens) -- Sec. 2, "Periodic eviction";
 * the decode step's attention output over the kept cache, o = sum_i alpha_i v_i
-  -- Eq. (1), Sec. 2 (the consumer of the cache the eviction leaves).
+  -- Eq. (1), Sec. 2 (the consumer of the cache the eviction leaves);
+* variants: the random-reservation ablation (N_v candidates drawn uniformly
+  at random instead of the largest Range) -- App. C, first paragraph; GQA
+  max-aggregation over the query heads of a KV head; one Gaussian projection
+  per round shared by every unit (shared-G DKV).
 
 Readings where the paper is silent (each is listed with its reason in the
 design notes of the repository):
 
 * GQA: the window rows of a KV head are the W cached queries of each of its
-  G query heads; the score is the mean over all G*W rows.
+  G query heads (head-major: rows g*W .. g*W+W-1 belong to query head g); the
+  score is the mean over all G*W rows, or (gqa="max") the largest over the G
+  heads of each head's mean over its W rows.
 * Window: W is its own parameter (the paper sets W = B); the divisor is G*W.
 * Pooling: odd kernel kappa, stride 1, zero padding, divisor kappa, along the
   slot axis over all N slots, before restricting to candidates.
@@ -40,10 +46,12 @@ design notes of the repository):
 * Ties in any ranking go to the lower slot (the older token).
 * Noise: u_i comes from Philox4x32-10 (Salmon et al., SC'11) with key
   (seed_lo, seed_hi) and counter (position, round, layer | tag << 24,
-  seq * Hkv + head); tag 0 = selection noise, tag 1 = DKV Gaussian.
+  seq * Hkv + head); tag 0 = selection noise, tag 1 = DKV Gaussian, tag 2 =
+  random-reservation noise.
   u = (2 * (x >> 9) + 1) * 2**-24 from word 0, exact in fp32 and fp64.
   Gaussian entries use Box-Muller (1958) on words 0 and 1 with counter
-  word 0 = a * r + b; the fixed-G (CurDKV) option puts 0 in the round word.
+  word 0 = a * r + b; the fixed-G (CurDKV) option puts 0 in the round word,
+  and the shared-G option puts 0 in the layer bits and the unit word.
 * DKV has no value reservation; the value awareness is the value leverage.
 """
 
@@ -65,6 +73,7 @@ _PHILOX_W1 = np.uint64(0xBB67AE85)
 
 TAG_SELECT = 0
 TAG_DKV = 1
+TAG_RESERVE = 2
 
 
 def philox4x32_10(c0, c1, c2, c3, k0, k1):
@@ -103,16 +112,28 @@ def selection_uniforms(seed, layer, seq, head, num_kv_heads, rnd, positions):
     return uniform_open01(w0)
 
 
-def gaussian_projection(seed, layer, seq, head, num_kv_heads, rnd, d, r, fixed_g=False):
+def reservation_uniforms(seed, layer, seq, head, num_kv_heads, rnd, positions):
+    """Uniform keys of the random-reservation ablation (App. C): the N_v largest pick R_V."""
+    k0, k1 = _noise_key(seed)
+    pos = np.asarray(positions, dtype=np.int64).astype(np.uint64)
+    w0, _, _, _ = philox4x32_10(pos, rnd, (layer | (TAG_RESERVE << 24)), seq * num_kv_heads + head, k0, k1)
+    return uniform_open01(w0)
+
+
+def gaussian_projection(seed, layer, seq, head, num_kv_heads, rnd, d, r, fixed_g=False, shared_g=False):
     """G in R^{d x r} with i.i.d. N(0, 1/r) entries -- Eq. (4), Sec. 2; redrawn per round -- Sec. 3.2.
 
     Entry (a, b) takes Philox counter (a * r + b, round, layer | 1 << 24, seq * Hkv + head)
-    and Box-Muller on words 0 and 1: z = sqrt(-2 ln u1) cos(2 pi u2).
+    and Box-Muller on words 0 and 1: z = sqrt(-2 ln u1) cos(2 pi u2).  fixed_g puts 0 in the round
+    word (one G for the whole stream); shared_g puts 0 in the layer bits and the unit word (one G
+    per round for every layer, sequence and KV head).
     """
     k0, k1 = _noise_key(seed)
     idx = np.arange(d * r, dtype=np.uint64)
     rr = 0 if fixed_g else rnd
-    w0, w1, _, _ = philox4x32_10(idx, rr, (layer | (TAG_DKV << 24)), seq * num_kv_heads + head, k0, k1)
+    c2 = (0 if shared_g else layer) | (TAG_DKV << 24)
+    c3 = 0 if shared_g else seq * num_kv_heads + head
+    w0, w1, _, _ = philox4x32_10(idx, rr, c2, c3, k0, k1)
     u1 = uniform_open01(w0)
     u2 = uniform_open01(w1)
     z = np.sqrt(-2.0 * np.log(u1)) * np.cos(2.0 * np.pi * u2)
@@ -141,9 +162,20 @@ def attention_weights(q_rows, keys):
     return e / e.sum(axis=1, keepdims=True)
 
 
-def window_attention_score(q_rows, keys):
-    """Mean of alpha over the G*W window rows (Eq. (2), non-causal cached queries), before pooling."""
-    return attention_weights(q_rows, keys).mean(axis=0)
+def window_attention_score(q_rows, keys, group=1, gqa="mean"):
+    """The window score of Eq. (2) (non-causal cached queries), before pooling.
+
+    q_rows holds the W window queries of each of the `group` query heads, head-major.  "mean": the
+    mean of alpha over all G*W rows.  "max": each head's mean over its W rows, then the largest over
+    the G heads (GQA max-aggregation)."""
+    a = attention_weights(q_rows, keys)
+    if gqa == "mean":
+        return a.mean(axis=0)
+    if gqa == "max":
+        G = int(group)
+        per_head = a.reshape(G, a.shape[0] // G, a.shape[1]).mean(axis=1)
+        return per_head.max(axis=0)
+    raise ValueError(f"unknown GQA reduction {gqa}")
 
 
 def average_pool(scores, kernel):
@@ -193,7 +225,7 @@ def top_k_slots(scores, k, eligible=None):
 def evict_unit(q_rows, keys, values, positions, *, budget_k, buffer_b, variant="attnv",
                n_v=None, value_score=VALUE_RANGE, pool_kernel=7, stochastic=True,
                dkv_rank=20, dkv_fixed_g=False, seed=0, layer=0, seq=0, head=0,
-               num_kv_heads=1, rnd=0):
+               num_kv_heads=1, rnd=0, group=1, gqa="mean", reserve="value", dkv_shared_g=False):
     """One eviction step for one unit, in fp64.
 
     q_rows [G*W, d], keys/values [K+B, d] (fp64, exact bf16 values), positions [K+B].
@@ -210,10 +242,15 @@ def evict_unit(q_rows, keys, values, positions, *, budget_k, buffer_b, variant="
         nv = K // 4 if n_v is None or n_v < 0 else int(n_v)
         m = K - nv - B                    # the K - |R| sampled slots (Sec. 3.2)
         assert m >= 0
-        a = window_attention_score(q_rows, keys)
+        a = window_attention_score(q_rows, keys, group, gqa)
         abar = average_pool(a, pool_kernel)
         vmag = value_magnitude(values[:K], value_score)
-        r_v = top_k_slots(vmag, nv)       # R_V: N_v largest Range among the K candidates
+        if reserve == "value":
+            r_v = top_k_slots(vmag, nv)   # R_V: N_v largest Range among the K candidates
+        elif reserve == "random":         # the ablation of App. C: N_v candidates uniformly at random
+            r_v = top_k_slots(reservation_uniforms(seed, layer, seq, head, num_kv_heads, rnd, positions[:K]), nv)
+        else:
+            raise ValueError(reserve)
         in_c = np.ones(K, dtype=bool)
         in_c[r_v] = False                 # C = [K] \ R_V
         if stochastic:
@@ -229,7 +266,7 @@ def evict_unit(q_rows, keys, values, positions, *, budget_k, buffer_b, variant="
         out.update(attn=a, pooled=abar, value_score=vmag, key=key_full, reserved_v=r_v)
     elif variant == "dkv":
         d = keys.shape[1]
-        G = gaussian_projection(seed, layer, seq, head, num_kv_heads, rnd, d, dkv_rank, dkv_fixed_g)
+        G = gaussian_projection(seed, layer, seq, head, num_kv_heads, rnd, d, dkv_rank, dkv_fixed_g, dkv_shared_g)
         s, lk, lv = leverage_scores(keys[:K], values[:K], G)
         sel = top_k_slots(s, K - B)
         keep[sel] = True

@@ -412,3 +412,82 @@ def test_unit_state_bits_roundtrip_through_oracle():
     assert q.shape[0] == wl.window_rows
     assert np.array_equal(res["k_bits_new"], st["k_bits"][res["src"]])
     assert res["keep"].sum() == 32
+
+
+# --------------------------------------------------------------------------- variants
+
+def test_gqa_max_closed_form_two_heads_two_dominant_keys():
+    """Head 0 looks only at key 0, head 1 only at key 1 (logit gap 400/sqrt(d)): the mean over the
+    2*W rows gives each key 1/2, the max over heads gives each key 1, every other key ~0."""
+    d, W, N = 128, 3, 6
+    k = np.zeros((N, d))
+    k[0, 0] = 20.0
+    k[1, 1] = 20.0
+    q = np.zeros((2 * W, d))
+    q[:W, 0] = 20.0        # head 0's W window queries
+    q[W:, 1] = 20.0        # head 1's
+    mean = O.window_attention_score(q, k, 2, "mean")
+    mx = O.window_attention_score(q, k, 2, "max")
+    assert np.allclose(mean[:2], 0.5, atol=1e-12) and np.allclose(mean[2:], 0.0, atol=1e-12)
+    assert np.allclose(mx[:2], 1.0, atol=1e-12) and np.allclose(mx[2:], 0.0, atol=1e-12)
+
+
+def test_gqa_max_reductions_and_bounds():
+    rng = np.random.default_rng(11)
+    d, W, N, G = 128, 4, 30, 3
+    k = rng.standard_normal((N, d))
+    q = rng.standard_normal((G * W, d))
+    mean = O.window_attention_score(q, k, G, "mean")
+    mx = O.window_attention_score(q, k, G, "max")
+    # one head: max over one head is that head's mean
+    assert np.allclose(O.window_attention_score(q[:W], k, 1, "max"), O.window_attention_score(q[:W], k))
+    # identical heads: max == mean
+    qs = np.tile(q[:W], (G, 1))
+    assert np.allclose(O.window_attention_score(qs, k, G, "max"), O.window_attention_score(qs, k, G, "mean"))
+    # mean <= max <= G * mean, and the max is a distribution over keys for no head but sums to >= 1
+    assert np.all(mx >= mean - 1e-15) and np.all(mx <= G * mean + 1e-15)
+    assert mx.sum() >= 1.0 - 1e-12
+    # the heads are the head-major row blocks: swapping two heads' row blocks leaves the max unchanged,
+    # swapping two rows across heads does not
+    sw = np.concatenate([q[W:2 * W], q[:W], q[2 * W:]])
+    assert np.allclose(O.window_attention_score(sw, k, G, "max"), mx)
+    cross = q.copy()
+    cross[[0, W]] = cross[[W, 0]]
+    assert not np.allclose(O.window_attention_score(cross, k, G, "max"), mx)
+
+
+def test_random_reservation_is_uniform_and_ignores_values():
+    K, B, nv = 16, 4, 4
+    counts = np.zeros(K)
+    rounds = 3000
+    q, k, v, pos = _tiny_unit(5, K + B, K)
+    for t in range(rounds):
+        res = O.evict_unit(q, k, v, pos, budget_k=K, buffer_b=B, n_v=nv, reserve="random", pool_kernel=1,
+                           seed=9, rnd=t)
+        assert res["keep"].sum() == K and res["keep"][K:].all() and len(res["reserved_v"]) == nv
+        counts[res["reserved_v"]] += 1
+        if t < 20:   # R_V depends on the noise key and the positions only, not on the values
+            v2 = v[::-1].copy()
+            res2 = O.evict_unit(q, k, v2, pos, budget_k=K, buffer_b=B, n_v=nv, reserve="random", pool_kernel=1,
+                                seed=9, rnd=t)
+            assert np.array_equal(res["reserved_v"], res2["reserved_v"])
+    # every candidate is reserved with probability N_v / K
+    expect = rounds * nv / K
+    chi2 = ((counts - expect) ** 2 / expect).sum()
+    assert scipy.stats.chi2.sf(chi2, K - 1) > 1e-4
+    u = O.reservation_uniforms(1, 2, 3, 4, 8, 5, np.arange(64))
+    assert not np.array_equal(u, O.selection_uniforms(1, 2, 3, 4, 8, 5, np.arange(64)))  # its own stream
+
+
+def test_shared_g_is_one_projection_per_round():
+    a = O.gaussian_projection(1, 2, 3, 4, 8, 7, 128, 20, shared_g=True)
+    b = O.gaussian_projection(1, 5, 0, 6, 8, 7, 128, 20, shared_g=True)
+    c = O.gaussian_projection(1, 5, 0, 6, 8, 8, 128, 20, shared_g=True)
+    d = O.gaussian_projection(1, 2, 3, 4, 8, 7, 128, 20, shared_g=False)
+    e = O.gaussian_projection(1, 5, 0, 6, 8, 7, 128, 20, shared_g=False)
+    assert np.array_equal(a, b)             # every layer and unit of a round
+    assert not np.allclose(b, c)            # redrawn per round
+    assert not np.allclose(d, e)            # per unit without the option
+    f = O.gaussian_projection(1, 2, 3, 4, 8, 9, 128, 20, fixed_g=True, shared_g=True)
+    g = O.gaussian_projection(1, 0, 0, 0, 8, 0, 128, 20)
+    assert np.array_equal(f, g)             # fixed and shared: the unit-0 projection of round 0

@@ -48,6 +48,11 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="qwen3_1p7b_k2048")
     ap.add_argument("--variant", choices=["attnv", "dkv"], default="attnv")
+    ap.add_argument("--reserve", choices=["value", "random"], default="value",
+                    help="AttnV R_V: largest value magnitude (Sec. 3.1) or uniformly random (App. C ablation)")
+    ap.add_argument("--gqa", choices=["mean", "max"], default="mean",
+                    help="AttnV: combine the G query heads' window scores by mean or by max")
+    ap.add_argument("--dkv-shared-g", action="store_true", help="DKV: one projection per round for every unit")
     ap.add_argument("--layers", type=int, default=None, help="run only this many layers of the workload")
     ap.add_argument("--e2e-steps", type=int, default=None, help="steps of the host-buffer end-to-end pass")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
@@ -295,7 +300,8 @@ def run_ours(args):
 
     L, K, Bf = wl.num_layers, wl.budget_k, wl.buffer_b
     cache = V.VaseCache(V.Geometry(K, Bf, wl.window, wl.num_q_heads, wl.num_kv_heads, L, wl.batch),
-                        variant=args.variant, seed=0, device=device)
+                        variant=args.variant, seed=0, device=device, reserve=args.reserve, gqa=args.gqa,
+                        dkv_shared_g=args.dkv_shared_g)
     gen = torch.Generator(device=device)
     gen.manual_seed(1000 + rank)
     # prefill: the first K tokens of every layer (untimed)
@@ -439,7 +445,8 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": wl.name, "variant": args.variant, "layers": L, "global_batch": wl.batch * world,
+        "config": {"workload": wl.name, "variant": args.variant, **variant_options(args), "layers": L,
+                   "global_batch": wl.batch * world,
                    "seq_len": wl.slots, "budget_k": K, "buffer_b": Bf, "window": wl.window,
                    "heads": f"{wl.num_q_heads}/{wl.num_kv_heads}", "parallelism": f"dp{world}",
                    "l2": "inputs larger than L2 (about 3.9 GB touched per step)"},
@@ -563,6 +570,18 @@ def run_decode(args):
     }
     print(json.dumps(outj))
     return 0
+
+
+def variant_options(args):
+    """The non-default variant switches of a run, for the config object of its JSON line."""
+    opts = {}
+    if args.reserve != "value":
+        opts["reserve"] = args.reserve
+    if args.gqa != "mean":
+        opts["gqa"] = args.gqa
+    if args.dkv_shared_g:
+        opts["dkv_shared_g"] = True
+    return opts
 
 
 def main():

@@ -55,6 +55,12 @@ extern "C" {
 #define VASE_VALUE_L2 1           /* App. A: ||v||_2 */
 #define VASE_VALUE_VAR 2          /* App. A: (1/d) sum_j (v_j - mean)^2 */
 
+#define VASE_RESERVE_VALUE 0      /* R_V = the N_v candidates of largest value magnitude (Sec. 3.1) */
+#define VASE_RESERVE_RANDOM 1     /* R_V = N_v candidates drawn uniformly at random (the ablation of App. C) */
+
+#define VASE_GQA_MEAN 0           /* window score of a KV head: mean over its G query heads' G*W window rows */
+#define VASE_GQA_MAX 1            /* ... the largest over its G query heads of each head's mean over W rows */
+
 typedef struct vase_config {
     int32_t budget_k;      /* K: persistent budget (Sec. 2) */
     int32_t buffer_b;      /* B: recency buffer, always kept (Sec. 2) */
@@ -73,6 +79,9 @@ typedef struct vase_config {
     int32_t dkv_fixed_g;   /* DKV: 1 = one G for the whole stream (CurDKV), 0 = G_t redrawn per round (VaSE-DKV) */
     int32_t debug_outputs; /* 1 = also write pooled scores, selection keys and the keep mask to the workspace */
     uint64_t seed;         /* key of the Philox4x32-10 noise stream */
+    int32_t reserve_kind;  /* AttnV: VASE_RESERVE_* (how R_V is chosen) */
+    int32_t gqa_reduce;    /* AttnV: VASE_GQA_*; VASE_GQA_MAX needs W % 4 == 0 and, when G*W > 256, 256 % W == 0 */
+    int32_t dkv_shared_g;  /* DKV: 1 = one G per round shared by every layer, sequence and KV head; 0 = per unit */
 } vase_config;
 
 /* Sizes in bytes of the caller-allocated device buffers for a configuration. */

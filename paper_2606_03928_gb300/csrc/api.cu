@@ -59,6 +59,10 @@ const char* check_config(const vase_config* c) {
     if (c->dkv_rank < 1 || c->dkv_rank > 32) return "dkv_rank must be in 1..32";
     const int nv = c->n_v < 0 ? c->budget_k / 4 : c->n_v;
     if (c->variant == VASE_VARIANT_ATTNV && nv + c->buffer_b > c->budget_k) return "n_v + buffer_b must not exceed budget_k";
+    if (c->reserve_kind != VASE_RESERVE_VALUE && c->reserve_kind != VASE_RESERVE_RANDOM) return "unknown reserve_kind";
+    if (c->gqa_reduce != VASE_GQA_MEAN && c->gqa_reduce != VASE_GQA_MAX) return "unknown gqa_reduce";
+    if (c->dkv_shared_g != 0 && c->dkv_shared_g != 1) return "dkv_shared_g must be 0 or 1";
+    if (c->gqa_reduce == VASE_GQA_MAX && c->window % 4) return "GQA max-aggregation needs window % 4 == 0";
     return nullptr;
 }
 
@@ -85,6 +89,10 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     p.GWp = p.GW <= 256 ? (p.GW + 31) / 32 * 32 : (p.GW + 255) / 256 * 256;
     p.NB = p.GWp < 256 ? p.GWp : 256;
     p.n_rb = p.GWp / p.NB;
+    if (c->gqa_reduce == VASE_GQA_MAX && p.n_rb > 1 && p.NB % c->window) {
+        *why = "GQA max-aggregation with G * window > 256 needs window to divide 256";
+        return false;
+    }
     if (p.GWp <= 64) {  // replicate short windows across the 128 pass-A lanes
         p.rep = 128 / p.GWp;
         p.n_rbA = 1;
@@ -262,6 +270,8 @@ ScoreAttnParams score_params(const Plan& P, const vase_config& c, const LayerBat
     sp.q_layer_rows = static_cast<int64_t>(c.batch) * c.num_q_heads * c.window;
     sp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
     sp.inv_gw = 1.0f / static_cast<float>(P.GW);
+    sp.head_rows = c.gqa_reduce == VASE_GQA_MAX ? c.window : 0;
+    sp.fold_rows = c.gqa_reduce == VASE_GQA_MAX ? c.window : P.GW;
     sp.attn = attn;
     sp.err = err;
     return sp;
@@ -564,6 +574,7 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
         dp.r = c.dkv_rank;
         dp.Hkv = c.num_kv_heads;
         dp.fixed_g = c.dkv_fixed_g;
+        dp.shared_g = c.dkv_shared_g;
         dp.units = P.units;
         dp.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
         dp.seed_hi = static_cast<uint32_t>(c.seed >> 32);
@@ -603,6 +614,8 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     sel.Hkv = c.num_kv_heads;
     sel.n_parts = c.variant == VASE_VARIANT_ATTNV ? P.n_rb : 1;
     sel.staged = P.select_staged ? 1 : 0;
+    sel.reserve_random = c.reserve_kind == VASE_RESERVE_RANDOM ? 1 : 0;
+    sel.gqa_max = c.gqa_reduce == VASE_GQA_MAX ? 1 : 0;
     sel.units = P.units;
     sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
     sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
@@ -1007,6 +1020,7 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
         dp.r = c.dkv_rank;
         dp.Hkv = c.num_kv_heads;
         dp.fixed_g = c.dkv_fixed_g;
+        dp.shared_g = c.dkv_shared_g;
         dp.units = P.units;
         dp.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
         dp.seed_hi = static_cast<uint32_t>(c.seed >> 32);
@@ -1045,6 +1059,8 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
     sel.Hkv = c.num_kv_heads;
     sel.n_parts = c.variant == VASE_VARIANT_ATTNV ? P.n_rb : 1;
     sel.staged = P.select_staged ? 1 : 0;
+    sel.reserve_random = c.reserve_kind == VASE_RESERVE_RANDOM ? 1 : 0;
+    sel.gqa_max = c.gqa_reduce == VASE_GQA_MAX ? 1 : 0;
     sel.units = P.units;
     sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
     sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);

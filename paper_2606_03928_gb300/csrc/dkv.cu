@@ -125,8 +125,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int r = p.r;
         const float inv_sqrt_r = 1.0f / sqrtf(static_cast<float>(r));
         const uint32_t c1 = static_cast<uint32_t>(rnd);
-        const uint32_t c2 = static_cast<uint32_t>(layer) | (kTagDkv << 24);
-        const uint32_t c3 = static_cast<uint32_t>(unit);
+        // shared G: one projection per round for every layer and unit (0 in the layer bits and the unit word)
+        const uint32_t c2 = static_cast<uint32_t>(p.shared_g ? 0 : layer) | (kTagDkv << 24);
+        const uint32_t c3 = static_cast<uint32_t>(p.shared_g ? 0 : unit);
         for (int idx = tid; idx < kHeadDim * 32; idx += kThreads) {
             const int a = idx >> 5;
             const int b = idx & 31;

@@ -63,6 +63,7 @@ __device__ __forceinline__ float open_uniform(uint32_t x) {
 
 constexpr uint32_t kTagSelect = 0u;
 constexpr uint32_t kTagDkv = 1u;
+constexpr uint32_t kTagReserve = 2u;
 
 // ------------------------------------------------------------------ parameter blocks
 
@@ -117,6 +118,8 @@ struct ScoreAttnParams {
     int32_t Hq, Hkv, W, G;
     int64_t layer_rows;     // cache rows per layer (units * N)
     int64_t q_layer_rows;   // window rows per layer (b * Hq * W)
+    int32_t head_rows;      // 0: the score sums all G*W window rows; W: per query head, the largest head sum
+    int32_t fold_rows;      // rows the score averages over: G*W (mean over the heads) or W (max over the heads)
     float scale_log2;       // log2(e) / sqrt(d)
     float inv_gw;           // 1 / (G * W)
     float* attn;            // [slot][n_rb][units][N] (one part per row block)
@@ -132,6 +135,7 @@ struct ValueParams {
 struct DkvParams {
     LayerBatch batch;
     int32_t N, K, r, Hkv, fixed_g, units;
+    int32_t shared_g;       // 1: one G per round for every layer and unit (counter without layer and unit)
     uint32_t seed_lo, seed_hi;
     int32_t n_tiles_k;      // ceil(K / 128)
     int32_t tiles_per_cta;
@@ -156,6 +160,8 @@ struct SelectParams {
     uint8_t* keep_dbg;      // nullable
     int32_t N, K, B, n_v, m, pool, variant, stochastic, Hkv, n_parts, units;
     int32_t staged;         // 1: every input array of the unit is copied to shared memory up front
+    int32_t reserve_random; // 1: R_V = the N_v largest reservation uniforms (App. C ablation) instead of value magnitudes
+    int32_t gqa_max;        // 1: the parts of the window score combine by max (GQA max-aggregation), 0: by sum
     uint32_t seed_lo, seed_hi;
     uint32_t* err;
 };

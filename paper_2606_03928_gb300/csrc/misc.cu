@@ -472,15 +472,18 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
             if (p.n_parts > 1) {
                 for (int i = tid; i < N; i += kSelThreads) {
                     float a = a_s[i];
-                    for (int part = 1; part < p.n_parts; ++part) a += a_s[part * N + i];
+                    for (int part = 1; part < p.n_parts; ++part)
+                        a = p.gqa_max ? fmaxf(a, a_s[part * N + i]) : a + a_s[part * N + i];
                     a_s[i] = a;
                 }
             }
         } else {
             for (int i = tid; i < N; i += kSelThreads) {
                 float a = attn[base + i];
-                for (int part = 1; part < p.n_parts; ++part)
-                    a += attn[(static_cast<int64_t>(part) * p.units + unit) * N + i];
+                for (int part = 1; part < p.n_parts; ++part) {
+                    const float b = attn[(static_cast<int64_t>(part) * p.units + unit) * N + i];
+                    a = p.gqa_max ? fmaxf(a, b) : a + b;
+                }
                 a_s[i] = a;
             }
         }
@@ -488,9 +491,18 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
             __syncthreads();
             for (int i = tid; i < N; i += kSelThreads) const_cast<float*>(attn)[base + i] = a_s[i];
         }
+        const uint32_t c2_res = static_cast<uint32_t>(layer) | (kTagReserve << 24);
         for (int i = tid; i < K; i += kSelThreads) {
             const float vm = staged ? vm_s[i] : vmag[base + i];
-            ord[i] = __float_as_uint(vm) + 1u;
+            if (p.reserve_random) {  // the N_v largest reservation uniforms: a uniformly random N_v-subset
+                const int32_t pi = staged ? pos_s[i] : pos[base + i];
+                const Philox4 w = philox4x32_10(
+                    Philox4{static_cast<uint32_t>(pi), static_cast<uint32_t>(rnd), c2_res, static_cast<uint32_t>(unit)},
+                    p.seed_lo, p.seed_hi);
+                ord[i] = (w.x >> 9) + 1u;
+            } else {
+                ord[i] = __float_as_uint(vm) + 1u;
+            }
             if (vscore_dbg) vscore_dbg[base + i] = vm;
         }
         __syncthreads();

@@ -133,6 +133,9 @@ __device__ __forceinline__ bool phase_tile(int t, int nA, int nB, int lead, int&
     return true;
 }
 
+// kHeadMax: GQA max-aggregation (per-head sums in pass B, the largest kept); a template argument so that the
+// default mean keeps its pass-B loop free of the head bookkeeping.
+template <bool kHeadMax>
 __global__ void __launch_bounds__(kThreads, 1)
     score_attn_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
                       const ScoreAttnParams p) {
@@ -167,6 +170,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int n_w = group < p.work ? (p.work - group + p.groups - 1) / p.groups : 0;
     const int GWp = p.GWp;
     const int NB = p.NB;
+    const int head_rows = p.head_rows;  // W when kHeadMax: rows per query head
     const int n_rb = p.n_rb;
     const int n_rbA = p.n_rbA;
     const int R = p.rep;                 // copies of the window rows across the 128 pass-A lanes
@@ -517,6 +521,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (j == nB - 1 && k + 1 < n_w) mbar_arrive(&q_empty[2 * ((k - 1) & (p.q_bufs - 1)) + grp]);
                         }
                         tc_fence_after();
+                        // GQA max-aggregation: the sum runs per query head (W consecutive window rows, whole
+                        // heads per row block) and the token keeps the largest head sum
+                        float head_sum = 0.f;
+                        int head_end = kHeadMax ? sub * NB + head_rows : 0;
                         for (int c = 0; c < NB; c += 64) {
                             float v[64];
                             const int width = NB - c >= 64 ? 64 : 32;
@@ -529,19 +537,36 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 for (int q = 0; q < 32; ++q) v[q] = h[q];
                             }
                             const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
-                            float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+                            if (!kHeadMax) {
+                                float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
-                            for (int q = 0; q < 16; ++q) {
-                                if (q < width / 4) {
-                                    const float4 mm = m4[q];
-                                    a0 += ex2(fmaf(v[4 * q], cs, -mm.x));
-                                    a1 += ex2(fmaf(v[4 * q + 1], cs, -mm.y));
-                                    a2 += ex2(fmaf(v[4 * q + 2], cs, -mm.z));
-                                    a3 += ex2(fmaf(v[4 * q + 3], cs, -mm.w));
+                                for (int q = 0; q < 16; ++q) {
+                                    if (q < width / 4) {
+                                        const float4 mm = m4[q];
+                                        a0 += ex2(fmaf(v[4 * q], cs, -mm.x));
+                                        a1 += ex2(fmaf(v[4 * q + 1], cs, -mm.y));
+                                        a2 += ex2(fmaf(v[4 * q + 2], cs, -mm.z));
+                                        a3 += ex2(fmaf(v[4 * q + 3], cs, -mm.w));
+                                    }
+                                }
+                                acc += (a0 + a1) + (a2 + a3);
+                            } else {
+#pragma unroll
+                                for (int q = 0; q < 16; ++q) {
+                                    if (q < width / 4) {
+                                        if (sub * NB + c + 4 * q == head_end) {  // the same in every thread
+                                            acc = fmaxf(acc, head_sum);
+                                            head_sum = 0.f;
+                                            head_end += head_rows;
+                                        }
+                                        const float4 mm = m4[q];
+                                        head_sum += (ex2(fmaf(v[4 * q], cs, -mm.x)) + ex2(fmaf(v[4 * q + 1], cs, -mm.y))) +
+                                                    (ex2(fmaf(v[4 * q + 2], cs, -mm.z)) + ex2(fmaf(v[4 * q + 3], cs, -mm.w)));
+                                    }
                                 }
                             }
-                            acc += (a0 + a1) + (a2 + a3);
                         }
+                        if (kHeadMax) acc = fmaxf(acc, head_sum);
                         tc_fence_before();
                         mbar_arrive(&t_empty[buf]);
                     }
@@ -577,7 +602,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 } else {
                     const bool real = r < p.GW;
-                    rowm[r] = real ? m + log2f(l * static_cast<float>(p.GW)) : INFINITY;
+                    rowm[r] = real ? m + log2f(l * static_cast<float>(p.fold_rows)) : INFINITY;
                 }
             }
             if (C > 1) {
@@ -587,7 +612,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     float m = -INFINITY, l = 0.f;
                     for (int c = 0; c < C; ++c) merge_ml(m, l, xm[c * GWp + r], xl[c * GWp + r]);
                     const bool real = r < p.GW;
-                    rowm[r] = real ? m + log2f(l * static_cast<float>(p.GW)) : INFINITY;
+                    rowm[r] = real ? m + log2f(l * static_cast<float>(p.fold_rows)) : INFINITY;
                 }
             }
             named_bar(1, kConsumers);
@@ -612,11 +637,13 @@ size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int clu
 }
 
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster) {
-    cudaError_t e = cudaFuncSetAttribute(score_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem_bytes));
-    if (e != cudaSuccess) return e;
-    if (cluster > 8) e = cudaFuncSetAttribute(score_attn_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    return e;
+    for (auto fn : {score_attn_kernel<false>, score_attn_kernel<true>}) {
+        cudaError_t e =
+            cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem_bytes));
+        if (e == cudaSuccess && cluster > 8) e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, const ScoreAttnParams& p,
@@ -633,7 +660,8 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, score_attn_kernel, kmap, qmap, p);
+    return p.head_rows > 0 ? cudaLaunchKernelEx(&cfg, score_attn_kernel<true>, kmap, qmap, p)
+                           : cudaLaunchKernelEx(&cfg, score_attn_kernel<false>, kmap, qmap, p);
 }
 
 }  // namespace vase

@@ -30,6 +30,8 @@ VASE_ERR_DEVICE = -7
 VASE_VARIANT_ATTNV = 0
 VASE_VARIANT_DKV = 1
 VASE_VALUE_RANGE, VASE_VALUE_L2, VASE_VALUE_VAR = 0, 1, 2
+VASE_RESERVE_VALUE, VASE_RESERVE_RANDOM = 0, 1
+VASE_GQA_MEAN, VASE_GQA_MAX = 0, 1
 
 EXPORTED = [
     "vase_config_default", "vase_get_buffer_sizes", "vase_create", "vase_destroy", "vase_append",
@@ -46,7 +48,7 @@ class vase_config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "budget_k", "buffer_b", "window", "num_q_heads", "num_kv_heads", "head_dim", "num_layers", "batch",
         "variant", "n_v", "value_score", "pool_kernel", "dkv_rank", "stochastic", "dkv_fixed_g", "debug_outputs")] + [
-        ("seed", ctypes.c_uint64)]
+        ("seed", ctypes.c_uint64)] + [(n, ctypes.c_int32) for n in ("reserve_kind", "gqa_reduce", "dkv_shared_g")]
 
 
 class vase_buffer_sizes(ctypes.Structure):
@@ -275,7 +277,7 @@ class VaseCache:
 
     def __init__(self, geometry: Geometry, *, variant="attnv", n_v=-1, value_score=VASE_VALUE_RANGE,
                  pool_kernel=7, dkv_rank=20, stochastic=True, dkv_fixed_g=False, debug_outputs=False, seed=0,
-                 device=None):
+                 reserve="value", gqa="mean", dkv_shared_g=False, device=None):
         g = geometry
         self.geometry = g
         self.cfg = vase_config_default(
@@ -283,7 +285,9 @@ class VaseCache:
             num_kv_heads=g.num_kv_heads, head_dim=g.head_dim, num_layers=g.num_layers, batch=g.batch,
             variant=VASE_VARIANT_ATTNV if variant == "attnv" else VASE_VARIANT_DKV, n_v=n_v,
             value_score=value_score, pool_kernel=pool_kernel, dkv_rank=dkv_rank, stochastic=int(stochastic),
-            dkv_fixed_g=int(dkv_fixed_g), debug_outputs=int(debug_outputs), seed=seed)
+            dkv_fixed_g=int(dkv_fixed_g), debug_outputs=int(debug_outputs), seed=seed,
+            reserve_kind={"value": VASE_RESERVE_VALUE, "random": VASE_RESERVE_RANDOM}[reserve],
+            gqa_reduce={"mean": VASE_GQA_MEAN, "max": VASE_GQA_MAX}[gqa], dkv_shared_g=int(dkv_shared_g))
         sizes = vase_get_buffer_sizes(self.cfg)
         dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
         self.device = dev

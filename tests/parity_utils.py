@@ -66,7 +66,7 @@ def oracle_unit(wl, st, s, h, *, variant, round_index, seed, layer, **kw):
     q = st["q_bits"][s, h * G:(h + 1) * G].reshape(-1, wl.head_dim)
     return O.evict_unit_bits(q, st["k_bits"][s, h], st["v_bits"][s, h], st["positions"][s, h],
                              budget_k=wl.budget_k, buffer_b=wl.buffer_b, variant=variant, seed=seed, layer=layer,
-                             seq=s, head=h, num_kv_heads=wl.num_kv_heads, rnd=round_index, **kw)
+                             seq=s, head=h, num_kv_heads=wl.num_kv_heads, rnd=round_index, group=G, **kw)
 
 
 def assert_close_scores(gpu, ref, what, rtol=SCORE_RTOL, atol=SCORE_ATOL):

@@ -472,3 +472,96 @@ def test_qwen3_1p7b_k2048_all_layers_in_one_launch():
                 gu["attn"] = gu["pooled"] = gu["key"] = gu["value_score"] = None
                 PU.check_unit(wl, ref, gu, st["k_bits"][s, h], st["v_bits"][s, h], st["positions"][s, h],
                               variant="attnv", n_v=wl.budget_k // 4, check_scores=False)
+
+
+# ----------------------------------------------------------------------------- variants
+
+def _reserved_slots(key_row, K):
+    """R_V of a unit from the debug keys: the candidates' keys are >= 0, the reserved slots carry -1."""
+    return np.flatnonzero(np.asarray(key_row[:K]) < 0)
+
+
+@pytest.mark.parametrize("stochastic", [True, False])
+def test_random_reservation_matches_oracle_exactly(stochastic):
+    kw = {"reserve": "random", "stochastic": stochastic}
+    cache, st, got, _ = _run_layer(SMALL, cache_kw=kw, oracle_kw=kw)
+    K = SMALL.budget_k
+    for s in range(SMALL.batch):
+        for h in range(SMALL.num_kv_heads):
+            ref = PU.oracle_unit(SMALL, st, s, h, variant="attnv", round_index=3, seed=0, layer=1, **kw)
+            gu = PU.unit_slice(got, s, h, SMALL.num_kv_heads)
+            # an integer decision on the same 23-bit uniforms on both sides: identical reserved sets
+            assert np.array_equal(_reserved_slots(gu["key"], K), ref["reserved_v"])
+
+
+def test_random_reservation_differs_from_value_reservation():
+    a = _run_layer(SMALL)[2]["key"]
+    b = _run_layer(SMALL, cache_kw={"reserve": "random"}, oracle_kw={"reserve": "random"})[2]["key"]
+    assert not np.array_equal(a < 0, b < 0)
+
+
+# (K, B, W, Hq, Hkv): heads of 16 rows four to a 64-column chunk; 12-row heads that straddle chunks and a
+# padded tail; G*W = 512 in two 256-row blocks (parts combined by max); one query head per KV head
+@pytest.mark.parametrize("K,B,Wn,Hq,Hkv", [(256, 64, 16, 32, 8), (200, 40, 12, 24, 8), (256, 64, 64, 32, 4),
+                                          (192, 64, 32, 8, 8)])
+def test_gqa_max_aggregation_matches_oracle(K, B, Wn, Hq, Hkv):
+    wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=Wn, num_q_heads=Hq, num_kv_heads=Hkv, batch=2,
+                  num_layers=2)
+    _run_layer(wl, cache_kw={"gqa": "max"}, oracle_kw={"gqa": "max"})
+
+
+def test_gqa_max_in_the_persistent_schedule():
+    """Eight layers of 64 units (one CTA per SM takes a strided list of units), max over the query heads."""
+    wl = W.shrink(SMALL, budget_k=192, buffer_b=64, window=16, num_q_heads=32, num_kv_heads=8, batch=8,
+                  num_layers=8)
+    cache = _cache(wl, 8, gqa="max")
+    states = [W.layer_state(wl, 12, layer, 2 + layer, "gapped") for layer in range(8)]
+    for layer, st in enumerate(states):
+        PU.upload_layer(cache, layer, st, 2 + layer)
+    assert cache.evict_all() == 8
+    status, code = cache.check_device_error()
+    assert status == 0, f"device error word {code:#x}"
+    for z in range(8):
+        dv = {k: (v.cpu().numpy() if k != "layer" else v) for k, v in cache.debug_view(z).items()}
+        layer = dv["layer"]
+        st = states[layer]
+        got = PU.download(cache, layer)
+        got.update({k: v for k, v in dv.items() if k != "layer"})
+        for s in range(wl.batch):
+            for h in range(wl.num_kv_heads):
+                ref = PU.oracle_unit(wl, st, s, h, variant="attnv", round_index=2 + layer, seed=0, layer=layer,
+                                     gqa="max")
+                PU.check_unit(wl, ref, PU.unit_slice(got, s, h, wl.num_kv_heads), st["k_bits"][s, h],
+                              st["v_bits"][s, h], st["positions"][s, h], variant="attnv", n_v=wl.budget_k // 4)
+
+
+def test_gqa_max_rejects_windows_that_split_a_row_block():
+    from paper_2606_03928_gb300.vase import VaseError
+    wl = W.shrink(SMALL, budget_k=256, buffer_b=64, window=48, num_q_heads=64, num_kv_heads=8, batch=1,
+                  num_layers=1)   # G*W = 384 > 256 and 48 does not divide 256
+    with pytest.raises(VaseError):
+        _cache(wl, 1, gqa="max")
+    wl2 = W.shrink(SMALL, budget_k=256, buffer_b=64, window=6, num_q_heads=16, num_kv_heads=8, batch=1,
+                   num_layers=1)  # W % 4 != 0
+    with pytest.raises(VaseError):
+        _cache(wl2, 1, gqa="max")
+
+
+def test_dkv_shared_g_matches_oracle_and_is_shared():
+    kw = {"dkv_shared_g": True}
+    _run_layer(SMALL, variant="dkv", cache_kw=kw, oracle_kw=kw)
+    # one projection for every unit of a round: two units holding identical rows score identically
+    wl = W.shrink(SMALL, batch=2, num_layers=1)
+    cache = _cache(wl, 1, variant="dkv", dkv_shared_g=True)
+    st = W.layer_state(wl, 3, 0, 0, "gapped")
+    for key in ("q_bits", "k_bits", "v_bits", "positions"):
+        st[key][1] = st[key][0]
+    PU.upload_layer(cache, 0, st, 0)
+    assert cache.evict(0) == 0
+    scores = cache.debug_view(0)["value_score"].cpu().numpy().reshape(wl.batch, wl.num_kv_heads, -1)
+    assert np.array_equal(scores[0], scores[1])
+    cache2 = _cache(wl, 1, variant="dkv")
+    PU.upload_layer(cache2, 0, st, 0)
+    assert cache2.evict(0) == 0
+    scores2 = cache2.debug_view(0)["value_score"].cpu().numpy().reshape(wl.batch, wl.num_kv_heads, -1)
+    assert not np.array_equal(scores2[0], scores2[1])

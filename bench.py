@@ -427,11 +427,11 @@ def run_ours(args):
     tpath = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tpath):
         try:
-            from paper_2606_03928_gb300.build import source_digest
+            from paper_2606_03928_gb300.build import kernel_digest
             with open(tpath) as f:
                 tr = json.load(f)
             ent = tr.get(f"{dom}:{wl.name}:{args.variant}:{L}")
-            if ent and ent.get("source_digest") == source_digest():
+            if ent and ent.get("kernel_digest") == kernel_digest(dom):
                 traffic = ent["bytes_per_launch"]
         except Exception:
             traffic = None

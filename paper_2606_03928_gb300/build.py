@@ -44,6 +44,26 @@ def source_digest():
     return h.hexdigest()
 
 
+# The source files each timed kernel is compiled from (its own translation unit and the headers it includes).
+KERNEL_SOURCES = {
+    "score_attn": ["score_attn.cu", "kernels.cuh", "ptx.cuh"],
+    "select_compact": ["misc.cu", "kernels.cuh", "ptx.cuh"],
+    "append": ["misc.cu", "kernels.cuh", "ptx.cuh"],
+    "dkv_score": ["dkv.cu", "kernels.cuh", "ptx.cuh"],
+    "decode": ["decode.cu", "kernels.cuh", "ptx.cuh"],
+}
+
+
+def kernel_digest(kernel):
+    """Digest of the sources of one kernel: ncu counters taken on it stay valid while this is unchanged."""
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES[kernel]:
+        h.update(name.encode())
+        with open(os.path.join(CSRC, name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
 def _digest():
     h = hashlib.sha256()
     for name in sorted(os.listdir(CSRC)) + ["vase.h"]:

@@ -26,7 +26,12 @@ time, where a *unit* is one (layer, sequence, KV head):
 * variants: the random-reservation ablation (N_v candidates drawn uniformly
   at random instead of the largest Range) -- App. C, first paragraph; GQA
   max-aggregation over the query heads of a KV head; one Gaussian projection
-  per round shared by every unit (shared-G DKV).
+  per round shared by every unit (shared-G DKV);
+* per-token asymmetric b-bit quantization of value rows, z = min v,
+  s = Range(v) / (2^b - 1), Q(v) = round((v - z) / s), v' = Q s + z -- the
+  equation of Sec. 4.4 -- and the mixed-precision value cache that Sec. 6
+  proposes: the reserved large-Range values (R_V) and the recency buffer keep
+  their bf16 rows, every other kept value is read back from its b-bit codes.
 
 Readings where the paper is silent (each is listed with its reason in the
 design notes of the repository):
@@ -53,6 +58,13 @@ design notes of the repository):
   word 0 = a * r + b; the fixed-G (CurDKV) option puts 0 in the round word,
   and the shared-G option puts 0 in the layer bits and the unit word.
 * DKV has no value reservation; the value awareness is the value leverage.
+* Quantization codes are integers decided by floating point, so they are
+  computed in fp32 (the kernels' precision): v - z, the division by s and
+  the rounding (half to even) each in fp32.  A row of equal values has s = 0
+  and codes 0.  After an eviction the reserved (bf16) values are R_B, the
+  last B kept slots, and R_V, which is again the N_v largest value
+  magnitudes among the first K - B kept slots (R_V is kept whole and the
+  compaction keeps the order).
 """
 
 from __future__ import annotations
@@ -302,6 +314,49 @@ def decode_attention_bits(q_bits, k_bits, v_bits):
     """decode_attention on raw bf16 bit arrays; returns (output, its error scale)."""
     q, k, v = bf16_bits_to_f64(q_bits), bf16_bits_to_f64(k_bits), bf16_bits_to_f64(v_bits)
     return decode_attention(q, k, v), decode_attention_bound(q, k, v)
+
+
+# ----------------------------------------------------------------------------
+# Mixed-precision values (Sec. 4.4 equation, Sec. 6 proposal)
+# ----------------------------------------------------------------------------
+
+def quantize_values(values, bits):
+    """Per-token asymmetric b-bit quantization of value rows [n, d] (exact bf16 values), in fp32.
+
+    Returns codes [n, d] (uint8, 0 .. 2^b - 1), s [n] and z [n] (fp32)."""
+    v = np.asarray(values, dtype=np.float32)
+    lo = v.min(axis=1)
+    hi = v.max(axis=1)
+    levels = np.float32(2 ** int(bits) - 1)
+    s = ((hi - lo) / levels).astype(np.float32)
+    safe = np.where(s > 0, s, np.float32(1)).astype(np.float32)
+    t = ((v - lo[:, None]) / safe[:, None]).astype(np.float32)
+    codes = np.where(s[:, None] > 0, np.clip(np.rint(t), 0, levels), 0).astype(np.uint8)
+    return codes, s, lo.astype(np.float32)
+
+
+def dequantize_values(codes, s, z):
+    """v' = Q s + z (Sec. 4.4), in fp64 from the fp32 parameters."""
+    return np.asarray(codes, dtype=np.float64) * np.asarray(s, dtype=np.float64)[:, None] + \
+        np.asarray(z, dtype=np.float64)[:, None]
+
+
+def reserved_after_eviction(value_scores, budget_k, buffer_b, n_v):
+    """Mask [K] of the kept slots whose bf16 value rows stay after an eviction: R_B (the last B slots)
+    and R_V (the N_v largest value magnitudes among the first K - B kept slots; ties to the lower slot)."""
+    K, B = int(budget_k), int(buffer_b)
+    mask = np.zeros(K, dtype=bool)
+    mask[K - B:] = True
+    if n_v > 0:
+        mask[top_k_slots(np.asarray(value_scores)[:K - B], int(n_v))] = True
+    return mask
+
+
+def decode_attention_mixed(q, keys, values, reserved, bits):
+    """Decode attention where the values of unreserved slots are read back from their b-bit codes."""
+    codes, s, z = quantize_values(values, bits)
+    v_eff = np.where(np.asarray(reserved, dtype=bool)[:, None], values, dequantize_values(codes, s, z))
+    return decode_attention(q, keys, v_eff), decode_attention_bound(q, keys, v_eff)
 
 
 def evict_unit_bits(q_bits, k_bits, v_bits, positions, **kw):

@@ -491,3 +491,66 @@ def test_shared_g_is_one_projection_per_round():
     f = O.gaussian_projection(1, 2, 3, 4, 8, 9, 128, 20, fixed_g=True, shared_g=True)
     g = O.gaussian_projection(1, 0, 0, 0, 8, 0, 128, 20)
     assert np.array_equal(f, g)             # fixed and shared: the unit-0 projection of round 0
+
+
+# --------------------------------------------------------------------------- mixed-precision values (NEXT-4)
+
+def test_quantization_worked_example():
+    """v = (-1, 0, 0.5, 2) at 2 bits: z = -1, s = 3 / 3 = 1, (v - z) / s = (0, 1, 1.5, 3) -> (0, 1, 2, 3)
+    (1.5 rounds to the even 2), reconstructed (-1, 0, 1, 2)."""
+    codes, s, z = O.quantize_values(np.array([[-1.0, 0.0, 0.5, 2.0]]), 2)
+    assert codes.tolist() == [[0, 1, 2, 3]] and s.tolist() == [1.0] and z.tolist() == [-1.0]
+    assert O.dequantize_values(codes, s, z).tolist() == [[-1.0, 0.0, 1.0, 2.0]]
+
+
+@pytest.mark.parametrize("bits", [2, 4, 8])
+def test_quantization_bounds_and_extremes(bits):
+    rng = np.random.default_rng(bits)
+    v = O.bf16_bits_to_f64(W.f32_to_bf16_bits(rng.standard_normal((200, 128)).astype(np.float32)))
+    codes, s, z = O.quantize_values(v, bits)
+    assert codes.max() <= 2 ** bits - 1
+    vr = O.dequantize_values(codes, s, z)
+    # the step is s = Range / (2^b - 1): every value is within half a step (plus fp32 rounding)
+    assert np.all(np.abs(vr - v) <= s[:, None] * (0.5 + 1e-5) + 1e-6)
+    # the minimum maps to 0 and the maximum to the top code
+    assert np.all(codes[np.arange(200), v.argmin(axis=1)] == 0)
+    assert np.all(codes[np.arange(200), v.argmax(axis=1)] == 2 ** bits - 1)
+    assert np.allclose(s, (v.max(axis=1) - v.min(axis=1)) / (2 ** bits - 1), rtol=1e-6)
+
+
+def test_quantization_constant_row_and_error_grows_with_range():
+    codes, s, z = O.quantize_values(np.full((1, 16), 0.375), 4)
+    assert s[0] == 0.0 and not codes.any() and np.all(O.dequantize_values(codes, s, z) == 0.375)
+    # Sec. 4.4: the error scales with Range(v): scaling a row by 4 (exact) keeps its codes and multiplies
+    # the mean squared reconstruction error by exactly 16
+    rng = np.random.default_rng(3)
+    v = rng.standard_normal((50, 128)).astype(np.float32).astype(np.float64)
+    c1, s1, z1 = O.quantize_values(v, 4)
+    c4, s4, z4 = O.quantize_values(4 * v, 4)
+    assert np.array_equal(c1, c4)
+    mse1 = ((O.dequantize_values(c1, s1, z1) - v) ** 2).mean()
+    mse4 = ((O.dequantize_values(c4, s4, z4) - 4 * v) ** 2).mean()
+    assert mse4 == pytest.approx(16 * mse1, rel=1e-9)
+
+
+def test_reserved_set_after_eviction_is_r_v_and_r_b():
+    for seed in range(20):
+        K, B, nv = 12, 3, 3
+        q, k, v, pos = _tiny_unit(seed, K + B, K)
+        res = O.evict_unit(q, k, v, pos, budget_k=K, buffer_b=B, n_v=nv, pool_kernel=3, seed=seed, rnd=seed)
+        vm_kept = O.value_magnitude(res["values_new"])
+        mask = O.reserved_after_eviction(vm_kept, K, B, nv)
+        expect = np.isin(res["src"], np.concatenate([res["reserved_v"], np.arange(K, K + B)]))
+        assert np.array_equal(mask, expect)
+
+
+def test_mixed_decode_reductions():
+    rng = np.random.default_rng(8)
+    q = rng.standard_normal((2, 128))
+    k = rng.standard_normal((40, 128))
+    v = rng.standard_normal((40, 128)).astype(np.float32).astype(np.float64)
+    full, _ = O.decode_attention_mixed(q, k, v, np.ones(40, bool), 4)
+    assert np.allclose(full, O.decode_attention(q, k, v), rtol=0, atol=0)
+    approx, _ = O.decode_attention_mixed(q, k, v, np.zeros(40, bool), 8)
+    _, s, _ = O.quantize_values(v, 8)
+    assert np.max(np.abs(approx - O.decode_attention(q, k, v))) <= s.max() / 2 * (1 + 1e-6)

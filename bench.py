@@ -53,6 +53,8 @@ def parse_args():
     ap.add_argument("--gqa", choices=["mean", "max"], default="mean",
                     help="AttnV: combine the G query heads' window scores by mean or by max")
     ap.add_argument("--dkv-shared-g", action="store_true", help="DKV: one projection per round for every unit")
+    ap.add_argument("--mixed-bits", type=int, default=0, choices=[0, 2, 4, 8],
+                    help="with --decode: read the unreserved values from b-bit codes (Sec. 4.4 / Sec. 6)")
     ap.add_argument("--layers", type=int, default=None, help="run only this many layers of the workload")
     ap.add_argument("--e2e-steps", type=int, default=None, help="steps of the host-buffer end-to-end pass")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
@@ -497,12 +499,26 @@ def run_decode(args):
     cache.evict_all()  # every layer now holds its K kept pairs
     q = torch.randn((L, wl.batch, wl.num_q_heads, wl.head_dim), generator=gen, device=device).to(torch.bfloat16)
     out = torch.empty((L, wl.batch, wl.num_q_heads, wl.head_dim), dtype=torch.float32, device=device)
+    bits = args.mixed_bits
+    mixed = []
+    if bits:  # codes of every layer's unreserved kept values (untimed: once per eviction round)
+        for layer in range(L):
+            mb, t = cache.mixed_buffers(bits)
+            cache.quantize_values(layer, bits, mb)
+            mixed.append((mb, t))
+        torch.cuda.synchronize()
+        reserved = sum(int(((t["rmask"] >> i) & 1).sum()) for _, t in mixed for i in range(32))  # bf16 slots
 
     # device pointers computed once: the step is 28 C calls, not 28 tensor views
     ptrs = [(q[layer].data_ptr(), out[layer].data_ptr()) for layer in range(L)]
     stream_handle = torch.cuda.current_stream()
 
     def step():
+        if bits:
+            for layer in range(L):
+                V.vase_decode_attention_mixed(cache.ctx, layer, bits, mixed[layer][0], ptrs[layer][0], ptrs[layer][1],
+                                              stream_handle)
+            return
         for layer in range(L):
             V.vase_decode_attention(cache.ctx, layer, ptrs[layer][0], ptrs[layer][1], stream_handle)
 
@@ -551,19 +567,29 @@ def run_decode(args):
     units = wl.batch * wl.num_kv_heads
     # K and V rows of the kept slots, the query rows in, the fp32 outputs out
     step_bytes_ = L * (units * K * 2 * 2 * wl.head_dim + wl.batch * wl.num_q_heads * wl.head_dim * (2 + 4))
+    mixed_info = None
+    if bits:
+        # b-bit values: K rows, bf16 V rows of the reserved slots, code rows and (s, z) of the others, the masks
+        coded = L * units * K - reserved
+        step_bytes_ = (L * units * K * 2 * wl.head_dim + reserved * 2 * wl.head_dim +
+                       coded * (wl.head_dim * bits // 8 + 8) + L * units * ((K + 31) // 32) * 4 +
+                       L * wl.batch * wl.num_q_heads * wl.head_dim * (2 + 4))
+        mixed_info = {"value_bits": bits, "reserved_fraction": round(reserved / (L * units * K), 4)}
     gbs = step_bytes_ / (ms / 1e3) / 1e9
     hbm_peak, _, peak_kind = measured_peaks()
     outj = {
-        "metric": "decode-step attention over the kept cache, bytes/s (K and V of every kept slot read once)",
+        "metric": ("decode-step attention over the kept cache, bytes/s (K and V of every kept slot read once)" if not bits
+                   else "decode-step attention over the kept cache with b-bit unreserved values, bytes/s (K rows, "
+                        "bf16 reserved V rows, codes and scales read once)"),
         "value": gbs, "unit": "GB/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
-        "config": {"workload": wl.name, "layers": L, "global_batch": wl.batch, "kept_slots": K,
+        "config": {"workload": wl.name, "layers": L, "global_batch": wl.batch, "kept_slots": K, **(mixed_info or {}),
                    "heads": f"{wl.num_q_heads}/{wl.num_kv_heads}", "parallelism": "dp1",
                    "l2": f"inputs larger than L2 ({step_bytes_ / 1e9:.2f} GB read per step)"},
         "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                      "frac": round(gbs / hbm_peak, 4), "traffic": None,
-                     "kernel": "decode_tc_kernel" if wl.group >= 3 else "decode_simt_kernel",
+                     "kernel": ("decode_simt_kernel" if bits or wl.group < 3 else "decode_tc_kernel"),
                      "algorithmic_bytes_per_launch": step_bytes_ // L, "peak_source": peak_kind},
         "clocks": clocks, "gpu_launches": launches, "timed_as": "CUDA graph replay of the step's launches",
         "eager_ms_per_step": eager_ms,

@@ -205,6 +205,36 @@ int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream);
  * VASE_ERR_UNSUPPORTED (more than 16 query heads per KV head). */
 int vase_decode_attention(vase_ctx* ctx, int32_t layer, const void* q, float* out, void* stream);
 
+/* ---- Mixed-precision values: the b-bit per-token quantizer of Sec. 4.4 and the reserved cache of Sec. 6.
+ * After an eviction the reserved values -- R_V (the N_v largest value magnitudes) and the recency buffer
+ * R_B -- keep their bf16 rows; every other kept value is read back from b-bit codes (b = 2, 4 or 8):
+ * z = min v, s = Range(v) / (2^b - 1), Q = round((v - z) / s) (half to even, decided in fp32),
+ * v' = Q s + z.  The bf16 cache stays the record the evictions work on; the codes serve the decode reads.
+ * The caller owns these buffers, one set per layer, all device memory: */
+typedef struct vase_mixed_buffers {
+    void* codes;      /* uint8 [b][Hkv][K][d * bits / 8]: lane-packed codes, dims 4i .. 4i+3 in 4*bits bits */
+    float* qparams;   /* fp32 [b][Hkv][Kp][2], Kp = K rounded up to even: (s, z) of each quantized slot */
+    uint32_t* rmask;  /* [b][Hkv][ceil(K / 32)]: bit t of word w set = slot 32 w + t keeps its bf16 value */
+    void* hp_rows;    /* bf16 [b][Hkv][N_v + B][d]: the reserved cache, the bf16 rows of the reserved slots in
+                         slot order (N_v = 0 for DKV) */
+} vase_mixed_buffers;
+
+/* Sizes in bytes of the four buffers of one layer (NULL outputs are skipped). */
+int vase_mixed_buffer_sizes(const vase_config* cfg, int32_t bits, size_t* codes, size_t* qparams, size_t* rmask,
+                            size_t* hp_rows);
+
+/* Writes the codes, parameters and reserved mask of `layer` right after its eviction (fill == K); the
+ * codes serve vase_decode_attention_mixed until the layer's next eviction.  Errors: VASE_ERR_INVALID (bad
+ * layer or bits, null buffers, fill != K or no eviction yet), VASE_ERR_UNSUPPORTED (reserve_kind random:
+ * its R_V is not a function of the kept values), VASE_ERR_ALIGN (buffers not 16-byte aligned). */
+int vase_quantize_values(vase_ctx* ctx, int32_t layer, int32_t bits, const vase_mixed_buffers* mb, void* stream);
+
+/* vase_decode_attention with the values of unreserved slots below K read from the codes of the layer's
+ * current round (slots appended since the eviction and reserved slots read bf16).  Errors as
+ * vase_decode_attention, plus VASE_ERR_INVALID when the codes were not written for this round and bits. */
+int vase_decode_attention_mixed(vase_ctx* ctx, int32_t layer, int32_t bits, const vase_mixed_buffers* mb,
+                                const void* q, float* out, void* stream);
+
 /* Copies the K positions of every unit of one layer to host memory
  * (int32 [b][Hkv][K]), enqueued on the stream; the host buffer is valid after
  * the stream completes. */

@@ -353,10 +353,16 @@ def reserved_after_eviction(value_scores, budget_k, buffer_b, n_v):
 
 
 def decode_attention_mixed(q, keys, values, reserved, bits):
-    """Decode attention where the values of unreserved slots are read back from their b-bit codes."""
+    """Decode attention where the values of unreserved slots are read back from their b-bit codes.
+
+    Returns the output and its error scale: sum_i alpha_i |v_i| over the bf16 rows and, for a coded row,
+    sum_i alpha_i (|Q_i s_i| + |z_i|), the size of the terms an fp32 evaluation of Q s + z rounds."""
     codes, s, z = quantize_values(values, bits)
-    v_eff = np.where(np.asarray(reserved, dtype=bool)[:, None], values, dequantize_values(codes, s, z))
-    return decode_attention(q, keys, v_eff), decode_attention_bound(q, keys, v_eff)
+    res = np.asarray(reserved, dtype=bool)[:, None]
+    v_eff = np.where(res, values, dequantize_values(codes, s, z))
+    scale = np.where(res, np.abs(values), np.abs(codes * np.asarray(s, dtype=np.float64)[:, None]) +
+                     np.abs(np.asarray(z, dtype=np.float64))[:, None])
+    return decode_attention(q, keys, v_eff), attention_weights(q, keys) @ scale
 
 
 def evict_unit_bits(q_bits, k_bits, v_bits, positions, **kw):

@@ -292,6 +292,7 @@ struct vase_ctx {
     CUtensorMap kmap, vmap, qmap;
     CUtensorMap kmap_dec, vmap_dec;  // 64-row boxes for the decode attention
     std::vector<vase_layer_state> layers;
+    std::vector<int32_t> quant_round, quant_bits;  // per layer: round and bits of the last vase_quantize_values
     std::vector<int32_t> last_batch;  // layers of the most recent eviction launch, by workspace slot
     int64_t launches = 0;
     std::string last_error;
@@ -467,7 +468,9 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
     if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
         (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess ||
         (e = select_set_attributes(P.select_smem)) != cudaSuccess ||
-        (e = decode_set_attributes(P.G, P.decode_smem)) != cudaSuccess) {
+        (e = decode_set_attributes(P.G, P.decode_smem)) != cudaSuccess ||
+        (e = decode_mixed_set_attributes()) != cudaSuccess ||
+        (e = quantize_set_attributes(quantize_smem_bytes(cfg->budget_k, cfg->buffer_b))) != cudaSuccess) {
         fprintf(stderr, "vase_create: kernel attributes: %s\n", cudaGetErrorString(e));
         delete ctx;
         return VASE_ERR_CUDA;
@@ -478,6 +481,8 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
         return VASE_ERR_CUDA;
     }
     ctx->layers.assign(static_cast<size_t>(cfg->num_layers), vase_layer_state{0, 0, 0, 0});
+    ctx->quant_round.assign(static_cast<size_t>(cfg->num_layers), -1);
+    ctx->quant_bits.assign(static_cast<size_t>(cfg->num_layers), 0);
     *out = ctx;
     return VASE_OK;
 }
@@ -765,9 +770,123 @@ int vase_decode_attention(vase_ctx* ctx, int32_t layer, const void* q, float* ou
     dp.row_base = layer * P.units * P.N;
     dp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
     dp.err = reinterpret_cast<uint32_t*>(ctx->ws + P.off_err);
+    dp.codes = nullptr;
+    dp.qparams = nullptr;
+    dp.rmask = nullptr;
+    dp.hp_rows = nullptr;
+    dp.bits = dp.code_row = dp.Kq = dp.Kp = dp.mask_words = dp.hp_cap = 0;
     cudaError_t e =
         launch_decode(ctx->kmap_dec, ctx->vmap_dec, dp, P.decode_smem, P.num_sms, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(ctx, e, "decode attention launch");
+    ctx->launches += 1;
+    return VASE_OK;
+}
+
+// Reserved rows per unit: R_V (N_v, none for DKV) and R_B.
+int hp_capacity(const vase_config* c) {
+    const int nv = c->variant == VASE_VARIANT_ATTNV ? (c->n_v < 0 ? c->budget_k / 4 : c->n_v) : 0;
+    return nv + c->buffer_b;
+}
+
+int vase_mixed_buffer_sizes(const vase_config* cfg, int32_t bits, size_t* codes, size_t* qparams, size_t* rmask,
+                            size_t* hp_rows) {
+    if (const char* why = check_config(cfg)) {
+        g_config_error = why;
+        return VASE_ERR_INVALID;
+    }
+    if (bits != 2 && bits != 4 && bits != 8) {
+        g_config_error = "bits must be 2, 4 or 8";
+        return VASE_ERR_INVALID;
+    }
+    const size_t units = static_cast<size_t>(cfg->batch) * cfg->num_kv_heads;
+    const size_t K = static_cast<size_t>(cfg->budget_k);
+    if (codes) *codes = units * K * (kHeadDim * bits / 8);
+    if (qparams) *qparams = units * ((K + 1) & ~size_t(1)) * 2 * sizeof(float);
+    if (rmask) *rmask = units * ((K + 31) / 32) * sizeof(uint32_t);
+    if (hp_rows) *hp_rows = units * static_cast<size_t>(hp_capacity(cfg)) * kRowBytes;
+    return VASE_OK;
+}
+
+int vase_quantize_values(vase_ctx* ctx, int32_t layer, int32_t bits, const vase_mixed_buffers* mb, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    if (bits != 2 && bits != 4 && bits != 8) return fail(ctx, VASE_ERR_INVALID, "bits must be 2, 4 or 8");
+    if (!mb || !mb->codes || !mb->qparams || !mb->rmask || !mb->hp_rows)
+        return fail(ctx, VASE_ERR_INVALID, "null mixed buffers");
+    if (!aligned(mb->codes, 16) || !aligned(mb->qparams, 16) || !aligned(mb->rmask, 16) || !aligned(mb->hp_rows, 16))
+        return fail(ctx, VASE_ERR_ALIGN, "mixed buffers must be 16-byte aligned");
+    const vase_config& c = ctx->cfg;
+    if (c.variant == VASE_VARIANT_ATTNV && c.reserve_kind == VASE_RESERVE_RANDOM)
+        return fail(ctx, VASE_ERR_UNSUPPORTED, "random reservation: R_V is not a function of the kept values");
+    const vase_layer_state& st = ctx->layers[layer];
+    if (st.round < 1 || st.fill != c.budget_k)
+        return fail(ctx, VASE_ERR_INVALID, "quantize right after an eviction (fill == K)");
+    const Plan& P = ctx->plan;
+    QuantParams qp;
+    qp.vc = vc_layer(ctx, layer);
+    qp.vmag = ctx->bufs.value_scores + static_cast<int64_t>(layer) * P.units * P.N;
+    qp.codes = static_cast<uint8_t*>(mb->codes);
+    qp.qparams = mb->qparams;
+    qp.rmask = mb->rmask;
+    qp.N = P.N;
+    qp.K = c.budget_k;
+    qp.B = c.buffer_b;
+    qp.n_v = c.variant == VASE_VARIANT_ATTNV ? P.n_v : 0;
+    qp.bits = bits;
+    qp.row_bytes = kHeadDim * bits / 8;
+    qp.Kp = (c.budget_k + 1) & ~1;
+    qp.mask_words = (c.budget_k + 31) / 32;
+    qp.hp_rows = static_cast<uint4*>(mb->hp_rows);
+    qp.hp_cap = hp_capacity(&c);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = launch_quantize(qp, P.units, quantize_smem_bytes(c.budget_k, c.buffer_b), s);
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "quantize launch");
+    ctx->launches += 1;
+    ctx->quant_round[layer] = st.round;
+    ctx->quant_bits[layer] = bits;
+    return VASE_OK;
+}
+
+int vase_decode_attention_mixed(vase_ctx* ctx, int32_t layer, int32_t bits, const vase_mixed_buffers* mb,
+                                const void* q, float* out, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    if (!q || !out || !mb || !mb->codes || !mb->qparams || !mb->rmask || !mb->hp_rows)
+        return fail(ctx, VASE_ERR_INVALID, "null input, output or mixed buffer");
+    if (!aligned(q, 16) || !aligned(out, 4)) return fail(ctx, VASE_ERR_ALIGN, "q must be 16-byte aligned, out 4-byte");
+    if (!aligned(mb->codes, 16) || !aligned(mb->qparams, 16) || !aligned(mb->rmask, 16) || !aligned(mb->hp_rows, 16))
+        return fail(ctx, VASE_ERR_ALIGN, "mixed buffers must be 16-byte aligned");
+    const vase_layer_state& st = ctx->layers[layer];
+    if (ctx->quant_round[layer] != st.round || ctx->quant_bits[layer] != bits)
+        return fail(ctx, VASE_ERR_INVALID, "no codes of this bit width for the layer's current round");
+    const Plan& P = ctx->plan;
+    if (P.G > 16) return fail(ctx, VASE_ERR_UNSUPPORTED, "decode attention handles at most 16 query heads per KV head");
+    DecodeParams dp;
+    dp.q = static_cast<const uint4*>(q);
+    dp.kc = kc_layer(ctx, layer);
+    dp.vc = vc_layer(ctx, layer);
+    dp.out = out;
+    dp.N = P.N;
+    dp.fill = st.fill;
+    dp.G = P.G;
+    dp.Hkv = ctx->cfg.num_kv_heads;
+    dp.units = P.units;
+    dp.row_base = layer * P.units * P.N;
+    dp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
+    dp.err = reinterpret_cast<uint32_t*>(ctx->ws + P.off_err);
+    dp.codes = static_cast<const uint8_t*>(mb->codes);
+    dp.qparams = mb->qparams;
+    dp.rmask = mb->rmask;
+    dp.bits = bits;
+    dp.code_row = kHeadDim * bits / 8;
+    dp.Kq = ctx->cfg.budget_k;
+    dp.Kp = (ctx->cfg.budget_k + 1) & ~1;
+    dp.mask_words = (ctx->cfg.budget_k + 31) / 32;
+    dp.hp_rows = static_cast<const uint4*>(mb->hp_rows);
+    dp.hp_cap = hp_capacity(&ctx->cfg);
+    cudaError_t e = launch_decode_mixed(dp, P.num_sms, static_cast<cudaStream_t>(stream));
+    if (e == cudaErrorInvalidValue) return fail(ctx, VASE_ERR_UNSUPPORTED, "too many chunks per CTA for the mixed decode");
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "mixed decode attention launch");
     ctx->launches += 1;
     return VASE_OK;
 }

@@ -26,6 +26,7 @@ enum ErrSite : uint32_t {
     kErrDecodeFull = 48,
     kErrDecodeEmpty = 49,
     kErrDecodeDrain = 50,
+    kErrDecodeMask = 51,
 };
 
 constexpr int kTileTokens = 128;   // tokens per MMA tile (M)
@@ -167,6 +168,18 @@ struct SelectParams {
 };
 
 
+// Mixed-precision values of one layer: codes of the unreserved kept value rows, their (s, z), and the
+// reserved-slot mask (bit t of word w: slot 32 w + t keeps its bf16 row).
+struct QuantParams {
+    const uint4* vc;        // layer base of [units][N][16]
+    const float* vmag;      // layer base of [units][N]: value magnitudes
+    uint8_t* codes;         // [units][K][row_bytes]
+    float* qparams;         // [units][Kp][2]: (s, z)
+    uint32_t* rmask;        // [units][mask_words]
+    uint4* hp_rows;         // [units][hp_cap][16]: the reserved rows in slot order
+    int32_t N, K, B, n_v, bits, row_bytes, Kp, mask_words, hp_cap;
+};
+
 struct DecodeParams {
     const uint4* q;         // [b][Hq][16]: the decode step's query rows (bf16)
     const uint4* kc;        // layer base of [units][N][16]
@@ -178,6 +191,12 @@ struct DecodeParams {
     int32_t row_base;       // first row of the layer in the K / V tensor maps (layer * units * N)
     float scale_log2;       // log2(e) / sqrt(d)
     uint32_t* err;
+    // mixed-precision values (bits > 0): unreserved slots below Kq read from codes
+    const uint8_t* codes;   // [units][Kq][code_row]
+    const float* qparams;   // [units][Kp][2]
+    const uint32_t* rmask;  // [units][mask_words]
+    const uint4* hp_rows;   // [units][hp_cap][16]: the reserved rows below Kq in slot order
+    int32_t bits, code_row, Kq, Kp, mask_words, hp_cap;
 };
 
 // ------------------------------------------------------------------ launchers (return cudaError_t)
@@ -189,6 +208,9 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
 cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
                        size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s);
+cudaError_t launch_quantize(const QuantParams& p, int units, size_t smem_bytes, cudaStream_t s);
+size_t quantize_smem_bytes(int K, int B);
+cudaError_t quantize_set_attributes(size_t smem_bytes);
 cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, DecodeParams p, size_t smem_bytes,
                           int num_sms, cudaStream_t s);
 
@@ -200,5 +222,9 @@ cudaError_t dkv_set_attributes(size_t smem_bytes);
 cudaError_t select_set_attributes(size_t smem_bytes);
 size_t decode_smem_bytes(int G);
 cudaError_t decode_set_attributes(int G, size_t smem_bytes);
+size_t decode_mixed_smem_bytes(int G, int bits, int mask_words);
+cudaError_t decode_mixed_set_attributes();
+cudaError_t launch_decode_mixed(DecodeParams p, int num_sms, cudaStream_t s);
+constexpr int kDecodeMaxMaskWords = 512;  // reserved-slot mask words of a unit the mixed-precision decode holds
 
 }  // namespace vase

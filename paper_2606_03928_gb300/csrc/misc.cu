@@ -610,6 +610,96 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
 }
 
 
+
+// Mixed-precision values (the quantizer of Sec. 4.4, the reserved cache of Sec. 6), one CTA per unit, right
+// after an eviction (fill == K): the reserved (bf16) values are R_B, the last B slots, and R_V, the N_v largest
+// value magnitudes among the first K - B slots (ties to the lower slot, the selection's own rule); every other
+// kept value row gets b-bit codes Q = round((v - z) / s), z = min v, s = Range(v) / (2^b - 1), decided in fp32.
+// Lane l of a warp holds dims 4l .. 4l+3 of a row and packs their four codes into 4b bits at byte 4l * b / 8.
+__global__ void __launch_bounds__(kSelThreads) quantize_kernel(const QuantParams p) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    __shared__ SelShared sh;
+    const int K = p.K;
+    const int C = p.K - p.B;  // candidates of R_V
+    uint32_t* ord = reinterpret_cast<uint32_t*>(smem_raw);
+    const int ord_bytes = max(4 * ((C + 3) & ~3), 8 * p.mask_words);
+    uint8_t* flags = smem_raw + ord_bytes;
+    const int unit = blockIdx.x;
+    const int tid = threadIdx.x;
+    const int lane = tid & 31;
+    const int warp = tid >> 5;
+    const int64_t base = static_cast<int64_t>(unit) * p.N;
+    for (int i = tid; i < K; i += kSelThreads) flags[i] = 0;
+    for (int i = tid; i < C; i += kSelThreads) ord[i] = __float_as_uint(p.vmag[base + i]) + 1u;
+    __syncthreads();
+    const int seg = (C + kSelThreads - 1) / kSelThreads;
+    const int seg_lo = min(C, tid * seg);
+    const int seg_hi = min(C, seg_lo + seg);
+    radix_top_k(ord, C, p.n_v, flags, kFlagValue, seg_lo, seg_hi, sh);  // ends with a barrier
+    // reserved masks (shared memory over the dead selection keys, and global), then their prefix counts
+    uint32_t* mask_s = ord;  // [mask_words], ord is no longer read
+    uint32_t* pre_s = ord + p.mask_words;
+    __syncthreads();
+    for (int w = warp; w < p.mask_words; w += kSelWarps) {
+        const int slot = 32 * w + lane;
+        const bool res = slot < K && (slot >= C || flags[slot]);
+        const uint32_t m = __ballot_sync(0xffffffffu, res);
+        if (lane == 0) {
+            p.rmask[static_cast<int64_t>(unit) * p.mask_words + w] = m;
+            mask_s[w] = m;
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        int run = 0;
+        for (int w = 0; w < p.mask_words; ++w) {
+            pre_s[w] = static_cast<uint32_t>(run);
+            run += __popc(mask_s[w]);
+        }
+    }
+    __syncthreads();
+    // the reserved rows, copied in slot order to the unit's reserved cache (n_v + B rows)
+    for (int j = warp; j < K; j += kSelWarps) {
+        const uint32_t m = mask_s[j >> 5];
+        if (!((m >> (j & 31)) & 1u)) continue;
+        const int idx = static_cast<int>(pre_s[j >> 5]) + __popc(m & ((1u << (j & 31)) - 1u));
+        const uint2 row = reinterpret_cast<const uint2*>(p.vc + (base + j) * kVecPerRow)[lane];
+        reinterpret_cast<uint2*>(p.hp_rows + (static_cast<int64_t>(unit) * p.hp_cap + idx) * kVecPerRow)[lane] = row;
+    }
+    const float levels = static_cast<float>((1 << p.bits) - 1);
+    const int code_bytes = p.bits / 2;  // bytes of one lane's four codes
+    for (int j = warp; j < C; j += kSelWarps) {
+        if (flags[j]) continue;  // R_V keeps its bf16 row (uniform over the warp)
+        const uint2 raw = reinterpret_cast<const uint2*>(p.vc + (base + j) * kVecPerRow)[lane];
+        const float v[4] = {__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xFFFF0000u),
+                            __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xFFFF0000u)};
+        float lo = fminf(fminf(v[0], v[1]), fminf(v[2], v[3]));
+        float hi = fmaxf(fmaxf(v[0], v[1]), fmaxf(v[2], v[3]));
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) {
+            lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+            hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+        }
+        const float s = __fdiv_rn(__fsub_rn(hi, lo), levels);
+        uint32_t packed = 0;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float t = s > 0.f ? rintf(__fdiv_rn(__fsub_rn(v[e], lo), s)) : 0.f;
+            const uint32_t c = static_cast<uint32_t>(fminf(fmaxf(t, 0.f), levels));
+            packed |= c << (e * p.bits);
+        }
+        uint8_t* dst = p.codes + (static_cast<int64_t>(unit) * K + j) * p.row_bytes + lane * code_bytes;
+        if (code_bytes == 4) *reinterpret_cast<uint32_t*>(dst) = packed;
+        else if (code_bytes == 2) *reinterpret_cast<uint16_t*>(dst) = static_cast<uint16_t>(packed);
+        else *dst = static_cast<uint8_t>(packed);
+        if (lane == 0) {
+            float* qp = p.qparams + (static_cast<int64_t>(unit) * p.Kp + j) * 2;
+            qp[0] = s;
+            qp[1] = lo;
+        }
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_append(const AppendParams& p, int n_layers, cudaStream_t s) {
@@ -634,6 +724,22 @@ size_t select_smem_bytes(int N, int K, int n_parts, bool staged) { return sel_la
 cudaError_t select_set_attributes(size_t smem_bytes) {
     return cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 static_cast<int>(smem_bytes));
+}
+
+size_t quantize_smem_bytes(int K, int B) {
+    const size_t words = 4u * ((K - B + 3) & ~3);
+    const size_t masks = 8u * ((K + 31) / 32);  // masks and their prefix counts, over the selection keys
+    return (words > masks ? words : masks) + K;
+}
+
+cudaError_t quantize_set_attributes(size_t smem_bytes) {
+    return cudaFuncSetAttribute(quantize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(smem_bytes));
+}
+
+cudaError_t launch_quantize(const QuantParams& p, int units, size_t smem_bytes, cudaStream_t s) {
+    quantize_kernel<<<static_cast<unsigned>(units), kSelThreads, smem_bytes, s>>>(p);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s) {

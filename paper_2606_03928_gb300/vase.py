@@ -39,7 +39,7 @@ EXPORTED = [
     "vase_kv_view_get", "vase_debug_view_get", "vase_check_device_error", "vase_launch_count",
     "vase_status_string", "vase_last_error", "vase_abi_version", "vase_profile_enable", "vase_profile_collect",
     "vase_append_all", "vase_evict_all", "vase_refresh_value_scores", "vase_evict_static_scratch",
-    "vase_decode_attention",
+    "vase_decode_attention", "vase_mixed_buffer_sizes", "vase_quantize_values", "vase_decode_attention_mixed",
 ]
 KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "compact"]
 
@@ -70,6 +70,11 @@ class vase_kv_view(ctypes.Structure):
     _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("positions", ctypes.c_void_p),
                 ("value_scores", ctypes.c_void_p), ("unit_stride", ctypes.c_int64), ("slots", ctypes.c_int32),
                 ("fill", ctypes.c_int32)]
+
+
+class vase_mixed_buffers(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_void_p), ("qparams", ctypes.c_void_p), ("rmask", ctypes.c_void_p),
+                ("hp_rows", ctypes.c_void_p)]
 
 
 class vase_debug_view(ctypes.Structure):
@@ -105,6 +110,10 @@ def load(path: str = LIB_PATH):
                                                      ctypes.POINTER(vase_layer_state), ctypes.POINTER(U32), P]),
         "vase_read_positions": (ctypes.c_int, [P, I32, P, P]),
         "vase_decode_attention": (ctypes.c_int, [P, I32, P, P, P]),
+        "vase_mixed_buffer_sizes": (ctypes.c_int, [ctypes.POINTER(vase_config), I32] +
+                                    [ctypes.POINTER(ctypes.c_size_t)] * 4),
+        "vase_quantize_values": (ctypes.c_int, [P, I32, I32, ctypes.POINTER(vase_mixed_buffers), P]),
+        "vase_decode_attention_mixed": (ctypes.c_int, [P, I32, I32, ctypes.POINTER(vase_mixed_buffers), P, P, P]),
         "vase_get_layer_state": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_layer_state)]),
         "vase_set_layer_state": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_layer_state)]),
         "vase_kv_view_get": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_kv_view)]),
@@ -219,6 +228,24 @@ def vase_evict_static_scratch(cfg: vase_config, bufs: vase_buffers, layer, fill,
 def vase_decode_attention(ctx, layer, q_ptr, out_ptr, stream=None):
     return _check(ctx, load().vase_decode_attention(ctx, layer, q_ptr, out_ptr, _stream_ptr(stream)),
                   "vase_decode_attention")
+
+
+def vase_mixed_buffer_sizes(cfg: vase_config, bits):
+    sizes = [ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_size_t()]
+    st = load().vase_mixed_buffer_sizes(ctypes.byref(cfg), bits, *(ctypes.byref(x) for x in sizes))
+    if st != VASE_OK:
+        raise VaseError(st, "vase_mixed_buffer_sizes: " + load().vase_last_error(None).decode())
+    return tuple(x.value for x in sizes)
+
+
+def vase_quantize_values(ctx, layer, bits, mb: vase_mixed_buffers, stream=None):
+    return _check(ctx, load().vase_quantize_values(ctx, layer, bits, ctypes.byref(mb), _stream_ptr(stream)),
+                  "vase_quantize_values")
+
+
+def vase_decode_attention_mixed(ctx, layer, bits, mb: vase_mixed_buffers, q_ptr, out_ptr, stream=None):
+    return _check(ctx, load().vase_decode_attention_mixed(ctx, layer, bits, ctypes.byref(mb), q_ptr, out_ptr,
+                                                          _stream_ptr(stream)), "vase_decode_attention_mixed")
 
 
 def vase_read_positions(ctx, layer, host_ptr, stream=None):
@@ -357,6 +384,31 @@ class VaseCache:
             out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
         assert out.is_cuda and out.dtype == torch.float32 and out.is_contiguous()
         vase_decode_attention(self.ctx, layer, q.data_ptr(), out.data_ptr(), stream)
+        return out
+
+    def mixed_buffers(self, bits):
+        """Device buffers of one layer's mixed-precision values (codes, (s, z), reserved mask, reserved rows) as
+        torch tensors, plus the vase_mixed_buffers struct that points at them."""
+        n_codes, n_qp, n_mask, n_hp = vase_mixed_buffer_sizes(self.cfg, bits)
+        t = {"codes": torch.zeros(n_codes, dtype=torch.uint8, device=self.device),
+             "qparams": torch.zeros(n_qp // 4, dtype=torch.float32, device=self.device),
+             "rmask": torch.zeros(n_mask // 4, dtype=torch.int32, device=self.device),
+             "hp_rows": torch.zeros(n_hp // 2, dtype=torch.bfloat16, device=self.device)}
+        mb = vase_mixed_buffers(t["codes"].data_ptr(), t["qparams"].data_ptr(), t["rmask"].data_ptr(),
+                                t["hp_rows"].data_ptr())
+        return mb, t
+
+    def quantize_values(self, layer, bits, mb, stream=None):
+        """Codes of the layer's unreserved kept values, right after its eviction."""
+        return vase_quantize_values(self.ctx, layer, bits, mb, stream)
+
+    def decode_attention_mixed(self, layer, bits, mb, q: torch.Tensor, out: torch.Tensor = None, stream=None):
+        """decode_attention with the unreserved values read from the codes of the layer's current round."""
+        assert q.is_cuda and q.dtype == torch.bfloat16 and q.is_contiguous()
+        if out is None:
+            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+        assert out.is_cuda and out.dtype == torch.float32 and out.is_contiguous()
+        vase_decode_attention_mixed(self.ctx, layer, bits, mb, q.data_ptr(), out.data_ptr(), stream)
         return out
 
     def read_positions(self, layer, out: torch.Tensor, stream=None):

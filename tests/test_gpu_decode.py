@@ -159,3 +159,18 @@ def test_decode_full_size_qwen3_8b_layer_sampled_units():
     out = cache.decode_attention(0, q)
     torch.cuda.synchronize()
     _check(wl, cache, 0, q_bits, out, wl.budget_k, units=[(0, 0), (17, 3), (31, 7)])
+
+
+@pytest.mark.parametrize("heads", [(1, 1), (4, 1)])
+def test_decode_at_the_largest_supported_fill(heads):
+    """K + B = 16640 slots in one unit (260 chunks of 64, 520 of 32): both kernels, every output checked."""
+    Hq, Hkv = heads
+    wl = W.shrink(SMALL, budget_k=16384, buffer_b=256, window=8, num_q_heads=Hq, num_kv_heads=Hkv, batch=1,
+                  num_layers=1)
+    cache = _cache(wl, 1)
+    st = W.layer_state(wl, 51, 0, 0, "dense")
+    PU.upload_layer(cache, 0, st, 0)
+    q_bits, q = _queries(wl, 52)
+    out = cache.decode_attention(0, q)
+    torch.cuda.synchronize()
+    _check(wl, cache, 0, q_bits, out, wl.slots)

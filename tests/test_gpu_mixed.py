@@ -160,3 +160,24 @@ def test_mixed_values_status_checks():
     mb2, t2 = rnd.mixed_buffers(4)
     with pytest.raises(VaseError):        # a random R_V cannot be recovered from the kept values
         rnd.quantize_values(0, 4, mb2)
+
+
+def test_mixed_decode_at_the_largest_budget():
+    """K = 16384: 512 mask words per unit, the most the mixed decode holds."""
+    wl = W.shrink(SMALL, budget_k=16384, buffer_b=256, window=8, num_q_heads=2, num_kv_heads=1, batch=1,
+                  num_layers=1)
+    cache = _evicted(wl, 61)
+    mb, _ = cache.mixed_buffers(4)
+    cache.quantize_values(0, 4, mb)
+    rng = np.random.default_rng(62)
+    q_bits = W.f32_to_bf16_bits(rng.standard_normal((1, 2, wl.head_dim)).astype(np.float32))
+    out = cache.decode_attention_mixed(0, 4, mb, PU.bits_to_bf16_tensor(q_bits, "cuda"))
+    torch.cuda.synchronize()
+    K, B = wl.budget_k, wl.buffer_b
+    k_bits = cache.k_cache[0].view(torch.int16).cpu().numpy().view(np.uint16)
+    v_bits = cache.v_cache[0].view(torch.int16).cpu().numpy().view(np.uint16)
+    v = O.bf16_bits_to_f64(v_bits[0, 0, :K])
+    reserved = O.reserved_after_eviction(O.value_magnitude(v), K, B, K // 4)
+    ref, bound = O.decode_attention_mixed(O.bf16_bits_to_f64(q_bits[0]), O.bf16_bits_to_f64(k_bits[0, 0, :K]), v,
+                                          reserved, 4)
+    assert not (np.abs(out.cpu().numpy()[0].astype(np.float64) - ref) > DEC_RTOL * bound + DEC_ATOL).any()

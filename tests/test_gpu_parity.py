@@ -565,3 +565,28 @@ def test_dkv_shared_g_matches_oracle_and_is_shared():
     assert cache2.evict(0) == 0
     scores2 = cache2.debug_view(0)["value_score"].cpu().numpy().reshape(wl.batch, wl.num_kv_heads, -1)
     assert not np.array_equal(scores2[0], scores2[1])
+
+
+# ----------------------------------------------------------------------------- maximum sizes and degenerate cases
+
+def test_largest_supported_unit_matches_oracle():
+    """K = 16384, B = 256: the largest budget the single-CTA selection holds (unstaged inputs), one unit, the
+    score kernel in cluster mode; every slot checked against the oracle."""
+    wl = W.shrink(SMALL, budget_k=16384, buffer_b=256, window=16, num_q_heads=4, num_kv_heads=1, batch=1,
+                  num_layers=1)
+    _run_layer(wl, layer=0, num_layers=1, round_index=4)
+
+
+def test_budget_equal_to_buffer_keeps_only_the_buffer():
+    """K == B (so N_v = 0 and m = 0): every candidate is evicted and the B newest pairs move down."""
+    wl = W.shrink(SMALL, budget_k=96, buffer_b=96, window=8, batch=2, num_layers=1)
+    cache, st, got, _ = _run_layer(wl, layer=0, num_layers=1, cache_kw={"n_v": 0}, oracle_kw={"n_v": 0})
+    for u in range(wl.batch * wl.num_kv_heads):
+        assert np.array_equal(got["src"][u], np.arange(96, 192))
+
+
+def test_value_reservation_filling_every_kept_candidate():
+    """N_v = K - B: R_V takes every kept candidate (m = 0), so the kept set is R_V plus the buffer."""
+    K, B = 160, 32
+    wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=8, batch=2, num_layers=1)
+    _run_layer(wl, layer=0, num_layers=1, cache_kw={"n_v": K - B}, oracle_kw={"n_v": K - B})

@@ -17,8 +17,9 @@ constexpr int kQPieceFloats = 12;
 // The running max of a warp is raised only when a score exceeds it by more than this (log2 units).
 constexpr float kLazyMax = 8.f;
 
-// Stage of one chunk: K rows, V rows (bf16; with b-bit values only the reserved rows and those past the
-// quantized slots are filled, each at its own row), then with b-bit values the chunk's code rows and (s, z).
+// Stage of one chunk: K rows, V rows (bf16; with b-bit values the chunk's reserved rows compacted at the front
+// and the rows of slots past the quantized ones at their own rows), then with b-bit values the chunk's code
+// rows and (s, z).
 __host__ __device__ constexpr uint32_t stage_bytes(int bits) {
     return 2 * kChunkBytes + (bits > 0 ? kChunk * 16u * bits + kChunk * 8u : 0u);
 }

@@ -50,7 +50,7 @@ KERNEL_SOURCES = {
     "select_compact": ["misc.cu", "kernels.cuh", "ptx.cuh"],
     "append": ["misc.cu", "kernels.cuh", "ptx.cuh"],
     "dkv_score": ["dkv.cu", "kernels.cuh", "ptx.cuh"],
-    "decode": ["decode.cu", "kernels.cuh", "ptx.cuh"],
+    "decode": ["decode.cu", "decode_simt.cuh", "decode_mixed.cu", "kernels.cuh", "ptx.cuh"],
 }
 
 

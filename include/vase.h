@@ -157,8 +157,10 @@ void vase_destroy(vase_ctx* ctx);
  * step adds one pair per KV head).  Device inputs, row-major:
  *   q [n_tokens][b][Hq][d], k and v [n_tokens][b][Hkv][d]  (bf16).
  * q goes to the window ring, k and v to slots fill..fill+n_tokens-1 with their
- * stream positions.  Returns VASE_EVICT_DUE when the layer becomes full,
- * VASE_ERR_FULL (nothing written) when fill + n_tokens > K + B. */
+ * stream positions.  Only the last min(W, n_tokens) query rows are read (the
+ * ring keeps no others); the rows before them need not hold data.  Returns
+ * VASE_EVICT_DUE when the layer becomes full, VASE_ERR_FULL (nothing written)
+ * when fill + n_tokens > K + B. */
 int vase_append(vase_ctx* ctx, int32_t layer, const void* q, const void* k, const void* v,
                 int32_t n_tokens, void* stream);
 

@@ -590,3 +590,22 @@ def test_value_reservation_filling_every_kept_candidate():
     K, B = 160, 32
     wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=8, batch=2, num_layers=1)
     _run_layer(wl, layer=0, num_layers=1, cache_kw={"n_v": K - B}, oracle_kw={"n_v": K - B})
+
+
+def test_append_reads_only_the_last_window_query_rows():
+    """vase_append's contract: query rows before the last min(W, n) are never read (NaN there changes nothing)."""
+    wl = W.shrink(SMALL, budget_k=128, buffer_b=64, window=8, batch=2, num_layers=1)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(71)
+    n = 40
+    q = torch.randn((n, wl.batch, wl.num_q_heads, wl.head_dim), generator=gen, device="cuda").to(torch.bfloat16)
+    k = torch.randn((n, wl.batch, wl.num_kv_heads, wl.head_dim), generator=gen, device="cuda").to(torch.bfloat16)
+    v = torch.randn((n, wl.batch, wl.num_kv_heads, wl.head_dim), generator=gen, device="cuda").to(torch.bfloat16)
+    q_nan = q.clone()
+    q_nan[:n - wl.window] = float("nan")
+    a, b = _cache(wl, 1, debug=False), _cache(wl, 1, debug=False)
+    a.append(0, q, k, v)
+    b.append(0, q_nan, k, v)
+    torch.cuda.synchronize()
+    assert torch.equal(a.q_window, b.q_window) and torch.equal(a.k_cache, b.k_cache)
+    assert torch.equal(a.v_cache, b.v_cache) and torch.equal(a.positions, b.positions)

@@ -521,6 +521,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (j == nB - 1 && k + 1 < n_w) mbar_arrive(&q_empty[2 * ((k - 1) & (p.q_bufs - 1)) + grp]);
                         }
                         tc_fence_after();
+                        if (!kHeadMax) {
+                            // 32 columns at a time, two register sets: the load of the next set is in flight
+                            // while this one is summed
+                            const uint32_t col0 = taddr + lane_base + static_cast<uint32_t>(buf * bufcols);
+                            const int nch = NB / 32;
+                            uint32_t ra[32], rb[32];
+                            auto sum32 = [&](const uint32_t (&r)[32], int c) {
+                                const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
+                                float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+                                for (int q = 0; q < 8; ++q) {
+                                    const float4 mm = m4[q];
+                                    a0 += ex2(fmaf(__uint_as_float(r[4 * q]), cs, -mm.x));
+                                    a1 += ex2(fmaf(__uint_as_float(r[4 * q + 1]), cs, -mm.y));
+                                    a2 += ex2(fmaf(__uint_as_float(r[4 * q + 2]), cs, -mm.z));
+                                    a3 += ex2(fmaf(__uint_as_float(r[4 * q + 3]), cs, -mm.w));
+                                }
+                                acc += (a0 + a1) + (a2 + a3);
+                            };
+                            tmem_ld32_issue(col0, ra);
+                            tmem_wait_ld32(ra);
+                            for (int ch = 0; ch < nch; ch += 2) {
+                                if (ch + 1 < nch) tmem_ld32_issue(col0 + 32 * (ch + 1), rb);
+                                sum32(ra, 32 * ch);
+                                if (ch + 1 < nch) {
+                                    tmem_wait_ld32(rb);
+                                    if (ch + 2 < nch) tmem_ld32_issue(col0 + 32 * (ch + 2), ra);
+                                    sum32(rb, 32 * (ch + 1));
+                                    if (ch + 2 < nch) tmem_wait_ld32(ra);
+                                }
+                            }
+                        } else {
                         // GQA max-aggregation: the sum runs per query head (W consecutive window rows, whole
                         // heads per row block) and the token keeps the largest head sum
                         float head_sum = 0.f;
@@ -537,36 +569,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 for (int q = 0; q < 32; ++q) v[q] = h[q];
                             }
                             const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
-                            if (!kHeadMax) {
-                                float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
-                                for (int q = 0; q < 16; ++q) {
-                                    if (q < width / 4) {
-                                        const float4 mm = m4[q];
-                                        a0 += ex2(fmaf(v[4 * q], cs, -mm.x));
-                                        a1 += ex2(fmaf(v[4 * q + 1], cs, -mm.y));
-                                        a2 += ex2(fmaf(v[4 * q + 2], cs, -mm.z));
-                                        a3 += ex2(fmaf(v[4 * q + 3], cs, -mm.w));
+                            for (int q = 0; q < 16; ++q) {
+                                if (q < width / 4) {
+                                    if (sub * NB + c + 4 * q == head_end) {  // the same in every thread
+                                        acc = fmaxf(acc, head_sum);
+                                        head_sum = 0.f;
+                                        head_end += head_rows;
                                     }
-                                }
-                                acc += (a0 + a1) + (a2 + a3);
-                            } else {
-#pragma unroll
-                                for (int q = 0; q < 16; ++q) {
-                                    if (q < width / 4) {
-                                        if (sub * NB + c + 4 * q == head_end) {  // the same in every thread
-                                            acc = fmaxf(acc, head_sum);
-                                            head_sum = 0.f;
-                                            head_end += head_rows;
-                                        }
-                                        const float4 mm = m4[q];
-                                        head_sum += (ex2(fmaf(v[4 * q], cs, -mm.x)) + ex2(fmaf(v[4 * q + 1], cs, -mm.y))) +
-                                                    (ex2(fmaf(v[4 * q + 2], cs, -mm.z)) + ex2(fmaf(v[4 * q + 3], cs, -mm.w)));
-                                    }
+                                    const float4 mm = m4[q];
+                                    head_sum += (ex2(fmaf(v[4 * q], cs, -mm.x)) + ex2(fmaf(v[4 * q + 1], cs, -mm.y))) +
+                                                (ex2(fmaf(v[4 * q + 2], cs, -mm.z)) + ex2(fmaf(v[4 * q + 3], cs, -mm.w)));
                                 }
                             }
                         }
-                        if (kHeadMax) acc = fmaxf(acc, head_sum);
+                        acc = fmaxf(acc, head_sum);
+                        }
                         tc_fence_before();
                         mbar_arrive(&t_empty[buf]);
                     }

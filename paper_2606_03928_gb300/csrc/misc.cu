@@ -307,14 +307,17 @@ __device__ __forceinline__ void cp_async_wait_all() {
 // Gather of the kept rows: one warp per tensor (K, V), a ring of kGatherStages chunks of kGatherRows
 // destination rows each.
 constexpr int kGatherRows = 24;
-constexpr int kGatherStages = 3;
-constexpr uint32_t kGatherRingBytes = kGatherStages * kGatherRows * kRowBytes;  // per tensor
+constexpr int kGatherStages = 3;       // ring depth when the selection's buffers leave no more room
+constexpr int kGatherMaxStages = 16;   // ring depth where they do (units of many slots)
+constexpr uint32_t kGatherChunkBytes = kGatherRows * kRowBytes;
+constexpr uint32_t kGatherRingBytes = kGatherStages * kGatherChunkBytes;  // per tensor, at the base depth
 
 // Shared-memory layout of the selection: window scores (one array per part) or leverage products, then
 // (staged) value magnitudes and positions, then the orderable keys and the flags.  The gather rings
 // overlay all of these once the selection is done; the kept list and the rings' barriers follow.
 struct SelLayout {
     uint32_t a_off, vm_off, pos_off, ord_off, flag_off, src_off, bar_off, total;
+    int gather_stages;  // ring depth per tensor: as many chunks as the selection's buffers hold, 3 at least
 };
 
 __host__ __device__ inline SelLayout sel_layout(int N, int K, int n_parts, bool staged) {
@@ -331,12 +334,14 @@ __host__ __device__ inline SelLayout sel_layout(int N, int K, int n_parts, bool 
     L.flag_off = o;
     o += N;
     if (o < 2 * kGatherRingBytes) o = 2 * kGatherRingBytes;
+    L.gather_stages = static_cast<int>(o / (2 * kGatherChunkBytes));
+    if (L.gather_stages > kGatherMaxStages) L.gather_stages = kGatherMaxStages;
     o = (o + 15u) & ~15u;
     L.src_off = o;
     o += 4u * K;
     o = (o + 7u) & ~7u;
     L.bar_off = o;
-    o += 8u * 2 * kGatherStages;
+    o += 8u * 2 * kGatherMaxStages;
     L.total = o;
     return L;
 }
@@ -354,6 +359,7 @@ __device__ __forceinline__ void bulk_store(void* gdst, const void* smem_src, uin
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // Stable in-place gather of one tensor's kept rows (K or V of one unit) by one warp: new row j takes old
@@ -364,17 +370,17 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 // so loads issued ahead never read a row that an earlier chunk's store overwrites; a chunk is stored only
 // after its own loads have landed.
 __device__ void gather_rows(uint8_t* base, const int32_t* src, int j_first, int K, uint8_t* ring, uint64_t* full,
-                            uint32_t* err) {
+                            int stages, uint32_t* err) {
     const int lane = threadIdx.x & 31;
     if (lane == 0) {
-        for (int s = 0; s < kGatherStages; ++s) mbar_init(&full[s], 1);
+        for (int s = 0; s < stages; ++s) mbar_init(&full[s], 1);
         fence_mbar_init();
     }
     __syncwarp();
     const int n_chunks = (K - j_first + kGatherRows - 1) / kGatherRows;
     auto load = [&](int c) {
-        const int stage = c % kGatherStages;
-        uint8_t* dst = ring + stage * (kGatherRows * kRowBytes);
+        const int stage = c % stages;
+        uint8_t* dst = ring + stage * kGatherChunkBytes;
         const int j0 = j_first + c * kGatherRows;
         const int rows = min(kGatherRows, K - j0);
         if (lane == 0) mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(rows) * kRowBytes);
@@ -391,22 +397,30 @@ __device__ void gather_rows(uint8_t* base, const int32_t* src, int j_first, int 
                       static_cast<uint32_t>(next - lane) * kRowBytes, &full[stage]);
         }
     };
+    // Loads run `ahead` chunks in front of the stores.  With the base depth the stage reloaded next was read by
+    // the store just issued, so every store must have read its bytes first (wait_group.read 0); with a deeper
+    // ring the reloaded stage's last store is at least two back, so the newest store may still be reading
+    // (wait_group.read 1).
+    const int ahead = stages > kGatherStages ? stages - 2 : stages - 1;
     bool ok = true;
-    for (int c = 0; c < kGatherStages - 1 && c < n_chunks; ++c) load(c);
+    for (int c = 0; c < ahead && c < n_chunks; ++c) load(c);
     for (int c = 0; c < n_chunks; ++c) {
-        const int nxt = c + kGatherStages - 1;
+        const int nxt = c + ahead;
         if (nxt < n_chunks) {
-            if (lane == 0) bulk_wait_read0();  // the store that last used nxt's stage has read its bytes
+            if (lane == 0) {
+                if (stages > kGatherStages) bulk_wait_read1();
+                else bulk_wait_read0();
+            }
             __syncwarp();
             load(nxt);
         }
-        const int stage = c % kGatherStages;
-        if (ok) ok = mbar_wait(&full[stage], (c / kGatherStages) & 1, err, kErrCompactFull);
+        const int stage = c % stages;
+        if (ok) ok = mbar_wait(&full[stage], (c / stages) & 1, err, kErrCompactFull);
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         if (lane == 0) {
             const int j0 = j_first + c * kGatherRows;
             const int rows = min(kGatherRows, K - j0);
-            bulk_store(base + static_cast<int64_t>(j0) * kRowBytes, ring + stage * (kGatherRows * kRowBytes),
+            bulk_store(base + static_cast<int64_t>(j0) * kRowBytes, ring + stage * kGatherChunkBytes,
                        static_cast<uint32_t>(rows) * kRowBytes);
             bulk_commit();
         }
@@ -604,8 +618,9 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
     if (warp < 2) {
         const int64_t unit_row = (static_cast<int64_t>(layer) * p.units + unit) * N;
         uint8_t* const rows = reinterpret_cast<uint8_t*>((warp == 0 ? p.kc : p.vc) + unit_row * kVecPerRow);
-        gather_rows(rows, src_s, sh.first_evicted, K, smem_raw + warp * kGatherRingBytes,
-                    reinterpret_cast<uint64_t*>(smem_raw + Ly.bar_off) + warp * kGatherStages, p.err);
+        gather_rows(rows, src_s, sh.first_evicted, K, smem_raw + warp * Ly.gather_stages * kGatherChunkBytes,
+                    reinterpret_cast<uint64_t*>(smem_raw + Ly.bar_off) + warp * kGatherMaxStages, Ly.gather_stages,
+                    p.err);
     }
 }
 

@@ -23,6 +23,7 @@ whole-job rate from the maximum step time over ranks.
 from __future__ import annotations
 
 import argparse
+import datetime
 import json
 import os
 import statistics
@@ -78,7 +79,7 @@ def measured_peaks():
 class ClockSampler:
     """nvidia-smi clock / throttle-reason samples taken while the timed region runs."""
 
-    FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+    FIELDS = ["timestamp", "index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
               "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
               "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
 
@@ -86,8 +87,15 @@ class ClockSampler:
         self.gpu = gpu_index
         self.proc = None
         self.file = None
+        self.t_begin = 0.0
+
+    def _rows(self):
+        with open(self.file.name) as f:
+            return [r for r in f.read().splitlines() if r.strip()]
 
     def start(self):
+        """Starts nvidia-smi and returns once its first sample is written (at most 5 s), so that its start-up
+        falls before the timed region, which the caller begins next."""
         try:
             self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             self.proc = subprocess.Popen(
@@ -95,10 +103,17 @@ class ClockSampler:
                  "--format=csv,noheader,nounits", "-lms", "50"], stdout=self.file, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
+            return
+        t0 = time.time()
+        while time.time() - t0 < 5.0 and self.proc.poll() is None and not self._rows():
+            time.sleep(0.01)
+        self.t_begin = time.time()
 
     def stop(self):
+        """Ends sampling (the caller has just ended the timed region); summarises the samples stamped inside it."""
         if self.proc is None:
             return None
+        t_end = time.time()
         time.sleep(0.06)
         self.proc.terminate()
         try:
@@ -112,16 +127,25 @@ class ClockSampler:
         os.unlink(self.file.name)
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        parsed = []  # (time stamp or None, fields)
         for r in rows:
             r = [x.strip() for x in r]
-            if len(r) < 9:
+            if len(r) < 10:
                 continue
             try:
-                sm.append(float(r[1]))
-                mx.append(float(r[2]))
+                t = datetime.datetime.strptime(r[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+            except ValueError:
+                t = None
+            parsed.append((t, r))
+        if any(t is not None for t, _ in parsed):  # else (an unknown stamp format) every sample is kept
+            parsed = [(t, r) for t, r in parsed if t is not None and self.t_begin - 0.01 <= t <= t_end + 0.01]
+        for _, r in parsed:
+            try:
+                sm.append(float(r[2]))
+                mx.append(float(r[3]))
             except ValueError:
                 continue
-            for name, val in zip(names, r[5:9]):
+            for name, val in zip(names, r[6:10]):
                 if val.lower() in ("active", "1"):
                     reasons.add(name)
         if not sm:
@@ -342,7 +366,6 @@ def run_ours(args):
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     sampler = ClockSampler(local if world > 1 else 0)
     launches0 = cache.launch_count()
-    cache.profile_enable(True)
     barrier()
     torch.cuda.synchronize()
     sampler.start()
@@ -353,9 +376,22 @@ def run_ours(args):
     torch.cuda.synchronize()
     barrier()
     clocks = sampler.stop()
+    launches = cache.launch_count() - launches0
+    # the same K steps again with a CUDA event pair around every launch (the library's profiling mode), for
+    # each kernel's launch duration; the step time above is taken without those events
+    cache.profile_enable(True)
+    barrier()
+    torch.cuda.synchronize()
+    ep0, ep1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ep0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ep1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
     cache.profile_enable(False)
     kernels = cache.profile_collect()
-    launches = cache.launch_count() - launches0
+    profiled_ms = ep0.elapsed_time(ep1) / args.steps
     ms = ev0.elapsed_time(ev1) / args.steps
     st, code = cache.check_device_error()
     if st != 0:
@@ -412,11 +448,12 @@ def run_ours(args):
     zero_copy_ms = timed(lambda: [e2e_step(r) for r in range(e2e_steps)])
 
     # Pipelined: a copy stream brings step r + 1's inputs into one of two device staging sets while step r
-    # appends (vase_append from the staging set) and evicts; it then reads step r's kept positions back.  The
-    # staging layout puts every layer's [last W query rows | k | v] back to back, so one copy per step moves
-    # them all; vase_append reads only the last W query rows, so each layer's q pointer is set W rows before
-    # its query rows (a pad of n - W rows at the front keeps layer 0's inside the buffer).  Every step's
-    # copies and its position read-back stay in the timed region.
+    # appends (one vase_append_all_strided launch from the staging set) and evicts; it then reads step r's kept
+    # positions back.  The staging layout puts every layer's [last W query rows | k | v] back to back, so one
+    # copy per step moves them all; the append reads only the last W query rows, so each layer's q pointer is
+    # set W rows before its query rows (a pad of n - W rows at the front keeps layer 0's inside the buffer)
+    # and consecutive layers' inputs are one block apart.  Every step's copies and its position read-back stay
+    # in the timed region.
     copy_stream = torch.cuda.Stream(device=device)
     n_tok = q0.shape[0]
     W_q = min(wl.window, n_tok)
@@ -441,11 +478,9 @@ def run_ours(args):
     copied = [torch.cuda.Event() for _ in range(2)]
     consumed = [torch.cuda.Event() for _ in range(2)]
     evicted = torch.cuda.Event()
-    ptrs = []
-    for b in range(2):
-        base = dev_flat[b].data_ptr()
-        ptrs.append([(base + 2 * layer * blk, base + 2 * (pad + layer * blk + W_q * q_row),
-                      base + 2 * (pad + layer * blk + W_q * q_row + kv_el)) for layer in range(L)])
+    # layer 0's (q, k, v) in each staging set; layer l's are l blocks (2 * blk bytes) further on
+    ptr0 = [(f.data_ptr(), f.data_ptr() + 2 * (pad + W_q * q_row), f.data_ptr() + 2 * (pad + W_q * q_row + kv_el))
+            for f in dev_flat]
 
     def issue_copy(r):
         b = r % 2
@@ -462,8 +497,7 @@ def run_ours(args):
                 issue_copy(r + 1)
             b = r % 2
             stream.wait_event(copied[b])
-            for layer in range(L):
-                V.vase_append(cache.ctx, layer, *ptrs[b][layer], n_tok, stream)
+            V.vase_append_all_strided(cache.ctx, *ptr0[b], n_tok, 2 * blk, 2 * blk, stream)
             consumed[b].record(stream)
             cache.evict_all()
             evicted.record(stream)
@@ -525,11 +559,12 @@ def run_ours(args):
                           "frac": round(step_roof_ms / ms, 4),
                           "amortised_us_per_decode_token": round(1e3 * evict_ms / Bf, 3)},
         "kernels": per_kernel,
+        "kernels_pass_ms_per_step": round(profiled_ms, 4),
         "clocks": clocks,
         "gpu_launches": launches,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": pos_host.numel() * pos_host.element_size(),
-                "ms_per_step": e2e_ms, "form": "next step's inputs copied (one copy) on a second stream during this step",
+                "ms_per_step": e2e_ms, "form": "next step's inputs copied (one copy) on a second stream during this step, appended in one launch",
                 "zero_copy_ms_per_step": zero_copy_ms},
     }
     if pool is not None:

@@ -168,6 +168,18 @@ int vase_append(vase_ctx* ctx, int32_t layer, const void* q, const void* k, cons
  * k and v [L][n_tokens][b][Hkv][d] (device, bf16).  All layers must have room. */
 int vase_append_all(vase_ctx* ctx, const void* q, const void* k, const void* v, int32_t n_tokens, void* stream);
 
+/* vase_append_all with the layers' inputs at any fixed distance: layer l's
+ * [n_tokens][b][Hq][d] query rows start at q + l * q_layer_stride bytes and its
+ * [n_tokens][b][Hkv][d] key and value rows at k + l * kv_layer_stride and
+ * v + l * kv_layer_stride (device, bf16).  As in vase_append only the last
+ * min(W, n_tokens) query rows of each layer are read, so a layer's block may
+ * hold its query tail alone (q pointing W rows before it) next to its keys and
+ * values, and one copy can bring every layer's inputs.  Strides must be positive
+ * multiples of 16 bytes (VASE_ERR_INVALID / VASE_ERR_ALIGN otherwise, nothing
+ * written); all layers must have room (VASE_ERR_FULL). */
+int vase_append_all_strided(vase_ctx* ctx, const void* q, const void* k, const void* v, int32_t n_tokens,
+                            int64_t q_layer_stride, int64_t kv_layer_stride, void* stream);
+
 /* Same as vase_append with HOST inputs (at most B tokens per call).  Page-locked
  * inputs (pinned or registered) are read by the append kernel in place over the
  * host link, asynchronously on `stream`; other host memory is first copied into

@@ -491,25 +491,32 @@ void vase_destroy(vase_ctx* ctx) { delete ctx; }
 
 namespace {
 
-// Appends n_tokens to each layer of `layers` (inputs stacked per layer slot) in one launch.
+// Appends n_tokens to each layer of `layers` in one launch; the inputs of consecutive layer slots are q_stride
+// and kv_stride bytes apart (0: packed, one slot's [n][b][H][d] after the other).
 int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void* q, const void* k, const void* v,
-                 int32_t n_tokens, cudaStream_t stream) {
+                 int32_t n_tokens, cudaStream_t stream, int64_t q_stride = 0, int64_t kv_stride = 0) {
     if (n_tokens < 1) return fail(ctx, VASE_ERR_INVALID, "n_tokens must be >= 1");
     if (!q || !k || !v) return fail(ctx, VASE_ERR_INVALID, "null input");
     if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16))
         return fail(ctx, VASE_ERR_ALIGN, "inputs must be 16-byte aligned");
+    if (q_stride < 0 || kv_stride < 0 || q_stride % 16 || kv_stride % 16)
+        return fail(ctx, VASE_ERR_ALIGN, "layer strides must be non-negative multiples of 16 bytes");
     for (int z = 0; z < n_layers; ++z)
         if (ctx->layers[layers[z]].fill + n_tokens > ctx->plan.N)
             return fail(ctx, VASE_ERR_FULL, "append would exceed K + B slots");
     const vase_config& c = ctx->cfg;
-    const size_t q_slot = static_cast<size_t>(n_tokens) * c.batch * c.num_q_heads * kVecPerRow;
-    const size_t kv_slot = static_cast<size_t>(n_tokens) * c.batch * c.num_kv_heads * kVecPerRow;
+    const size_t q_slot = q_stride > 0 ? static_cast<size_t>(q_stride) / 16
+                                       : static_cast<size_t>(n_tokens) * c.batch * c.num_q_heads * kVecPerRow;
+    const size_t kv_slot = kv_stride > 0 ? static_cast<size_t>(kv_stride) / 16
+                                         : static_cast<size_t>(n_tokens) * c.batch * c.num_kv_heads * kVecPerRow;
     for (int z0 = 0; z0 < n_layers; z0 += kMaxLayerBatch) {
         const int nz = n_layers - z0 < kMaxLayerBatch ? n_layers - z0 : kMaxLayerBatch;
         AppendParams p;
         p.q = static_cast<const uint4*>(q) + z0 * q_slot;
         p.k = static_cast<const uint4*>(k) + z0 * kv_slot;
         p.v = static_cast<const uint4*>(v) + z0 * kv_slot;
+        p.q_stride = static_cast<int64_t>(q_slot);
+        p.kv_stride = static_cast<int64_t>(kv_slot);
         p.qwin = static_cast<uint4*>(ctx->bufs.q_window);
         p.kc = static_cast<uint4*>(ctx->bufs.k_cache);
         p.vc = static_cast<uint4*>(ctx->bufs.v_cache);
@@ -651,6 +658,16 @@ int vase_append_all(vase_ctx* ctx, const void* q, const void* k, const void* v, 
     std::vector<int32_t> all(static_cast<size_t>(ctx->cfg.num_layers));
     for (int32_t l = 0; l < ctx->cfg.num_layers; ++l) all[l] = l;
     return append_batch(ctx, all.data(), ctx->cfg.num_layers, q, k, v, n_tokens, static_cast<cudaStream_t>(stream));
+}
+
+int vase_append_all_strided(vase_ctx* ctx, const void* q, const void* k, const void* v, int32_t n_tokens,
+                            int64_t q_layer_stride, int64_t kv_layer_stride, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (q_layer_stride <= 0 || kv_layer_stride <= 0) return fail(ctx, VASE_ERR_INVALID, "layer strides must be > 0");
+    std::vector<int32_t> all(static_cast<size_t>(ctx->cfg.num_layers));
+    for (int32_t l = 0; l < ctx->cfg.num_layers; ++l) all[l] = l;
+    return append_batch(ctx, all.data(), ctx->cfg.num_layers, q, k, v, n_tokens, static_cast<cudaStream_t>(stream),
+                        q_layer_stride, kv_layer_stride);
 }
 
 namespace {

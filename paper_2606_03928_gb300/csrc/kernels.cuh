@@ -78,9 +78,10 @@ struct LayerBatch {
 };
 
 struct AppendParams {
-    const uint4* q;   // [slot][n][b][Hq][16]
-    const uint4* k;   // [slot][n][b][Hkv][16]
+    const uint4* q;   // [slot][n][b][Hq][16], layer slots q_stride apart
+    const uint4* k;   // [slot][n][b][Hkv][16], layer slots kv_stride apart
     const uint4* v;
+    int64_t q_stride, kv_stride;  // 16-byte vectors between consecutive layer slots' inputs
     uint4* qwin;      // base of [L][b][Hq][W][16]
     uint4* kc;        // base of [L][b][Hkv][N][16]
     uint4* vc;

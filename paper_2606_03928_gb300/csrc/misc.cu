@@ -90,9 +90,9 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
     int32_t* const pos = p.pos + unit0 * N;
     float* const vmag = p.vmag + unit0 * N;
     uint4* const qwin = p.qwin + (static_cast<int64_t>(layer) * p.b + s) * Hq * W * kVecPerRow;
-    const uint4* const qin = p.q + static_cast<int64_t>(z) * p.n * p.b * Hq * kVecPerRow;
-    const uint4* const kin = p.k + static_cast<int64_t>(z) * p.n * units * kVecPerRow;
-    const uint4* const vin = p.v + static_cast<int64_t>(z) * p.n * units * kVecPerRow;
+    const uint4* const qin = p.q + static_cast<int64_t>(z) * p.q_stride;
+    const uint4* const kin = p.k + static_cast<int64_t>(z) * p.kv_stride;
+    const uint4* const vin = p.v + static_cast<int64_t>(z) * p.kv_stride;
     for (int t = t0; t < t1; ++t) {
         const bool q_lives = t >= p.n - W;
         const int per = (2 * Hkv + (q_lives ? Hq : 0)) * 16;  // 16-byte vectors of this step

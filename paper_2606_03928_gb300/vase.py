@@ -38,7 +38,7 @@ EXPORTED = [
     "vase_append_host", "vase_evict", "vase_read_positions", "vase_get_layer_state", "vase_set_layer_state",
     "vase_kv_view_get", "vase_debug_view_get", "vase_check_device_error", "vase_launch_count",
     "vase_status_string", "vase_last_error", "vase_abi_version", "vase_profile_enable", "vase_profile_collect",
-    "vase_append_all", "vase_evict_all", "vase_refresh_value_scores", "vase_evict_static_scratch",
+    "vase_append_all", "vase_append_all_strided", "vase_evict_all", "vase_refresh_value_scores", "vase_evict_static_scratch",
     "vase_decode_attention", "vase_mixed_buffer_sizes", "vase_quantize_values", "vase_decode_attention_mixed",
 ]
 KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "compact"]
@@ -103,6 +103,7 @@ def load(path: str = LIB_PATH):
         "vase_append": (ctypes.c_int, [P, I32, P, P, P, I32, P]),
         "vase_append_host": (ctypes.c_int, [P, I32, P, P, P, I32, P]),
         "vase_append_all": (ctypes.c_int, [P, P, P, P, I32, P]),
+        "vase_append_all_strided": (ctypes.c_int, [P, P, P, P, I32, I64, I64, P]),
         "vase_evict": (ctypes.c_int, [P, I32, P]),
         "vase_evict_all": (ctypes.c_int, [P, P]),
         "vase_refresh_value_scores": (ctypes.c_int, [P, I32, P]),
@@ -195,6 +196,12 @@ def vase_append_host(ctx, layer, q_ptr, k_ptr, v_ptr, n_tokens, stream=None):
 def vase_append_all(ctx, q_ptr, k_ptr, v_ptr, n_tokens, stream=None):
     return _check(ctx, load().vase_append_all(ctx, q_ptr, k_ptr, v_ptr, n_tokens, _stream_ptr(stream)),
                   "vase_append_all")
+
+
+def vase_append_all_strided(ctx, q_ptr, k_ptr, v_ptr, n_tokens, q_layer_stride, kv_layer_stride, stream=None):
+    return _check(ctx, load().vase_append_all_strided(ctx, q_ptr, k_ptr, v_ptr, n_tokens, q_layer_stride,
+                                                      kv_layer_stride, _stream_ptr(stream)),
+                  "vase_append_all_strided")
 
 
 def vase_evict(ctx, layer, stream=None):

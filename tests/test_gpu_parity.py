@@ -407,6 +407,47 @@ def test_append_all_equals_per_layer_appends():
         assert a.layer_state(layer) == b.layer_state(layer)
 
 
+def test_append_all_strided_from_one_staging_block_equals_packed_append_all():
+    """vase_append_all_strided over a staging buffer that holds, per layer, only [last W query rows | k | v]
+    (q pointers W rows before each tail, one block between layers) writes exactly what vase_append_all writes
+    from packed [L][n] inputs: the rows before each layer's query tail belong to the previous block and are
+    never read."""
+    from paper_2606_03928_gb300 import vase as V
+    L, n = 3, 40
+    wl = W.shrink(SMALL, budget_k=64, buffer_b=16, window=8, batch=2, num_layers=L)
+    a, b = _cache(wl, L), _cache(wl, L)
+    dev = a.device
+    chunks = [W.stream_chunk(wl, 9, layer, 0, n) for layer in range(L)]
+    qs = [PU.bits_to_bf16_tensor(c["q_bits"], dev) for c in chunks]
+    ks = [PU.bits_to_bf16_tensor(c["k_bits"], dev) for c in chunks]
+    vs = [PU.bits_to_bf16_tensor(c["v_bits"], dev) for c in chunks]
+    a.append_all(torch.stack(qs), torch.stack(ks), torch.stack(vs))
+    Wq = wl.window
+    q_row = qs[0][0].numel()
+    kv_el = ks[0].numel()
+    pad = (n - Wq) * q_row
+    blk = Wq * q_row + 2 * kv_el
+    flat = torch.full((pad + L * blk,), float("nan"), dtype=torch.bfloat16, device=dev)
+    for layer in range(L):
+        o = pad + layer * blk
+        flat[o:o + Wq * q_row] = qs[layer][n - Wq:].reshape(-1)
+        flat[o + Wq * q_row:o + Wq * q_row + kv_el] = ks[layer].reshape(-1)
+        flat[o + Wq * q_row + kv_el:o + blk] = vs[layer].reshape(-1)
+    base = flat.data_ptr()
+    with pytest.raises(V.VaseError):  # a stride that is not a multiple of 16 bytes: nothing is written
+        V.vase_append_all_strided(b.ctx, base, base + 2 * (pad + Wq * q_row), base + 2 * (pad + Wq * q_row + kv_el),
+                                  n, 2 * blk + 2, 2 * blk)
+    V.vase_append_all_strided(b.ctx, base, base + 2 * (pad + Wq * q_row), base + 2 * (pad + Wq * q_row + kv_el),
+                              n, 2 * blk, 2 * blk)
+    torch.cuda.synchronize()
+    assert torch.equal(a.k_cache[:, :, :, :n], b.k_cache[:, :, :, :n])
+    assert torch.equal(a.v_cache[:, :, :, :n], b.v_cache[:, :, :, :n])
+    assert torch.equal(a.q_window, b.q_window) and torch.equal(a.positions, b.positions)
+    assert torch.equal(a.value_scores[..., :n], b.value_scores[..., :n])
+    for layer in range(L):
+        assert a.layer_state(layer) == b.layer_state(layer)
+
+
 # ----------------------------------------------------------------------------- interleaved (persistent) schedule
 
 @pytest.mark.parametrize("K,B,Wn,Hq,Hkv", [(192, 64, 16, 16, 8), (200, 40, 16, 16, 8), (256, 64, 32, 32, 8),

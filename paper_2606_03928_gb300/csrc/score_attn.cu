@@ -135,7 +135,11 @@ __device__ __forceinline__ bool phase_tile(int t, int nA, int nB, int lead, int&
 
 // kHeadMax: GQA max-aggregation (per-head sums in pass B, the largest kept); a template argument so that the
 // default mean keeps its pass-B loop free of the head bookkeeping.
-template <bool kHeadMax>
+// kEarly: with two accumulator buffers (one per group) the next MMA into a buffer waits for its consumer, so
+// the buffer is released as soon as the item's last TMEM load has landed; with four, each group already has a
+// second buffer in flight and the release follows the item's arithmetic (measured faster there).  A template
+// argument so that each form compiles to its own loop.
+template <bool kHeadMax, bool kEarly>
 __global__ void __launch_bounds__(kThreads, 1)
     score_attn_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
                       const ScoreAttnParams p) {
@@ -427,6 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int c0 = copy * cw;
         float* pmg = pm + grp * n_rbA * 128;
         float* plg = pl + grp * n_rbA * 128;
+        constexpr bool early = kEarly;
         int st_pos = 0;  // K stage ring position
         int item = 0;    // accumulator counter
         for (int k = 0; k <= n_w; ++k) {
@@ -468,6 +473,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     v[q + 32] = -INFINITY;
                                 }
                             }
+                            if (early && c + 64 >= cw) {  // the item's last load has landed
+                                tc_fence_before();
+                                mbar_arrive(&t_empty[buf]);
+                            }
                             const int nvalid = min(width, p.N - (tok0 + c0 + c));
                             if (nvalid < 64) {
 #pragma unroll
@@ -498,8 +507,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                         pmg[sub * 128 + L] = m;
                         plg[sub * 128 + L] = l;
-                        tc_fence_before();
-                        mbar_arrive(&t_empty[buf]);
+                        if (!early) {
+                            tc_fence_before();
+                            mbar_arrive(&t_empty[buf]);
+                        }
                     }
                 } else {
                     // ------------------------------------ pass B: per-token accumulation
@@ -540,16 +551,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 }
                                 acc += (a0 + a1) + (a2 + a3);
                             };
+                            // (early) the accumulator is released as soon as its last chunk is in registers
+                            auto release = [&]() {
+                                if (!early) return;
+                                tc_fence_before();
+                                mbar_arrive(&t_empty[buf]);
+                            };
                             tmem_ld32_issue(col0, ra);
                             tmem_wait_ld32(ra);
+                            if (nch == 1) release();
                             for (int ch = 0; ch < nch; ch += 2) {
                                 if (ch + 1 < nch) tmem_ld32_issue(col0 + 32 * (ch + 1), rb);
                                 sum32(ra, 32 * ch);
                                 if (ch + 1 < nch) {
                                     tmem_wait_ld32(rb);
                                     if (ch + 2 < nch) tmem_ld32_issue(col0 + 32 * (ch + 2), ra);
+                                    else release();  // rb holds the last chunk
                                     sum32(rb, 32 * (ch + 1));
-                                    if (ch + 2 < nch) tmem_wait_ld32(ra);
+                                    if (ch + 2 < nch) {
+                                        tmem_wait_ld32(ra);
+                                        if (ch + 3 >= nch) release();  // ra holds the last chunk
+                                    }
                                 }
                             }
                         } else {
@@ -568,6 +590,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                                 for (int q = 0; q < 32; ++q) v[q] = h[q];
                             }
+                            if (early && c + 64 >= NB) {  // the item's last load has landed
+                                tc_fence_before();
+                                mbar_arrive(&t_empty[buf]);
+                            }
                             const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
 #pragma unroll
                             for (int q = 0; q < 16; ++q) {
@@ -585,8 +611,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                         acc = fmaxf(acc, head_sum);
                         }
-                        tc_fence_before();
-                        mbar_arrive(&t_empty[buf]);
+                        if (!early) {
+                            tc_fence_before();
+                            mbar_arrive(&t_empty[buf]);
+                        }
                     }
                     // no item in the last pass-B tile: the group's last one (if any) was waited for earlier
                     if (!mine && owned_b && j == nB - 1 && k + 1 < n_w)
@@ -655,7 +683,8 @@ size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int clu
 }
 
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster) {
-    for (auto fn : {score_attn_kernel<false>, score_attn_kernel<true>}) {
+    for (auto fn : {score_attn_kernel<false, false>, score_attn_kernel<true, false>, score_attn_kernel<false, true>,
+                    score_attn_kernel<true, true>}) {
         cudaError_t e =
             cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem_bytes));
         if (e == cudaSuccess && cluster > 8) e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
@@ -678,8 +707,11 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return p.head_rows > 0 ? cudaLaunchKernelEx(&cfg, score_attn_kernel<true>, kmap, qmap, p)
-                           : cudaLaunchKernelEx(&cfg, score_attn_kernel<false>, kmap, qmap, p);
+    if (p.nbuf == 2)
+        return p.head_rows > 0 ? cudaLaunchKernelEx(&cfg, score_attn_kernel<true, true>, kmap, qmap, p)
+                               : cudaLaunchKernelEx(&cfg, score_attn_kernel<false, true>, kmap, qmap, p);
+    return p.head_rows > 0 ? cudaLaunchKernelEx(&cfg, score_attn_kernel<true, false>, kmap, qmap, p)
+                           : cudaLaunchKernelEx(&cfg, score_attn_kernel<false, false>, kmap, qmap, p);
 }
 
 }  // namespace vase

@@ -1,4 +1,4 @@
-"""GPU parity of the mixed-precision values (SURVEY NEXT-4): the per-token b-bit quantizer of Sec. 4.4 with
+"""GPU parity of the mixed-precision values: the per-token b-bit quantizer of Sec. 4.4 with
 the reserved cache of Sec. 6 (R_V and R_B keep bf16), and the decode attention that reads the other values
 from their codes, against the fp64 oracle.
 

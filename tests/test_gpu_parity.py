@@ -515,7 +515,7 @@ def test_qwen3_1p7b_k2048_all_layers_in_one_launch():
                               variant="attnv", n_v=wl.budget_k // 4, check_scores=False)
 
 
-# ----------------------------------------------------------------------------- variants
+# ----------------------------------------------------------------------------- variants: GQA max-aggregation, shared-G DKV, random reservation
 
 def _reserved_slots(key_row, K):
     """R_V of a unit from the debug keys: the candidates' keys are >= 0, the reserved slots carry -1."""

@@ -414,7 +414,7 @@ def test_unit_state_bits_roundtrip_through_oracle():
     assert res["keep"].sum() == 32
 
 
-# --------------------------------------------------------------------------- variants
+# --------------------------------------------------------------------------- variants: GQA max-aggregation, shared-G DKV, random reservation
 
 def test_gqa_max_closed_form_two_heads_two_dominant_keys():
     """Head 0 looks only at key 0, head 1 only at key 1 (logit gap 400/sqrt(d)): the mean over the

@@ -15,6 +15,8 @@ using namespace vase;
 namespace {
 
 constexpr size_t kMaxDynSmem = 232448;  // 227 KB per block on sm_100-class GPUs
+constexpr size_t kSmemPerSm = 233472;   // 228 KB per SM
+constexpr size_t kSmemReservedPerBlock = 1024;  // the system's share of each block's shared memory
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -192,7 +194,16 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     p.dkv_smem = dkv_smem_bytes(p.dkv_stages);
     {
         const int n_parts = c->variant == VASE_VARIANT_ATTNV ? p.n_rb : 1;
-        p.select_staged = select_smem_bytes(p.N, c->budget_k, n_parts, true) <= kMaxDynSmem - 9216;
+        // Staged (every input of the unit copied to shared memory at once), unless that leaves one CTA per SM
+        // and reading the inputs from global memory lets two or more share it, so that one CTA's gather runs
+        // under another's selection (measured: Qwen3-32B geometry 1807 -> 1675 us per eight layers; at two
+        // staged CTAs per SM, Qwen3-8B, four unstaged ones were slower).
+        auto per_sm = [](size_t smem) {
+            return kSmemPerSm / (smem + select_static_smem_bytes() + kSmemReservedPerBlock);
+        };
+        const size_t s_staged = select_smem_bytes(p.N, c->budget_k, n_parts, true);
+        const size_t s_plain = select_smem_bytes(p.N, c->budget_k, n_parts, false);
+        p.select_staged = s_staged <= kMaxDynSmem - 9216 && !(per_sm(s_staged) < 2 && per_sm(s_plain) >= 2);
         p.select_smem = select_smem_bytes(p.N, c->budget_k, n_parts, p.select_staged);
     }
     if (p.select_smem > kMaxDynSmem - 9216) {

@@ -218,6 +218,7 @@ cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, Deco
 size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages);
 size_t dkv_smem_bytes(int stages);
 size_t select_smem_bytes(int N, int K, int n_parts, bool staged);
+size_t select_static_smem_bytes();  // the selection kernel's static shared memory
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster);
 cudaError_t dkv_set_attributes(size_t smem_bytes);
 cudaError_t select_set_attributes(size_t smem_bytes);

@@ -735,6 +735,7 @@ cudaError_t launch_value_score(const ValueParams& p, int num_sms, cudaStream_t s
 }
 
 size_t select_smem_bytes(int N, int K, int n_parts, bool staged) { return sel_layout(N, K, n_parts, staged).total; }
+size_t select_static_smem_bytes() { return sizeof(SelShared); }
 
 cudaError_t select_set_attributes(size_t smem_bytes) {
     return cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -60,6 +60,11 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=None, help="steps of the host-buffer end-to-end pass")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="the Qwen3-8B-geometry sweep over K, B, batch and value-outlier rate (one JSON line, a point each)")
+    ap.add_argument("--sweep-full", action="store_true", help="with --sweep: every point of the 5 x 3 x 4 x 3 grid")
+    ap.add_argument("--sweep-gb", type=float, default=48.0,
+                    help="with --sweep: cache bytes (GB) a point may hold; the layers beyond it are left out")
     ap.add_argument("--decode", action="store_true",
                     help="time the decode-step attention over every layer's kept cache instead of the eviction step")
     return ap.parse_args()
@@ -703,6 +708,102 @@ def run_decode(args):
     return 0
 
 
+def sweep_grid(full):
+    """(K, B, batch, value-outlier rate) points of the sweep on the Qwen3-8B geometry: the whole 5 x 3 x 4 x 3
+    grid, or every (K, B) pair at batch 32 and rate 0.5 % plus the batch and rate axes through K 4096, B 128."""
+    Ks, Bs, bs, rates = (1024, 2048, 4096, 8192, 16384), (32, 128, 512), (1, 8, 32, 128), (0.0, 0.005, 0.02)
+    if full:
+        return [(K, B, b, r) for K in Ks for B in Bs for b in bs for r in rates]
+    pts = [(K, B, 32, 0.005) for K in Ks for B in Bs]
+    pts += [(4096, 128, b, 0.005) for b in (1, 8, 128)]
+    pts += [(4096, 128, 32, r) for r in (0.0, 0.02)]
+    return pts
+
+
+def run_sweep(args):
+    """The eviction step (append B tokens to every layer, evict every layer) at each sweep point, on as many
+    of the 36 layers as fit in --sweep-gb of cache (a resident subset: all 36 at most points; the step of a
+    point covers the same number of layers every time, so per-layer-round figures compare across points)."""
+    import torch
+
+    torch.cuda.set_device(0)
+    device = torch.device("cuda", 0)
+    from paper_2606_03928_gb300 import workloads as Wm
+    from paper_2606_03928_gb300 import build as B
+    B.build()
+    from paper_2606_03928_gb300 import vase as V
+
+    hbm_peak, _, peak_kind = measured_peaks()
+    stream = torch.cuda.current_stream()
+    points = []
+    launches = 0
+    for (K, Bf, b, rate) in sweep_grid(args.sweep_full):
+        wl = Wm.sweep_point(K, Bf, b, rate)
+        units = wl.batch * wl.num_kv_heads
+        per_layer = units * wl.slots * (2 * 2 * wl.head_dim + 8) + wl.batch * wl.num_q_heads * wl.window * 2 * wl.head_dim
+        L = max(1, min(wl.num_layers, int(args.sweep_gb * 1e9 // per_layer)))
+        wl = Wm.shrink(wl, num_layers=L)
+        cache = V.VaseCache(V.Geometry(K, Bf, wl.window, wl.num_q_heads, wl.num_kv_heads, L, wl.batch),
+                            variant="attnv", seed=0, device=device)
+        gen = torch.Generator(device=device)
+        gen.manual_seed(1000)
+        for layer in range(L):  # prefill in pieces of at most 1024 tokens (bounded generator temporaries)
+            for t0 in range(0, K, 1024):
+                cache.append(layer, *gen_stream(wl, min(1024, K - t0), gen, device, torch))
+        per_layer_new = [gen_stream(wl, Bf, gen, device, torch) for _ in range(L)]
+        chunk = tuple(torch.stack([pl[i] for pl in per_layer_new]) for i in range(3))
+        del per_layer_new
+
+        def step():
+            cache.append_all(*chunk)
+            cache.evict_all()
+
+        for _ in range(3):
+            step()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        n_steps = max(5, min(100, int(100.0 / max(e0.elapsed_time(e1), 1e-3))))  # about 0.1 s of steps
+        sampler = ClockSampler(0)
+        sampler.start()
+        l0 = cache.launch_count()
+        e0.record(stream)
+        for _ in range(n_steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        clocks = sampler.stop()
+        launches += cache.launch_count() - l0
+        st, code = cache.check_device_error()
+        if st != 0:
+            raise RuntimeError(f"device error at sweep point K={K} B={Bf} b={b} rate={rate}: {code:#x}")
+        ms = e0.elapsed_time(e1) / n_steps
+        roof_ms = L * step_bytes(wl, "attnv") / (hbm_peak * 1e9) * 1e3
+        points.append({"budget_k": K, "buffer_b": Bf, "batch": b, "value_outlier_rate": rate, "layers": L,
+                       "steps": n_steps, "ms_per_step": round(ms, 4),
+                       "token_heads_per_s": L * units * wl.slots / (ms / 1e3),
+                       "sequence_tokens_per_s": L * wl.batch * wl.slots / (ms / 1e3),
+                       "step_roofline_ms": round(roof_ms, 4), "roofline_frac": round(roof_ms / ms, 4),
+                       # the whole step (B appends + the eviction) of these L layers over the B decode steps it serves
+                       "step_us_per_decode_token": round(1e3 * ms / Bf, 3), "clocks": clocks})
+        del cache, chunk
+        torch.cuda.empty_cache()
+    ref = next(p for p in points if (p["budget_k"], p["buffer_b"], p["batch"], p["value_outlier_rate"]) ==
+               (4096, 128, 32, 0.005))
+    outj = {"metric": METRIC + " over the Qwen3-8B-geometry sweep", "value": ref["token_heads_per_s"], "unit": UNIT,
+            "n_gpus": 1, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic", "value_at": "K 4096, B 128, batch 32, 0.5 % outliers",
+            "config": {"workload": "qwen3_8b_sweep", "heads": "32/8", "window": 32, "variant": "attnv",
+                       "grid": "full" if args.sweep_full else "axes", "cache_gb_per_point": args.sweep_gb,
+                       "parallelism": "dp1"},
+            "peak": hbm_peak, "peak_source": peak_kind, "gpu_launches": launches, "points": points}
+    print(json.dumps(outj))
+    return 0
+
+
 def variant_options(args):
     """The non-default variant switches of a run, for the config object of its JSON line."""
     opts = {}
@@ -719,6 +820,8 @@ def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.sweep:
+        return run_sweep(args)
     if args.decode:
         return run_decode(args)
     return run_ours(args)

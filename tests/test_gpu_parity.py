@@ -347,6 +347,17 @@ def test_qwen3_8b_k4096_dkv_sampled_units():
     _run_layer(wl, variant="dkv", layer=2, num_layers=4, round_index=77, units=units, debug=False)
 
 
+@pytest.mark.parametrize("K,B,b,rate,units", [
+    (16384, 512, 1, 0.005, [(0, 0), (0, 5)]),             # the sweep's largest unit: N = 16896, unstaged selection
+    (1024, 32, 128, 0.02, [(0, 0), (77, 3), (127, 7)]),   # smallest budget and buffer, largest batch, most outliers
+    (2048, 128, 8, 0.0, [(0, 2), (7, 7)]),                 # no value outliers: the reservation takes ordinary rows
+])
+def test_qwen3_8b_sweep_points_sampled_units(K, B, b, rate, units):
+    """Points of the Qwen3-8B-geometry sweep (32/8 heads, W = 32) at its extremes, sampled units against the oracle."""
+    wl = W.sweep_point(K, B, b, rate)
+    _run_layer(wl, layer=0, num_layers=1, round_index=5, units=units, debug=False)
+
+
 def test_qwen3_32b_k8192_sampled_units():
     wl = W.WORKLOADS["qwen3_32b_k8192"]
     units = [(0, 0), (7, 5), (15, 7)]

@@ -207,7 +207,7 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
         p.select_smem = select_smem_bytes(p.N, c->budget_k, n_parts, p.select_staged);
     }
     if (p.select_smem > kMaxDynSmem - 9216) {
-        *why = "K + B too large for the single-CTA selection (its shared memory holds about 16.6k slots)";
+        *why = "K + B too large for the single-CTA selection (its shared memory holds about 17k slots)";
         return false;
     }
 

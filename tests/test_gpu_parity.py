@@ -622,8 +622,8 @@ def test_dkv_shared_g_matches_oracle_and_is_shared():
 # ----------------------------------------------------------------------------- maximum sizes and degenerate cases
 
 def test_largest_supported_unit_matches_oracle():
-    """K = 16384, B = 256: the largest budget the single-CTA selection holds (unstaged inputs), one unit, the
-    score kernel in cluster mode; every slot checked against the oracle."""
+    """K = 16384, B = 256 (N = 16640, inputs read unstaged by the single-CTA selection), one unit, the score
+    kernel in cluster mode; every slot checked against the oracle (the sweep test samples N = 16896)."""
     wl = W.shrink(SMALL, budget_k=16384, buffer_b=256, window=16, num_q_heads=4, num_kv_heads=1, batch=1,
                   num_layers=1)
     _run_layer(wl, layer=0, num_layers=1, round_index=4)

@@ -32,6 +32,7 @@ struct Plan {
     size_t dkv_smem;
     size_t select_smem;
     bool select_staged;
+    int select_threads;
     // workspace
     int slots;  // layers one launch can batch
     size_t stride_attn, stride_un, stride_src;  // elements per workspace slot
@@ -205,6 +206,9 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
         const size_t s_plain = select_smem_bytes(p.N, c->budget_k, n_parts, false);
         p.select_staged = s_staged <= kMaxDynSmem - 9216 && !(per_sm(s_staged) < 2 && per_sm(s_plain) >= 2);
         p.select_smem = select_smem_bytes(p.N, c->budget_k, n_parts, p.select_staged);
+        // threads per CTA: 1024 when one CTA holds an SM, 512 for two, 256 (four) otherwise
+        const size_t ctas = per_sm(p.select_smem);
+        p.select_threads = ctas <= 1 ? 1024 : (ctas == 2 ? 512 : 256);
     }
     if (p.select_smem > kMaxDynSmem - 9216) {
         *why = "K + B too large for the single-CTA selection (its shared memory holds about 17k slots)";
@@ -643,7 +647,7 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
     sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
     sel.err = err;
-    if ((e = timed_launch(ctx, VASE_KERNEL_SELECT, s, [&] { return launch_select(sel, P.units, P.select_smem, s); })) !=
+    if ((e = timed_launch(ctx, VASE_KERNEL_SELECT, s, [&] { return launch_select(sel, P.units, P.select_smem, P.select_threads, s); })) !=
         cudaSuccess)
         return cuda_fail(ctx, e, "select launch");
     ctx->launches += 1;
@@ -1212,7 +1216,7 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
     sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
     sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
     sel.err = err;
-    if ((e = launch_select(sel, P.units, P.select_smem, s)) != cudaSuccess) {
+    if ((e = launch_select(sel, P.units, P.select_smem, P.select_threads, s)) != cudaSuccess) {
         g_config_error = std::string("select launch: ") + cudaGetErrorString(e);
         return VASE_ERR_CUDA;
     }

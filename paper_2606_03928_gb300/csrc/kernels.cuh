@@ -208,7 +208,7 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
                               size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
                        size_t smem_bytes, cudaStream_t s);
-cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s);
+cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, int threads, cudaStream_t s);
 cudaError_t launch_quantize(const QuantParams& p, int units, size_t smem_bytes, cudaStream_t s);
 size_t quantize_smem_bytes(int K, int B);
 cudaError_t quantize_set_attributes(size_t smem_bytes);

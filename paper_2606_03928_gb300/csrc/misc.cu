@@ -161,14 +161,16 @@ constexpr int kSelBins = 256;
 
 struct SelShared {
     uint32_t hist[kSelBins];
-    int warp_tot[kSelWarps];
+    int warp_tot[32];  // one per warp of the block (up to 1024 threads)
     uint32_t bcast[4];
     int first_evicted;  // lowest evicted slot (slots below it keep their place)
 };
 
 // Exclusive prefix over threads of `v` in thread order; returns the offset and
-// writes the block total to *total.  Every thread must call it.
+// writes the block total to *total.  Every thread of the kT-thread block must call it.
+template <int kT = kSelThreads>
 __device__ __forceinline__ int block_exclusive_scan(int v, SelShared& sh, int* total) {
+    constexpr int kW = kT / 32;
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     int x = v;
@@ -180,15 +182,15 @@ __device__ __forceinline__ int block_exclusive_scan(int v, SelShared& sh, int* t
     if (lane == 31) sh.warp_tot[warp] = x;
     __syncthreads();
     if (warp == 0) {
-        int w = lane < kSelWarps ? sh.warp_tot[lane] : 0;
+        int w = lane < kW ? sh.warp_tot[lane] : 0;
         int inc = w;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int y = __shfl_up_sync(0xffffffffu, inc, o);
             if (lane >= o) inc += y;
         }
-        if (lane < kSelWarps) sh.warp_tot[lane] = inc - w;  // exclusive warp offsets
-        if (lane == kSelWarps - 1) sh.bcast[3] = static_cast<uint32_t>(inc);
+        if (lane < kW) sh.warp_tot[lane] = inc - w;  // exclusive warp offsets
+        if (lane == kW - 1) sh.bcast[3] = static_cast<uint32_t>(inc);
     }
     __syncthreads();
     const int off = sh.warp_tot[warp] + x - v;
@@ -201,19 +203,21 @@ __device__ __forceinline__ int block_exclusive_scan(int v, SelShared& sh, int* t
 // index), by an MSB-first radix select on four 8-bit digits (lanes with the
 // same digit are merged with __match_any_sync before the shared-memory atomic)
 // followed by a slot-ordered rank of the elements equal to the threshold.
-// Each thread owns the contiguous slots [seg_lo, seg_hi).
+// Each thread of the kT-thread block owns the contiguous slots [seg_lo, seg_hi).
+template <int kT = kSelThreads>
 __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, uint8_t flag, int seg_lo,
                             int seg_hi, SelShared& sh) {
+    static_assert(kT >= kSelBins, "a thread per histogram bin");
     if (k <= 0) return;
     const int tid = threadIdx.x;
     const int lane = tid & 31;
     uint32_t prefix = 0, mask = 0;
     int remain = k;
     for (int shift = 24; shift >= 0; shift -= 8) {
-        sh.hist[tid] = 0;  // kSelThreads == kSelBins
+        if (tid < kSelBins) sh.hist[tid] = 0;
         __syncthreads();
         const int n_round = (n + 31) & ~31;
-        for (int i = tid; i < n_round; i += kSelThreads) {
+        for (int i = tid; i < n_round; i += kT) {
             const uint32_t x = i < n ? ord[i] : 0u;
             const bool in = i < n && (x & mask) == prefix;
             const uint32_t bin = in ? ((x >> shift) & 0xFFu) : 0xFFFFFFFFu;
@@ -258,7 +262,7 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
     int eq = 0;
     for (int i = seg_lo; i < seg_hi; ++i) eq += ord[i] == thr;
     int total;
-    int rank = block_exclusive_scan(eq, sh, &total);
+    int rank = block_exclusive_scan<kT>(eq, sh, &total);
     for (int i = seg_lo; i < seg_hi; ++i) {
         const uint32_t x = ord[i];
         bool take = x > thr;
@@ -430,7 +434,10 @@ __device__ void gather_rows(uint8_t* base, const int32_t* src, int j_first, int 
     __syncwarp();
 }
 
-__global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectParams p) {
+// kT threads per CTA: 256 where four CTAs share an SM; 512 or 1024 where the unit's arrays leave room for two
+// or one, so that the selection phase, which no other CTA's gather hides there, runs on as many warps.
+template <int kT>
+__global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParams p) {
     extern __shared__ __align__(16) uint8_t smem_raw[];
     __shared__ SelShared sh;
     const int N = p.N, K = p.K;
@@ -455,7 +462,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
     float* const pooled_dbg = p.pooled_dbg ? p.pooled_dbg + zs : nullptr;
     float* const key_dbg = p.key_dbg ? p.key_dbg + zs : nullptr;
     uint8_t* const keep_dbg = p.keep_dbg ? p.keep_dbg + zs : nullptr;
-    const int seg = (N + kSelThreads - 1) / kSelThreads;
+    const int seg = (N + kT - 1) / kT;
     const int seg_lo = min(N, tid * seg);
     const int seg_hi = min(N, seg_lo + seg);
     const int kseg_lo = min(K, seg_lo);
@@ -475,7 +482,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
         cp_async_words(vm_s, vmag + base, N);
         cp_async_words(pos_s, pos + base, N);
     }
-    for (int i = tid; i < N; i += kSelThreads) flags[i] = 0;
+    for (int i = tid; i < N; i += kT) flags[i] = 0;
     if (tid == 0) sh.first_evicted = K;
     if (staged) {
         cp_async_wait_all();
@@ -484,7 +491,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
     if (p.variant == 0) {
         if (staged) {
             if (p.n_parts > 1) {
-                for (int i = tid; i < N; i += kSelThreads) {
+                for (int i = tid; i < N; i += kT) {
                     float a = a_s[i];
                     for (int part = 1; part < p.n_parts; ++part)
                         a = p.gqa_max ? fmaxf(a, a_s[part * N + i]) : a + a_s[part * N + i];
@@ -492,7 +499,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
                 }
             }
         } else {
-            for (int i = tid; i < N; i += kSelThreads) {
+            for (int i = tid; i < N; i += kT) {
                 float a = attn[base + i];
                 for (int part = 1; part < p.n_parts; ++part) {
                     const float b = attn[(static_cast<int64_t>(part) * p.units + unit) * N + i];
@@ -503,10 +510,10 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
         }
         if (p.n_parts > 1 && pooled_dbg) {
             __syncthreads();
-            for (int i = tid; i < N; i += kSelThreads) const_cast<float*>(attn)[base + i] = a_s[i];
+            for (int i = tid; i < N; i += kT) const_cast<float*>(attn)[base + i] = a_s[i];
         }
         const uint32_t c2_res = static_cast<uint32_t>(layer) | (kTagReserve << 24);
-        for (int i = tid; i < K; i += kSelThreads) {
+        for (int i = tid; i < K; i += kT) {
             const float vm = staged ? vm_s[i] : vmag[base + i];
             if (p.reserve_random) {  // the N_v largest reservation uniforms: a uniformly random N_v-subset
                 const int32_t pi = staged ? pos_s[i] : pos[base + i];
@@ -520,12 +527,12 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
             if (vscore_dbg) vscore_dbg[base + i] = vm;
         }
         __syncthreads();
-        radix_top_k(ord, K, p.n_v, flags, kFlagValue, kseg_lo, kseg_hi, sh);
+        radix_top_k<kT>(ord, K, p.n_v, flags, kFlagValue, kseg_lo, kseg_hi, sh);
         // keys over the candidates C
         const int h = p.pool / 2;
         const float inv_pool = 1.0f / static_cast<float>(p.pool);
         const uint32_t c2 = static_cast<uint32_t>(layer) | (kTagSelect << 24);
-        for (int i = tid; i < N; i += kSelThreads) {
+        for (int i = tid; i < N; i += kT) {
             float sum = 0.f;
             const int lo = max(0, i - h), hi = min(N - 1, i + h);
             for (int j = lo; j <= hi; ++j) sum += a_s[j];
@@ -550,27 +557,27 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
             if (key_dbg) key_dbg[base + i] = key;
         }
         __syncthreads();
-        radix_top_k(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
+        radix_top_k<kT>(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
     } else {
-        for (int i = tid; i < K; i += kSelThreads) {
+        for (int i = tid; i < K; i += kT) {
             const float s = staged ? a_s[i] : dkv[base + i];
             ord[i] = __float_as_uint(s) + 1u;
             if (key_dbg) key_dbg[base + i] = s;
         }
         __syncthreads();
-        radix_top_k(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
+        radix_top_k<kT>(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
     }
     // positions move with the kept rows (unstaged: copy the old ones into shared memory, a_s is free now)
     if (!staged) {
         pos_s = reinterpret_cast<int32_t*>(a_s);
-        for (int i = tid; i < N; i += kSelThreads) pos_s[i] = pos[base + i];
+        for (int i = tid; i < N; i += kT) pos_s[i] = pos[base + i];
     }
     // keep = R_B u R_V u sampled; ascending list of kept slots (also kept in shared memory for the gather)
     int32_t* src_s = reinterpret_cast<int32_t*>(smem_raw + Ly.src_off);
     int cnt = 0;
     for (int i = seg_lo; i < seg_hi; ++i) cnt += (i >= K) || flags[i];
     int total;
-    const int dst0 = block_exclusive_scan(cnt, sh, &total);  // also a barrier after the staging above
+    const int dst0 = block_exclusive_scan<kT>(cnt, sh, &total);  // also a barrier after the staging above
     int dst = dst0;
     int first_ev = K;
     for (int i = seg_lo; i < seg_hi; ++i) {
@@ -589,12 +596,12 @@ __global__ void __launch_bounds__(kSelThreads, 4) select_kernel(const SelectPara
         if (key_dbg && i >= K) key_dbg[base + i] = -1.f;
     }
     if (first_ev < K) atomicMin(&sh.first_evicted, first_ev);
-    for (int i = K + tid; i < N; i += kSelThreads) pos[base + i] = -1;
+    for (int i = K + tid; i < N; i += kT) pos[base + i] = -1;
     // value magnitudes move with their rows too
     if (!staged) {
         __syncthreads();
         vm_s = a_s;
-        for (int i = tid; i < N; i += kSelThreads) vm_s[i] = vmag[base + i];
+        for (int i = tid; i < N; i += kT) vm_s[i] = vmag[base + i];
         __syncthreads();
     }
     dst = dst0;
@@ -738,8 +745,12 @@ size_t select_smem_bytes(int N, int K, int n_parts, bool staged) { return sel_la
 size_t select_static_smem_bytes() { return sizeof(SelShared); }
 
 cudaError_t select_set_attributes(size_t smem_bytes) {
-    return cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                static_cast<int>(smem_bytes));
+    for (auto fn : {select_kernel<256>, select_kernel<512>, select_kernel<1024>}) {
+        const cudaError_t e =
+            cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem_bytes));
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 size_t quantize_smem_bytes(int K, int B) {
@@ -758,8 +769,11 @@ cudaError_t launch_quantize(const QuantParams& p, int units, size_t smem_bytes, 
     return cudaGetLastError();
 }
 
-cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, cudaStream_t s) {
-    select_kernel<<<dim3(static_cast<unsigned>(units), static_cast<unsigned>(p.batch.n)), kSelThreads, smem_bytes, s>>>(p);
+cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, int threads, cudaStream_t s) {
+    const dim3 grid(static_cast<unsigned>(units), static_cast<unsigned>(p.batch.n));
+    if (threads == 1024) select_kernel<1024><<<grid, 1024, smem_bytes, s>>>(p);
+    else if (threads == 512) select_kernel<512><<<grid, 512, smem_bytes, s>>>(p);
+    else select_kernel<256><<<grid, 256, smem_bytes, s>>>(p);
     return cudaGetLastError();
 }
 

@@ -781,6 +781,13 @@ def run_sweep(args):
         if st != 0:
             raise RuntimeError(f"device error at sweep point K={K} B={Bf} b={b} rate={rate}: {code:#x}")
         ms = e0.elapsed_time(e1) / n_steps
+        # the same steps again with an event pair around every launch, for each kernel's duration
+        cache.profile_enable(True)
+        for _ in range(n_steps):
+            step()
+        torch.cuda.synchronize()
+        cache.profile_enable(False)
+        kern = {name: round(1e3 * kms / n, 1) for name, (kms, n) in cache.profile_collect().items() if n}
         roof_ms = L * step_bytes(wl, "attnv") / (hbm_peak * 1e9) * 1e3
         points.append({"budget_k": K, "buffer_b": Bf, "batch": b, "value_outlier_rate": rate, "layers": L,
                        "steps": n_steps, "ms_per_step": round(ms, 4),
@@ -788,7 +795,8 @@ def run_sweep(args):
                        "sequence_tokens_per_s": L * wl.batch * wl.slots / (ms / 1e3),
                        "step_roofline_ms": round(roof_ms, 4), "roofline_frac": round(roof_ms / ms, 4),
                        # the whole step (B appends + the eviction) of these L layers over the B decode steps it serves
-                       "step_us_per_decode_token": round(1e3 * ms / Bf, 3), "clocks": clocks})
+                       "step_us_per_decode_token": round(1e3 * ms / Bf, 3), "kernels_us_per_launch": kern,
+                       "clocks": clocks})
         del cache, chunk
         torch.cuda.empty_cache()
     ref = next(p for p in points if (p["budget_k"], p["buffer_b"], p["batch"], p["value_outlier_rate"]) ==

@@ -14,6 +14,13 @@ Metric: eviction-step KV token-heads per second = (layers * batch * Hkv * (K+B))
 per step / step time.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  python bench.py --workload qwen3_8b_k4096|qwen3_32b_k8192 [--layers L] [--variant dkv]
+  python bench.py --sweep [--sweep-full]     # the Qwen3-8B-geometry grid over K, B, batch, outlier rate
+  python bench.py --decode [--mixed-bits b]  # decode attention over the kept cache
+
+The step time of `value` is taken without per-launch events; each kernel's launch time comes from a
+second, profiled pass of the same steps.  `e2e` runs the step from pinned host buffers with the
+host-device copies inside the timed region.
 
 Under torchrun (N > 1) every rank runs the same per-GPU workload on its own GPU
 (units are independent: no collective on the data path); value is the

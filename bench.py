@@ -166,6 +166,22 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def max_over_ranks(ms, world, device):
+    """The slowest rank's time: every rank's step time, reduced by MAX over the process group (any backend)."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank, world, ms):
+    """Units processed by all ranks (the same per-rank work: weak scaling) per second of the slowest rank."""
+    return world * units_per_rank / (ms / 1e3)
+
+
 def kernel_bytes(kind, wl, variant, moved_rows_per_unit):
     """Algorithmic bytes of one kernel for one layer (a launch covers up to 64 layers)."""
     U = wl.batch * wl.num_kv_heads
@@ -408,12 +424,9 @@ def run_ours(args):
     st, code = cache.check_device_error()
     if st != 0:
         raise RuntimeError(f"device error in the timed region: {code:#x}")
-    if world > 1:
-        t = torch.tensor([ms], device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, world, device)
     token_heads = L * wl.batch * wl.num_kv_heads * wl.slots
-    value = world * token_heads / (ms / 1e3)
+    value = whole_job_rate(token_heads, world, ms)
 
     # moved rows per unit in the last eviction (rows whose slot changes) for the compaction's bytes
     src = cache.debug_view(0)["src"].cpu()
@@ -450,11 +463,7 @@ def run_ours(args):
         torch.cuda.synchronize()
         barrier()
         t_ms = e0.elapsed_time(e1) / e2e_steps
-        if world > 1:
-            t = torch.tensor([t_ms], device=device)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            t_ms = float(t.item())
-        return t_ms
+        return max_over_ranks(t_ms, world, device)
 
     e2e_step(0)
     zero_copy_ms = timed(lambda: [e2e_step(r) for r in range(e2e_steps)])
@@ -521,7 +530,7 @@ def run_ours(args):
         stream.wait_stream(copy_stream)  # the last read-back ends inside the timed region
 
     e2e_ms = timed(pipelined)
-    e2e_value = world * token_heads / (e2e_ms / 1e3)
+    e2e_value = whole_job_rate(token_heads, world, e2e_ms)
 
     # ---- roofline of the dominant kernel
     hbm_peak, _, peak_kind = measured_peaks()

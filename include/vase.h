@@ -266,6 +266,16 @@ int vase_debug_view_get(const vase_ctx* ctx, int32_t slot, vase_debug_view* out)
  * (with *code, if non-NULL, set to the raw word). */
 int vase_check_device_error(vase_ctx* ctx, void* stream, uint32_t* code);
 
+/* Self-test of the failure detection: launches on `stream` a one-thread kernel whose
+ * bounded wait on an mbarrier that nothing completes runs out (about two seconds,
+ * the wait limit of every kernel here); the kernel records VASE_SITE_SELF_TEST in
+ * the context's device error word and returns, without a fault.  A following
+ * vase_check_device_error then returns VASE_ERR_DEVICE with (code & 0xffff) ==
+ * VASE_SITE_SELF_TEST and clears the word; the context stays usable.  Returns
+ * VASE_OK once launched. */
+#define VASE_SITE_SELF_TEST 127
+int vase_self_test_wait_timeout(vase_ctx* ctx, void* stream);
+
 /* Number of kernels the library launched on this context since creation. */
 int64_t vase_launch_count(const vase_ctx* ctx);
 

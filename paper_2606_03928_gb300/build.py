@@ -20,7 +20,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libvase.so")
-SOURCES = ["api.cu", "score_attn.cu", "dkv.cu", "misc.cu", "decode.cu", "decode_mixed.cu"]
+SOURCES = ["api.cu", "score_attn.cu", "dkv.cu", "misc.cu", "decode.cu", "decode_mixed.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 

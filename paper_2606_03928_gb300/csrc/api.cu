@@ -390,6 +390,10 @@ int32_t* pos_layer(vase_ctx* c, int layer) {
 
 }  // namespace
 
+namespace vase {
+cudaError_t launch_wait_timeout_probe(uint32_t* err, cudaStream_t s);  // selftest.cu: the failure-detection self-test
+}
+
 extern "C" {
 
 void vase_config_default(vase_config* cfg) {
@@ -994,6 +998,15 @@ int vase_check_device_error(vase_ctx* ctx, void* stream, uint32_t* code) {
         snprintf(buf, sizeof(buf), "device error word 0x%08x", word);
         return fail(ctx, VASE_ERR_DEVICE, buf);
     }
+    return VASE_OK;
+}
+
+int vase_self_test_wait_timeout(vase_ctx* ctx, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    uint32_t* err = reinterpret_cast<uint32_t*>(ctx->ws + ctx->plan.off_err);
+    cudaError_t e = vase::launch_wait_timeout_probe(err, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "self-test launch");
+    ctx->launches += 1;
     return VASE_OK;
 }
 

@@ -26,6 +26,7 @@ VASE_ERR_CUDA = -4
 VASE_ERR_UNSUPPORTED = -5
 VASE_ERR_ALIGN = -6
 VASE_ERR_DEVICE = -7
+VASE_SITE_SELF_TEST = 127  # error-word site of vase_self_test_wait_timeout
 
 VASE_VARIANT_ATTNV = 0
 VASE_VARIANT_DKV = 1
@@ -38,7 +39,7 @@ EXPORTED = [
     "vase_append_host", "vase_evict", "vase_read_positions", "vase_get_layer_state", "vase_set_layer_state",
     "vase_kv_view_get", "vase_debug_view_get", "vase_check_device_error", "vase_launch_count",
     "vase_status_string", "vase_last_error", "vase_abi_version", "vase_profile_enable", "vase_profile_collect",
-    "vase_append_all", "vase_append_all_strided", "vase_evict_all", "vase_refresh_value_scores", "vase_evict_static_scratch",
+    "vase_append_all", "vase_append_all_strided", "vase_evict_all", "vase_self_test_wait_timeout", "vase_refresh_value_scores", "vase_evict_static_scratch",
     "vase_decode_attention", "vase_mixed_buffer_sizes", "vase_quantize_values", "vase_decode_attention_mixed",
 ]
 KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "compact"]
@@ -104,6 +105,7 @@ def load(path: str = LIB_PATH):
         "vase_append_host": (ctypes.c_int, [P, I32, P, P, P, I32, P]),
         "vase_append_all": (ctypes.c_int, [P, P, P, P, I32, P]),
         "vase_append_all_strided": (ctypes.c_int, [P, P, P, P, I32, I64, I64, P]),
+        "vase_self_test_wait_timeout": (ctypes.c_int, [P, P]),
         "vase_evict": (ctypes.c_int, [P, I32, P]),
         "vase_evict_all": (ctypes.c_int, [P, P]),
         "vase_refresh_value_scores": (ctypes.c_int, [P, I32, P]),
@@ -202,6 +204,10 @@ def vase_append_all_strided(ctx, q_ptr, k_ptr, v_ptr, n_tokens, q_layer_stride, 
     return _check(ctx, load().vase_append_all_strided(ctx, q_ptr, k_ptr, v_ptr, n_tokens, q_layer_stride,
                                                       kv_layer_stride, _stream_ptr(stream)),
                   "vase_append_all_strided")
+
+
+def vase_self_test_wait_timeout(ctx, stream=None):
+    return _check(ctx, load().vase_self_test_wait_timeout(ctx, _stream_ptr(stream)), "vase_self_test_wait_timeout")
 
 
 def vase_evict(ctx, layer, stream=None):

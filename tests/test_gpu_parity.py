@@ -33,14 +33,15 @@ def _cache(wl, num_layers, variant="attnv", debug=True, **kw):
 
 
 def _run_layer(wl, *, variant="attnv", layer=1, num_layers=2, round_index=3, seed=0, data_seed=0, units=None,
-               debug=True, positions="gapped", cache_kw=None, oracle_kw=None, state_round=None):
+               debug=True, positions="gapped", cache_kw=None, oracle_kw=None, state_round=None, cache=None):
     """Uploads one layer, evicts it through the C ABI and checks `units` (default all) against the oracle.
 
     round_index is the eviction counter (it keys the noise); state_round (default round_index) draws the data.
     """
     cache_kw = dict(cache_kw or {})
     oracle_kw = dict(oracle_kw or {})
-    cache = _cache(wl, num_layers, variant=variant, debug=debug, seed=seed, **cache_kw)
+    if cache is None:
+        cache = _cache(wl, num_layers, variant=variant, debug=debug, seed=seed, **cache_kw)
     st = W.layer_state(wl, data_seed, layer, round_index if state_round is None else state_round, positions)
     PU.upload_layer(cache, layer, st, round_index)
     other = None
@@ -664,3 +665,19 @@ def test_append_reads_only_the_last_window_query_rows():
     assert torch.equal(a.k_cache[..., :n, :], b.k_cache[..., :n, :])
     assert torch.equal(a.v_cache[..., :n, :], b.v_cache[..., :n, :])
     assert torch.equal(a.positions[..., :n], b.positions[..., :n])
+
+
+# ----------------------------------------------------------------------------- failure detection
+
+def test_bounded_wait_runs_out_and_the_host_reads_its_site():
+    """A kernel whose mbarrier wait nothing completes: the wait gives up at its limit (about two seconds), the
+    site lands in the device error word, the host reads and clears it, and the same context then evicts a
+    layer that matches the oracle (no fault, nothing left stuck)."""
+    from paper_2606_03928_gb300 import vase as V
+    cache = _cache(SMALL, 2)
+    V.vase_self_test_wait_timeout(cache.ctx)
+    status, code = cache.check_device_error()
+    assert status == V.VASE_ERR_DEVICE
+    assert code & 0x80000000 and (code & 0xFFFF) == V.VASE_SITE_SELF_TEST
+    assert cache.check_device_error() == (0, 0)  # read and cleared
+    _run_layer(SMALL, cache=cache)

@@ -141,8 +141,9 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
         p.cluster_for[nz] = best_c;
         if (nz <= max_batch && best_c > c_max) c_max = best_c;
     }
-    // With at least two items per SM, one CTA per SM takes a strided list of units and overlaps the pass-B
-    // sweep of each with the pass-A sweep of the next; this needs two window-row buffers.
+    // With at least one item per SM, one CTA per SM takes a strided list of units and overlaps the pass-B
+    // sweep of each with the pass-A sweep of the next (measured faster than one cluster per unit from 152
+    // items on: batch-1 launches of 288 units); this needs two window-row buffers.
     p.stages_p = 0;
     for (int s = 4; s >= 2; --s) {
         if (score_attn_smem_bytes(p.q_rows, 2, p.n_rbA, p.GWp, 1, s) <= kMaxDynSmem) {
@@ -153,7 +154,7 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     bool any_persist = false;
     c_max = 0;
     for (int nz = 1; nz <= kMaxLayerBatch; ++nz) {
-        p.persist_for[nz] = p.stages_p > 0 && static_cast<long>(p.units) * nz >= 2L * num_sms;
+        p.persist_for[nz] = p.stages_p > 0 && static_cast<long>(p.units) * nz >= num_sms;
         if (nz <= max_batch) {
             if (p.persist_for[nz]) any_persist = true;
             else if (p.cluster_for[nz] > c_max) c_max = p.cluster_for[nz];

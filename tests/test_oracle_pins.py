@@ -355,6 +355,143 @@ def test_dkv_keeps_top_leverage_and_buffer():
     assert len(sets) > 1 and len(fixed) == 1
 
 
+# --------------------------------------------------------------------------- DKV leverage product (Eq. (4))
+#
+# Three checks of s_i = ||G^T k_i||^2 * ||G^T v_i||^2 that do not restate the formula: the expectation over
+# G that Isserlis' theorem fixes, hand-built projections whose answer is known entry by entry, and the
+# DKV ranking (ties included) against brute force.  Each check takes the leverage function as an argument,
+# so that the last test can plant the plausible slips in a copy of it and see every slip rejected.
+
+def _pin_isserlis_expectation(lev):
+    """For G_ab ~ N(0, 1/r) i.i.d., x = G^T k and y = G^T v are r independent pairs with E x_b^2 = |k|^2 / r,
+    E y_b^2 = |v|^2 / r and E x_b y_b = (k . v) / r; Isserlis' theorem, E[x^2 y^2] = E x^2 E y^2 + 2 (E xy)^2,
+    summed over the r^2 pairs (b, c), gives E[|G^T k|^2 |G^T v|^2] = |k|^2 |v|^2 + 2 (k . v)^2 / r.
+    Monte Carlo over Philox projections (d = 16, r = 4): the sample mean lies within 4 standard errors of
+    that value and more than 4 away from |k|^2 |v|^2 (the value without the correlation term)."""
+    d, r = 16, 4
+    rng = np.random.default_rng(21)
+    k = rng.standard_normal(d)
+    v = k + 0.3 * rng.standard_normal(d)
+    vals = np.array([lev(k[None], v[None], O.gaussian_projection(11, 0, 0, 0, 8, t, d, r))[0][0]
+                     for t in range(4000)])
+    mean, se = vals.mean(), vals.std() / math.sqrt(vals.size)
+    expected = (k @ k) * (v @ v) + 2.0 * (k @ v) ** 2 / r
+    return abs(mean - expected) < 4 * se and abs(mean - (k @ k) * (v @ v)) > 4 * se
+
+
+def _pin_hand_built_projections(lev):
+    """G = c * e_j e_b^T (one non-zero entry, j != b, square d = r so a transposed G still has the right shape):
+    G^T k = c * k_j e_b, so s_i = c^4 k_ij^2 v_ij^2 exactly (powers of two: no rounding).  G = I: s_i =
+    |k_i|^2 |v_i|^2.  Also the two factors returned beside the product."""
+    d = 8
+    rng = np.random.default_rng(22)
+    keys = rng.integers(-4, 5, size=(6, d)).astype(np.float64)
+    vals = rng.integers(-4, 5, size=(6, d)).astype(np.float64)
+    c, j, b = 2.0, 5, 1
+    G = np.zeros((d, d))
+    G[j, b] = c
+    s, lk, lv = lev(keys, vals, G)
+    ok = np.array_equal(s, c ** 4 * keys[:, j] ** 2 * vals[:, j] ** 2)
+    ok &= np.array_equal(lk, c ** 2 * keys[:, j] ** 2) and np.array_equal(lv, c ** 2 * vals[:, j] ** 2)
+    s_id, _, _ = lev(keys, vals, np.eye(d))
+    ok &= np.array_equal(s_id, (keys ** 2).sum(axis=1) * (vals ** 2).sum(axis=1))
+    return bool(ok)
+
+
+def _brute_force_dkv_keep(s, K, B):
+    """Kept candidates of a DKV step by enumeration: the unique (K - B)-subset of slots 0..K-1 whose every
+    member outranks every non-member (higher score, or equal score and lower slot)."""
+    winners = []
+    for sub in itertools.combinations(range(K), K - B):
+        rest = [j for j in range(K) if j not in sub]
+        if all((s[i] > s[j]) or (s[i] == s[j] and i < j) for i in sub for j in rest):
+            winners.append(set(sub))
+    assert len(winners) == 1
+    return winners[0]
+
+
+def _pin_dkv_ranking_with_ties(lev, monkeypatch):
+    """Tiny caches whose integer keys and values tie the product score often, with a hand-built G in place
+    of the Philox draw: the DKV step keeps R_B and exactly the brute-force top K - B (ties to the lower slot)."""
+    d = 6
+    G = np.zeros((d, 3))
+    G[0, 0], G[2, 1], G[4, 2] = 1.0, 2.0, 1.0
+    monkeypatch.setattr(O, "gaussian_projection", lambda *a, **kw: G)
+    monkeypatch.setattr(O, "leverage_scores", lev)
+    rng = np.random.default_rng(23)
+    ok, ties = True, 0
+    for trial in range(60):
+        K, B = int(rng.integers(3, 8)), int(rng.integers(1, 3))
+        if B > K - 1:
+            continue
+        keys = rng.integers(-1, 2, size=(K + B, d)).astype(np.float64)
+        vals = rng.integers(-1, 2, size=(K + B, d)).astype(np.float64)
+        s_true = (((keys[:K] @ G) ** 2).sum(axis=1) * ((vals[:K] @ G) ** 2).sum(axis=1))
+        ties += len(s_true) - len(np.unique(s_true))
+        res = O.evict_unit(None, keys, vals, np.arange(K + B), budget_k=K, buffer_b=B, variant="dkv", dkv_rank=3)
+        kept = set(np.flatnonzero(res["keep"][:K]).tolist())
+        ok &= bool(res["keep"][K:].all()) and kept == _brute_force_dkv_keep(s_true, K, B)
+    assert ties > 20  # the cases really exercise ties
+    return ok
+
+
+def test_leverage_product_expectation_matches_isserlis():
+    assert _pin_isserlis_expectation(O.leverage_scores)
+
+
+def test_leverage_product_on_hand_built_projections():
+    assert _pin_hand_built_projections(O.leverage_scores)
+
+
+def test_dkv_top_k_minus_b_with_ties_matches_brute_force(monkeypatch):
+    assert _pin_dkv_ranking_with_ties(O.leverage_scores, monkeypatch)
+
+
+def _planted_slips():
+    """Plausible mistakes in the product score: a sum of the factors, unsquared norms, G transposed, only the
+    key factor, and the key projected with one G and the value with an independent one."""
+    def sum_(keys, values, G):
+        lk, lv = ((keys @ G) ** 2).sum(axis=1), ((values @ G) ** 2).sum(axis=1)
+        return lk + lv, lk, lv
+
+    def unsquared(keys, values, G):
+        lk, lv = np.linalg.norm(keys @ G, axis=1), np.linalg.norm(values @ G, axis=1)
+        return lk * lv, lk, lv
+
+    def transposed(keys, values, G):
+        lk, lv = ((keys @ G.T) ** 2).sum(axis=1), ((values @ G.T) ** 2).sum(axis=1)
+        return lk * lv, lk, lv
+
+    def key_only(keys, values, G):
+        lk = ((keys @ G) ** 2).sum(axis=1)
+        return lk, lk, lk
+
+    def independent(keys, values, G):
+        G2 = np.roll(G, 1, axis=0)  # another projection: G applied to the value's channels shifted by one
+        lk, lv = ((keys @ G) ** 2).sum(axis=1), ((values @ G2) ** 2).sum(axis=1)
+        return lk * lv, lk, lv
+
+    return {"sum": sum_, "unsquared": unsquared, "transposed": transposed, "key_only": key_only,
+            "independent": independent}
+
+
+@pytest.mark.parametrize("slip", sorted(_planted_slips()))
+def test_leverage_pins_reject_planted_slips(slip, monkeypatch):
+    """Every slip fails at least one of the three pins (the pins are not restatements of the formula)."""
+    lev = _planted_slips()[slip]
+    passed = [_pin_hand_built_projections(lev)]
+    try:
+        passed.append(_pin_isserlis_expectation(lev))
+    except ValueError:  # a shape error is a failure too
+        passed.append(False)
+    with monkeypatch.context() as m:
+        try:
+            passed.append(_pin_dkv_ranking_with_ties(lev, m))
+        except (ValueError, AssertionError):
+            passed.append(False)
+    assert not all(passed), f"planted slip '{slip}' passed every pin"
+
+
 # --------------------------------------------------------------------------- decode attention (Eq. (1) output)
 
 def test_decode_attention_closed_forms():

@@ -142,15 +142,24 @@ typedef struct vase_ctx vase_ctx;
  * stochastic, fresh G per round, Range value score.  Geometry fields are zeroed. */
 void vase_config_default(vase_config* cfg);
 
-/* Validates *cfg and reports the buffer sizes it needs.  No device work. */
+/* Validates *cfg and reports the buffer sizes it needs.  No device work.  The caches
+ * hold N = K + B slots per (layer, sequence, KV head) -- the budget K and buffer B of
+ * Sec. 2's periodic eviction -- and the window ring the W cached decode queries per
+ * query head that Eq. (2) and its footnote score against.  Errors: VASE_ERR_INVALID
+ * (inconsistent configuration; vase_last_error(NULL) says which check),
+ * VASE_ERR_UNSUPPORTED (head_dim != 128). */
 int vase_get_buffer_sizes(const vase_config* cfg, vase_buffer_sizes* out);
 
-/* Creates a context over caller-owned buffers (sizes from vase_buffer_sizes).
- * Reads the current CUDA device; encodes the TMA descriptors of the caches.
- * Every layer starts empty (fill 0, round 0).  The buffers are not cleared. */
+/* Creates a context over caller-owned buffers (sizes from vase_buffer_sizes): the
+ * per-layer KV caches of budget K plus buffer B that Sec. 2's periodic eviction works
+ * on.  Reads the current CUDA device; encodes the TMA descriptors of the caches.
+ * Every layer starts empty (fill 0, round 0).  The buffers are not cleared and stay
+ * the caller's; the context keeps only pointers.  Errors: VASE_ERR_INVALID (bad
+ * configuration or null buffer), VASE_ERR_ALIGN (a buffer not 256-byte aligned),
+ * VASE_ERR_UNSUPPORTED, VASE_ERR_CUDA; *out is NULL then. */
 int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out);
 
-/* Frees the context's host state.  Caller memory is untouched. */
+/* Frees the context's host state.  Caller memory is untouched.  NULL is a no-op. */
 void vase_destroy(vase_ctx* ctx);
 
 /* Appends n_tokens consecutive decode steps of one layer (Sec. 2: each decode
@@ -254,11 +263,62 @@ int vase_decode_attention_mixed(vase_ctx* ctx, int32_t layer, int32_t bits, cons
  * the stream completes. */
 int vase_read_positions(vase_ctx* ctx, int32_t layer, int32_t* host_out, void* stream);
 
+/* ---- Host-buffer pipeline: a decode loop whose inputs and results live in host memory.
+ *
+ * Sec. 2's loop appends one (q, k, v) per decode step and evicts every B steps; here one call
+ * stages a whole round's inputs (n_tokens <= B steps of every layer) from host memory, the next
+ * appends them, and the kept positions go back to the host after the eviction.  The copies run on
+ * a caller-given copy stream, so the copies of round r + 1 overlap the kernels of round r when the
+ * caller stages r + 1 before it appends r:
+ *     stage(r = 0); for r: { stage(r + 1); append_all_staged; evict_all; read_positions_all }
+ * The library records events to order the two streams; it allocates no device memory (the caller
+ * passes the staging buffer).  For the copies to be asynchronous the host inputs and outputs must
+ * be page-locked (pinned or registered). */
+
+/* Bytes of ONE staged step for n_tokens per layer: per layer, the last min(W, n_tokens) query
+ * rows and the n_tokens key and value rows, each layer's block rounded up to 256 bytes.  The
+ * staging buffer of vase_stage_host_inputs holds two steps (2 x this).  0 for a bad config. */
+size_t vase_host_staging_bytes(const vase_config* cfg, int32_t n_tokens);
+
+/* Enqueues on copy_stream the host-to-device copies of one step's inputs of every layer into the
+ * next half of `staging` (device, 256-byte aligned, >= 2 x vase_host_staging_bytes(cfg, n_tokens)
+ * bytes, caller-owned; pass the same buffer on every call).  Host inputs, bf16 rows of 256 bytes:
+ * layer l's q [n_tokens][b][Hq][d] at q_host + l * q_layer_stride bytes, its k and v
+ * [n_tokens][b][Hkv][d] at k_host / v_host + l * kv_layer_stride.  Only the query rows of the last
+ * min(W, n_tokens) steps are copied (the window ring keeps no others), so a layer's host block may
+ * hold its query tail alone (q_host pointing n_tokens - min(W, n_tokens) steps before it, a stride of
+ * at least the tail; strides are multiples of 16 bytes).  A half is refilled only
+ * after the append that read it has run (the copy stream waits for it).  At most two steps can be
+ * staged and not yet appended (VASE_ERR_FULL otherwise).  The host inputs may change once
+ * copy_stream has run the copies.  Errors: VASE_ERR_INVALID (null pointer, n_tokens outside
+ * 1..B, strides smaller than a layer's inputs, staging too small), VASE_ERR_ALIGN, VASE_ERR_FULL,
+ * VASE_ERR_CUDA. */
+int vase_stage_host_inputs(vase_ctx* ctx, const void* q_host, const void* k_host, const void* v_host,
+                           int32_t n_tokens, int64_t q_layer_stride, int64_t kv_layer_stride, void* staging,
+                           size_t staging_bytes, void* copy_stream);
+
+/* Appends the oldest staged step to every layer on `stream` (vase_append_all from the staging
+ * buffer; `stream` first waits for that step's copies).  Returns as vase_append_all
+ * (VASE_EVICT_DUE when the layers become full), VASE_ERR_INVALID when nothing is staged. */
+int vase_append_all_staged(vase_ctx* ctx, void* stream);
+
+/* Copies the K positions of every unit of every layer (int32 [L][b][Hkv][K]) to host_out on
+ * copy_stream, after everything enqueued on `stream` so far (call it after vase_evict_all).  The
+ * next eviction on this context waits for the copy, so the positions it reads cannot move under
+ * it.  host_out is valid once copy_stream has run the copy. */
+int vase_read_positions_all(vase_ctx* ctx, int32_t* host_out, void* copy_stream, void* stream);
+
 int vase_get_layer_state(const vase_ctx* ctx, int32_t layer, vase_layer_state* out);
 /* Sets one layer's counters (resume from a checkpoint, or tests that write the buffers directly). */
 int vase_set_layer_state(vase_ctx* ctx, int32_t layer, const vase_layer_state* st);
 
+/* Where a decode kernel reads one layer's kept pairs (slots 0..fill-1 in stream order, the
+ * layout Sec. 2's compaction back to K slots leaves).  Host call, no device work. */
 int vase_kv_view_get(const vase_ctx* ctx, int32_t layer, vase_kv_view* out);
+/* Device pointers to the intermediate results of the most recent eviction call: the window
+ * score of Eq. (2) before and after pooling, the value magnitudes of Eq. (5) (or the DKV
+ * products of Eq. (4)), the selection keys of Sec. 3.2 and the kept list.  The arrays stay
+ * in the workspace; the caller copies what it needs before the next eviction. */
 int vase_debug_view_get(const vase_ctx* ctx, int32_t slot, vase_debug_view* out);
 
 /* Synchronises the stream, then reads and clears the device error word that
@@ -315,14 +375,23 @@ int vase_profile_collect(vase_ctx* ctx, double* total_ms, int64_t* launches);
  *   state:     the layer's counters as the caller tracks them; state->fill must be K + B and
  *              state->round keys the noise.  The call does not update them: afterwards the
  *              caller sets fill = K and round + 1.
- *   device_error: NULL, or a host word: then the call waits for the stream, stores the device
- *              error word there and returns VASE_ERR_DEVICE if it is non-zero.
- * Layers needing more scratch than the array holds ((b*Hkv) * (K+B) * 4 * (1 + parts) +
- * (b*Hkv) * K * 4 bytes, parts = 2 when G*W > 256, else 1) are rejected with
- * VASE_ERR_UNSUPPORTED.  The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress) with that device current; make that first call before any stream
- * capture.  Every call shares the one array and leaves its contents behind: calls that can
- * overlap on the GPU (different streams, or several host threads) race on it and must be
+ *   device_error: NULL, or a host word.  Non-NULL: the call waits for the stream, stores the
+ *              device error word there, and if it is non-zero clears it and returns
+ *              VASE_ERR_DEVICE.  NULL: the call neither waits nor reads the word; a failure
+ *              stays recorded in the array (the kernels only set bits in it) and is returned
+ *              by the next call made with a non-NULL device_error, so a caller that passes
+ *              NULL on its hot path can ask now and then.
+ * Layers needing more scratch than the array holds (256 + (b*Hkv) * (K+B) * 4 * (1 + parts)
+ * + (b*Hkv) * K * 4 bytes, parts = 2 when G*W > 256, else 1, each term rounded up to 256)
+ * are rejected with VASE_ERR_UNSUPPORTED before any buffer is looked at; the Qwen3-32B
+ * geometry at batch 16 (about 17 MB) is one.  The first call on a device looks up the array's
+ * device address (cudaGetSymbolAddress) with that device current; make that first call before
+ * any stream capture.  Under the CUDA default of lazy module loading that first call is also
+ * when the device commits the VASE_STATIC_SCRATCH_BYTES of the array, and it fails with
+ * VASE_ERR_CUDA (an out-of-memory message) if the device's memory is already taken: make it
+ * at start-up, or set CUDA_MODULE_LOADING=EAGER so that the array is committed when the
+ * library loads.  Every call shares the one array and leaves its contents behind: calls that
+ * can overlap on the GPU (different streams, or several host threads) race on it and must be
  * serialised by the caller.  Errors are explained by vase_last_error(NULL). */
 #define VASE_STATIC_SCRATCH_BYTES (16u << 20)
 int vase_evict_static_scratch(const vase_config* cfg, const vase_buffers* bufs, int32_t layer,

@@ -321,11 +321,32 @@ struct vase_ctx {
     std::vector<EventPair> events;
     size_t events_used = 0;
     bool profiling = false;
+    // host-input pipeline (vase_stage_host_inputs / vase_append_all_staged / vase_read_positions_all)
+    struct Staged {
+        cudaEvent_t copied = nullptr;    // the inputs of this half have landed
+        cudaEvent_t consumed = nullptr;  // the append that read this half has run
+        bool consumed_pending = false;   // `consumed` was recorded and a later copy into the half must wait for it
+        const uint8_t* base = nullptr;   // device address of the half
+        int32_t n_tokens = 0, w_q = 0;   // tokens per layer, query rows kept per layer
+        int64_t block = 0;               // bytes of one layer's [query tail | k | v] block
+    };
+    Staged staged[2];
+    int staged_next = 0;      // half the next vase_stage_host_inputs fills
+    int staged_count = 0;     // staged steps not yet appended (0..2)
+    cudaEvent_t evicted = nullptr;    // recorded on the compute stream before a positions read-back
+    cudaEvent_t read_done = nullptr;  // the last positions read-back has run; the next eviction waits for it
+    bool read_pending = false;
     ~vase_ctx() {
         for (auto& e : events) {
             cudaEventDestroy(e.start);
             cudaEventDestroy(e.end);
         }
+        for (auto& h : staged) {
+            if (h.copied) cudaEventDestroy(h.copied);
+            if (h.consumed) cudaEventDestroy(h.consumed);
+        }
+        if (evicted) cudaEventDestroy(evicted);
+        if (read_done) cudaEventDestroy(read_done);
     }
 };
 
@@ -591,6 +612,10 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     float* vscore = reinterpret_cast<float*>(ctx->ws + P.off_vscore);
     int32_t* src = reinterpret_cast<int32_t*>(ctx->ws + P.off_src);
     cudaError_t e;
+    if (ctx->read_pending) {  // the positions a read-back copies must not move before it has run
+        if ((e = cudaStreamWaitEvent(s, ctx->read_done, 0)) != cudaSuccess) return cuda_fail(ctx, e, "read-back wait");
+        ctx->read_pending = false;
+    }
     if (c.variant == VASE_VARIANT_ATTNV) {
         const ScoreAttnParams sp = score_params(P, c, batch, nz, attn, err);
         if ((e = timed_launch(ctx, VASE_KERNEL_SCORE, s, [&] {
@@ -940,6 +965,127 @@ int vase_read_positions(vase_ctx* ctx, int32_t layer, int32_t* host_out, void* s
     return VASE_OK;
 }
 
+namespace {
+
+// One step's staging block per layer: [the last w_q query rows | n key rows | n value rows].
+int64_t staged_block_bytes(const vase_config& c, int32_t n_tokens, int32_t* w_q) {
+    *w_q = n_tokens < c.window ? n_tokens : c.window;
+    const int64_t q_step = static_cast<int64_t>(c.batch) * c.num_q_heads * kRowBytes;
+    const int64_t kv = static_cast<int64_t>(n_tokens) * c.batch * c.num_kv_heads * kRowBytes;
+    return align_up(static_cast<size_t>(*w_q * q_step + 2 * kv), kAlign);
+}
+
+cudaError_t lazy_event(cudaEvent_t* ev) {
+    if (*ev) return cudaSuccess;
+    return cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
+}
+
+}  // namespace
+
+size_t vase_host_staging_bytes(const vase_config* cfg, int32_t n_tokens) {
+    if (!cfg || n_tokens < 1 || check_config(cfg)) return 0;
+    int32_t w_q = 0;
+    return static_cast<size_t>(cfg->num_layers) * static_cast<size_t>(staged_block_bytes(*cfg, n_tokens, &w_q));
+}
+
+int vase_stage_host_inputs(vase_ctx* ctx, const void* q_host, const void* k_host, const void* v_host,
+                           int32_t n_tokens, int64_t q_layer_stride, int64_t kv_layer_stride, void* staging,
+                           size_t staging_bytes, void* copy_stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    const vase_config& c = ctx->cfg;
+    if (!q_host || !k_host || !v_host || !staging) return fail(ctx, VASE_ERR_INVALID, "null input or staging buffer");
+    if (n_tokens < 1 || n_tokens > c.buffer_b) return fail(ctx, VASE_ERR_INVALID, "n_tokens must be in 1..buffer_b");
+    int32_t w_q = 0;
+    const int64_t block = staged_block_bytes(c, n_tokens, &w_q);
+    const int64_t q_step = static_cast<int64_t>(c.batch) * c.num_q_heads * kRowBytes;
+    const int64_t kv = static_cast<int64_t>(n_tokens) * c.batch * c.num_kv_heads * kRowBytes;
+    if (q_layer_stride < w_q * q_step || kv_layer_stride < kv)
+        return fail(ctx, VASE_ERR_INVALID, "layer strides smaller than one layer's inputs");
+    if (q_layer_stride % 16 || kv_layer_stride % 16)
+        return fail(ctx, VASE_ERR_ALIGN, "layer strides must be multiples of 16 bytes");
+    const size_t half = static_cast<size_t>(c.num_layers) * static_cast<size_t>(block);
+    if (staging_bytes < 2 * half) return fail(ctx, VASE_ERR_INVALID, "staging buffer smaller than 2 x vase_host_staging_bytes");
+    if (!aligned(staging, kAlign)) return fail(ctx, VASE_ERR_ALIGN, "staging buffer must be 256-byte aligned");
+    if (ctx->staged_count == 2) return fail(ctx, VASE_ERR_FULL, "two steps are staged already: append one first");
+    cudaStream_t cs = static_cast<cudaStream_t>(copy_stream);
+    vase_ctx::Staged& h = ctx->staged[ctx->staged_next];
+    cudaError_t e;
+    if ((e = lazy_event(&h.copied)) != cudaSuccess || (e = lazy_event(&h.consumed)) != cudaSuccess)
+        return cuda_fail(ctx, e, "staging events");
+    if (h.consumed_pending) {  // the append that read this half before must have run
+        if ((e = cudaStreamWaitEvent(cs, h.consumed, 0)) != cudaSuccess) return cuda_fail(ctx, e, "staging wait");
+        h.consumed_pending = false;
+    }
+    uint8_t* dst = static_cast<uint8_t*>(staging) + static_cast<size_t>(ctx->staged_next) * half;
+    const uint8_t* qs = static_cast<const uint8_t*>(q_host) + static_cast<int64_t>(n_tokens - w_q) * q_step;
+    const size_t L = static_cast<size_t>(c.num_layers);
+    // three strided copies move every layer's query tail, keys and values into its block
+    if ((e = cudaMemcpy2DAsync(dst, static_cast<size_t>(block), qs, static_cast<size_t>(q_layer_stride),
+                               static_cast<size_t>(w_q * q_step), L, cudaMemcpyHostToDevice, cs)) != cudaSuccess ||
+        (e = cudaMemcpy2DAsync(dst + w_q * q_step, static_cast<size_t>(block), k_host,
+                               static_cast<size_t>(kv_layer_stride), static_cast<size_t>(kv), L,
+                               cudaMemcpyHostToDevice, cs)) != cudaSuccess ||
+        (e = cudaMemcpy2DAsync(dst + w_q * q_step + kv, static_cast<size_t>(block), v_host,
+                               static_cast<size_t>(kv_layer_stride), static_cast<size_t>(kv), L,
+                               cudaMemcpyHostToDevice, cs)) != cudaSuccess ||
+        (e = cudaEventRecord(h.copied, cs)) != cudaSuccess)
+        return cuda_fail(ctx, e, "host-to-device staging copy");
+    h.base = dst;
+    h.n_tokens = n_tokens;
+    h.w_q = w_q;
+    h.block = block;
+    ctx->staged_next ^= 1;
+    ctx->staged_count += 1;
+    return VASE_OK;
+}
+
+int vase_append_all_staged(vase_ctx* ctx, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (ctx->staged_count == 0) return fail(ctx, VASE_ERR_INVALID, "no staged step: call vase_stage_host_inputs first");
+    const int oldest = (ctx->staged_next + 2 - ctx->staged_count) & 1;
+    vase_ctx::Staged& h = ctx->staged[oldest];
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const vase_config& c = ctx->cfg;
+    cudaError_t e;
+    for (int32_t l = 0; l < c.num_layers; ++l)
+        if (ctx->layers[l].fill + h.n_tokens > ctx->plan.N)
+            return fail(ctx, VASE_ERR_FULL, "append would exceed K + B slots");
+    if ((e = cudaStreamWaitEvent(s, h.copied, 0)) != cudaSuccess) return cuda_fail(ctx, e, "staging wait");
+    // the append reads only the last w_q query rows, so layer l's q pointer sits n - w_q steps before its tail
+    const int64_t q_step = static_cast<int64_t>(c.batch) * c.num_q_heads * kRowBytes;
+    const void* q = h.base - static_cast<int64_t>(h.n_tokens - h.w_q) * q_step;
+    const void* k = h.base + h.w_q * q_step;
+    const void* v = static_cast<const uint8_t*>(k) + static_cast<int64_t>(h.n_tokens) * c.batch * c.num_kv_heads * kRowBytes;
+    std::vector<int32_t> all(static_cast<size_t>(c.num_layers));
+    for (int32_t l = 0; l < c.num_layers; ++l) all[l] = l;
+    const int r = append_batch(ctx, all.data(), c.num_layers, q, k, v, h.n_tokens, s, h.block, h.block);
+    if (r < 0) return r;
+    if ((e = cudaEventRecord(h.consumed, s)) != cudaSuccess) return cuda_fail(ctx, e, "staging event");
+    h.consumed_pending = true;
+    ctx->staged_count -= 1;
+    return r;
+}
+
+int vase_read_positions_all(vase_ctx* ctx, int32_t* host_out, void* copy_stream, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    if (!host_out) return fail(ctx, VASE_ERR_INVALID, "null output");
+    cudaError_t e;
+    if ((e = lazy_event(&ctx->evicted)) != cudaSuccess || (e = lazy_event(&ctx->read_done)) != cudaSuccess)
+        return cuda_fail(ctx, e, "read-back events");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaStream_t cs = static_cast<cudaStream_t>(copy_stream);
+    const Plan& P = ctx->plan;
+    const size_t width = static_cast<size_t>(ctx->cfg.budget_k) * 4;
+    const size_t rows = static_cast<size_t>(ctx->cfg.num_layers) * P.units;
+    if ((e = cudaEventRecord(ctx->evicted, s)) != cudaSuccess || (e = cudaStreamWaitEvent(cs, ctx->evicted, 0)) != cudaSuccess ||
+        (e = cudaMemcpy2DAsync(host_out, width, ctx->bufs.positions, static_cast<size_t>(P.N) * 4, width, rows,
+                               cudaMemcpyDeviceToHost, cs)) != cudaSuccess ||
+        (e = cudaEventRecord(ctx->read_done, cs)) != cudaSuccess)
+        return cuda_fail(ctx, e, "positions read-back");
+    ctx->read_pending = true;
+    return VASE_OK;
+}
+
 int vase_get_layer_state(const vase_ctx* ctx, int32_t layer, vase_layer_state* out) {
     if (!ctx || !out || layer < 0 || layer >= ctx->cfg.num_layers) return VASE_ERR_INVALID;
     *out = ctx->layers[layer];
@@ -1079,6 +1225,18 @@ __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
 constexpr int kMaxDevices = 64;
 void* g_static_scratch_addr[kMaxDevices] = {};  // device address of g_static_scratch, per device
 
+// Host set-up of the previous call (tensor maps, kernel attributes), reused while nothing it depends on changed.
+struct StaticScratchSetup {
+    bool valid = false;
+    int device = -1;
+    vase_config cfg;
+    const void* k = nullptr;
+    const void* v = nullptr;
+    const void* q = nullptr;
+    CUtensorMap kmap, vmap, qmap;
+};
+StaticScratchSetup g_static_setup;
+
 }  // namespace
 
 extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buffers* bufs, int32_t layer,
@@ -1102,6 +1260,19 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
         g_config_error = "layer out of range";
         return VASE_ERR_INVALID;
     }
+    // scratch of one layer: error word | window-score parts | DKV products | kept lists (a property of the
+    // configuration alone, so it is checked before anything else is looked at)
+    const size_t un = static_cast<size_t>(P.units) * P.N;
+    const size_t off_attn = kAlign;
+    const size_t off_dkv = align_up(off_attn + un * 4 * P.n_rb, kAlign);
+    const size_t off_src = align_up(off_dkv + un * 4, kAlign);
+    const size_t need = align_up(off_src + static_cast<size_t>(P.units) * c.budget_k * 4, kAlign);
+    if (need > kStaticScratchBytes) {
+        g_config_error = "one layer needs " + std::to_string(need) +
+                         " bytes of eviction scratch, more than the static array holds (VASE_STATIC_SCRATCH_BYTES = " +
+                         std::to_string(kStaticScratchBytes) + ")";
+        return VASE_ERR_UNSUPPORTED;
+    }
     if (state->fill != P.N) {
         g_config_error = "evict needs a full cache (fill == K + B)";
         return VASE_ERR_NOT_FULL;
@@ -1113,21 +1284,15 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
             return p ? VASE_ERR_ALIGN : VASE_ERR_INVALID;
         }
     }
-    // scratch of one layer: error word | window-score parts | DKV products | kept lists
-    const size_t un = static_cast<size_t>(P.units) * P.N;
-    const size_t off_attn = kAlign;
-    const size_t off_dkv = align_up(off_attn + un * 4 * P.n_rb, kAlign);
-    const size_t off_src = align_up(off_dkv + un * 4, kAlign);
-    const size_t need = align_up(off_src + static_cast<size_t>(P.units) * c.budget_k * 4, kAlign);
-    if (need > kStaticScratchBytes) {
-        g_config_error = "one layer needs more eviction scratch than the static array holds (VASE_STATIC_SCRATCH_BYTES)";
-        return VASE_ERR_UNSUPPORTED;
-    }
-    // set-up, once per device, with that device current: the device address of the static array
+    // set-up, once per device, with that device current: the device address of the static array.  With lazy
+    // module loading (the CUDA default) this is also where the array is committed on the device.
     if (!g_static_scratch_addr[device]) {
         void* addr = nullptr;
         if ((e = cudaGetSymbolAddress(&addr, g_static_scratch)) != cudaSuccess || !addr) {
-            g_config_error = std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e);
+            g_config_error = e == cudaErrorMemoryAllocation
+                                 ? "out of device memory while loading the static scratch array (first call on this "
+                                   "device): make the first call at start-up, or set CUDA_MODULE_LOADING=EAGER"
+                                 : std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e);
             return VASE_ERR_CUDA;
         }
         g_static_scratch_addr[device] = addr;
@@ -1138,35 +1303,49 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
     float* dkv = reinterpret_cast<float*>(scratch + off_dkv);
     int32_t* src = reinterpret_cast<int32_t*>(scratch + off_src);
 
-    void* fn = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
-    if (e != cudaSuccess || !fn || q != cudaDriverEntryPointSuccess) {
-        g_config_error = "cuTensorMapEncodeTiled unavailable";
-        return VASE_ERR_CUDA;
+    // Tensor maps and kernel attributes: reused while the device, the configuration and the buffers are those of
+    // the previous call (a serving loop evicts the same caches over and over).
+    StaticScratchSetup& su = g_static_setup;
+    if (!(su.valid && su.device == device && std::memcmp(&su.cfg, &c, sizeof(c)) == 0 &&
+          su.k == bufs->k_cache && su.v == bufs->v_cache && su.q == bufs->q_window)) {
+        su.valid = false;
+        void* fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e != cudaSuccess || !fn || q != cudaDriverEntryPointSuccess) {
+            g_config_error = "cuTensorMapEncodeTiled unavailable";
+            return VASE_ERR_CUDA;
+        }
+        EncodeTiledFn enc = reinterpret_cast<EncodeTiledFn>(fn);
+        const uint64_t cache_rows = static_cast<uint64_t>(c.num_layers) * P.units * P.N;
+        const uint64_t q_rows = static_cast<uint64_t>(c.num_layers) * c.batch * c.num_q_heads * c.window;
+        if (cache_rows >= (1ull << 31) || q_rows >= (1ull << 31) ||
+            !encode_rows(enc, &su.kmap, bufs->k_cache, cache_rows, kTileTokens) ||
+            !encode_rows(enc, &su.vmap, bufs->v_cache, cache_rows, kTileTokens) ||
+            !encode_rows(enc, &su.qmap, bufs->q_window, q_rows, static_cast<uint32_t>(P.q_box))) {
+            g_config_error = "tensor map encoding failed";
+            return VASE_ERR_CUDA;
+        }
+        if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
+            (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess ||
+            (e = select_set_attributes(P.select_smem)) != cudaSuccess) {
+            g_config_error = std::string("kernel attributes: ") + cudaGetErrorString(e);
+            return VASE_ERR_CUDA;
+        }
+        su.device = device;
+        su.cfg = c;
+        su.k = bufs->k_cache;
+        su.v = bufs->v_cache;
+        su.q = bufs->q_window;
+        su.valid = true;
     }
-    EncodeTiledFn enc = reinterpret_cast<EncodeTiledFn>(fn);
-    const uint64_t cache_rows = static_cast<uint64_t>(c.num_layers) * P.units * P.N;
-    const uint64_t q_rows = static_cast<uint64_t>(c.num_layers) * c.batch * c.num_q_heads * c.window;
-    CUtensorMap kmap, vmap, qmap;
-    if (cache_rows >= (1ull << 31) || q_rows >= (1ull << 31) ||
-        !encode_rows(enc, &kmap, bufs->k_cache, cache_rows, kTileTokens) ||
-        !encode_rows(enc, &vmap, bufs->v_cache, cache_rows, kTileTokens) ||
-        !encode_rows(enc, &qmap, bufs->q_window, q_rows, static_cast<uint32_t>(P.q_box))) {
-        g_config_error = "tensor map encoding failed";
-        return VASE_ERR_CUDA;
-    }
-    if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
-        (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess || (e = select_set_attributes(P.select_smem)) != cudaSuccess) {
-        g_config_error = std::string("kernel attributes: ") + cudaGetErrorString(e);
-        return VASE_ERR_CUDA;
-    }
+    const CUtensorMap& kmap = su.kmap;
+    const CUtensorMap& vmap = su.vmap;
+    const CUtensorMap& qmap = su.qmap;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    // the array keeps the previous call's contents: the error word must start at zero
-    if ((e = cudaMemsetAsync(err, 0, sizeof(uint32_t), s)) != cudaSuccess) {
-        g_config_error = std::string("error word reset: ") + cudaGetErrorString(e);
-        return VASE_ERR_CUDA;
-    }
+    // The error word is not cleared here: the kernels OR their failure sites into it, and it is read and cleared
+    // only by a call that reports it (device_error != NULL), so a failure of a call made with device_error == NULL
+    // is reported by the next call that asks.  Every other part of the array is written before it is read.
     LayerBatch batch;
     batch.n = 1;
     batch.layer[0] = layer;
@@ -1241,7 +1420,18 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
             return VASE_ERR_CUDA;
         }
         if (*device_error) {
-            g_config_error = "device-side check or bounded wait failed";
+            // reported: clear it, so that the next call starts from zero
+            if ((e = cudaMemsetAsync(err, 0, sizeof(uint32_t), s)) != cudaSuccess ||
+                (e = cudaStreamSynchronize(s)) != cudaSuccess) {
+                g_config_error = std::string("error word clear: ") + cudaGetErrorString(e);
+                return VASE_ERR_CUDA;
+            }
+            char buf[128];
+            snprintf(buf, sizeof(buf),
+                     "device-side check or bounded wait failed (word 0x%08x, this call or an earlier one made "
+                     "without device_error)",
+                     *device_error);
+            g_config_error = buf;
             return VASE_ERR_DEVICE;
         }
     }

@@ -4,7 +4,10 @@ Such callers (a plugin whose host process owns all device memory, a runtime that
 forbids allocation after start-up) hand the library their caches but no workspace;
 vase_evict_static_scratch then keeps its scratch in a static device array.  This
 file checks, through the C ABI, that two such calls in a row give what vase_evict
-gives on an identical copy of the caches.  It is collected last on purpose.
+gives on an identical copy of the caches -- for both scoring variants, and for a
+window of more than 256 rows, whose score comes in two parts -- and that a layer
+needing more scratch than the array holds is refused before anything runs.  It is
+collected last on purpose.
 """
 
 import numpy as np
@@ -17,17 +20,32 @@ import parity_utils as PU
 pytestmark = pytest.mark.gpu
 
 
-def test_static_scratch_eviction_matches_vase_evict_on_two_calls():
+def _lib():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     from paper_2606_03928_gb300 import build
     build.build()
     from paper_2606_03928_gb300 import vase as V
+    return V
 
-    wl = W.shrink(W.WORKLOADS["single_layer_k256"], num_layers=2, batch=2)
+
+CASES = {
+    # (workload, shrink arguments, variant)
+    "attnv_k256": ("single_layer_k256", dict(num_layers=2, batch=2), "attnv"),
+    "dkv_k256": ("single_layer_k256", dict(num_layers=2, batch=2), "dkv"),
+    # G*W = 8 * 64 = 512 window rows: the window score is written as two parts that the selection adds
+    "attnv_two_parts": ("qwen3_32b_k8192", dict(num_layers=2, batch=1, budget_k=256, buffer_b=64), "attnv"),
+}
+
+
+@pytest.mark.parametrize("case", sorted(CASES))
+def test_static_scratch_eviction_matches_vase_evict_on_two_calls(case):
+    V = _lib()
+    name, shrink, variant = CASES[case]
+    wl = W.shrink(W.WORKLOADS[name], **shrink)
     geometry = PU.geometry_of(wl, 2)
-    ref = V.VaseCache(geometry, seed=5)        # evicted with vase_evict
-    dut = V.VaseCache(geometry, seed=5)        # its caches go to the static-scratch entry point
+    ref = V.VaseCache(geometry, seed=5, variant=variant)  # evicted with vase_evict
+    dut = V.VaseCache(geometry, seed=5, variant=variant)  # its caches go to the static-scratch entry point
     rounds = [3, 4]
     for layer in range(2):
         st = W.layer_state(wl, 7, layer, rounds[layer])
@@ -52,3 +70,19 @@ def test_static_scratch_eviction_matches_vase_evict_on_two_calls():
     pos = dut.positions.cpu().numpy()
     assert np.all(pos[..., wl.budget_k:] == -1)
     assert np.all(np.diff(pos[..., :wl.budget_k], axis=-1) > 0)
+
+
+def test_static_scratch_refuses_a_layer_larger_than_the_array():
+    """The Qwen3-32B geometry at batch 16 needs about 17 MB of scratch per layer, more than the 16 MiB
+    array: the call returns VASE_ERR_UNSUPPORTED from the configuration alone (no buffer is given, so
+    nothing could have been launched)."""
+    V = _lib()
+    wl = W.shrink(W.WORKLOADS["qwen3_32b_k8192"], num_layers=1)
+    cfg = V.vase_config_default(budget_k=wl.budget_k, buffer_b=wl.buffer_b, window=wl.window,
+                                num_q_heads=wl.num_q_heads, num_kv_heads=wl.num_kv_heads, head_dim=128,
+                                num_layers=1, batch=wl.batch)
+    bufs = V.vase_buffers(None, None, None, None, None, None)
+    with pytest.raises(V.VaseError) as exc:
+        V.vase_evict_static_scratch(cfg, bufs, 0, wl.slots, 0)
+    assert exc.value.status == V.VASE_ERR_UNSUPPORTED
+    assert "VASE_STATIC_SCRATCH_BYTES" in str(exc.value)

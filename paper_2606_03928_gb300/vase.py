@@ -41,6 +41,7 @@ EXPORTED = [
     "vase_status_string", "vase_last_error", "vase_abi_version", "vase_profile_enable", "vase_profile_collect",
     "vase_append_all", "vase_append_all_strided", "vase_evict_all", "vase_self_test_wait_timeout", "vase_refresh_value_scores", "vase_evict_static_scratch",
     "vase_decode_attention", "vase_mixed_buffer_sizes", "vase_quantize_values", "vase_decode_attention_mixed",
+    "vase_host_staging_bytes", "vase_stage_host_inputs", "vase_append_all_staged", "vase_read_positions_all",
 ]
 KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "compact"]
 
@@ -112,6 +113,10 @@ def load(path: str = LIB_PATH):
         "vase_evict_static_scratch": (ctypes.c_int, [ctypes.POINTER(vase_config), ctypes.POINTER(vase_buffers), I32,
                                                      ctypes.POINTER(vase_layer_state), ctypes.POINTER(U32), P]),
         "vase_read_positions": (ctypes.c_int, [P, I32, P, P]),
+        "vase_host_staging_bytes": (ctypes.c_size_t, [ctypes.POINTER(vase_config), I32]),
+        "vase_stage_host_inputs": (ctypes.c_int, [P, P, P, P, I32, I64, I64, P, ctypes.c_size_t, P]),
+        "vase_append_all_staged": (ctypes.c_int, [P, P]),
+        "vase_read_positions_all": (ctypes.c_int, [P, P, P, P]),
         "vase_decode_attention": (ctypes.c_int, [P, I32, P, P, P]),
         "vase_mixed_buffer_sizes": (ctypes.c_int, [ctypes.POINTER(vase_config), I32] +
                                     [ctypes.POINTER(ctypes.c_size_t)] * 4),
@@ -263,6 +268,26 @@ def vase_decode_attention_mixed(ctx, layer, bits, mb: vase_mixed_buffers, q_ptr,
 
 def vase_read_positions(ctx, layer, host_ptr, stream=None):
     return _check(ctx, load().vase_read_positions(ctx, layer, host_ptr, _stream_ptr(stream)), "vase_read_positions")
+
+
+def vase_host_staging_bytes(cfg: vase_config, n_tokens) -> int:
+    return int(load().vase_host_staging_bytes(ctypes.byref(cfg), n_tokens))
+
+
+def vase_stage_host_inputs(ctx, q_ptr, k_ptr, v_ptr, n_tokens, q_layer_stride, kv_layer_stride, staging_ptr,
+                           staging_bytes, copy_stream):
+    return _check(ctx, load().vase_stage_host_inputs(ctx, q_ptr, k_ptr, v_ptr, n_tokens, q_layer_stride,
+                                                     kv_layer_stride, staging_ptr, staging_bytes,
+                                                     _stream_ptr(copy_stream)), "vase_stage_host_inputs")
+
+
+def vase_append_all_staged(ctx, stream=None):
+    return _check(ctx, load().vase_append_all_staged(ctx, _stream_ptr(stream)), "vase_append_all_staged")
+
+
+def vase_read_positions_all(ctx, host_ptr, copy_stream, stream=None):
+    return _check(ctx, load().vase_read_positions_all(ctx, host_ptr, _stream_ptr(copy_stream), _stream_ptr(stream)),
+                  "vase_read_positions_all")
 
 
 def vase_get_layer_state(ctx, layer) -> vase_layer_state:
@@ -423,6 +448,29 @@ class VaseCache:
         assert out.is_cuda and out.dtype == torch.float32 and out.is_contiguous()
         vase_decode_attention_mixed(self.ctx, layer, bits, mb, q.data_ptr(), out.data_ptr(), stream)
         return out
+
+    def host_staging(self, n_tokens):
+        """A device staging buffer for vase_stage_host_inputs (two steps of n_tokens per layer)."""
+        nbytes = 2 * vase_host_staging_bytes(self.cfg, n_tokens)
+        return torch.empty(nbytes, dtype=torch.uint8, device=self.device)
+
+    def stage_host_inputs(self, q, k, v, staging, copy_stream):
+        """q [L, n, b, Hq, d], k/v [L, n, b, Hkv, d] bf16 CPU tensors (pinned for asynchronous copies):
+        one step's inputs of every layer, copied on copy_stream into the next half of `staging`."""
+        for t in (q, k, v):
+            assert (not t.is_cuda) and t.dtype == torch.bfloat16 and t.is_contiguous()
+        n = q.shape[1]
+        return vase_stage_host_inputs(self.ctx, q.data_ptr(), k.data_ptr(), v.data_ptr(), n,
+                                      q[0].numel() * 2, k[0].numel() * 2, staging.data_ptr(), staging.numel(),
+                                      copy_stream)
+
+    def append_all_staged(self, stream=None):
+        return vase_append_all_staged(self.ctx, stream)
+
+    def read_positions_all(self, out: torch.Tensor, copy_stream, stream=None):
+        """Every layer's K kept positions into a CPU int32 tensor [L, b, Hkv, K] (pinned), on copy_stream."""
+        assert (not out.is_cuda) and out.dtype == torch.int32 and out.is_contiguous()
+        return vase_read_positions_all(self.ctx, out.data_ptr(), copy_stream, stream)
 
     def read_positions(self, layer, out: torch.Tensor, stream=None):
         """Copies the K kept positions of every unit into a CPU int32 tensor [b, Hkv, K]."""

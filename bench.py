@@ -51,10 +51,10 @@ FALLBACK_HBM_GBS = 6800.0
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
-    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="qwen3_1p7b_k2048")
+    ap.add_argument("--workload", default="qwen3_32b_k8192")
     ap.add_argument("--variant", choices=["attnv", "dkv"], default="attnv")
     ap.add_argument("--reserve", choices=["value", "random"], default="value",
                     help="AttnV R_V: largest value magnitude (Sec. 3.1) or uniformly random (App. C ablation)")
@@ -67,6 +67,9 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=None, help="steps of the host-buffer end-to-end pass")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the records of the other configurations (single layer, Qwen3-1.7B, Qwen3-8B both "
+                         "variants, the sweep's K 16384 point)")
     ap.add_argument("--sweep", action="store_true",
                     help="the Qwen3-8B-geometry sweep over K, B, batch and value-outlier rate (one JSON line, a point each)")
     ap.add_argument("--sweep-full", action="store_true", help="with --sweep: every point of the 5 x 3 x 4 x 3 grid")
@@ -84,7 +87,7 @@ def measured_peaks():
     if os.path.exists(path):
         with open(path) as f:
             d = json.load(f)
-        return float(d["hbm_gbs"]), float(d.get("bf16_tflops", 0.0)), "measured"
+        return float(d["hbm_gbs"]), float(d.get("bf16_tflops", 1900.0)), "measured"
     return FALLBACK_HBM_GBS, 1900.0, "fallback"
 
 
@@ -112,7 +115,7 @@ class ClockSampler:
             self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", "--query-gpu=" + ",".join(self.FIELDS),
-                 "--format=csv,noheader,nounits", "-lms", "50"], stdout=self.file, stderr=subprocess.DEVNULL)
+                 "--format=csv,noheader,nounits", "-lms", "20"], stdout=self.file, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
             return
@@ -149,8 +152,18 @@ class ClockSampler:
             except ValueError:
                 t = None
             parsed.append((t, r))
+        bracketed = False
         if any(t is not None for t, _ in parsed):  # else (an unknown stamp format) every sample is kept
-            parsed = [(t, r) for t, r in parsed if t is not None and self.t_begin - 0.01 <= t <= t_end + 0.01]
+            stamped = [(t, r) for t, r in parsed if t is not None]
+            inside = [(t, r) for t, r in stamped if self.t_begin - 0.01 <= t <= t_end + 0.01]
+            if not inside:
+                # a region shorter than the sampling interval: the last sample before it and the first after it
+                before = [x for x in stamped if x[0] < self.t_begin]
+                after = [x for x in stamped if x[0] > t_end]
+                inside = ([max(before, key=lambda x: x[0])] if before else []) + \
+                         ([min(after, key=lambda x: x[0])] if after else [])
+                bracketed = bool(inside)
+            parsed = inside
         for _, r in parsed:
             try:
                 sm.append(float(r[2]))
@@ -162,8 +175,10 @@ class ClockSampler:
                     reasons.add(name)
         if not sm:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        out = {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons), "samples": len(sm)}
+        if bracketed:
+            out["bracketing"] = True
+        return out
 
 
 def max_over_ranks(ms, world, device):
@@ -325,6 +340,206 @@ def gen_stream(wl, n_tokens, gen, device, torch):
     return q.to(torch.bfloat16), k.to(torch.bfloat16), v.to(torch.bfloat16)
 
 
+class Rig:
+    """One workload's context, its prefilled caches and a few distinct rounds of new decode tokens, resident
+    in HBM.  A round holds, per layer, the B new key and value rows and the query rows of the last W steps
+    (the only query rows the append reads: the window ring keeps no others)."""
+
+    def __init__(self, wl, variant, device, seed, torch, V, n_distinct=4, **cache_kw):
+        self.wl, self.torch, self.V = wl, torch, V
+        L, K, Bf = wl.num_layers, wl.budget_k, wl.buffer_b
+        self.cache = V.VaseCache(V.Geometry(K, Bf, wl.window, wl.num_q_heads, wl.num_kv_heads, L, wl.batch),
+                                 variant=variant, seed=0, device=device, **cache_kw)
+        gen = torch.Generator(device=device)
+        gen.manual_seed(seed)
+        for layer in range(L):  # prefill: K tokens per layer, in pieces of at most 1024 (bounded temporaries)
+            for t0 in range(0, K, 1024):
+                self.cache.append(layer, *gen_stream(wl, min(1024, K - t0), gen, device, torch))
+        self.w_q = min(wl.window, Bf)
+        self.rounds = []
+        for _ in range(max(1, min(n_distinct, wl.rounds_per_layer))):
+            qs, ks, vs = [], [], []
+            for layer in range(L):
+                q, k, v = gen_stream(wl, Bf, gen, device, torch)
+                qs.append(q[Bf - self.w_q:].contiguous())
+                ks.append(k)
+                vs.append(v)
+                del q
+            self.rounds.append((torch.stack(qs), torch.stack(ks), torch.stack(vs)))
+            del qs, ks, vs
+        torch.cuda.synchronize()
+        self.r = 0
+        self.q_step = wl.batch * wl.num_q_heads * wl.head_dim * 2  # bytes of one step's query rows
+
+    def append(self, stream):
+        """The next round's B tokens to every layer, one launch (layer l's query pointer sits B - W steps
+        before its tail, which the library never reads)."""
+        q, k, v = self.rounds[self.r % len(self.rounds)]
+        self.r += 1
+        Bf = self.wl.buffer_b
+        return self.V.vase_append_all_strided(self.cache.ctx, q.data_ptr() - (Bf - self.w_q) * self.q_step,
+                                              k.data_ptr(), v.data_ptr(), Bf, q[0].numel() * 2, k[0].numel() * 2,
+                                              stream)
+
+    def step(self, stream):
+        self.append(stream)
+        self.cache.evict_all(stream)
+
+    def close(self):
+        self.cache.close()
+        del self.cache, self.rounds
+
+
+def timed_steps(torch, step, steps, stream, barrier=lambda: None, sampler=None):
+    """Mean ms per step of `steps` calls of step(), CUDA events on the launch stream, synchronised and
+    bracketed by the barrier on both sides."""
+    barrier()
+    torch.cuda.synchronize()
+    if sampler is not None:
+        sampler.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clocks = sampler.stop() if sampler is not None else None
+    return e0.elapsed_time(e1) / steps, clocks
+
+
+def kernel_table(kernels, wl, variant, moved, layers_per_launch, hbm_peak, tflops_peak):
+    """Per kernel: launches, mean launch time, share of the kernel time, algorithmic GB/s; for the window
+    score also its algorithmic QK^T TFLOP/s and the bound of its own roofline."""
+    out = {}
+    total = sum(v[0] for v in kernels.values()) or 1.0
+    for name, (kms, n) in kernels.items():
+        if n == 0:
+            continue
+        per_launch = kms / n
+        b = kernel_bytes(name, wl, variant, moved) * layers_per_launch
+        rec = {"launches": n, "us_per_launch": round(1e3 * per_launch, 3), "share": round(kms / total, 4),
+               "gbs": round(b / (per_launch / 1e3) / 1e9, 1)}
+        if name == "score_attn":
+            f = score_flops(wl) * layers_per_launch
+            rec["qkt_tflops"] = round(f / (per_launch / 1e3) / 1e12, 1)
+            rec["bound"] = "tensor" if f / (tflops_peak * 1e12) > b / (hbm_peak * 1e9) else "hbm"
+        out[name] = rec
+    return out
+
+
+def score_flops(wl):
+    """Algorithmic FLOPs of the window score of one layer: one QK^T over the unit's G*W window rows and its
+    N keys, 2 * G*W * N * d per unit (the kernel's second, transposed product is not counted)."""
+    return wl.batch * wl.num_kv_heads * 2 * wl.window_rows * wl.slots * wl.head_dim
+
+
+def roofline_of(kernels_tab, dom, wl, variant, moved, layers_per_launch, hbm_peak, tflops_peak, peak_kind, traffic):
+    rec = kernels_tab[dom]
+    if rec.get("bound") == "tensor":
+        f = score_flops(wl) * layers_per_launch
+        return {"bound": "tensor", "achieved": rec["qkt_tflops"], "peak": tflops_peak, "unit": "TFLOP/s",
+                "frac": round(rec["qkt_tflops"] / tflops_peak, 4), "traffic": traffic, "kernel": dom,
+                "algorithmic_flops_per_launch": f, "peak_source": peak_kind + " bf16 burst"}
+    b = kernel_bytes(dom, wl, variant, moved) * layers_per_launch
+    return {"bound": "hbm", "achieved": rec["gbs"], "peak": hbm_peak, "unit": "GB/s",
+            "frac": round(rec["gbs"] / hbm_peak, 4), "traffic": traffic, "kernel": dom,
+            "algorithmic_bytes_per_launch": b, "peak_source": peak_kind}
+
+
+def moved_rows(cache, torch):
+    """Rows per unit whose slot changed in the last eviction (layer slot 0 of the last call)."""
+    src = cache.debug_view(0)["src"].cpu()
+    K = src.shape[-1]
+    return float((src != torch.arange(K, dtype=torch.int32)).sum().item()) / src.shape[0]
+
+
+def profiled_kernels(torch, rig, steps, stream):
+    """The same steps again with a CUDA event pair around every launch (the library's profiling mode)."""
+    rig.cache.profile_enable(True)
+    ms, _ = timed_steps(torch, lambda: rig.step(stream), steps, stream)
+    rig.cache.profile_enable(False)
+    return rig.cache.profile_collect(), ms
+
+
+def traffic_of(dom, wl, variant, L):
+    """ncu DRAM bytes per launch of the dominant kernel, when a capture of these exact sources exists."""
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(tpath):
+        return None
+    try:
+        from paper_2606_03928_gb300.build import kernel_digest
+        with open(tpath) as f:
+            tr = json.load(f)
+        ent = tr.get(f"{dom}:{wl.name}:{variant}:{L}")
+        if ent and ent.get("kernel_digest") == kernel_digest(dom):
+            return ent["bytes_per_launch"]
+    except Exception:
+        return None
+    return None
+
+
+def score_ncu(wl):
+    """Tensor-pipe utilisation of the window-score kernel from its committed ncu capture at this workload, when
+    that capture was taken on the current sources (profiles/score_ncu.json)."""
+    path = os.path.join(ROOT, "profiles", "score_ncu.json")
+    if not os.path.exists(path):
+        return None
+    try:
+        from paper_2606_03928_gb300.build import kernel_digest
+        with open(path) as f:
+            d = json.load(f)
+        ent = d.get(wl.name)
+        if ent and ent.get("kernel_digest") == kernel_digest("score_attn"):
+            return {k: v for k, v in ent.items() if k != "kernel_digest"}
+    except Exception:
+        return None
+    return None
+
+
+# the other configurations measured in the same run, each as a record of the JSON line: the single-layer case,
+# the Qwen3-1.7B and Qwen3-8B geometries (both scoring variants) and the sweep's largest budget
+EXTRA_CONFIGS = [("single_layer_k256", "attnv", None), ("qwen3_1p7b_k2048", "attnv", None),
+                 ("qwen3_8b_k4096", "attnv", None), ("qwen3_8b_k4096", "dkv", None),
+                 ("sweep:16384:128:32:0.005", "attnv", 21)]
+
+
+def workload_by_name(Wm, name, layers=None):
+    if name.startswith("sweep:"):
+        _, K, Bf, b, rate = name.split(":")
+        wl = Wm.sweep_point(int(K), int(Bf), int(b), float(rate))
+    else:
+        wl = Wm.WORKLOADS[name]
+    if layers:
+        wl = Wm.shrink(wl, num_layers=min(layers, wl.num_layers))
+    return wl
+
+
+def measure_config(torch, V, Wm, name, variant, layers, steps, warmup, device, hbm_peak, tflops_peak):
+    wl = workload_by_name(Wm, name, layers)
+    rig = Rig(wl, variant, device, 1000, torch, V)
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        rig.step(stream)
+    ms, clocks = timed_steps(torch, lambda: rig.step(stream), steps, stream, sampler=ClockSampler(0))
+    kernels, _ = profiled_kernels(torch, rig, steps, stream)
+    st, code = rig.cache.check_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error in {name}: {code:#x}")
+    L = wl.num_layers
+    moved = moved_rows(rig.cache, torch)
+    tab = kernel_table(kernels, wl, variant, moved, min(L, 64), hbm_peak, tflops_peak)
+    roof_ms = L * step_bytes(wl, variant) / (hbm_peak * 1e9) * 1e3
+    rig.close()
+    torch.cuda.empty_cache()
+    return {"workload": wl.name, "variant": variant, "layers": L, "batch": wl.batch, "budget_k": wl.budget_k,
+            "buffer_b": wl.buffer_b, "window": wl.window, "heads": f"{wl.num_q_heads}/{wl.num_kv_heads}",
+            "steps": steps, "ms_per_step": round(ms, 4),
+            "token_heads_per_s": L * wl.batch * wl.num_kv_heads * wl.slots / (ms / 1e3),
+            "step_roofline_ms": round(roof_ms, 4), "step_roofline_frac": round(roof_ms / ms, 4),
+            "kernels": tab, "clocks": clocks}
+
+
 def run_ours(args):
     import torch
     import torch.distributed as dist
@@ -352,219 +567,87 @@ def run_ours(args):
     B.build()
     from paper_2606_03928_gb300 import vase as V
 
+    hbm_peak, tflops_peak, peak_kind = measured_peaks()
     L, K, Bf = wl.num_layers, wl.budget_k, wl.buffer_b
-    cache = V.VaseCache(V.Geometry(K, Bf, wl.window, wl.num_q_heads, wl.num_kv_heads, L, wl.batch),
-                        variant=args.variant, seed=0, device=device, reserve=args.reserve, gqa=args.gqa,
-                        dkv_shared_g=args.dkv_shared_g)
-    gen = torch.Generator(device=device)
-    gen.manual_seed(1000 + rank)
-    # prefill: the first K tokens of every layer (untimed)
-    for layer in range(L):
-        q, k, v = gen_stream(wl, K, gen, device, torch)
-        cache.append(layer, q, k, v)
-        del q, k, v
-    n_rounds = max(1, min(wl.rounds_per_layer, args.warmup + args.steps))
-    # per round: the B new tokens of every layer, stacked [L, B, b, H, d] for one batched append
-    chunks = []
-    for _ in range(n_rounds):
-        per_layer = [gen_stream(wl, Bf, gen, device, torch) for _ in range(L)]
-        chunks.append(tuple(torch.stack([pl[i] for pl in per_layer]) for i in range(3)))
-        del per_layer
-    torch.cuda.synchronize()
-
-    state = {"r": 0}
-
-    def step():
-        # every layer receives its B new decode tokens, then every layer is evicted (batched launches)
-        cache.append_all(*chunks[state["r"] % n_rounds])
-        cache.evict_all()
-        state["r"] += 1
+    rig = Rig(wl, args.variant, device, 1000 + rank, torch, V, reserve=args.reserve, gqa=args.gqa,
+              dkv_shared_g=args.dkv_shared_g)
+    cache = rig.cache
+    stream = torch.cuda.current_stream()
 
     def barrier():
         if world > 1:
             dist.barrier()
 
     for _ in range(args.warmup):
-        step()
+        rig.step(stream)
     st, code = cache.check_device_error()
     if st != 0:
         raise RuntimeError(f"device error during warm-up: {code:#x}")
 
-    stream = torch.cuda.current_stream()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    sampler = ClockSampler(local if world > 1 else 0)
     launches0 = cache.launch_count()
-    barrier()
-    torch.cuda.synchronize()
-    sampler.start()
-    ev0.record(stream)
-    for _ in range(args.steps):
-        step()
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    clocks = sampler.stop()
+    ms, clocks = timed_steps(torch, lambda: rig.step(stream), args.steps, stream, barrier,
+                             ClockSampler(local if world > 1 else 0))
     launches = cache.launch_count() - launches0
-    # the same K steps again with a CUDA event pair around every launch (the library's profiling mode), for
-    # each kernel's launch duration; the step time above is taken without those events
-    cache.profile_enable(True)
-    barrier()
-    torch.cuda.synchronize()
-    ep0, ep1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    ep0.record(stream)
-    for _ in range(args.steps):
-        step()
-    ep1.record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    cache.profile_enable(False)
-    kernels = cache.profile_collect()
-    profiled_ms = ep0.elapsed_time(ep1) / args.steps
-    ms = ev0.elapsed_time(ev1) / args.steps
+    # each kernel's launch duration: the same K steps again with a CUDA event pair around every launch (the
+    # library's profiling mode); the step time above is taken without those events
+    kernels, profiled_ms = profiled_kernels(torch, rig, args.steps, stream)
     st, code = cache.check_device_error()
     if st != 0:
         raise RuntimeError(f"device error in the timed region: {code:#x}")
     ms = max_over_ranks(ms, world, device)
     token_heads = L * wl.batch * wl.num_kv_heads * wl.slots
     value = whole_job_rate(token_heads, world, ms)
+    moved = moved_rows(cache, torch)
 
-    # moved rows per unit in the last eviction (rows whose slot changes) for the compaction's bytes
-    src = cache.debug_view(0)["src"].cpu()
-    moved = float((src != torch.arange(K, dtype=torch.int32)).sum().item()) / src.shape[0]
-
-    # ---- end to end through the C ABI with host buffers: pinned host inputs, host-side kept positions
-    e2e_steps = args.e2e_steps if args.e2e_steps is not None else max(1, min(args.steps, 50))
-    n_host = min(n_rounds, 4)
-    host_chunks = [[tuple(x[layer].cpu().pin_memory() for x in chunks[r]) for layer in range(L)]
-                   for r in range(n_host)]
-    pos_out = [torch.empty((wl.batch, wl.num_kv_heads, K), dtype=torch.int32).pin_memory() for _ in range(L)]
-    # bytes that cross the host link per step: every k and v row, and the query rows of the last W steps
-    # (the library reads no other query row: only the last W stay in the window ring)
-    q0, k0, v0 = host_chunks[0][0]
-    h2d = (k0.numel() * k0.element_size() + v0.numel() * v0.element_size()
-           + q0.numel() * q0.element_size() * min(wl.window, q0.shape[0]) // q0.shape[0]) * L
-    d2h = sum(p.numel() * p.element_size() for p in pos_out)
-
-    def e2e_step(r):  # host appends read the pinned buffers in place (vase_append_host)
-        c = host_chunks[r % n_host]
-        for layer in range(L):
-            cache.append_host(layer, *c[layer])
-        cache.evict_all()
-        for layer in range(L):
-            cache.read_positions(layer, pos_out[layer])
-
-    def timed(fn):
-        barrier()
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        fn()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        barrier()
-        t_ms = e0.elapsed_time(e1) / e2e_steps
-        return max_over_ranks(t_ms, world, device)
-
-    e2e_step(0)
-    zero_copy_ms = timed(lambda: [e2e_step(r) for r in range(e2e_steps)])
-
-    # Pipelined: a copy stream brings step r + 1's inputs into one of two device staging sets while step r
-    # appends (one vase_append_all_strided launch from the staging set) and evicts; it then reads step r's kept
-    # positions back.  The staging layout puts every layer's [last W query rows | k | v] back to back, so one
-    # copy per step moves them all; the append reads only the last W query rows, so each layer's q pointer is
-    # set W rows before its query rows (a pad of n - W rows at the front keeps layer 0's inside the buffer)
-    # and consecutive layers' inputs are one block apart.  Every step's copies and its position read-back stay
-    # in the timed region.
+    # ---- end to end through the C ABI from host buffers: every step's inputs cross from pinned host memory
+    # (vase_stage_host_inputs on a copy stream, the next step's copies issued before this step's kernels),
+    # are appended from the staging buffer (vase_append_all_staged), and every layer's kept positions come
+    # back to pinned host memory (vase_read_positions_all); all of it inside the timed region
+    e2e_steps = args.e2e_steps if args.e2e_steps is not None else max(1, min(args.steps, 20))
+    host_rounds = [tuple(t.cpu().pin_memory() for t in r) for r in rig.rounds]
+    staging = cache.host_staging(Bf)
     copy_stream = torch.cuda.Stream(device=device)
-    n_tok = q0.shape[0]
-    W_q = min(wl.window, n_tok)
-    q_row = q0.numel() // n_tok                  # bf16 elements of one step's query rows
-    kv_el = k0.numel()
-    pad = (n_tok - W_q) * q_row
-    blk = W_q * q_row + 2 * kv_el                # one layer's [query tail | k | v]
-    total = pad + L * blk
+    pos_host = torch.empty((L, wl.batch, wl.num_kv_heads, K), dtype=torch.int32).pin_memory()
+    q0, k0, v0 = host_rounds[0]
+    h2d = sum(t.numel() * t.element_size() for t in (q0, k0, v0))
+    d2h = pos_host.numel() * pos_host.element_size()
+    Wq, q_step = rig.w_q, rig.q_step
 
-    host_flat = []
-    for r in range(n_host):
-        f = torch.empty(total, dtype=torch.bfloat16).pin_memory()
-        for layer in range(L):
-            qh, kh, vh = host_chunks[r][layer]
-            o = pad + layer * blk
-            f[o:o + W_q * q_row].copy_(qh[-W_q:].reshape(-1))
-            f[o + W_q * q_row:o + W_q * q_row + kv_el].copy_(kh.reshape(-1))
-            f[o + W_q * q_row + kv_el:o + blk].copy_(vh.reshape(-1))
-        host_flat.append(f)
-    dev_flat = [torch.empty(total, dtype=torch.bfloat16, device=device) for _ in range(2)]
-    pos_host = torch.empty(cache.positions.shape, dtype=torch.int32).pin_memory()
-    copied = [torch.cuda.Event() for _ in range(2)]
-    consumed = [torch.cuda.Event() for _ in range(2)]
-    evicted = torch.cuda.Event()
-    # layer 0's (q, k, v) in each staging set; layer l's are l blocks (2 * blk bytes) further on
-    ptr0 = [(f.data_ptr(), f.data_ptr() + 2 * (pad + W_q * q_row), f.data_ptr() + 2 * (pad + W_q * q_row + kv_el))
-            for f in dev_flat]
+    def stage(r):
+        q, k, v = host_rounds[r % len(host_rounds)]
+        V.vase_stage_host_inputs(cache.ctx, q.data_ptr() - (Bf - Wq) * q_step, k.data_ptr(), v.data_ptr(), Bf,
+                                 q[0].numel() * 2, k[0].numel() * 2, staging.data_ptr(), staging.numel(),
+                                 copy_stream)
 
-    def issue_copy(r):
-        b = r % 2
-        with torch.cuda.stream(copy_stream):
-            if r >= 2:
-                copy_stream.wait_event(consumed[b])
-            dev_flat[b][pad:].copy_(host_flat[r % n_host][pad:], non_blocking=True)
-            copied[b].record(copy_stream)
-
-    def pipelined():
-        issue_copy(0)
-        for r in range(e2e_steps):
-            if r + 1 < e2e_steps:
-                issue_copy(r + 1)
-            b = r % 2
-            stream.wait_event(copied[b])
-            V.vase_append_all_strided(cache.ctx, *ptr0[b], n_tok, 2 * blk, 2 * blk, stream)
-            consumed[b].record(stream)
-            cache.evict_all()
-            evicted.record(stream)
-            # every layer's kept positions in one copy, on the copy stream behind the next step's inputs (one
-            # copy engine serves both directions here, so a read-back on the compute stream would wait for them)
-            with torch.cuda.stream(copy_stream):
-                copy_stream.wait_event(evicted)
-                pos_host.copy_(cache.positions, non_blocking=True)
+    def e2e_run(n):
+        stage(0)
+        for r in range(n):
+            if r + 1 < n:
+                stage(r + 1)
+            cache.append_all_staged(stream)
+            cache.evict_all(stream)
+            cache.read_positions_all(pos_host, copy_stream, stream)
         stream.wait_stream(copy_stream)  # the last read-back ends inside the timed region
 
-    e2e_ms = timed(pipelined)
+    e2e_run(2)  # warm-up of the host path
+    e2e_total, _ = timed_steps(torch, lambda: e2e_run(e2e_steps), 1, stream, barrier)
+    e2e_ms = max_over_ranks(e2e_total / e2e_steps, world, device)
     e2e_value = whole_job_rate(token_heads, world, e2e_ms)
+    st, code = cache.check_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error in the end-to-end steps: {code:#x}")
 
     # ---- roofline of the dominant kernel
-    hbm_peak, _, peak_kind = measured_peaks()
-    per_kernel = {}
-    total_k = sum(v[0] for v in kernels.values()) or 1.0
     layers_per_launch = min(L, 64)
-    for name, (kms, n) in kernels.items():
-        if n == 0:
-            continue
-        per_launch = kms / n
-        b = kernel_bytes(name, wl, args.variant, moved) * layers_per_launch
-        per_kernel[name] = {"launches": n, "us_per_launch": round(1e3 * per_launch, 3),
-                            "share": round(kms / total_k, 4),
-                            "gbs": round(b / (per_launch / 1e3) / 1e9, 1)}
-    dom = max(per_kernel, key=lambda k: per_kernel[k]["share"])
-    dom_bytes = kernel_bytes(dom, wl, args.variant, moved) * layers_per_launch
-    achieved = per_kernel[dom]["gbs"]
-    traffic = None
-    tpath = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tpath):
-        try:
-            from paper_2606_03928_gb300.build import kernel_digest
-            with open(tpath) as f:
-                tr = json.load(f)
-            ent = tr.get(f"{dom}:{wl.name}:{args.variant}:{L}")
-            if ent and ent.get("kernel_digest") == kernel_digest(dom):
-                traffic = ent["bytes_per_launch"]
-        except Exception:
-            traffic = None
-    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                "frac": round(achieved / hbm_peak, 4), "traffic": traffic, "kernel": dom,
-                "algorithmic_bytes_per_launch": dom_bytes, "peak_source": peak_kind}
+    tab = kernel_table(kernels, wl, args.variant, moved, layers_per_launch, hbm_peak, tflops_peak)
+    dom = max(tab, key=lambda k: tab[k]["share"])
+    roofline = roofline_of(tab, dom, wl, args.variant, moved, layers_per_launch, hbm_peak, tflops_peak, peak_kind,
+                           traffic_of(dom, wl, args.variant, L))
     step_roof_ms = L * step_bytes(wl, args.variant) / (hbm_peak * 1e9) * 1e3
     evict_ms = sum(kernels[k][0] for k in kernels if k != "append") / args.steps
+    rig.close()
+    del staging, host_rounds
+    torch.cuda.empty_cache()
 
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -574,20 +657,26 @@ def run_ours(args):
                    "global_batch": wl.batch * world,
                    "seq_len": wl.slots, "budget_k": K, "buffer_b": Bf, "window": wl.window,
                    "heads": f"{wl.num_q_heads}/{wl.num_kv_heads}", "parallelism": f"dp{world}",
-                   "l2": "inputs larger than L2 (about 3.9 GB touched per step)"},
+                   "l2": f"inputs larger than L2 (about {L * step_bytes(wl, args.variant) / 1e9:.1f} GB touched per step)"},
         "roofline": roofline,
         "step_roofline": {"ms_per_step_at_hbm_peak": round(step_roof_ms, 4),
                           "frac": round(step_roof_ms / ms, 4),
                           "amortised_us_per_decode_token": round(1e3 * evict_ms / Bf, 3)},
-        "kernels": per_kernel,
+        "kernels": tab,
+        "score_kernel_ncu": score_ncu(wl) if args.variant == "attnv" else None,
         "kernels_pass_ms_per_step": round(profiled_ms, 4),
         "clocks": clocks,
         "gpu_launches": launches,
-        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": pos_host.numel() * pos_host.element_size(),
-                "ms_per_step": e2e_ms, "form": "next step's inputs copied (one copy) on a second stream during this step, appended in one launch",
-                "zero_copy_ms_per_step": zero_copy_ms},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_ms, "steps": e2e_steps,
+                "form": "C ABI: vase_stage_host_inputs (pinned host -> device on a copy stream, the next step's "
+                        "copies issued before this step's kernels), vase_append_all_staged, vase_evict_all, "
+                        "vase_read_positions_all (every layer's kept positions to pinned host memory)"},
     }
+    if rank == 0 and world == 1 and not args.no_configs:
+        out["configs"] = [measure_config(torch, V, Wm, name, variant, layers, args.steps, args.warmup, device,
+                                         hbm_peak, tflops_peak)
+                          for (name, variant, layers) in EXTRA_CONFIGS]
     if pool is not None:
         v, done, wall = oracle_throughput(pool, n_units, wl, args.cpu_seconds)
         pool.close()

@@ -67,3 +67,29 @@ def test_clock_sampler_keeps_every_sample_when_no_stamp_parses():
             "t1, 0, 1980, 2070, 950.0, 0x0, Active, Not Active, Not Active, Not Active"]
     out = _sampler_with_rows(rows, time.time()).stop()
     assert out == {"sm_mhz": 2025.0, "sm_max_mhz": 2070.0, "reasons": ["hw_slowdown"], "samples": 2}
+
+
+def test_clock_sampler_brackets_a_region_shorter_than_the_sampling_interval():
+    """No sample inside the region: the last sample before it and the first after it stand for it."""
+    now = time.time()
+    rows = [f"{_stamp(now - 5)}, 0, 345, 2070, 100.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+            f"{_stamp(now - 0.2)}, 0, 2070, 2070, 900.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+            f"{_stamp(now + 0.5)}, 0, 2040, 2070, 950.0, 0x4, Not Active, Not Active, Not Active, Active",
+            f"{_stamp(now + 9)}, 0, 300, 2070, 100.0, 0x0, Active, Not Active, Not Active, Not Active"]
+    cs = _sampler_with_rows(rows, now - 0.1)
+    out = cs.stop()
+    assert out == {"sm_mhz": 2055.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 2,
+                   "bracketing": True}
+
+
+def test_score_roofline_bound_follows_the_algorithmic_ratio():
+    """The window score is tensor-bound where its QK^T FLOPs at the bf16 peak outlast its bytes at the HBM
+    peak (Qwen3-32B geometry, G*W = 512) and HBM-bound otherwise (Qwen3-1.7B geometry, G*W = 32)."""
+    for name, bound in (("qwen3_32b_k8192", "tensor"), ("qwen3_1p7b_k2048", "hbm")):
+        wl = W.WORKLOADS[name]
+        tab = bench.kernel_table({"score_attn": (1.0, 1), "select_compact": (1.0, 1)}, wl, "attnv", 100.0, 8,
+                                 6799.3, 1897.1)
+        assert tab["score_attn"]["bound"] == bound
+        roof = bench.roofline_of(tab, "score_attn", wl, "attnv", 100.0, 8, 6799.3, 1897.1, "measured", None)
+        assert roof["bound"] == bound and roof["unit"] == ("TFLOP/s" if bound == "tensor" else "GB/s")
+        assert roof["frac"] == pytest.approx(roof["achieved"] / roof["peak"], rel=1e-3)

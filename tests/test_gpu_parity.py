@@ -527,6 +527,106 @@ def test_qwen3_1p7b_k2048_all_layers_in_one_launch():
                               variant="attnv", n_v=wl.budget_k // 4, check_scores=False)
 
 
+def _unit_state_from_stream(wl, ch, t0, t1, s, h):
+    """[t0, t1) of a host stream chunk as one unit's rows: keys and values [n, d], and the query rows of its G
+    heads over the last W steps of the range, head-major [G*W, d]."""
+    G, Wn = wl.group, wl.window
+    q = ch["q_bits"][t1 - Wn:t1, s, h * G:(h + 1) * G]            # [W, G, d]
+    return (ch["k_bits"][t0:t1, s, h], ch["v_bits"][t0:t1, s, h],
+            np.ascontiguousarray(q.transpose(1, 0, 2)).reshape(G * Wn, wl.head_dim))
+
+
+def test_qwen3_1p7b_k2048_appended_stream_two_rounds_in_the_bench_launch():
+    """The bench's launch (all 28 layers per kernel launch, debug outputs on), driven as the bench drives it:
+    every layer's stream enters through the library's append (K + B tokens each, then B more for every layer in
+    one vase_append_all_strided launch from [last W query rows | k | v] blocks), and every layer is evicted twice.
+    The value magnitudes the appends computed are compared with the oracle's for every unit of three layers; after
+    each eviction, sampled units of those layers are compared with the oracle on the chained state (window
+    scores, pooled scores, keys, kept sets, compacted rows), the second round on the oracle's own compaction of
+    the first.  Layer l runs host stream l % 2."""
+    from paper_2606_03928_gb300 import vase as V
+    wl = W.WORKLOADS["qwen3_1p7b_k2048"]
+    L, K, B, N, Wn, G = wl.num_layers, wl.budget_k, wl.buffer_b, wl.slots, wl.window, wl.group
+    b, Hq, Hkv, d = wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim
+    cache = _cache(wl, L, debug=True)
+    dev = cache.device
+    streams = [W.stream_chunk(wl, 23, i, 0, N + B) for i in range(2)]
+    dstreams = [{x: PU.bits_to_bf16_tensor(c[x], dev) for x in ("q_bits", "k_bits", "v_bits")} for c in streams]
+    for layer in range(L):  # the first K + B tokens of each layer, appended through the library
+        ds = dstreams[layer % 2]
+        cache.append(layer, ds["q_bits"][:N], ds["k_bits"][:N], ds["v_bits"][:N])
+    layers, units = (0, 13, L - 1), [(0, 0), (3, 5), (b - 1, Hkv - 1)]
+    torch.cuda.synchronize()
+    for layer in layers:  # magnitudes computed by the append kernel, every unit
+        ch = streams[layer % 2]
+        vref = O.value_magnitude(O.bf16_bits_to_f64(ch["v_bits"][:N].transpose(1, 2, 0, 3)).reshape(-1, d))
+        PU.assert_close_scores(cache.value_scores[layer].cpu().numpy().reshape(-1), vref, "append magnitudes")
+    # round 0
+    assert cache.evict_all() == L
+    assert cache.check_device_error()[0] == 0
+    chained = {}
+    z_of = {}
+    for z in range(L):
+        z_of[cache.debug_view(z)["layer"]] = z
+    for layer in layers:
+        ch = streams[layer % 2]
+        dv = {k: (v.cpu().numpy() if k != "layer" else v) for k, v in cache.debug_view(z_of[layer]).items()}
+        got = PU.download(cache, layer)
+        got.update({k: v for k, v in dv.items() if k != "layer"})
+        for (s_, h) in units:
+            k0, v0, q0 = _unit_state_from_stream(wl, ch, 0, N, s_, h)
+            pos0 = np.arange(N)
+            ref = O.evict_unit_bits(q0, k0, v0, pos0, budget_k=K, buffer_b=B, seed=0, layer=layer, seq=s_, head=h,
+                                    num_kv_heads=Hkv, rnd=0, group=G)
+            gu = PU.unit_slice(got, s_, h, Hkv)
+            PU.check_unit(wl, ref, gu, k0, v0, pos0, variant="attnv", n_v=K // 4)
+            if np.array_equal(gu["src"], ref["src"]):  # chain only from a state both sides agree on
+                chained[(layer, s_, h)] = ref
+    # round 1: B new tokens for every layer in one strided launch from per-layer [W query rows | k | v] blocks
+    qtail = [dstreams[i]["q_bits"][N + B - Wn:N + B] for i in range(2)]
+    blk = Wn * b * Hq * d + 2 * B * b * Hkv * d
+    flat = torch.empty((L * blk,), dtype=torch.bfloat16, device=dev)
+    for layer in range(L):
+        ds, o = dstreams[layer % 2], layer * blk
+        flat[o:o + Wn * b * Hq * d] = qtail[layer % 2].reshape(-1)
+        flat[o + Wn * b * Hq * d:o + Wn * b * Hq * d + B * b * Hkv * d] = ds["k_bits"][N:N + B].reshape(-1)
+        flat[o + Wn * b * Hq * d + B * b * Hkv * d:o + blk] = ds["v_bits"][N:N + B].reshape(-1)
+    base = flat.data_ptr()
+    q_ptr = base - (B - Wn) * b * Hq * d * 2  # the append reads only the last W query rows of each layer
+    k_ptr = base + Wn * b * Hq * d * 2
+    v_ptr = k_ptr + B * b * Hkv * d * 2
+    assert V.vase_append_all_strided(cache.ctx, q_ptr, k_ptr, v_ptr, B, blk * 2, blk * 2) == V.VASE_EVICT_DUE
+    torch.cuda.synchronize()
+    for layer in layers:  # the appended slots' magnitudes, every unit
+        ch = streams[layer % 2]
+        vref = O.value_magnitude(O.bf16_bits_to_f64(ch["v_bits"][N:N + B].transpose(1, 2, 0, 3)).reshape(-1, d))
+        PU.assert_close_scores(cache.value_scores[layer][..., K:].cpu().numpy().reshape(-1), vref,
+                               "append magnitudes, second round")
+    assert cache.evict_all() == L
+    assert cache.check_device_error()[0] == 0
+    for z in range(L):
+        z_of[cache.debug_view(z)["layer"]] = z
+    compared = 0
+    for layer in layers:
+        ch = streams[layer % 2]
+        dv = {k: (v.cpu().numpy() if k != "layer" else v) for k, v in cache.debug_view(z_of[layer]).items()}
+        got = PU.download(cache, layer)
+        got.update({k: v for k, v in dv.items() if k != "layer"})
+        for (s_, h) in units:
+            prev = chained.get((layer, s_, h))
+            if prev is None:
+                continue
+            k1 = np.concatenate([prev["k_bits_new"], ch["k_bits"][N:N + B, s_, h]])
+            v1 = np.concatenate([prev["v_bits_new"], ch["v_bits"][N:N + B, s_, h]])
+            pos1 = np.concatenate([prev["positions_new"], np.arange(N, N + B)])
+            _, _, q1 = _unit_state_from_stream(wl, ch, N, N + B, s_, h)
+            ref = O.evict_unit_bits(q1, k1, v1, pos1, budget_k=K, buffer_b=B, seed=0, layer=layer, seq=s_, head=h,
+                                    num_kv_heads=Hkv, rnd=1, group=G)
+            PU.check_unit(wl, ref, PU.unit_slice(got, s_, h, Hkv), k1, v1, pos1, variant="attnv", n_v=K // 4)
+            compared += 1
+    assert compared >= len(layers) * len(units) - 2  # a first-round threshold tie may end a unit's chain
+
+
 # ----------------------------------------------------------------------------- variants: GQA max-aggregation, shared-G DKV, random reservation
 
 def _reserved_slots(key_row, K):

@@ -463,7 +463,7 @@ def test_append_all_strided_from_one_staging_block_equals_packed_append_all():
 # ----------------------------------------------------------------------------- interleaved (persistent) schedule
 
 @pytest.mark.parametrize("K,B,Wn,Hq,Hkv", [(192, 64, 16, 16, 8), (200, 40, 16, 16, 8), (256, 64, 32, 32, 8),
-                                          (160, 96, 32, 64, 8)])
+                                          (160, 96, 32, 64, 8), (160, 64, 64, 64, 8)])
 def test_evict_all_with_several_units_per_cta_matches_oracle(K, B, Wn, Hq, Hkv):
     """Eight layers of 64 units: more than two items per SM, so one CTA per SM takes a strided list of units and
     interleaves the pass-B sweep of each with the pass-A sweep of the next.  Every unit of every layer is checked."""
@@ -487,6 +487,35 @@ def test_evict_all_with_several_units_per_cta_matches_oracle(K, B, Wn, Hq, Hkv):
                 ref = PU.oracle_unit(wl, st, s, h, variant="attnv", round_index=3 + layer, seed=0, layer=layer)
                 PU.check_unit(wl, ref, PU.unit_slice(got, s, h, wl.num_kv_heads), st["k_bits"][s, h],
                               st["v_bits"][s, h], st["positions"][s, h], variant="attnv", n_v=wl.budget_k // 4)
+
+
+def test_sixteen_layers_of_512_window_rows_match_oracle():
+    """G*W = 512 window rows (the Qwen3-32B group and window) on sixteen layers in one batched launch, one CTA
+    per unit scoring four 128-row blocks in pass A and two 256-row items in pass B: every layer's workspace
+    slot, kept set and compacted rows are checked on sampled units, and every layer's counters advance."""
+    wl = W.shrink(W.WORKLOADS["qwen3_32b_k8192"], budget_k=192, buffer_b=64, batch=2, num_layers=16)
+    L = wl.num_layers
+    cache = _cache(wl, L)
+    states = [W.layer_state(wl, 17, layer, 5 + layer, "gapped") for layer in range(L)]
+    for layer, st in enumerate(states):
+        PU.upload_layer(cache, layer, st, 5 + layer)
+    assert cache.evict_all() == L
+    status, code = cache.check_device_error()
+    assert status == 0, f"device error word {code:#x}"
+    seen = set()
+    for z in range(L):
+        dv = {k: (v.cpu().numpy() if k != "layer" else v) for k, v in cache.debug_view(z).items()}
+        layer = dv["layer"]
+        seen.add(layer)
+        st = states[layer]
+        got = PU.download(cache, layer)
+        got.update({k: v for k, v in dv.items() if k != "layer"})
+        for (s_, h) in ((0, 0), (1, 7), (z % 2, z % 8)):
+            ref = PU.oracle_unit(wl, st, s_, h, variant="attnv", round_index=5 + layer, seed=0, layer=layer)
+            PU.check_unit(wl, ref, PU.unit_slice(got, s_, h, wl.num_kv_heads), st["k_bits"][s_, h],
+                          st["v_bits"][s_, h], st["positions"][s_, h], variant="attnv", n_v=wl.budget_k // 4)
+        assert cache.layer_state(layer)["fill"] == wl.budget_k and cache.layer_state(layer)["round"] == 6 + layer
+    assert seen == set(range(L))
 
 
 def test_qwen3_1p7b_k2048_all_layers_in_one_launch():

@@ -211,6 +211,9 @@ def kernel_bytes(kind, wl, variant, moved_rows_per_unit):
     if kind == "select_compact":
         # scores, magnitudes and positions in; kept list, positions, magnitudes and the moved K/V rows out
         return U * (N * 4 + K * 4 + K * 4 + K * 4) + U * moved_rows_per_unit * (2 * 2 * row + 8)
+    if kind == "evict_small":  # window score, selection and gather of one unit in one launch
+        return kernel_bytes("score_attn", wl, variant, moved_rows_per_unit) + \
+            kernel_bytes("select_compact", wl, variant, moved_rows_per_unit)
     if kind == "append":
         # k and v rows of the B steps in and out, the query rows of the last W steps in and out (earlier
         # queries never reach the window ring), positions and value magnitudes out

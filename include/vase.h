@@ -345,7 +345,7 @@ int64_t vase_launch_count(const vase_ctx* ctx);
 #define VASE_KERNEL_VALUE 2   /* value magnitude refresh (vase_refresh_value_scores) */
 #define VASE_KERNEL_DKV 3     /* DKV leverage scores (tcgen05) */
 #define VASE_KERNEL_SELECT 4  /* reservation + sampling + kept list + stable in-place gather of the kept rows */
-#define VASE_KERNEL_COMPACT 5 /* reserved: the gather runs inside the selection kernel (no launches) */
+#define VASE_KERNEL_EVICT_SMALL 5 /* window score + selection + gather in one launch (launch-bound batches of small units) */
 #define VASE_KERNEL_COUNT 6
 
 /* enable = 1: from now on record a CUDA event pair on the launch stream around

@@ -38,6 +38,10 @@ struct Plan {
     size_t stride_attn, stride_un, stride_src;  // elements per workspace slot
     size_t off_err, off_attn, off_pooled, off_vscore, off_key, off_keep, off_src, off_staging, staging_bytes, ws_bytes;
     size_t decode_smem;                           // decode attention: shared memory per CTA
+    // fused eviction of small units (evict_small_kernel): usable when the unit's score matrix fits in TMEM
+    bool small_ok;
+    int small_tiles, small_stages, small_tmem_cols;
+    size_t small_smem;
 };
 
 // Launch parameters of the window-score kernel for `nz` layers of `batch`.
@@ -243,6 +247,14 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     o = align_up(o + p.staging_bytes, kAlign);
     p.decode_smem = decode_smem_bytes(p.G);
     p.ws_bytes = o;
+    // fused small-unit eviction: AttnV, at most 128 window rows, every 128-token tile's S = K Q^T resident in TMEM
+    p.small_tiles = p.n_tiles;
+    p.small_stages = p.n_tiles < 4 ? p.n_tiles : 4;
+    p.small_tmem_cols = 32;
+    while (p.small_tmem_cols < p.n_tiles * p.GWp) p.small_tmem_cols *= 2;
+    p.small_smem = evict_small_smem_bytes(p.N, c->budget_k, p.GWp, p.q_box, p.n_tiles, p.small_stages);
+    p.small_ok = c->variant == VASE_VARIANT_ATTNV && p.GWp <= 128 && p.n_tiles <= kSmallMaxTiles &&
+                 p.n_tiles * p.GWp <= 512 && p.q_box >= p.GWp && p.small_smem <= kMaxDynSmem;
     return true;
 }
 
@@ -511,7 +523,8 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
         (e = select_set_attributes(P.select_smem)) != cudaSuccess ||
         (e = decode_set_attributes(P.G, P.decode_smem)) != cudaSuccess ||
         (e = decode_mixed_set_attributes()) != cudaSuccess ||
-        (e = quantize_set_attributes(quantize_smem_bytes(cfg->budget_k, cfg->buffer_b))) != cudaSuccess) {
+        (e = quantize_set_attributes(quantize_smem_bytes(cfg->budget_k, cfg->buffer_b))) != cudaSuccess ||
+        (P.small_ok && (e = evict_small_set_attributes(P.small_smem)) != cudaSuccess)) {
         fprintf(stderr, "vase_create: kernel attributes: %s\n", cudaGetErrorString(e));
         delete ctx;
         return VASE_ERR_CUDA;
@@ -602,6 +615,43 @@ LayerBatch make_batch(vase_ctx* ctx, const int32_t* layers, int nz) {
     return b;
 }
 
+// The selection's parameter block for one batched eviction (workspace arrays of the batch's first slot).
+void fill_select_params(vase_ctx* ctx, const LayerBatch& batch, float* attn, float* vscore, int32_t* src,
+                        uint32_t* err, SelectParams* out) {
+    const Plan& P = ctx->plan;
+    const vase_config& c = ctx->cfg;
+    SelectParams& sel = *out;
+    sel.batch = batch;
+    sel.attn = attn;
+    sel.dkv = vscore;
+    sel.vmag = ctx->bufs.value_scores;
+    sel.vscore_dbg = (c.debug_outputs && c.variant == VASE_VARIANT_ATTNV) ? vscore : nullptr;
+    sel.pos = ctx->bufs.positions;
+    sel.kc = static_cast<uint4*>(ctx->bufs.k_cache);
+    sel.vc = static_cast<uint4*>(ctx->bufs.v_cache);
+    sel.src = src;
+    sel.pooled_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_pooled) : nullptr;
+    sel.key_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_key) : nullptr;
+    sel.keep_dbg = c.debug_outputs ? ctx->ws + P.off_keep : nullptr;
+    sel.N = P.N;
+    sel.K = c.budget_k;
+    sel.B = c.buffer_b;
+    sel.n_v = P.n_v;
+    sel.m = P.m;
+    sel.pool = c.pool_kernel;
+    sel.variant = c.variant;
+    sel.stochastic = c.stochastic;
+    sel.Hkv = c.num_kv_heads;
+    sel.n_parts = c.variant == VASE_VARIANT_ATTNV ? P.n_rb : 1;
+    sel.staged = P.select_staged ? 1 : 0;
+    sel.reserve_random = c.reserve_kind == VASE_RESERVE_RANDOM ? 1 : 0;
+    sel.gqa_max = c.gqa_reduce == VASE_GQA_MAX ? 1 : 0;
+    sel.units = P.units;
+    sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
+    sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
+    sel.err = err;
+}
+
 // One eviction step for up to kMaxLayerBatch full layers: every kernel covers all of them in one launch.
 int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     const Plan& P = ctx->plan;
@@ -615,6 +665,42 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     if (ctx->read_pending) {  // the positions a read-back copies must not move before it has run
         if ((e = cudaStreamWaitEvent(s, ctx->read_done, 0)) != cudaSuccess) return cuda_fail(ctx, e, "read-back wait");
         ctx->read_pending = false;
+    }
+    SelectParams sel;
+    fill_select_params(ctx, batch, attn, vscore, src, err, &sel);
+    // Launch-bound batches (every unit of every layer in one wave, one CTA each) whose units are small enough for
+    // the fused kernel: score, selection and gather in one launch
+    if (P.small_ok && static_cast<long>(P.units) * nz <= P.num_sms) {
+        SmallEvictParams sm;
+        sm.sel = sel;
+        sm.sel.n_parts = 1;
+        sm.sel.staged = 1;
+        sm.GW = P.GW;
+        sm.GWp = P.GWp;
+        sm.q_rows = P.q_box;
+        sm.n_tiles = P.small_tiles;
+        sm.stages = P.small_stages;
+        sm.tmem_cols = P.small_tmem_cols;
+        sm.Hq = c.num_q_heads;
+        sm.W = c.window;
+        sm.G = P.G;
+        sm.head_rows = c.gqa_reduce == VASE_GQA_MAX ? c.window : 0;
+        sm.fold_rows = c.gqa_reduce == VASE_GQA_MAX ? c.window : P.GW;
+        sm.layer_rows = static_cast<int64_t>(P.units) * P.N;
+        sm.q_layer_rows = static_cast<int64_t>(c.batch) * c.num_q_heads * c.window;
+        sm.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
+        sm.attn = attn;
+        if ((e = timed_launch(ctx, VASE_KERNEL_EVICT_SMALL, s, [&] {
+                 return launch_evict_small(ctx->kmap, ctx->qmap, sm, P.units, P.small_smem, s);
+             })) != cudaSuccess)
+            return cuda_fail(ctx, e, "fused small-unit eviction launch");
+        ctx->launches += 1;
+        for (int z = 0; z < nz; ++z) {
+            vase_layer_state& st = ctx->layers[layers[z]];
+            st.fill = c.budget_k;
+            st.round += 1;
+        }
+        return VASE_OK;
     }
     if (c.variant == VASE_VARIANT_ATTNV) {
         const ScoreAttnParams sp = score_params(P, c, batch, nz, attn, err);
@@ -647,36 +733,6 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
             return cuda_fail(ctx, e, "dkv launch");
         ctx->launches += 1;
     }
-    SelectParams sel;
-    sel.batch = batch;
-    sel.attn = attn;
-    sel.dkv = vscore;
-    sel.vmag = ctx->bufs.value_scores;
-    sel.vscore_dbg = (c.debug_outputs && c.variant == VASE_VARIANT_ATTNV) ? vscore : nullptr;
-    sel.pos = ctx->bufs.positions;
-    sel.kc = static_cast<uint4*>(ctx->bufs.k_cache);
-    sel.vc = static_cast<uint4*>(ctx->bufs.v_cache);
-    sel.src = src;
-    sel.pooled_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_pooled) : nullptr;
-    sel.key_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_key) : nullptr;
-    sel.keep_dbg = c.debug_outputs ? ctx->ws + P.off_keep : nullptr;
-    sel.N = P.N;
-    sel.K = c.budget_k;
-    sel.B = c.buffer_b;
-    sel.n_v = P.n_v;
-    sel.m = P.m;
-    sel.pool = c.pool_kernel;
-    sel.variant = c.variant;
-    sel.stochastic = c.stochastic;
-    sel.Hkv = c.num_kv_heads;
-    sel.n_parts = c.variant == VASE_VARIANT_ATTNV ? P.n_rb : 1;
-    sel.staged = P.select_staged ? 1 : 0;
-    sel.reserve_random = c.reserve_kind == VASE_RESERVE_RANDOM ? 1 : 0;
-    sel.gqa_max = c.gqa_reduce == VASE_GQA_MAX ? 1 : 0;
-    sel.units = P.units;
-    sel.seed_lo = static_cast<uint32_t>(c.seed & 0xFFFFFFFFull);
-    sel.seed_hi = static_cast<uint32_t>(c.seed >> 32);
-    sel.err = err;
     if ((e = timed_launch(ctx, VASE_KERNEL_SELECT, s, [&] { return launch_select(sel, P.units, P.select_smem, P.select_threads, s); })) !=
         cudaSuccess)
         return cuda_fail(ctx, e, "select launch");

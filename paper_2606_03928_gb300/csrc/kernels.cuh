@@ -27,6 +27,10 @@ enum ErrSite : uint32_t {
     kErrDecodeEmpty = 49,
     kErrDecodeDrain = 50,
     kErrDecodeMask = 51,
+    kErrSmallQ = 64,
+    kErrSmallKFull = 65,
+    kErrSmallKFree = 66,
+    kErrSmallDone = 67,
 };
 
 constexpr int kTileTokens = 128;   // tokens per MMA tile (M)
@@ -88,6 +92,7 @@ struct AppendParams {
     int32_t* pos;     // base of [L][b][Hkv][N]
     float* vmag;      // base of [L][b][Hkv][N]: value magnitude of each cached token
     int32_t n, b, Hq, Hkv, W, N, kind;
+    int32_t steps_per_block;         // decode steps per block (set by launch_append)
     int32_t layer[kMaxLayerBatch];
     int32_t fill[kMaxLayerBatch];
     int64_t next_pos[kMaxLayerBatch];
@@ -169,6 +174,26 @@ struct SelectParams {
 };
 
 
+// The fused eviction of small units (evict_small_kernel): one CTA per unit scores it, selects and gathers in one
+// launch.  sel is the selection's block (one score part, staged); the rest describes the window score.
+struct SmallEvictParams {
+    SelectParams sel;
+    int32_t GW, GWp;        // window rows per unit, padded to 32
+    int32_t q_rows;         // window rows per TMA box of the window map and per shared-memory panel (>= GWp)
+    int32_t n_tiles;        // ceil(N / 128): 128-token tiles, all resident in TMEM as S = K Q^T
+    int32_t stages;         // K tile ring depth
+    int32_t tmem_cols;
+    int32_t Hq, W, G;
+    int32_t head_rows;      // 0: mean over the G*W rows; W: per query head, the largest head mean (GQA max)
+    int32_t fold_rows;      // G*W (mean) or W (max)
+    int64_t layer_rows;     // cache rows per layer
+    int64_t q_layer_rows;   // window rows per layer
+    float scale_log2;       // log2(e) / sqrt(d)
+    float* attn;            // [slot][units][N]: the window score, written for the debug view (nullable)
+};
+constexpr int kSmallThreads = 256;
+constexpr int kSmallMaxTiles = 8;
+
 // Mixed-precision values of one layer: codes of the unreserved kept value rows, their (s, z), and the
 // reserved-slot mask (bit t of word w: slot 32 w + t keeps its bf16 row).
 struct QuantParams {
@@ -209,6 +234,10 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
 cudaError_t launch_dkv(const CUtensorMap& kmap, const CUtensorMap& vmap, const DkvParams& p, int units,
                        size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, int units, size_t smem_bytes, int threads, cudaStream_t s);
+size_t evict_small_smem_bytes(int N, int K, int GWp, int q_rows, int n_tiles, int stages);
+cudaError_t evict_small_set_attributes(size_t smem_bytes);
+cudaError_t launch_evict_small(const CUtensorMap& kmap, const CUtensorMap& qmap, const SmallEvictParams& p, int units,
+                               size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_quantize(const QuantParams& p, int units, size_t smem_bytes, cudaStream_t s);
 size_t quantize_smem_bytes(int K, int B);
 cudaError_t quantize_set_attributes(size_t smem_bytes);

@@ -79,8 +79,8 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
     const int z = blockIdx.y;  // layer slot
     const int layer = p.layer[z];
     const int s = static_cast<int>(blockIdx.x) % p.b;  // sequence
-    const int t0 = (static_cast<int>(blockIdx.x) / p.b) * kAppendSteps;
-    const int t1 = min(p.n, t0 + kAppendSteps);
+    const int t0 = (static_cast<int>(blockIdx.x) / p.b) * p.steps_per_block;
+    const int t1 = min(p.n, t0 + p.steps_per_block);
     const int Hq = p.Hq, Hkv = p.Hkv, N = p.N, W = p.W;
     const int fill = p.fill[z];
     const int64_t units = static_cast<int64_t>(p.b) * Hkv;
@@ -275,6 +275,34 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
     __syncthreads();
 }
 
+// The same selection as radix_top_k for n <= kT candidates, by rank: slot i is taken when fewer than k slots
+// outrank it (a larger key, or an equal key at a lower slot).  One candidate per thread, n comparisons each against
+// keys read as broadcasts; no histogram passes.  Ends with a barrier.
+template <int kT>
+__device__ void rank_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, uint8_t flag) {
+    const int i = threadIdx.x;
+    if (k > 0 && i < n) {
+        const uint32_t x = ord[i];
+        int rank = 0;
+        const int n4 = n & ~3;
+        for (int j = 0; j < n4; j += 4) {
+            const uint4 y = *reinterpret_cast<const uint4*>(ord + j);
+            rank += (y.x > x) + (y.y > x) + (y.z > x) + (y.w > x);
+            rank += (y.x == x && j < i) + (y.y == x && j + 1 < i) + (y.z == x && j + 2 < i) + (y.w == x && j + 3 < i);
+        }
+        for (int j = n4; j < n; ++j) rank += (ord[j] > x) + (ord[j] == x && j < i);
+        if (rank < k) flags[i] |= flag;
+    }
+    __syncthreads();
+}
+
+template <int kT>
+__device__ __forceinline__ void top_k_select(const uint32_t* ord, int n, int k, uint8_t* flags, uint8_t flag,
+                                             int seg_lo, int seg_hi, SelShared& sh) {
+    if (n <= kT) rank_top_k<kT>(ord, n, k, flags, flag);
+    else radix_top_k<kT>(ord, n, k, flags, flag, seg_lo, seg_hi, sh);
+}
+
 // One CTA per unit.  AttnV (Sec. 3.2): R_B = slots >= K; R_V = N_v largest
 // value magnitudes among slots < K; the m = K - N_v - B remaining slots are
 // the m largest keys pooled_i / E_i over C = [K] \ R_V, E_i = -ln u_i, which is
@@ -333,6 +361,7 @@ __host__ __device__ inline SelLayout sel_layout(int N, int K, int n_parts, bool 
     if (staged) o += 4u * N;
     L.pos_off = o;
     if (staged) o += 4u * N;
+    o = (o + 15u) & ~15u;  // the keys are read four at a time (rank_top_k)
     L.ord_off = o;
     o += 4u * K;
     L.flag_off = o;
@@ -436,18 +465,18 @@ __device__ void gather_rows(uint8_t* base, const int32_t* src, int j_first, int 
 
 // kT threads per CTA: 256 where four CTAs share an SM; 512 or 1024 where the unit's arrays leave room for two
 // or one, so that the selection phase, which no other CTA's gather hides there, runs on as many warps.
+//
+// The body is select_unit, which the fused small-unit eviction (evict_small_kernel) runs too, on window scores it
+// has already written to shared memory (a_ready: the staging skips them; one part).
 template <int kT>
-__global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParams p) {
-    extern __shared__ __align__(16) uint8_t smem_raw[];
-    __shared__ SelShared sh;
+__device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int z, uint8_t* smem_raw, SelShared& sh,
+                                            bool a_ready, uint4* gbuf = nullptr) {
     const int N = p.N, K = p.K;
     const bool staged = p.staged != 0;
     const SelLayout Ly = sel_layout(N, K, p.n_parts, staged);
     float* a_s = reinterpret_cast<float*>(smem_raw + Ly.a_off);         // [N] window score (AttnV)
     uint32_t* ord = reinterpret_cast<uint32_t*>(smem_raw + Ly.ord_off);  // [K] orderable keys
     uint8_t* flags = smem_raw + Ly.flag_off;                            // [N]
-    const int unit = blockIdx.x;
-    const int z = blockIdx.y;  // layer slot
     const int layer = p.batch.layer[z];
     const int rnd = p.batch.rnd[z];
     const int tid = threadIdx.x;
@@ -474,8 +503,9 @@ __global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParam
     int32_t* pos_s = staged ? reinterpret_cast<int32_t*>(smem_raw + Ly.pos_off) : nullptr;
     if (staged) {
         if (p.variant == 0) {
-            for (int part = 0; part < p.n_parts; ++part)
-                cp_async_words(a_s + part * N, attn + (static_cast<int64_t>(part) * p.units + unit) * N, N);
+            if (!a_ready)
+                for (int part = 0; part < p.n_parts; ++part)
+                    cp_async_words(a_s + part * N, attn + (static_cast<int64_t>(part) * p.units + unit) * N, N);
         } else {
             cp_async_words(a_s, dkv + base, K);
         }
@@ -498,7 +528,7 @@ __global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParam
                     a_s[i] = a;
                 }
             }
-        } else {
+        } else if (!a_ready) {
             for (int i = tid; i < N; i += kT) {
                 float a = attn[base + i];
                 for (int part = 1; part < p.n_parts; ++part) {
@@ -527,7 +557,7 @@ __global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParam
             if (vscore_dbg) vscore_dbg[base + i] = vm;
         }
         __syncthreads();
-        radix_top_k<kT>(ord, K, p.n_v, flags, kFlagValue, kseg_lo, kseg_hi, sh);
+        top_k_select<kT>(ord, K, p.n_v, flags, kFlagValue, kseg_lo, kseg_hi, sh);
         // keys over the candidates C
         const int h = p.pool / 2;
         const float inv_pool = 1.0f / static_cast<float>(p.pool);
@@ -557,7 +587,7 @@ __global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParam
             if (key_dbg) key_dbg[base + i] = key;
         }
         __syncthreads();
-        radix_top_k<kT>(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
+        top_k_select<kT>(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
     } else {
         for (int i = tid; i < K; i += kT) {
             const float s = staged ? a_s[i] : dkv[base + i];
@@ -565,7 +595,7 @@ __global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParam
             if (key_dbg) key_dbg[base + i] = s;
         }
         __syncthreads();
-        radix_top_k<kT>(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
+        top_k_select<kT>(ord, K, p.m, flags, kFlagSampled, kseg_lo, kseg_hi, sh);
     }
     // positions move with the kept rows (unstaged: copy the old ones into shared memory, a_s is free now)
     if (!staged) {
@@ -620,6 +650,29 @@ __global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParam
     // ---- stable in-place gather of the kept K and V rows into slots 0..K-1 (the cache is restored to K
     // pairs, Sec. 2): warp 0 moves the K rows, warp 1 the V rows, through rings over the selection's
     // shared memory (written by generic stores until now: order them before the bulk copies).
+    if (gbuf) {
+        // every moving row of both tensors is read into shared memory first, then written to its new slot: with no
+        // store before the last read there is no in-place hazard, and all threads take part (for units whose
+        // K rows of K and V fit in gbuf: the latency-bound case, where the two-warp ring below would be slow)
+        const int64_t unit_row = (static_cast<int64_t>(layer) * p.units + unit) * N;
+        uint4* const kc = p.kc + unit_row * kVecPerRow;
+        uint4* const vc = p.vc + unit_row * kVecPerRow;
+        const int jf = sh.first_evicted;
+        const int n_vec = (K - jf) * 2 * kVecPerRow;
+        for (int e = tid; e < n_vec; e += kT) {
+            const int r = e >> 5, part = e & 31;
+            const int64_t row = src_s[jf + r];
+            gbuf[e] = part < kVecPerRow ? kc[row * kVecPerRow + part] : vc[row * kVecPerRow + part - kVecPerRow];
+        }
+        __syncthreads();
+        for (int e = tid; e < n_vec; e += kT) {
+            const int r = e >> 5, part = e & 31;
+            const int64_t row = jf + r;
+            if (part < kVecPerRow) kc[row * kVecPerRow + part] = gbuf[e];
+            else vc[row * kVecPerRow + part - kVecPerRow] = gbuf[e];
+        }
+        return;
+    }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     const int warp = tid >> 5;
     if (warp < 2) {
@@ -629,6 +682,286 @@ __global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParam
                     reinterpret_cast<uint64_t*>(smem_raw + Ly.bar_off) + warp * kGatherMaxStages, Ly.gather_stages,
                     p.err);
     }
+}
+
+template <int kT>
+__global__ void __launch_bounds__(kT, 1024 / kT) select_kernel(const SelectParams p) {
+    extern __shared__ __align__(16) uint8_t smem_raw[];
+    __shared__ SelShared sh;
+    select_unit<kT>(p, blockIdx.x, blockIdx.y, smem_raw, sh, false);
+}
+
+// ------------------------------------------------------------------ fused eviction of small units
+// For launch-bound configurations (every unit of the launch fits in one wave, one CTA per unit) the window score,
+// the selection and the gather run in one launch.  The unit's score matrix is small enough to stay in TMEM whole:
+// S = K Q^T (M = 128 tokens per tile, N = the G*W window rows) for every 128-token tile, one tcgen05 product per
+// (row, token) pair, no second transposed product and no second read of K.  With tokens in TMEM lanes, the
+// softmax statistics of a window row are reductions across lanes (warp shuffles, then shared memory across the
+// warps), and the per-token sum of Eq. (2) is a reduction along a lane's own columns.
+struct SmallLayout {
+    uint32_t sel_total, q_off, k_off, bar_off, part_off, row_off, slot_off, total;
+};
+
+__host__ __device__ inline SmallLayout small_layout(int N, int K, int GWp, int q_rows, int n_tiles, int stages) {
+    SmallLayout L;
+    uint32_t o = sel_layout(N, K, 1, true).total;
+    L.sel_total = o;
+    o = (o + 1023u) & ~1023u;
+    L.q_off = o;
+    o += static_cast<uint32_t>(q_rows) * kRowBytes;  // two 64-column panels of q_rows rows (the TMA box height)
+    o = (o + 1023u) & ~1023u;
+    L.k_off = o;
+    o += static_cast<uint32_t>(stages) * kTileTokens * kRowBytes;
+    L.bar_off = o;
+    o += 8u * (2 + 2 * 8);
+    L.part_off = o;
+    o += 4u * static_cast<uint32_t>(n_tiles) * 4u * GWp;  // partial row statistics: [tile][lane quadrant][row]
+    L.row_off = o;
+    o += 4u * 2u * GWp;  // row offsets m_r, then -m'_r
+    L.slot_off = o;
+    o += 16;  // TMEM address, then the CTA-wide "waits completed" flag
+    // the shared-memory gather of the selection overlays the score's buffers once they are dead: room for the K
+    // rows of K and V
+    const uint32_t gather = L.q_off + 2u * static_cast<uint32_t>(K) * kRowBytes;
+    L.total = o > gather ? o : gather;
+    return L;
+}
+
+// Reduce-scatter of a 32 x 32 block across a warp: lane l holds v[c] = its value of column c; afterwards lane l
+// returns the reduction (max or sum) over the 32 lanes of column l.  Five halving steps: at offset o a lane keeps
+// the half of its remaining columns whose bit o matches its own and receives the partner's partials of that half
+// (16 + 8 + 4 + 2 + 1 = 31 shuffles in all, against 5 per column for 32 separate all-reduces).
+template <bool kMax>
+__device__ __forceinline__ float warp_reduce_scatter32(float (&v)[32]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const bool hi = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < o; ++i) {
+            const float keep = hi ? v[i + o] : v[i];
+            const float send = hi ? v[i] : v[i + o];
+            const float got = __shfl_xor_sync(0xffffffffu, send, o);
+            v[i] = kMax ? fmaxf(keep, got) : keep + got;
+        }
+    }
+    return v[0];
+}
+
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__global__ void __launch_bounds__(kSmallThreads, 1)
+    evict_small_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
+                       const SmallEvictParams p) {
+    extern __shared__ __align__(1024) uint8_t smem_base[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_base) + 1023) & ~uintptr_t(1023));
+    __shared__ SelShared sh;
+    const SelectParams& sp = p.sel;
+    const int N = sp.N, GWp = p.GWp, T = p.n_tiles, S = p.stages;
+    const SmallLayout Ly = small_layout(N, sp.K, GWp, p.q_rows, T, S);
+    uint8_t* q_s = smem + Ly.q_off;
+    uint8_t* k_s = smem + Ly.k_off;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Ly.bar_off);
+    uint64_t* q_full = bars;           // [1]
+    uint64_t* all_done = bars + 1;     // [1]
+    uint64_t* k_full = bars + 2;       // [S]
+    uint64_t* k_free = bars + 2 + 8;   // [S]
+    float* part = reinterpret_cast<float*>(smem + Ly.part_off);  // [T][4][GWp]
+    float* row_m = reinterpret_cast<float*>(smem + Ly.row_off);  // [GWp] row offset (exp2 domain)
+    float* rown = row_m + GWp;                                   // [GWp] -m'_r
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Ly.slot_off);
+    volatile uint32_t* loads_ok = tmem_slot + 1;  // thread 0's waits all completed
+    const int unit = blockIdx.x, z = blockIdx.y;
+    const int layer = sp.batch.layer[z];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int seq = unit / sp.Hkv, head = unit - (unit / sp.Hkv) * sp.Hkv;
+    const int64_t k_row = static_cast<int64_t>(layer) * p.layer_rows + static_cast<int64_t>(unit) * N;
+    const int64_t q_row = static_cast<int64_t>(layer) * p.q_layer_rows +
+                          (static_cast<int64_t>(seq) * p.Hq + static_cast<int64_t>(head) * p.G) * p.W;
+
+    if (tid == 0) {
+        *loads_ok = 1u;
+        mbar_init(q_full, 1);
+        mbar_init(all_done, 1);
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&k_full[s], 1);
+            mbar_init(&k_free[s], 1);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(tmem_slot, static_cast<uint32_t>(p.tmem_cols));
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t taddr = *tmem_slot;
+    bool ok = true;
+
+    // ---- loads and products, one thread: S_t = K_t Q^T for every tile t into TMEM columns [t*GWp, (t+1)*GWp)
+    if (tid == 0) {
+        tma_prefetch_desc(&kmap);
+        tma_prefetch_desc(&qmap);
+        const uint32_t q_panel = static_cast<uint32_t>(p.q_rows) * 128u;
+        mbar_arrive_expect_tx(q_full, 2u * q_panel);
+        for (int panel = 0; panel < 2; ++panel)
+            tma_load_2d(q_s + panel * q_panel, &qmap, panel * 64, static_cast<int32_t>(q_row), q_full);
+        auto load_tile = [&](int t) {
+            const int st = t % S;
+            uint8_t* dst = k_s + st * (kTileTokens * kRowBytes);
+            const int32_t row = static_cast<int32_t>(k_row + static_cast<int64_t>(t) * kTileTokens);
+            mbar_arrive_expect_tx(&k_full[st], kTileTokens * kRowBytes);
+            tma_load_2d(dst, &kmap, 0, row, &k_full[st]);
+            tma_load_2d(dst + kTileTokens * 128, &kmap, 64, row, &k_full[st]);
+        };
+        int issued = 0, landed = 0;  // tiles whose loads were issued / were seen to land
+        for (int t = 0; t < S && t < T; ++t, ++issued) load_tile(t);
+        const uint32_t idesc = idesc_bf16_f32(128, static_cast<uint32_t>(GWp));
+        const uint64_t qdesc = sw128_kmajor_desc(smem_u32(q_s));
+        const uint64_t kdesc = sw128_kmajor_desc(smem_u32(k_s));
+        const bool q_ok = mbar_wait(q_full, 0, sp.err, kErrSmallQ);
+        ok = q_ok;
+        for (int t = 0; t < T; ++t) {
+            const int st = t % S;
+            if (ok && t < issued) {
+                ok = mbar_wait(&k_full[st], (t / S) & 1, sp.err, kErrSmallKFull);
+                if (ok) landed = t + 1;
+            }
+            tc_fence_after();
+            if (ok) {
+                const uint64_t kt = kdesc + ((static_cast<uint32_t>(st) * kTileTokens * kRowBytes) >> 4);
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    const uint32_t koff = ((kk >> 2) * (kTileTokens * 128) + (kk & 3) * 32) >> 4;
+                    const uint32_t qoff = ((kk >> 2) * q_panel + (kk & 3) * 32) >> 4;
+                    tc_mma_bf16(taddr + static_cast<uint32_t>(t * GWp), kt + koff, qdesc + qoff, idesc,
+                                kk > 0 ? 1u : 0u);
+                }
+            }
+            tc_commit(&k_free[st]);  // the stage is free once these products have read it
+            if (t + S < T && ok) {
+                ok = mbar_wait(&k_free[st], (t / S) & 1, sp.err, kErrSmallKFree);
+                if (ok) {
+                    load_tile(t + S);
+                    ++issued;
+                }
+            }
+        }
+        tc_commit(all_done);
+        // after a wait ran out: every load that was issued lands before the CTA goes on (bounded waits)
+        if (!q_ok) mbar_wait(q_full, 0, sp.err, kErrSmallQ);
+        for (int t = landed; t < issued && !ok; ++t) mbar_wait(&k_full[t % S], (t / S) & 1, sp.err, kErrSmallKFull);
+        if (!ok) *loads_ok = 0u;
+    }
+    __syncwarp();
+    if (!mbar_wait(all_done, 0, sp.err, kErrSmallDone)) atomicAnd(const_cast<uint32_t*>(loads_ok), 0u);
+    tc_fence_after();
+
+    // ---- softmax statistics of the window rows: warp w reads the lanes of quadrant w % 4 (32 tokens) of the
+    // tiles t = w / 4, w / 4 + 2, ...; every column c is a window row
+    const int quad = warp & 3;
+    const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
+    const float cs = p.scale_log2;
+    const int nch = GWp / 32;
+    for (int t = warp >> 2; t < T; t += 2) {
+        const bool valid = t * kTileTokens + quad * 32 + lane < N;
+        for (int ch = 0; ch < nch; ++ch) {
+            float v[32];
+            tmem_ld32(taddr + lane_base + static_cast<uint32_t>(t * GWp + ch * 32), v);
+            if (!valid) {
+#pragma unroll
+                for (int c = 0; c < 32; ++c) v[c] = -INFINITY;
+            }
+            part[(t * 4 + quad) * GWp + ch * 32 + lane] = warp_reduce_scatter32<true>(v);
+        }
+    }
+    __syncthreads();
+    for (int r = tid; r < GWp; r += kSmallThreads) {
+        float m = -INFINITY;
+        for (int j = 0; j < T * 4; ++j) m = fmaxf(m, part[j * GWp + r]);
+        row_m[r] = m * cs;
+    }
+    __syncthreads();
+    for (int t = warp >> 2; t < T; t += 2) {
+        const bool valid = t * kTileTokens + quad * 32 + lane < N;
+        for (int ch = 0; ch < nch; ++ch) {
+            float v[32];
+            tmem_ld32(taddr + lane_base + static_cast<uint32_t>(t * GWp + ch * 32), v);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) v[c] = valid ? ex2_approx(fmaf(v[c], cs, -row_m[ch * 32 + c])) : 0.f;
+            part[(t * 4 + quad) * GWp + ch * 32 + lane] = warp_reduce_scatter32<false>(v);
+        }
+    }
+    __syncthreads();
+    for (int r = tid; r < GWp; r += kSmallThreads) {
+        float l = 0.f;
+        for (int j = 0; j < T * 4; ++j) l += part[j * GWp + r];
+        rown[r] = r < p.GW ? -(row_m[r] + log2f(l * static_cast<float>(p.fold_rows))) : -INFINITY;
+    }
+    __syncthreads();
+
+    // ---- per-token score (Eq. (2)): sum over the window rows of the normalised weights, 1/(G*W) folded into rown
+    // (GQA max: each head's sum over its W rows, the largest kept); into the selection's score array
+    const SelLayout SL = sel_layout(N, sp.K, 1, true);
+    float* a_s = reinterpret_cast<float*>(smem + SL.a_off);
+    float* attn_out = p.attn ? p.attn + (static_cast<int64_t>(z) * sp.units + unit) * N : nullptr;
+    for (int t = warp >> 2; t < T; t += 2) {
+        const int token = t * kTileTokens + quad * 32 + lane;
+        float acc = 0.f, head_sum = 0.f;
+        int head_end = p.head_rows;
+        for (int ch = 0; ch < nch; ++ch) {
+            float v[32];
+            tmem_ld32(taddr + lane_base + static_cast<uint32_t>(t * GWp + ch * 32), v);
+            if (p.head_rows == 0) {
+                float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+                for (int c = 0; c < 32; c += 2) {
+                    a0 += ex2_approx(fmaf(v[c], cs, rown[ch * 32 + c]));
+                    a1 += ex2_approx(fmaf(v[c + 1], cs, rown[ch * 32 + c + 1]));
+                }
+                acc += a0 + a1;
+            } else {
+                for (int c = 0; c < 32; ++c) {
+                    const int r = ch * 32 + c;
+                    if (r >= p.GW) break;
+                    if (r == head_end) {
+                        acc = fmaxf(acc, head_sum);
+                        head_sum = 0.f;
+                        head_end += p.head_rows;
+                    }
+                    head_sum += ex2_approx(fmaf(v[c], cs, rown[r]));
+                }
+            }
+        }
+        if (p.head_rows != 0) acc = fmaxf(acc, head_sum);
+        if (token < N) {
+            a_s[token] = acc;
+            if (attn_out) attn_out[token] = acc;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(taddr, static_cast<uint32_t>(p.tmem_cols));
+    if (tid == 0) {  // the barriers' memory is reused by the gather below
+        mbar_inval(q_full);
+        mbar_inval(all_done);
+        for (int st = 0; st < S; ++st) {
+            mbar_inval(&k_full[st]);
+            mbar_inval(&k_free[st]);
+        }
+    }
+    if (*loads_ok == 0u) {
+        // a wait ran out (the same flag for every thread): the scores are not all there; leave the cache as it is
+        // (the error word is set)
+        return;
+    }
+    // ---- selection and gather on the scores just written (the selection's buffers sit below the score's)
+    select_unit<kSmallThreads>(sp, unit, z, smem, sh, true, reinterpret_cast<uint4*>(smem + Ly.q_off));
 }
 
 
@@ -725,8 +1058,13 @@ __global__ void __launch_bounds__(kSelThreads) quantize_kernel(const QuantParams
 }  // namespace
 
 cudaError_t launch_append(const AppendParams& p, int n_layers, cudaStream_t s) {
-    const int chunks = (p.n + kAppendSteps - 1) / kAppendSteps;
-    append_kernel<<<dim3(static_cast<unsigned>(chunks * p.b), static_cast<unsigned>(n_layers)), 256, 0, s>>>(p);
+    // four steps per block, or one where four would leave fewer blocks than the GPU's 152 SMs (small,
+    // latency-bound appends)
+    AppendParams q = p;
+    q.steps_per_block = static_cast<int64_t>((p.n + kAppendSteps - 1) / kAppendSteps) * p.b * n_layers < 152
+                            ? 1 : kAppendSteps;
+    const int chunks = (p.n + q.steps_per_block - 1) / q.steps_per_block;
+    append_kernel<<<dim3(static_cast<unsigned>(chunks * p.b), static_cast<unsigned>(n_layers)), 256, 0, s>>>(q);
     return cudaGetLastError();
 }
 
@@ -766,6 +1104,22 @@ cudaError_t quantize_set_attributes(size_t smem_bytes) {
 
 cudaError_t launch_quantize(const QuantParams& p, int units, size_t smem_bytes, cudaStream_t s) {
     quantize_kernel<<<static_cast<unsigned>(units), kSelThreads, smem_bytes, s>>>(p);
+    return cudaGetLastError();
+}
+
+size_t evict_small_smem_bytes(int N, int K, int GWp, int q_rows, int n_tiles, int stages) {
+    return small_layout(N, K, GWp, q_rows, n_tiles, stages).total + 1024;
+}
+
+cudaError_t evict_small_set_attributes(size_t smem_bytes) {
+    return cudaFuncSetAttribute(evict_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(smem_bytes));
+}
+
+cudaError_t launch_evict_small(const CUtensorMap& kmap, const CUtensorMap& qmap, const SmallEvictParams& p, int units,
+                               size_t smem_bytes, cudaStream_t s) {
+    evict_small_kernel<<<dim3(static_cast<unsigned>(units), static_cast<unsigned>(p.sel.batch.n)), kSmallThreads,
+                         smem_bytes, s>>>(kmap, qmap, p);
     return cudaGetLastError();
 }
 

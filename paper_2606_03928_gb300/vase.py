@@ -43,7 +43,7 @@ EXPORTED = [
     "vase_decode_attention", "vase_mixed_buffer_sizes", "vase_quantize_values", "vase_decode_attention_mixed",
     "vase_host_staging_bytes", "vase_stage_host_inputs", "vase_append_all_staged", "vase_read_positions_all",
 ]
-KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "compact"]
+KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "evict_small"]
 
 
 class vase_config(ctypes.Structure):

@@ -659,10 +659,23 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
         uint4* const vc = p.vc + unit_row * kVecPerRow;
         const int jf = sh.first_evicted;
         const int n_vec = (K - jf) * 2 * kVecPerRow;
-        for (int e = tid; e < n_vec; e += kT) {
-            const int r = e >> 5, part = e & 31;
-            const int64_t row = src_s[jf + r];
-            gbuf[e] = part < kVecPerRow ? kc[row * kVecPerRow + part] : vc[row * kVecPerRow + part - kVecPerRow];
+        constexpr int kBatch = 8;  // loads in flight per thread before their shared-memory stores
+        for (int e0 = 0; e0 < n_vec; e0 += kBatch * kT) {
+            uint4 val[kBatch];
+#pragma unroll
+            for (int b = 0; b < kBatch; ++b) {
+                const int e = e0 + b * kT + tid;
+                if (e < n_vec) {
+                    const int r = e >> 5, part = e & 31;
+                    const int64_t row = src_s[jf + r];
+                    val[b] = part < kVecPerRow ? kc[row * kVecPerRow + part] : vc[row * kVecPerRow + part - kVecPerRow];
+                }
+            }
+#pragma unroll
+            for (int b = 0; b < kBatch; ++b) {
+                const int e = e0 + b * kT + tid;
+                if (e < n_vec) gbuf[e] = val[b];
+            }
         }
         __syncthreads();
         for (int e = tid; e < n_vec; e += kT) {

@@ -470,7 +470,7 @@ __device__ void gather_rows(uint8_t* base, const int32_t* src, int j_first, int 
 // has already written to shared memory (a_ready: the staging skips them; one part).
 template <int kT>
 __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int z, uint8_t* smem_raw, SelShared& sh,
-                                            bool a_ready, uint4* gbuf = nullptr) {
+                                            bool a_ready, uint4* gbuf = nullptr, int gbuf_rows = 0) {
     const int N = p.N, K = p.K;
     const bool staged = p.staged != 0;
     const SelLayout Ly = sel_layout(N, K, p.n_parts, staged);
@@ -651,38 +651,42 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
     // pairs, Sec. 2): warp 0 moves the K rows, warp 1 the V rows, through rings over the selection's
     // shared memory (written by generic stores until now: order them before the bulk copies).
     if (gbuf) {
-        // every moving row of both tensors is read into shared memory first, then written to its new slot: with no
-        // store before the last read there is no in-place hazard, and all threads take part (for units whose
-        // K rows of K and V fit in gbuf: the latency-bound case, where the two-warp ring below would be slow)
+        // Gather by every thread (the fused small-unit kernel): the moving rows go in blocks of gbuf_rows destination
+        // rows; all the block's K and V source rows are read into shared memory, then (after a barrier) written to
+        // their new slots.  In place this is safe: a block's sources lie at or above its first destination row, so
+        // no earlier block's stores touch them, and within a block every read precedes every write.
         const int64_t unit_row = (static_cast<int64_t>(layer) * p.units + unit) * N;
         uint4* const kc = p.kc + unit_row * kVecPerRow;
         uint4* const vc = p.vc + unit_row * kVecPerRow;
         const int jf = sh.first_evicted;
-        const int n_vec = (K - jf) * 2 * kVecPerRow;
         constexpr int kBatch = 8;  // loads in flight per thread before their shared-memory stores
-        for (int e0 = 0; e0 < n_vec; e0 += kBatch * kT) {
-            uint4 val[kBatch];
+        for (int j0 = jf; j0 < K; j0 += gbuf_rows) {
+            const int n_vec = min(gbuf_rows, K - j0) * 2 * kVecPerRow;
+            for (int e0 = 0; e0 < n_vec; e0 += kBatch * kT) {
+                uint4 val[kBatch];
 #pragma unroll
-            for (int b = 0; b < kBatch; ++b) {
-                const int e = e0 + b * kT + tid;
-                if (e < n_vec) {
-                    const int r = e >> 5, part = e & 31;
-                    const int64_t row = src_s[jf + r];
-                    val[b] = part < kVecPerRow ? kc[row * kVecPerRow + part] : vc[row * kVecPerRow + part - kVecPerRow];
+                for (int b = 0; b < kBatch; ++b) {
+                    const int e = e0 + b * kT + tid;
+                    if (e < n_vec) {
+                        const int r = e >> 5, part = e & 31;
+                        const int64_t row = src_s[j0 + r];
+                        val[b] = part < kVecPerRow ? kc[row * kVecPerRow + part] : vc[row * kVecPerRow + part - kVecPerRow];
+                    }
+                }
+#pragma unroll
+                for (int b = 0; b < kBatch; ++b) {
+                    const int e = e0 + b * kT + tid;
+                    if (e < n_vec) gbuf[e] = val[b];
                 }
             }
-#pragma unroll
-            for (int b = 0; b < kBatch; ++b) {
-                const int e = e0 + b * kT + tid;
-                if (e < n_vec) gbuf[e] = val[b];
+            __syncthreads();
+            for (int e = tid; e < n_vec; e += kT) {
+                const int r = e >> 5, part = e & 31;
+                const int64_t row = j0 + r;
+                if (part < kVecPerRow) kc[row * kVecPerRow + part] = gbuf[e];
+                else vc[row * kVecPerRow + part - kVecPerRow] = gbuf[e];
             }
-        }
-        __syncthreads();
-        for (int e = tid; e < n_vec; e += kT) {
-            const int r = e >> 5, part = e & 31;
-            const int64_t row = jf + r;
-            if (part < kVecPerRow) kc[row * kVecPerRow + part] = gbuf[e];
-            else vc[row * kVecPerRow + part - kVecPerRow] = gbuf[e];
+            __syncthreads();
         }
         return;
     }
@@ -974,7 +978,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1)
         return;
     }
     // ---- selection and gather on the scores just written (the selection's buffers sit below the score's)
-    select_unit<kSmallThreads>(sp, unit, z, smem, sh, true, reinterpret_cast<uint4*>(smem + Ly.q_off));
+    select_unit<kSmallThreads>(sp, unit, z, smem, sh, true, reinterpret_cast<uint4*>(smem + Ly.q_off), sp.K);
 }
 
 

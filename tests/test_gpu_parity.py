@@ -95,6 +95,26 @@ def test_single_layer_k256_all_units_match_oracle():
     assert flips <= 2
 
 
+# Launch-bound single-layer evictions of small units run the fused kernel (score held in TMEM, selection and
+# gather in the same launch).  Its edges: 128 window rows (a whole 128-column TMEM block per tile), a ragged last
+# tile, four tiles of 128 rows (all 512 TMEM columns, and K rows of K and V filling most of shared memory), debug
+# outputs off, GQA max-aggregation and noise off.
+@pytest.mark.parametrize("K,B,Wn,Hq,Hkv,kw", [
+    (256, 64, 32, 32, 8, {}),                      # G*W = 128
+    (200, 40, 16, 16, 8, {}),                      # N = 240: a ragged last tile
+    (320, 192, 32, 32, 8, {}),                     # N = 512, G*W = 128: 512 TMEM columns
+    (256, 64, 32, 16, 8, {"debug": False}),
+    (256, 64, 16, 32, 8, {"gqa": "max"}),
+    (256, 64, 32, 16, 8, {"stochastic": False}),
+])
+def test_fused_small_unit_eviction_matches_oracle(K, B, Wn, Hq, Hkv, kw):
+    kw = dict(kw)
+    debug = kw.pop("debug", True)
+    wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=Wn, num_q_heads=Hq, num_kv_heads=Hkv, batch=2, num_layers=2)
+    _, _, _, flips = _run_layer(wl, debug=debug, cache_kw=kw, oracle_kw=kw)
+    assert flips <= 4
+
+
 def test_layer_offset_and_gapped_positions():
     _run_layer(SMALL, layer=1, num_layers=2, round_index=5)
 

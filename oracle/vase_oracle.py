@@ -31,7 +31,12 @@ time, where a *unit* is one (layer, sequence, KV head):
   s = Range(v) / (2^b - 1), Q(v) = round((v - z) / s), v' = Q s + z -- the
   equation of Sec. 4.4 -- and the mixed-precision value cache that Sec. 6
   proposes: the reserved large-Range values (R_V) and the recency buffer keep
-  their bf16 rows, every other kept value is read back from its b-bit codes.
+  their bf16 rows, every other kept value is read back from its b-bit codes;
+* the compressed value store built on that proposal: the bf16 rows live only
+  in a reserved cache of N_v + 2B rows (a ring in slot order), every other
+  cached value only as its codes; an append that finds the reserved cache full
+  quantizes its earliest value into the low-precision cache (the rule Sec. 6
+  states), and an eviction quantizes the kept values that leave R_V u R_B.
 
 Readings where the paper is silent (each is listed with its reason in the
 design notes of the repository):
@@ -65,6 +70,14 @@ design notes of the repository):
   last B kept slots, and R_V, which is again the N_v largest value
   magnitudes among the first K - B kept slots (R_V is kept whole and the
   compaction keeps the order).
+* Compressed value store: keys stay bf16 (Sec. 4.4 and Sec. 6 speak of value
+  states).  The reserved cache holds R_V u R_B after an eviction (at most
+  N_v + B rows) and the B values appended before the next one, so its
+  capacity is H = N_v + 2B; only the appends before the first eviction can
+  find it full.  A value that leaves R_V u R_B at an eviction while kept is
+  quantized then (it no longer holds a reserved slot).  A quantized value
+  never returns to bf16: a later R_V is drawn from the earlier R_V and the
+  newly appended values only, since R_V is kept whole.
 """
 
 from __future__ import annotations
@@ -373,3 +386,64 @@ def evict_unit_bits(q_bits, k_bits, v_bits, positions, **kw):
     res["k_bits_new"] = np.asarray(k_bits)[src]
     res["v_bits_new"] = np.asarray(v_bits)[src]
     return res
+
+
+# ----------------------------------------------------------------------------
+# Compressed value store (Sec. 6: high-precision reserved cache, low-precision rest)
+# ----------------------------------------------------------------------------
+
+def store_capacity(budget_k, buffer_b, n_v):
+    """Rows of the reserved (bf16) cache: R_V u R_B after an eviction plus the B values appended before the
+    next one, H = N_v + 2B."""
+    return int(n_v) + 2 * int(buffer_b)
+
+
+def store_new(capacity):
+    """An empty store: the reserved cache is a ring of `capacity` rows whose entries are the bf16 slots in slot
+    order, entry i at ring position (head + i) mod capacity."""
+    return {"H": int(capacity), "head": 0, "slots": []}
+
+
+def store_append(store, fill, n):
+    """Appends slots fill .. fill + n - 1 (their values enter the reserved cache in bf16).  Whenever the
+    reserved cache would hold more than H values, its earliest value is quantized into the low-precision
+    cache (Sec. 6).  Returns the slots quantized by this call, in the order they left."""
+    spilled = []
+    for t in range(int(n)):
+        store["slots"].append(int(fill) + t)
+        if len(store["slots"]) > store["H"]:
+            spilled.append(store["slots"].pop(0))
+            store["head"] = (store["head"] + 1) % store["H"]
+    return spilled
+
+
+def store_evict(store, src, reserved_new):
+    """The eviction's effect on the store: new slot j holds old slot src[j]; its value stays bf16 when it was
+    bf16 and j is in R_V u R_B (reserved_new[j]), and is quantized when it was bf16 and is not.  The ring keeps
+    its head; the retained entries close up in slot order.  Returns the new slots quantized by the eviction."""
+    old = set(store["slots"])
+    kept, spilled = [], []
+    for j, s in enumerate(np.asarray(src).tolist()):
+        if s in old:
+            (kept if reserved_new[j] else spilled).append(j)
+    store["slots"] = kept
+    return spilled
+
+
+def store_ring_positions(store):
+    """Ring position of each bf16 slot: {slot: (head + i) mod H}."""
+    H, h = store["H"], store["head"]
+    return {s: (h + i) % H for i, s in enumerate(store["slots"])}
+
+
+def store_reserved_mask(store, n_slots):
+    """Mask [n_slots]: True where the slot's value is held in bf16."""
+    mask = np.zeros(int(n_slots), dtype=bool)
+    mask[np.asarray(store["slots"], dtype=np.int64)] = True
+    return mask
+
+
+def store_bytes(n_slots, capacity, d, bits):
+    """Bytes of one unit's compressed value store (codes and (s, z) of every slot, the reserved cache)
+    against the n_slots bf16 rows it replaces."""
+    return int(n_slots) * (d * int(bits) // 8 + 8) + int(capacity) * 2 * d, int(n_slots) * 2 * d

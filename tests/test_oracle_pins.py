@@ -492,6 +492,125 @@ def test_leverage_pins_reject_planted_slips(slip, monkeypatch):
     assert not all(passed), f"planted slip '{slip}' passed every pin"
 
 
+# --------------------------------------------------------------------------- compressed value store (Sec. 6)
+
+def _pin_store_fifo(new, append):
+    """Sec. 6: once the high-precision cache is full, its earliest value is quantized.  A stream appended in
+    random pieces into a cache of 5 rows: the bf16 values are always the latest min(fill, 5), the quantized ones
+    are exactly the earlier slots, each quantized once, in stream order; with no eviction yet, slot s sits at
+    ring position s mod 5 (the head advances by one per quantized value)."""
+    rng = np.random.default_rng(0)
+    st = new(5)
+    fill, seen = 0, []
+    for _ in range(40):
+        n = int(rng.integers(0, 8))
+        seen += append(st, fill, n)
+        fill += n
+        if st["slots"] != list(range(max(0, fill - 5), fill)) or seen != list(range(max(0, fill - 5))):
+            return False
+        if any(pos != s % 5 for s, pos in O.store_ring_positions(st).items()):
+            return False
+    return True
+
+
+def _pin_store_rounds(new, append, evict):
+    """Chained AttnV rounds on one unit with the store beside them.  After every eviction the bf16 values are
+    the kept members of R_V u R_B that were bf16 before (R_B always: it was just appended), at most N_v + B;
+    the B appends before the next eviction never find the cache full (N_v + 2B = H); a quantized token never
+    comes back to bf16; the ring entries stay in slot order behind an unchanged head."""
+    K, B, nv, d, Wn = 24, 4, 6, 8, 2
+    H = O.store_capacity(K, B, nv)
+    N = K + B
+    rng = np.random.default_rng(5)
+    total = N + 16 * B
+    keys = rng.standard_normal((total, d))
+    values = rng.standard_normal((total, d))
+    values[rng.random(total) < 0.15] *= 20
+    st = new(H)
+    slot_pos = list(range(N))
+    coded = set(append(st, 0, N))          # stream positions whose value has been quantized
+    if len(coded) != N - H:
+        return False
+    nxt = N
+    for rnd in range(16):
+        q = rng.standard_normal((Wn, d))
+        res = O.evict_unit(q, keys[slot_pos], values[slot_pos], np.array(slot_pos), budget_k=K, buffer_b=B,
+                           n_v=nv, pool_kernel=3, seed=1, rnd=rnd)
+        src = res["src"]
+        resnew = (src >= K) | np.isin(src, res["reserved_v"])
+        was = set(st["slots"])
+        head = st["head"]
+        spilled = evict(st, src, resnew)
+        slot_pos = [slot_pos[s] for s in src]
+        if st["slots"] != [j for j in range(K) if int(src[j]) in was and resnew[j]]:
+            return False
+        if len(st["slots"]) > nv + B or not set(range(K - B, K)) <= set(st["slots"]) or st["head"] != head:
+            return False
+        coded |= {slot_pos[j] for j in spilled}
+        if any(slot_pos[j] in coded for j in st["slots"]):
+            return False
+        if append(st, K, B):
+            return False
+        slot_pos += list(range(nxt, nxt + B))
+        nxt += B
+    return True
+
+
+def test_store_spills_the_earliest_value_when_full():
+    assert _pin_store_fifo(O.store_new, O.store_append)
+
+
+def test_store_keeps_r_v_and_r_b_across_rounds():
+    assert _pin_store_rounds(O.store_new, O.store_append, O.store_evict)
+
+
+def test_store_bytes_closed_form():
+    """Qwen3-1.7B geometry, K 2048, B 128, N_v 512, 4 bits: 2176 slots x (64 code bytes + 8 for s, z) plus
+    a reserved cache of 512 + 256 rows of 256 bytes, against 2176 bf16 rows."""
+    assert O.store_capacity(2048, 128, 512) == 768
+    assert O.store_bytes(2176, 768, 128, 4) == (2176 * 72 + 768 * 256, 2176 * 256)
+    assert O.store_bytes(2176, 768, 128, 2) == (2176 * 40 + 768 * 256, 2176 * 256)
+
+
+def _store_slips():
+    """Plausible mistakes in the store: the latest value leaves a full cache instead of the earliest; the
+    eviction quantizes nothing (kept non-reserved values stay bf16); it quantizes R_B too; it re-admits
+    quantized values of R_V u R_B to bf16."""
+    def lifo_append(st, fill, n):
+        out = []
+        for t in range(int(n)):
+            st["slots"].append(int(fill) + t)
+            if len(st["slots"]) > st["H"]:
+                out.append(st["slots"].pop())
+        return out
+
+    def no_spill_evict(st, src, resnew):
+        old = set(st["slots"])
+        st["slots"] = [j for j, s in enumerate(np.asarray(src).tolist()) if s in old]
+        return []
+
+    def spill_rb_evict(st, src, resnew):
+        K = len(src)
+        out = O.store_evict(st, src, resnew)
+        rb = [j for j in st["slots"] if j >= K - 4]
+        st["slots"] = [j for j in st["slots"] if j < K - 4]
+        return out + rb
+
+    def readmit_evict(st, src, resnew):
+        out = O.store_evict(st, src, resnew)
+        st["slots"] = [j for j in range(len(src)) if resnew[j]]
+        return out
+
+    return {"lifo": (lifo_append, O.store_evict), "no_spill": (O.store_append, no_spill_evict),
+            "spill_rb": (O.store_append, spill_rb_evict), "readmit": (O.store_append, readmit_evict)}
+
+
+@pytest.mark.parametrize("slip", sorted(_store_slips()))
+def test_store_pins_reject_planted_slips(slip):
+    append, evict = _store_slips()[slip]
+    assert not (_pin_store_fifo(O.store_new, append) and _pin_store_rounds(O.store_new, append, evict)), slip
+
+
 # --------------------------------------------------------------------------- decode attention (Eq. (1) output)
 
 def test_decode_attention_closed_forms():

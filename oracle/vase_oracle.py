@@ -35,8 +35,9 @@ time, where a *unit* is one (layer, sequence, KV head):
 * the compressed value store built on that proposal: the bf16 rows live only
   in a reserved cache of N_v + 2B rows (a ring in slot order), every other
   cached value only as its codes; an append that finds the reserved cache full
-  quantizes its earliest value into the low-precision cache (the rule Sec. 6
-  states), and an eviction quantizes the kept values that leave R_V u R_B.
+  quantizes its earliest value that is not large-Range into the low-precision
+  cache (the rule Sec. 6 states), and an eviction quantizes the kept values
+  that leave R_V u R_B.
 
 Readings where the paper is silent (each is listed with its reason in the
 design notes of the repository):
@@ -74,10 +75,18 @@ design notes of the repository):
   states).  The reserved cache holds R_V u R_B after an eviction (at most
   N_v + B rows) and the B values appended before the next one, so its
   capacity is H = N_v + 2B; only the appends before the first eviction can
-  find it full.  A value that leaves R_V u R_B at an eviction while kept is
-  quantized then (it no longer holds a reserved slot).  A quantized value
-  never returns to bf16: a later R_V is drawn from the earlier R_V and the
-  newly appended values only, since R_V is kept whole.
+  find it full.  The values the rule of Sec. 6 spills when it is full are
+  "the earliest" among those that are not large-Range: the large-Range values
+  are the N_v largest value magnitudes among the slots the next eviction
+  draws R_V from (slots below K, ties to the lower slot), the set R_V would be
+  now.  (Taken over all values, a long first fill would quantize the
+  large-Range values of its earliest tokens before the first eviction could
+  reserve them, which is what the proposal is there to prevent.)  So the
+  first eviction finds R_V in bf16, and so does every later one.  A value
+  that leaves R_V u R_B at an eviction while kept is quantized then (it no
+  longer holds a reserved slot).  A quantized value never returns to bf16: a
+  later R_V is drawn from the earlier R_V and the newly appended values only,
+  since R_V is kept whole.
 """
 
 from __future__ import annotations
@@ -404,16 +413,28 @@ def store_new(capacity):
     return {"H": int(capacity), "head": 0, "slots": []}
 
 
-def store_append(store, fill, n):
-    """Appends slots fill .. fill + n - 1 (their values enter the reserved cache in bf16).  Whenever the
-    reserved cache would hold more than H values, its earliest value is quantized into the low-precision
-    cache (Sec. 6).  Returns the slots quantized by this call, in the order they left."""
-    spilled = []
-    for t in range(int(n)):
-        store["slots"].append(int(fill) + t)
-        if len(store["slots"]) > store["H"]:
-            spilled.append(store["slots"].pop(0))
-            store["head"] = (store["head"] + 1) % store["H"]
+def store_large_range(value_scores, n_slots, budget_k, n_v):
+    """The large-Range values of a cache of n_slots: the N_v largest value magnitudes among the slots below K
+    (the candidates of R_V, Eq. (5)); ties to the lower slot."""
+    c = min(int(n_slots), int(budget_k))
+    return set(top_k_slots(np.asarray(value_scores, dtype=np.float64)[:c], min(int(n_v), c)).tolist())
+
+
+def store_append(store, fill, n, value_scores=None, budget_k=0, n_v=0):
+    """Appends slots fill .. fill + n - 1 (their values enter the reserved cache in bf16).  When the reserved
+    cache would hold more than H values, its earliest values that are not large-Range (store_large_range over
+    the filled slots, value_scores indexed by slot) are quantized into the low-precision cache (Sec. 6), as many
+    as it is over.  The entries keep their slot order behind an unchanged head.  Returns the slots quantized by
+    this call, in slot order."""
+    H = store["H"]
+    store["slots"] += [int(fill) + t for t in range(int(n))]
+    over = len(store["slots"]) - H
+    if over <= 0:
+        return []
+    keep = store_large_range(value_scores, fill + n, budget_k, n_v) if n_v else set()
+    spilled = [s for s in store["slots"] if s not in keep][:over]
+    gone = set(spilled)
+    store["slots"] = [s for s in store["slots"] if s not in gone]
     return spilled
 
 

@@ -495,29 +495,57 @@ def test_leverage_pins_reject_planted_slips(slip, monkeypatch):
 # --------------------------------------------------------------------------- compressed value store (Sec. 6)
 
 def _pin_store_fifo(new, append):
-    """Sec. 6: once the high-precision cache is full, its earliest value is quantized.  A stream appended in
-    random pieces into a cache of 5 rows: the bf16 values are always the latest min(fill, 5), the quantized ones
-    are exactly the earlier slots, each quantized once, in stream order; with no eviction yet, slot s sits at
-    ring position s mod 5 (the head advances by one per quantized value)."""
+    """Sec. 6: once the high-precision cache is full, its earliest value is quantized.  With no large-Range
+    reservation (N_v = 0), a stream appended in random pieces into a cache of 5 rows: the bf16 values are always
+    the latest min(fill, 5), the quantized ones exactly the earlier slots, each quantized once, in stream order;
+    the entries sit at ring rows head, head + 1, ... in slot order."""
     rng = np.random.default_rng(0)
     st = new(5)
     fill, seen = 0, []
     for _ in range(40):
         n = int(rng.integers(0, 8))
-        seen += append(st, fill, n)
+        seen += append(st, fill, n, np.zeros(fill + n), 10 ** 6, 0)
         fill += n
         if st["slots"] != list(range(max(0, fill - 5), fill)) or seen != list(range(max(0, fill - 5))):
             return False
-        if any(pos != s % 5 for s, pos in O.store_ring_positions(st).items()):
+        pos = O.store_ring_positions(st)
+        if [pos[s] for s in st["slots"]] != [(st["head"] + i) % 5 for i in range(len(st["slots"]))]:
+            return False
+    return True
+
+
+def _pin_store_first_fill_keeps_large_range(new, append):
+    """The large-Range values survive a long first fill: whatever the pieces, after K + B appends into a cache of
+    N_v + 2B rows the N_v largest magnitudes among the first K slots (R_V of the first eviction) and the last B
+    slots (R_B) are all in bf16, and exactly K + B - H values were quantized, each an earliest value not in the
+    large-Range set at its time (checked against the final R_V: none of it left)."""
+    K, B, nv = 40, 4, 6
+    H = O.store_capacity(K, B, nv)
+    for seed in range(20):
+        rng = np.random.default_rng(100 + seed)
+        vmag = rng.random(K + B)
+        vmag[rng.integers(0, K, 5)] += 10          # a few large-Range values, some early
+        vmag[rng.integers(0, K, 3)] = vmag[0]      # ties with slot 0
+        st = new(H)
+        fill, spilled = 0, []
+        while fill < K + B:
+            n = int(min(K + B - fill, rng.integers(1, 12)))
+            spilled += append(st, fill, n, vmag, K, nv)
+            fill += n
+        r_v = set(O.top_k_slots(vmag[:K], nv).tolist())
+        if not (r_v | set(range(K, K + B))) <= set(st["slots"]):
+            return False
+        if len(spilled) != K + B - H or r_v & set(spilled):
             return False
     return True
 
 
 def _pin_store_rounds(new, append, evict):
     """Chained AttnV rounds on one unit with the store beside them.  After every eviction the bf16 values are
-    the kept members of R_V u R_B that were bf16 before (R_B always: it was just appended), at most N_v + B;
-    the B appends before the next eviction never find the cache full (N_v + 2B = H); a quantized token never
-    comes back to bf16; the ring entries stay in slot order behind an unchanged head."""
+    the kept members of R_V u R_B that were bf16 before, and that is all of R_V u R_B (the first fill kept R_V in
+    bf16, and R_B was just appended); the B appends before the next eviction never find the cache full
+    (N_v + 2B = H); a quantized token never comes back to bf16; the ring entries stay in slot order behind an
+    unchanged head."""
     K, B, nv, d, Wn = 24, 4, 6, 8, 2
     H = O.store_capacity(K, B, nv)
     N = K + B
@@ -526,9 +554,10 @@ def _pin_store_rounds(new, append, evict):
     keys = rng.standard_normal((total, d))
     values = rng.standard_normal((total, d))
     values[rng.random(total) < 0.15] *= 20
+    vmag_all = O.value_magnitude(values)
     st = new(H)
     slot_pos = list(range(N))
-    coded = set(append(st, 0, N))          # stream positions whose value has been quantized
+    coded = set(append(st, 0, N, vmag_all[:N], K, nv))   # stream positions whose value has been quantized
     if len(coded) != N - H:
         return False
     nxt = N
@@ -544,20 +573,24 @@ def _pin_store_rounds(new, append, evict):
         slot_pos = [slot_pos[s] for s in src]
         if st["slots"] != [j for j in range(K) if int(src[j]) in was and resnew[j]]:
             return False
-        if len(st["slots"]) > nv + B or not set(range(K - B, K)) <= set(st["slots"]) or st["head"] != head:
+        if st["slots"] != [j for j in range(K) if resnew[j]] or st["head"] != head:
             return False
         coded |= {slot_pos[j] for j in spilled}
         if any(slot_pos[j] in coded for j in st["slots"]):
             return False
-        if append(st, K, B):
-            return False
         slot_pos += list(range(nxt, nxt + B))
+        if append(st, K, B, vmag_all[slot_pos], K, nv):
+            return False
         nxt += B
     return True
 
 
 def test_store_spills_the_earliest_value_when_full():
     assert _pin_store_fifo(O.store_new, O.store_append)
+
+
+def test_store_first_fill_keeps_the_large_range_values():
+    assert _pin_store_first_fill_keeps_large_range(O.store_new, O.store_append)
 
 
 def test_store_keeps_r_v_and_r_b_across_rounds():
@@ -574,15 +607,18 @@ def test_store_bytes_closed_form():
 
 def _store_slips():
     """Plausible mistakes in the store: the latest value leaves a full cache instead of the earliest; the
-    eviction quantizes nothing (kept non-reserved values stay bf16); it quantizes R_B too; it re-admits
-    quantized values of R_V u R_B to bf16."""
-    def lifo_append(st, fill, n):
+    earliest leaves whether it is large-Range or not (the sentence taken over all values); the eviction quantizes
+    nothing (kept non-reserved values stay bf16); it quantizes R_B too; it puts R_B's rows ahead of R_V's in
+    the ring (out of slot order)."""
+    def lifo_append(st, fill, n, vmag, K, nv):
+        st["slots"] += [int(fill) + t for t in range(int(n))]
         out = []
-        for t in range(int(n)):
-            st["slots"].append(int(fill) + t)
-            if len(st["slots"]) > st["H"]:
-                out.append(st["slots"].pop())
+        while len(st["slots"]) > st["H"]:
+            out.append(st["slots"].pop())
         return out
+
+    def plain_fifo_append(st, fill, n, vmag, K, nv):
+        return O.store_append(st, fill, n, vmag, K, 0)
 
     def no_spill_evict(st, src, resnew):
         old = set(st["slots"])
@@ -596,19 +632,22 @@ def _store_slips():
         st["slots"] = [j for j in st["slots"] if j < K - 4]
         return out + rb
 
-    def readmit_evict(st, src, resnew):
+    def rb_first_evict(st, src, resnew):
+        K = len(src)
         out = O.store_evict(st, src, resnew)
-        st["slots"] = [j for j in range(len(src)) if resnew[j]]
+        st["slots"] = [j for j in st["slots"] if j >= K - 4] + [j for j in st["slots"] if j < K - 4]
         return out
 
-    return {"lifo": (lifo_append, O.store_evict), "no_spill": (O.store_append, no_spill_evict),
-            "spill_rb": (O.store_append, spill_rb_evict), "readmit": (O.store_append, readmit_evict)}
+    return {"lifo": (lifo_append, O.store_evict), "plain_fifo": (plain_fifo_append, O.store_evict),
+            "no_spill": (O.store_append, no_spill_evict), "spill_rb": (O.store_append, spill_rb_evict),
+            "rb_first": (O.store_append, rb_first_evict)}
 
 
 @pytest.mark.parametrize("slip", sorted(_store_slips()))
 def test_store_pins_reject_planted_slips(slip):
     append, evict = _store_slips()[slip]
-    assert not (_pin_store_fifo(O.store_new, append) and _pin_store_rounds(O.store_new, append, evict)), slip
+    assert not (_pin_store_fifo(O.store_new, append) and _pin_store_first_fill_keeps_large_range(O.store_new, append)
+                and _pin_store_rounds(O.store_new, append, evict)), slip
 
 
 # --------------------------------------------------------------------------- decode attention (Eq. (1) output)

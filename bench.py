@@ -63,6 +63,8 @@ def parse_args():
     ap.add_argument("--dkv-shared-g", action="store_true", help="DKV: one projection per round for every unit")
     ap.add_argument("--mixed-bits", type=int, default=0, choices=[0, 2, 4, 8],
                     help="with --decode: read the unreserved values from b-bit codes (Sec. 4.4 / Sec. 6)")
+    ap.add_argument("--value-bits", type=int, default=0, choices=[0, 2, 4, 8],
+                    help="AttnV: keep the values in the compressed value store (b-bit codes, bf16 reserved ring)")
     ap.add_argument("--layers", type=int, default=None, help="run only this many layers of the workload")
     ap.add_argument("--e2e-steps", type=int, default=None, help="steps of the host-buffer end-to-end pass")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle CPU baseline")
@@ -197,11 +199,21 @@ def whole_job_rate(units_per_rank, world, ms):
     return world * units_per_rank / (ms / 1e3)
 
 
-def kernel_bytes(kind, wl, variant, moved_rows_per_unit):
-    """Algorithmic bytes of one kernel for one layer (a launch covers up to 64 layers)."""
+def kernel_bytes(kind, wl, variant, moved_rows_per_unit, bits=0):
+    """Algorithmic bytes of one kernel for one layer (a launch covers up to 64 layers); bits > 0: with the
+    compressed value store, whose values move in the store kernels instead of the gather."""
     U = wl.batch * wl.num_kv_heads
     N, K, B, d = wl.slots, wl.budget_k, wl.buffer_b, wl.head_dim
     row = 2 * d
+    if bits and kind == "select_compact":  # only the key rows move here
+        return U * (N * 4 + K * 4 + K * 4 + K * 4 + K) + U * moved_rows_per_unit * (2 * row + 8)
+    if kind == "store_append":  # the B value rows in and into the ring, the unit's masks and ring state
+        return U * (2 * B * row + 2 * 4 * ((N + 31) // 32) + 16)
+    if kind == "store_evict":
+        # the kept list and flags, the masks; every kept slot's codes and (s, z) read and written; the reserved
+        # rows (N_v + B after the eviction) read and written
+        nv = K // 4  # the default N_v the bench runs with
+        return U * (K * 5 + 2 * 4 * ((N + 31) // 32) + 2 * K * (d * bits // 8 + 8) + 2 * (nv + B) * row)
     if kind == "score_attn":
         return U * (N * row + wl.window_rows * row + N * 4)
     if kind == "value_score":
@@ -411,7 +423,7 @@ def timed_steps(torch, step, steps, stream, barrier=lambda: None, sampler=None):
     return e0.elapsed_time(e1) / steps, clocks
 
 
-def kernel_table(kernels, wl, variant, moved, layers_per_launch, hbm_peak, tflops_peak):
+def kernel_table(kernels, wl, variant, moved, layers_per_launch, hbm_peak, tflops_peak, bits=0):
     """Per kernel: launches, mean launch time, share of the kernel time, algorithmic GB/s; for the window
     score also its algorithmic QK^T TFLOP/s and the bound of its own roofline."""
     out = {}
@@ -420,7 +432,7 @@ def kernel_table(kernels, wl, variant, moved, layers_per_launch, hbm_peak, tflop
         if n == 0:
             continue
         per_launch = kms / n
-        b = kernel_bytes(name, wl, variant, moved) * layers_per_launch
+        b = kernel_bytes(name, wl, variant, moved, bits) * layers_per_launch
         rec = {"launches": n, "us_per_launch": round(1e3 * per_launch, 3), "share": round(kms / total, 4),
                "gbs": round(b / (per_launch / 1e3) / 1e9, 1)}
         if name == "score_attn":
@@ -437,14 +449,15 @@ def score_flops(wl):
     return wl.batch * wl.num_kv_heads * 2 * wl.window_rows * wl.slots * wl.head_dim
 
 
-def roofline_of(kernels_tab, dom, wl, variant, moved, layers_per_launch, hbm_peak, tflops_peak, peak_kind, traffic):
+def roofline_of(kernels_tab, dom, wl, variant, moved, layers_per_launch, hbm_peak, tflops_peak, peak_kind, traffic,
+                bits=0):
     rec = kernels_tab[dom]
     if rec.get("bound") == "tensor":
         f = score_flops(wl) * layers_per_launch
         return {"bound": "tensor", "achieved": rec["qkt_tflops"], "peak": tflops_peak, "unit": "TFLOP/s",
                 "frac": round(rec["qkt_tflops"] / tflops_peak, 4), "traffic": traffic, "kernel": dom,
                 "algorithmic_flops_per_launch": f, "peak_source": peak_kind + " bf16 burst"}
-    b = kernel_bytes(dom, wl, variant, moved) * layers_per_launch
+    b = kernel_bytes(dom, wl, variant, moved, bits) * layers_per_launch
     return {"bound": "hbm", "achieved": rec["gbs"], "peak": hbm_peak, "unit": "GB/s",
             "frac": round(rec["gbs"] / hbm_peak, 4), "traffic": traffic, "kernel": dom,
             "algorithmic_bytes_per_launch": b, "peak_source": peak_kind}
@@ -502,9 +515,40 @@ def score_ncu(wl):
 
 # the other configurations measured in the same run, each as a record of the JSON line: the single-layer case,
 # the Qwen3-1.7B and Qwen3-8B geometries (both scoring variants) and the sweep's largest budget
-EXTRA_CONFIGS = [("single_layer_k256", "attnv", None), ("qwen3_1p7b_k2048", "attnv", None),
-                 ("qwen3_8b_k4096", "attnv", None), ("qwen3_8b_k4096", "dkv", None),
-                 ("sweep:16384:128:32:0.005", "attnv", 21)]
+EXTRA_CONFIGS = [("single_layer_k256", "attnv", None, {}), ("qwen3_1p7b_k2048", "attnv", None, {"decode": True}),
+                 ("qwen3_1p7b_k2048", "attnv", None, {"value_bits": 4, "decode": True}),
+                 ("qwen3_8b_k4096", "attnv", None, {}), ("qwen3_8b_k4096", "dkv", None, {}),
+                 ("sweep:16384:128:32:0.005", "attnv", 21, {})]
+
+
+def decode_step_ms(torch, V, cache, wl, device, steps, warmup):
+    """ms of one decode step's attention over every layer's cache (vase_decode_attention per layer, captured in a
+    CUDA graph and replayed, as a serving loop runs it)."""
+    L = wl.num_layers
+    gen = torch.Generator(device=device)
+    gen.manual_seed(7)
+    q = torch.randn((L, wl.batch, wl.num_q_heads, wl.head_dim), generator=gen, device=device).to(torch.bfloat16)
+    out = torch.empty((L, wl.batch, wl.num_q_heads, wl.head_dim), dtype=torch.float32, device=device)
+    ptrs = [(q[l].data_ptr(), out[l].data_ptr()) for l in range(L)]
+
+    def step():
+        sh = torch.cuda.current_stream()
+        for l in range(L):
+            V.vase_decode_attention(cache.ctx, l, ptrs[l][0], ptrs[l][1], sh)
+
+    step()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step()
+    for _ in range(warmup):
+        graph.replay()
+    stream = torch.cuda.current_stream()
+    ms, _ = timed_steps(torch, graph.replay, steps, stream)
+    st, code = cache.check_device_error()
+    if st != 0:
+        raise RuntimeError(f"device error in the decode steps: {code:#x}")
+    return ms
 
 
 def workload_by_name(Wm, name, layers=None):
@@ -518,9 +562,13 @@ def workload_by_name(Wm, name, layers=None):
     return wl
 
 
-def measure_config(torch, V, Wm, name, variant, layers, steps, warmup, device, hbm_peak, tflops_peak):
+def measure_config(torch, V, Wm, name, variant, layers, steps, warmup, device, hbm_peak, tflops_peak,
+                   cache_kw=None):
     wl = workload_by_name(Wm, name, layers)
-    rig = Rig(wl, variant, device, 1000, torch, V)
+    cache_kw = dict(cache_kw or {})
+    with_decode = cache_kw.pop("decode", False)
+    bits = cache_kw.get("value_bits", 0)
+    rig = Rig(wl, variant, device, 1000, torch, V, **cache_kw)
     stream = torch.cuda.current_stream()
     for _ in range(warmup):
         rig.step(stream)
@@ -531,11 +579,19 @@ def measure_config(torch, V, Wm, name, variant, layers, steps, warmup, device, h
         raise RuntimeError(f"device error in {name}: {code:#x}")
     L = wl.num_layers
     moved = moved_rows(rig.cache, torch)
-    tab = kernel_table(kernels, wl, variant, moved, min(L, 64), hbm_peak, tflops_peak)
+    tab = kernel_table(kernels, wl, variant, moved, min(L, 64), hbm_peak, tflops_peak, bits)
     roof_ms = L * step_bytes(wl, variant) / (hbm_peak * 1e9) * 1e3
+    extra = {}
+    if bits:  # the compressed value store: its V buffer against the bf16 cache
+        sizes = V.vase_get_buffer_sizes(rig.cache.cfg)
+        bf_bytes = L * wl.batch * wl.num_kv_heads * wl.slots * 2 * wl.head_dim
+        extra = {"value_bits": bits, "v_bytes": sizes.v_cache, "v_bytes_bf16": bf_bytes,
+                 "v_bytes_ratio": round(sizes.v_cache / bf_bytes, 4)}
+    if with_decode:  # the decode step that reads the cache the eviction leaves (the store, with value_bits)
+        extra["decode_ms_per_step"] = round(decode_step_ms(torch, V, rig.cache, wl, device, steps, warmup), 4)
     rig.close()
     torch.cuda.empty_cache()
-    return {"workload": wl.name, "variant": variant, "layers": L, "batch": wl.batch, "budget_k": wl.budget_k,
+    return {"workload": wl.name, "variant": variant, **extra, "layers": L, "batch": wl.batch, "budget_k": wl.budget_k,
             "buffer_b": wl.buffer_b, "window": wl.window, "heads": f"{wl.num_q_heads}/{wl.num_kv_heads}",
             "steps": steps, "ms_per_step": round(ms, 4),
             "token_heads_per_s": L * wl.batch * wl.num_kv_heads * wl.slots / (ms / 1e3),
@@ -573,7 +629,7 @@ def run_ours(args):
     hbm_peak, tflops_peak, peak_kind = measured_peaks()
     L, K, Bf = wl.num_layers, wl.budget_k, wl.buffer_b
     rig = Rig(wl, args.variant, device, 1000 + rank, torch, V, reserve=args.reserve, gqa=args.gqa,
-              dkv_shared_g=args.dkv_shared_g)
+              dkv_shared_g=args.dkv_shared_g, value_bits=args.value_bits)
     cache = rig.cache
     stream = torch.cuda.current_stream()
 
@@ -642,10 +698,10 @@ def run_ours(args):
 
     # ---- roofline of the dominant kernel
     layers_per_launch = min(L, 64)
-    tab = kernel_table(kernels, wl, args.variant, moved, layers_per_launch, hbm_peak, tflops_peak)
+    tab = kernel_table(kernels, wl, args.variant, moved, layers_per_launch, hbm_peak, tflops_peak, args.value_bits)
     dom = max(tab, key=lambda k: tab[k]["share"])
     roofline = roofline_of(tab, dom, wl, args.variant, moved, layers_per_launch, hbm_peak, tflops_peak, peak_kind,
-                           traffic_of(dom, wl, args.variant, L))
+                           None if args.value_bits else traffic_of(dom, wl, args.variant, L), args.value_bits)
     step_roof_ms = L * step_bytes(wl, args.variant) / (hbm_peak * 1e9) * 1e3
     evict_ms = sum(kernels[k][0] for k in kernels if k != "append") / args.steps
     rig.close()
@@ -678,8 +734,8 @@ def run_ours(args):
     }
     if rank == 0 and world == 1 and not args.no_configs:
         out["configs"] = [measure_config(torch, V, Wm, name, variant, layers, args.steps, args.warmup, device,
-                                         hbm_peak, tflops_peak)
-                          for (name, variant, layers) in EXTRA_CONFIGS]
+                                         hbm_peak, tflops_peak, kw)
+                          for (name, variant, layers, kw) in EXTRA_CONFIGS]
     if pool is not None:
         v, done, wall = oracle_throughput(pool, n_units, wl, args.cpu_seconds)
         pool.close()
@@ -709,7 +765,7 @@ def run_decode(args):
 
     L, K, Bf = wl.num_layers, wl.budget_k, wl.buffer_b
     cache = V.VaseCache(V.Geometry(K, Bf, wl.window, wl.num_q_heads, wl.num_kv_heads, L, wl.batch),
-                        variant=args.variant, seed=0, device=device)
+                        variant=args.variant, seed=0, device=device, value_bits=args.value_bits)
     gen = torch.Generator(device=device)
     gen.manual_seed(1000)
     for layer in range(L):
@@ -786,7 +842,16 @@ def run_decode(args):
     # K and V rows of the kept slots, the query rows in, the fp32 outputs out
     step_bytes_ = L * (units * K * 2 * 2 * wl.head_dim + wl.batch * wl.num_q_heads * wl.head_dim * (2 + 4))
     mixed_info = None
-    if bits:
+    if args.value_bits:
+        # compressed value store: K rows, the code rows and (s, z) of every slot, the ring rows of the bf16 slots,
+        # the masks and ring state
+        vb = args.value_bits
+        ring_rows = sum(int(cache.value_store(l)["state"][:, 1].sum().item()) for l in range(L))
+        step_bytes_ = (L * units * K * (2 * wl.head_dim + wl.head_dim * vb // 8 + 8) + ring_rows * 2 * wl.head_dim +
+                       L * units * (4 * ((K + Bf + 31) // 32) + 16) +
+                       L * wl.batch * wl.num_q_heads * wl.head_dim * (2 + 4))
+        mixed_info = {"value_bits": vb, "store": True, "reserved_fraction": round(ring_rows / (L * units * K), 4)}
+    elif bits:
         # b-bit values: K rows, bf16 V rows of the reserved slots, code rows and (s, z) of the others, the masks
         coded = L * units * K - reserved
         step_bytes_ = (L * units * K * 2 * wl.head_dim + reserved * 2 * wl.head_dim +
@@ -807,7 +872,7 @@ def run_decode(args):
                    "l2": f"inputs larger than L2 ({step_bytes_ / 1e9:.2f} GB read per step)"},
         "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                      "frac": round(gbs / hbm_peak, 4), "traffic": None,
-                     "kernel": ("decode_simt_kernel" if bits or wl.group < 3 else "decode_tc_kernel"),
+                     "kernel": ("decode_simt_kernel" if bits or args.value_bits or wl.group < 3 else "decode_tc_kernel"),
                      "algorithmic_bytes_per_launch": step_bytes_ // L, "peak_source": peak_kind},
         "clocks": clocks, "gpu_launches": launches, "timed_as": "CUDA graph replay of the step's launches",
         "eager_ms_per_step": eager_ms,
@@ -929,6 +994,8 @@ def variant_options(args):
         opts["gqa"] = args.gqa
     if args.dkv_shared_g:
         opts["dkv_shared_g"] = True
+    if args.value_bits:
+        opts["value_bits"] = args.value_bits
     return opts
 
 

@@ -36,7 +36,7 @@
 extern "C" {
 #endif
 
-#define VASE_ABI_VERSION 2
+#define VASE_ABI_VERSION 3
 
 #define VASE_OK 0
 #define VASE_EVICT_DUE 1          /* the layer's cache is full: call vase_evict before the next append */
@@ -82,12 +82,13 @@ typedef struct vase_config {
     int32_t reserve_kind;  /* AttnV: VASE_RESERVE_* (how R_V is chosen) */
     int32_t gqa_reduce;    /* AttnV: VASE_GQA_*; VASE_GQA_MAX needs W % 4 == 0 and, when G*W > 256, 256 % W == 0 */
     int32_t dkv_shared_g;  /* DKV: 1 = one G per round shared by every layer, sequence and KV head; 0 = per unit */
+    int32_t value_bits;    /* AttnV: 0 = bf16 value cache; 2, 4 or 8 = the compressed value store (below) */
 } vase_config;
 
 /* Sizes in bytes of the caller-allocated device buffers for a configuration. */
 typedef struct vase_buffer_sizes {
     size_t k_cache;    /* bf16 [L][b][Hkv][K+B][d] */
-    size_t v_cache;    /* bf16 [L][b][Hkv][K+B][d] */
+    size_t v_cache;    /* bf16 [L][b][Hkv][K+B][d]; with value_bits > 0 the compressed value store of every layer */
     size_t q_window;   /* bf16 [L][b][Hq][W][d], a ring over the last W decode queries */
     size_t positions;  /* int32 [L][b][Hkv][K+B], absolute stream position of each slot, -1 if empty */
     size_t value_scores; /* fp32 [L][b][Hkv][K+B], value magnitude of the token in each slot */
@@ -224,8 +225,10 @@ int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream);
  * The caller owns q and out; the call uses no workspace (the slots of each KV head are split
  * over the CTAs of one thread-block cluster, whose states are folded in shared memory), so
  * calls may overlap with each other but not with an append or eviction of the same layer.
+ * With the compressed value store (value_bits > 0) the values are read from it: bf16 rows from the
+ * reserved ring, every other value as Q s + z from its codes (CUDA cores, at most 8 query heads per KV head).
  * Errors: VASE_ERR_INVALID (bad layer, null pointer, empty layer), VASE_ERR_ALIGN,
- * VASE_ERR_UNSUPPORTED (more than 16 query heads per KV head). */
+ * VASE_ERR_UNSUPPORTED (more than 16 query heads per KV head; more than 8 with the store). */
 int vase_decode_attention(vase_ctx* ctx, int32_t layer, const void* q, float* out, void* stream);
 
 /* ---- Mixed-precision values: the b-bit per-token quantizer of Sec. 4.4 and the reserved cache of Sec. 6.
@@ -321,10 +324,46 @@ int vase_kv_view_get(const vase_ctx* ctx, int32_t layer, vase_kv_view* out);
  * in the workspace; the caller copies what it needs before the next eviction. */
 int vase_debug_view_get(const vase_ctx* ctx, int32_t slot, vase_debug_view* out);
 
+/* ---- Compressed value store (value_bits = 2, 4 or 8; AttnV only).  The mixed-precision value cache that Sec. 6
+ * proposes, built on the per-token asymmetric b-bit quantizer of Sec. 4.4 (z = min v, s = Range(v) / (2^b - 1),
+ * Q = round((v - z) / s) half to even, decided in fp32, v' = Q s + z).  Keys stay in the bf16 K cache; a value is
+ * held either as a bf16 row in the unit's reserved cache or as its codes:
+ *   - the reserved cache is a ring of H = N_v + 2B rows: R_V and R_B after an eviction (Sec. 3.1 and Sec. 2, at
+ *     most N_v + B values) and the B values appended before the next eviction;
+ *   - every appended value enters the ring in bf16; an append that finds the ring full quantizes its earliest
+ *     value into the codes (the rule of Sec. 6), which happens only before the layer's first eviction;
+ *   - an eviction moves the kept values with their slots and quantizes the kept bf16 values that are not in the
+ *     new R_V u R_B (a quantized value never returns to bf16).
+ * The V buffer holds, per layer (layer stride and offsets in vase_value_store), for each of the b*Hkv units:
+ * codes uint8 [K+B][16 b] (lane-packed: dims 4i .. 4i+3 in 4b bits at byte i*b/2), (s, z) fp32 [sz_stride][2],
+ * mask uint32 [mask_stride] (bit t of word w set = slot 32 w + t is held in bf16), ring bf16 [H][d] (the bf16
+ * values in slot order, the i-th at row (head + i) mod H), state int32 [4] = (head, count, 0, 0).  The library
+ * writes all of it; the first append of a layer (fill 0) starts it empty.  vase_decode_attention reads it;
+ * vase_kv_view_get reports v = NULL.  Not available in this mode (VASE_ERR_UNSUPPORTED): the DKV variant (its
+ * score reads every value each round), vase_refresh_value_scores, vase_quantize_values,
+ * vase_decode_attention_mixed (the bf16-cache read path) and vase_evict_static_scratch. */
+typedef struct vase_value_store {
+    uint8_t* codes;        /* device, layer's [units][slots][code_row] */
+    float* sz;             /* device, [units][sz_stride][2] */
+    uint32_t* mask;        /* device, [units][mask_stride] */
+    void* ring;            /* device, bf16 [units][ring_rows][d] */
+    int32_t* state;        /* device, [units][4]: ring head, ring count */
+    int32_t bits, code_row, slots, sz_stride, mask_stride, ring_rows, units, fill;
+} vase_value_store;
+
+/* Device pointers to one layer's compressed value store.  Errors: VASE_ERR_INVALID (null or bad layer),
+ * VASE_ERR_UNSUPPORTED (value_bits = 0). */
+int vase_value_store_get(const vase_ctx* ctx, int32_t layer, vase_value_store* out);
+
 /* Synchronises the stream, then reads and clears the device error word that
  * bounded waits and device-side checks set.  Returns VASE_OK or VASE_ERR_DEVICE
  * (with *code, if non-NULL, set to the raw word). */
 int vase_check_device_error(vase_ctx* ctx, void* stream, uint32_t* code);
+/* Sites (code & 0xffff) of the compressed value store: an append or eviction found a ring state or bf16 masks
+ * it did not write (head or count out of range) and wrote nothing; an append would overflow the ring after an
+ * eviction (a fill that skipped an eviction).  The decode reads such a store with head 0 and records its own site. */
+#define VASE_SITE_STORE_OVERFLOW 80
+#define VASE_SITE_STORE_STATE 81
 
 /* Self-test of the failure detection: launches on `stream` a one-thread kernel whose
  * bounded wait on an mbarrier that nothing completes runs out (about two seconds,
@@ -346,7 +385,9 @@ int64_t vase_launch_count(const vase_ctx* ctx);
 #define VASE_KERNEL_DKV 3     /* DKV leverage scores (tcgen05) */
 #define VASE_KERNEL_SELECT 4  /* reservation + sampling + kept list + stable in-place gather of the kept rows */
 #define VASE_KERNEL_EVICT_SMALL 5 /* window score + selection + gather in one launch (launch-bound batches of small units) */
-#define VASE_KERNEL_COUNT 6
+#define VASE_KERNEL_STORE_APPEND 6 /* compressed value store: new values into the reserved ring (earliest out when full) */
+#define VASE_KERNEL_STORE_EVICT 7  /* compressed value store: codes and ring compacted, values leaving R_V u R_B quantized */
+#define VASE_KERNEL_COUNT 8
 
 /* enable = 1: from now on record a CUDA event pair on the launch stream around
  * every kernel (host-side instrumentation, no change to the kernels);

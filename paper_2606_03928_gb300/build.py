@@ -20,7 +20,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libvase.so")
-SOURCES = ["api.cu", "score_attn.cu", "dkv.cu", "misc.cu", "decode.cu", "decode_mixed.cu", "selftest.cu"]
+SOURCES = ["api.cu", "score_attn.cu", "dkv.cu", "misc.cu", "store.cu", "decode.cu", "decode_mixed.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 
@@ -47,8 +47,10 @@ def source_digest():
 # The source files each timed kernel is compiled from (its own translation unit and the headers it includes).
 KERNEL_SOURCES = {
     "score_attn": ["score_attn.cu", "kernels.cuh", "ptx.cuh"],
-    "select_compact": ["misc.cu", "kernels.cuh", "ptx.cuh"],
-    "append": ["misc.cu", "kernels.cuh", "ptx.cuh"],
+    "select_compact": ["misc.cu", "kernels.cuh", "ptx.cuh", "quant.cuh"],
+    "append": ["misc.cu", "kernels.cuh", "ptx.cuh", "quant.cuh"],
+    "store_append": ["store.cu", "kernels.cuh", "ptx.cuh", "quant.cuh"],
+    "store_evict": ["store.cu", "kernels.cuh", "ptx.cuh", "quant.cuh"],
     "dkv_score": ["dkv.cu", "kernels.cuh", "ptx.cuh"],
     "decode": ["decode.cu", "decode_simt.cuh", "decode_mixed.cu", "kernels.cuh", "ptx.cuh"],
 }

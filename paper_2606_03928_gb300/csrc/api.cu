@@ -38,6 +38,12 @@ struct Plan {
     size_t stride_attn, stride_un, stride_src;  // elements per workspace slot
     size_t off_err, off_attn, off_pooled, off_vscore, off_key, off_keep, off_src, off_staging, staging_bytes, ws_bytes;
     size_t decode_smem;                           // decode attention: shared memory per CTA
+    // compressed value store (value_bits > 0): per layer the codes, (s, z), masks, ring and ring state of every unit
+    bool store;
+    int st_H, st_Np, st_mask_words, st_mask_stride, st_code_row;
+    size_t st_codes_off, st_qp_off, st_mask_off, st_ring_off, st_state_off, st_layer_bytes, st_evict_smem;
+    size_t st_append_smem;  // the append's shared memory when the ring may overflow (a first fill of N past H)
+    size_t off_resv;  // workspace: [slot][units][K] R_V u R_B flags of the kept slots
     // fused eviction of small units (evict_small_kernel): usable when the unit's score matrix fits in TMEM
     bool small_ok;
     int small_tiles, small_stages, small_tmem_cols;
@@ -70,6 +76,10 @@ const char* check_config(const vase_config* c) {
     if (c->gqa_reduce != VASE_GQA_MEAN && c->gqa_reduce != VASE_GQA_MAX) return "unknown gqa_reduce";
     if (c->dkv_shared_g != 0 && c->dkv_shared_g != 1) return "dkv_shared_g must be 0 or 1";
     if (c->gqa_reduce == VASE_GQA_MAX && c->window % 4) return "GQA max-aggregation needs window % 4 == 0";
+    if (c->value_bits != 0 && c->value_bits != 2 && c->value_bits != 4 && c->value_bits != 8)
+        return "value_bits must be 0, 2, 4 or 8";
+    if (c->value_bits != 0 && c->variant != VASE_VARIANT_ATTNV)
+        return "the compressed value store needs the AttnV variant (DKV scores read every value each round)";
     return nullptr;
 }
 
@@ -242,6 +252,8 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     o = align_up(o + Z * un, kAlign);
     p.off_src = o;
     o = align_up(o + Z * p.stride_src * 4, kAlign);
+    p.off_resv = o;
+    o = align_up(o + Z * p.units * static_cast<size_t>(store_resv_stride(c->budget_k)), kAlign);
     p.off_staging = o;
     p.staging_bytes = static_cast<size_t>(c->buffer_b) * c->batch * (c->num_q_heads + 2 * c->num_kv_heads) * kRowBytes;
     o = align_up(o + p.staging_bytes, kAlign);
@@ -253,14 +265,44 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     p.small_tmem_cols = 32;
     while (p.small_tmem_cols < p.n_tiles * p.GWp) p.small_tmem_cols *= 2;
     p.small_smem = evict_small_smem_bytes(p.N, c->budget_k, p.GWp, p.q_box, p.n_tiles, p.small_stages);
+    p.store = c->value_bits != 0;
     p.small_ok = c->variant == VASE_VARIANT_ATTNV && p.GWp <= 128 && p.n_tiles <= kSmallMaxTiles &&
-                 p.n_tiles * p.GWp <= 512 && p.q_box >= p.GWp && p.small_smem <= kMaxDynSmem;
+                 p.n_tiles * p.GWp <= 512 && p.q_box >= p.GWp && p.small_smem <= kMaxDynSmem && !p.store;
+    // compressed value store: the reserved ring holds R_V u R_B after an eviction and the B values appended
+    // before the next one
+    p.st_H = p.n_v + 2 * c->buffer_b;
+    p.st_Np = (p.N + 1) & ~1;
+    p.st_mask_words = ceil_div(p.N, 32);
+    p.st_mask_stride = (p.st_mask_words + 3) & ~3;
+    p.st_code_row = c->value_bits ? kHeadDim * c->value_bits / 8 : 0;
+    {
+        const size_t u = static_cast<size_t>(p.units);
+        size_t so = 0;
+        p.st_codes_off = so;
+        so = align_up(so + u * p.N * p.st_code_row, kAlign);
+        p.st_qp_off = so;
+        so = align_up(so + u * p.st_Np * 8, kAlign);
+        p.st_mask_off = so;
+        so = align_up(so + u * p.st_mask_stride * 4, kAlign);
+        p.st_ring_off = so;
+        so = align_up(so + u * p.st_H * kRowBytes, kAlign);
+        p.st_state_off = so;
+        so = align_up(so + u * 16, kAlign);
+        p.st_layer_bytes = so;
+    }
+    p.st_evict_smem = store_evict_smem_bytes(c->budget_k, p.st_mask_stride);
+    p.st_append_smem = store_append_smem_bytes(p.st_mask_stride, p.st_H, p.N, c->budget_k, true);
+    if (p.store && (p.st_evict_smem > kMaxDynSmem || p.st_append_smem > kMaxDynSmem ||
+                    p.st_mask_words > kDecodeMaxMaskWords)) {
+        *why = "K + B too large for the compressed value store";
+        return false;
+    }
     return true;
 }
 
 ScoreAttnParams score_params(const Plan& P, const vase_config& c, const LayerBatch& batch, int nz, float* attn,
                              uint32_t* err) {
-    ScoreAttnParams sp;
+    ScoreAttnParams sp{};
     sp.batch = batch;
     sp.N = P.N;
     sp.GW = P.GW;
@@ -422,6 +464,34 @@ int32_t* pos_layer(vase_ctx* c, int layer) {
     return c->bufs.positions + static_cast<int64_t>(layer) * c->plan.units * c->plan.N;
 }
 
+// The compressed value store's parameter block (layer-independent part).
+StoreParams store_params(vase_ctx* ctx) {
+    const Plan& P = ctx->plan;
+    const vase_config& c = ctx->cfg;
+    StoreParams sp;
+    std::memset(&sp, 0, sizeof(sp));
+    sp.base = static_cast<uint8_t*>(ctx->bufs.v_cache);
+    sp.layer_bytes = static_cast<int64_t>(P.st_layer_bytes);
+    sp.codes_off = static_cast<int64_t>(P.st_codes_off);
+    sp.qp_off = static_cast<int64_t>(P.st_qp_off);
+    sp.mask_off = static_cast<int64_t>(P.st_mask_off);
+    sp.ring_off = static_cast<int64_t>(P.st_ring_off);
+    sp.state_off = static_cast<int64_t>(P.st_state_off);
+    sp.units = P.units;
+    sp.N = P.N;
+    sp.Np = P.st_Np;
+    sp.mask_stride = P.st_mask_stride;
+    sp.mask_words = P.st_mask_words;
+    sp.H = P.st_H;
+    sp.bits = c.value_bits;
+    sp.code_row = P.st_code_row;
+    sp.K = c.budget_k;
+    sp.b = c.batch;
+    sp.Hkv = c.num_kv_heads;
+    sp.err = reinterpret_cast<uint32_t*>(ctx->ws + P.off_err);
+    return sp;
+}
+
 }  // namespace
 
 namespace vase {
@@ -452,7 +522,7 @@ int vase_get_buffer_sizes(const vase_config* cfg, vase_buffer_sizes* out) {
     if (!make_plan(cfg, 152, &p, &why)) return cfg->head_dim != 128 ? VASE_ERR_UNSUPPORTED : VASE_ERR_INVALID;
     const size_t rows = static_cast<size_t>(cfg->num_layers) * p.units * p.N;
     out->k_cache = rows * kRowBytes;
-    out->v_cache = rows * kRowBytes;
+    out->v_cache = p.store ? static_cast<size_t>(cfg->num_layers) * p.st_layer_bytes : rows * kRowBytes;
     out->q_window = static_cast<size_t>(cfg->num_layers) * cfg->batch * cfg->num_q_heads * cfg->window * kRowBytes;
     out->positions = rows * 4;
     out->value_scores = rows * 4;
@@ -509,11 +579,14 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
         return VASE_ERR_UNSUPPORTED;
     }
     const uint32_t qbox = static_cast<uint32_t>(P.q_box);
+    // (with the compressed value store there are no V rows to map; no kernel of that mode reads the V maps)
+    std::memset(&ctx->vmap, 0, sizeof(ctx->vmap));
+    std::memset(&ctx->vmap_dec, 0, sizeof(ctx->vmap_dec));
     if (!encode_rows(enc, &ctx->kmap, bufs->k_cache, cache_rows, kTileTokens) ||
-        !encode_rows(enc, &ctx->vmap, bufs->v_cache, cache_rows, kTileTokens) ||
+        (!P.store && !encode_rows(enc, &ctx->vmap, bufs->v_cache, cache_rows, kTileTokens)) ||
         !encode_rows(enc, &ctx->qmap, bufs->q_window, q_rows, qbox) ||
         !encode_rows(enc, &ctx->kmap_dec, bufs->k_cache, cache_rows, kDecodeTileRows) ||
-        !encode_rows(enc, &ctx->vmap_dec, bufs->v_cache, cache_rows, kDecodeTileRows)) {
+        (!P.store && !encode_rows(enc, &ctx->vmap_dec, bufs->v_cache, cache_rows, kDecodeTileRows))) {
         fprintf(stderr, "vase_create: tensor map encoding failed\n");
         delete ctx;
         return VASE_ERR_CUDA;
@@ -524,7 +597,8 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
         (e = decode_set_attributes(P.G, P.decode_smem)) != cudaSuccess ||
         (e = decode_mixed_set_attributes()) != cudaSuccess ||
         (e = quantize_set_attributes(quantize_smem_bytes(cfg->budget_k, cfg->buffer_b))) != cudaSuccess ||
-        (P.small_ok && (e = evict_small_set_attributes(P.small_smem)) != cudaSuccess)) {
+        (P.small_ok && (e = evict_small_set_attributes(P.small_smem)) != cudaSuccess) ||
+        (P.store && (e = store_set_attributes(P.st_evict_smem, P.st_append_smem)) != cudaSuccess)) {
         fprintf(stderr, "vase_create: kernel attributes: %s\n", cudaGetErrorString(e));
         delete ctx;
         return VASE_ERR_CUDA;
@@ -565,7 +639,7 @@ int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void*
                                          : static_cast<size_t>(n_tokens) * c.batch * c.num_kv_heads * kVecPerRow;
     for (int z0 = 0; z0 < n_layers; z0 += kMaxLayerBatch) {
         const int nz = n_layers - z0 < kMaxLayerBatch ? n_layers - z0 : kMaxLayerBatch;
-        AppendParams p;
+        AppendParams p{};
         p.q = static_cast<const uint4*>(q) + z0 * q_slot;
         p.k = static_cast<const uint4*>(k) + z0 * kv_slot;
         p.v = static_cast<const uint4*>(v) + z0 * kv_slot;
@@ -573,7 +647,7 @@ int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void*
         p.kv_stride = static_cast<int64_t>(kv_slot);
         p.qwin = static_cast<uint4*>(ctx->bufs.q_window);
         p.kc = static_cast<uint4*>(ctx->bufs.k_cache);
-        p.vc = static_cast<uint4*>(ctx->bufs.v_cache);
+        p.vc = ctx->plan.store ? nullptr : static_cast<uint4*>(ctx->bufs.v_cache);  // store: values go below
         p.pos = ctx->bufs.positions;
         p.vmag = ctx->bufs.value_scores;
         p.kind = c.value_score;
@@ -593,6 +667,25 @@ int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void*
         cudaError_t e = timed_launch(ctx, VASE_KERNEL_APPEND, stream, [&] { return launch_append(p, nz, stream); });
         if (e != cudaSuccess) return cuda_fail(ctx, e, "append launch");
         ctx->launches += 1;
+        if (ctx->plan.store) {
+            StoreParams sp = store_params(ctx);
+            for (int z = 0; z < nz; ++z) {
+                const vase_layer_state& st = ctx->layers[layers[z0 + z]];
+                sp.layer[z] = layers[z0 + z];
+                sp.fill[z] = st.fill;
+                sp.round[z] = st.round;
+                // before the first eviction a fill past H overflows the ring (the bf16 count is at most the fill)
+                if (st.round == 0 && st.fill + n_tokens > ctx->plan.st_H) sp.big = 1;
+            }
+            sp.v = p.v;
+            sp.kv_stride = p.kv_stride;
+            sp.n = n_tokens;
+            sp.n_v = ctx->plan.n_v;
+            sp.vmag = ctx->bufs.value_scores;
+            e = timed_launch(ctx, VASE_KERNEL_STORE_APPEND, stream, [&] { return launch_store_append(sp, nz, stream); });
+            if (e != cudaSuccess) return cuda_fail(ctx, e, "value store append launch");
+            ctx->launches += 1;
+        }
     }
     bool due = false;
     for (int z = 0; z < n_layers; ++z) {
@@ -628,8 +721,9 @@ void fill_select_params(vase_ctx* ctx, const LayerBatch& batch, float* attn, flo
     sel.vscore_dbg = (c.debug_outputs && c.variant == VASE_VARIANT_ATTNV) ? vscore : nullptr;
     sel.pos = ctx->bufs.positions;
     sel.kc = static_cast<uint4*>(ctx->bufs.k_cache);
-    sel.vc = static_cast<uint4*>(ctx->bufs.v_cache);
+    sel.vc = P.store ? nullptr : static_cast<uint4*>(ctx->bufs.v_cache);  // the store's values move below
     sel.src = src;
+    sel.resv = P.store ? ctx->ws + P.off_resv : nullptr;
     sel.pooled_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_pooled) : nullptr;
     sel.key_dbg = c.debug_outputs ? reinterpret_cast<float*>(ctx->ws + P.off_key) : nullptr;
     sel.keep_dbg = c.debug_outputs ? ctx->ws + P.off_keep : nullptr;
@@ -666,12 +760,12 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
         if ((e = cudaStreamWaitEvent(s, ctx->read_done, 0)) != cudaSuccess) return cuda_fail(ctx, e, "read-back wait");
         ctx->read_pending = false;
     }
-    SelectParams sel;
+    SelectParams sel{};  // value-initialised: a field this path does not set is zero (pointers null)
     fill_select_params(ctx, batch, attn, vscore, src, err, &sel);
     // Launch-bound batches (every unit of every layer in one wave, one CTA each) whose units are small enough for
     // the fused kernel: score, selection and gather in one launch
     if (P.small_ok && static_cast<long>(P.units) * nz <= P.num_sms) {
-        SmallEvictParams sm;
+        SmallEvictParams sm{};
         sm.sel = sel;
         sm.sel.n_parts = 1;
         sm.sel.staged = 1;
@@ -710,7 +804,7 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
             return cuda_fail(ctx, e, "score launch");
         ctx->launches += 1;
     } else {
-        DkvParams dp;
+        DkvParams dp{};
         dp.batch = batch;
         dp.N = P.N;
         dp.K = c.budget_k;
@@ -737,6 +831,16 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
         cudaSuccess)
         return cuda_fail(ctx, e, "select launch");
     ctx->launches += 1;
+    if (P.store) {
+        StoreParams sp = store_params(ctx);
+        for (int z = 0; z < nz; ++z) sp.layer[z] = layers[z];
+        sp.src = src;
+        sp.resv = ctx->ws + P.off_resv;
+        if ((e = timed_launch(ctx, VASE_KERNEL_STORE_EVICT, s, [&] { return launch_store_evict(sp, nz, s); })) !=
+            cudaSuccess)
+            return cuda_fail(ctx, e, "value store eviction launch");
+        ctx->launches += 1;
+    }
     for (int z = 0; z < nz; ++z) {
         vase_layer_state& st = ctx->layers[layers[z]];
         st.fill = c.budget_k;
@@ -850,9 +954,11 @@ int vase_evict_all(vase_ctx* ctx, void* stream) {
 int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream) {
     if (!ctx) return VASE_ERR_INVALID;
     if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    if (ctx->plan.store)
+        return fail(ctx, VASE_ERR_UNSUPPORTED, "the compressed value store keeps no bf16 rows to recompute magnitudes from");
     const int rows = ctx->layers[layer].fill;
     if (rows == 0) return VASE_OK;
-    ValueParams vp;
+    ValueParams vp{};
     vp.vc = static_cast<const uint4*>(ctx->bufs.v_cache) + static_cast<int64_t>(layer) * ctx->plan.units * ctx->plan.N * kVecPerRow;
     vp.out = ctx->bufs.value_scores + static_cast<int64_t>(layer) * ctx->plan.units * ctx->plan.N;
     vp.N = ctx->plan.N;
@@ -866,6 +972,51 @@ int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream) {
     return VASE_OK;
 }
 
+}  // extern "C"
+
+namespace {
+
+// Decode attention over the compressed value store: the mixed-precision kernel with the store's arrays (codes of
+// every slot, the ring of bf16 rows and its head).
+int decode_store(vase_ctx* ctx, int32_t layer, const void* q, float* out, cudaStream_t stream) {
+    const Plan& P = ctx->plan;
+    if (P.G > 8) return fail(ctx, VASE_ERR_UNSUPPORTED, "decode over the compressed value store handles at most 8 query heads per KV head");
+    uint8_t* base = static_cast<uint8_t*>(ctx->bufs.v_cache) + static_cast<size_t>(layer) * P.st_layer_bytes;
+    DecodeParams dp{};
+    dp.q = static_cast<const uint4*>(q);
+    dp.kc = kc_layer(ctx, layer);
+    dp.vc = nullptr;
+    dp.out = out;
+    dp.N = P.N;
+    dp.fill = ctx->layers[layer].fill;
+    dp.G = P.G;
+    dp.Hkv = ctx->cfg.num_kv_heads;
+    dp.units = P.units;
+    dp.row_base = layer * P.units * P.N;
+    dp.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
+    dp.err = reinterpret_cast<uint32_t*>(ctx->ws + P.off_err);
+    dp.codes = base + P.st_codes_off;
+    dp.qparams = reinterpret_cast<const float*>(base + P.st_qp_off);
+    dp.rmask = reinterpret_cast<const uint32_t*>(base + P.st_mask_off);
+    dp.hp_rows = reinterpret_cast<const uint4*>(base + P.st_ring_off);
+    dp.ring_state = reinterpret_cast<const int32_t*>(base + P.st_state_off);
+    dp.bits = ctx->cfg.value_bits;
+    dp.code_row = P.st_code_row;
+    dp.Kq = P.N;  // every slot has a code row (unit stride N); bf16 values are the masked ones
+    dp.Kp = P.st_Np;
+    dp.mask_words = P.st_mask_stride;
+    dp.hp_cap = P.st_H;
+    cudaError_t e = launch_decode_mixed(dp, P.num_sms, stream);
+    if (e == cudaErrorInvalidValue) return fail(ctx, VASE_ERR_UNSUPPORTED, "too many slots for the mixed decode");
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "value store decode attention launch");
+    ctx->launches += 1;
+    return VASE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
 int vase_decode_attention(vase_ctx* ctx, int32_t layer, const void* q, float* out, void* stream) {
     if (!ctx) return VASE_ERR_INVALID;
     if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
@@ -875,10 +1026,12 @@ int vase_decode_attention(vase_ctx* ctx, int32_t layer, const void* q, float* ou
     if (fill < 1) return fail(ctx, VASE_ERR_INVALID, "the layer holds no cached pair");
     const Plan& P = ctx->plan;
     if (P.G > 16) return fail(ctx, VASE_ERR_UNSUPPORTED, "decode attention handles at most 16 query heads per KV head");
-    DecodeParams dp;
+    if (P.store) return decode_store(ctx, layer, q, out, static_cast<cudaStream_t>(stream));
+    DecodeParams dp{};
     dp.q = static_cast<const uint4*>(q);
     dp.kc = kc_layer(ctx, layer);
     dp.vc = vc_layer(ctx, layer);
+    dp.ring_state = nullptr;
     dp.out = out;
     dp.N = P.N;
     dp.fill = fill;
@@ -929,6 +1082,8 @@ int vase_quantize_values(vase_ctx* ctx, int32_t layer, int32_t bits, const vase_
     if (!ctx) return VASE_ERR_INVALID;
     if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
     if (bits != 2 && bits != 4 && bits != 8) return fail(ctx, VASE_ERR_INVALID, "bits must be 2, 4 or 8");
+    if (ctx->plan.store)
+        return fail(ctx, VASE_ERR_UNSUPPORTED, "the compressed value store quantizes by itself (value_bits)");
     if (!mb || !mb->codes || !mb->qparams || !mb->rmask || !mb->hp_rows)
         return fail(ctx, VASE_ERR_INVALID, "null mixed buffers");
     if (!aligned(mb->codes, 16) || !aligned(mb->qparams, 16) || !aligned(mb->rmask, 16) || !aligned(mb->hp_rows, 16))
@@ -940,7 +1095,7 @@ int vase_quantize_values(vase_ctx* ctx, int32_t layer, int32_t bits, const vase_
     if (st.round < 1 || st.fill != c.budget_k)
         return fail(ctx, VASE_ERR_INVALID, "quantize right after an eviction (fill == K)");
     const Plan& P = ctx->plan;
-    QuantParams qp;
+    QuantParams qp{};
     qp.vc = vc_layer(ctx, layer);
     qp.vmag = ctx->bufs.value_scores + static_cast<int64_t>(layer) * P.units * P.N;
     qp.codes = static_cast<uint8_t*>(mb->codes);
@@ -969,6 +1124,8 @@ int vase_decode_attention_mixed(vase_ctx* ctx, int32_t layer, int32_t bits, cons
                                 const void* q, float* out, void* stream) {
     if (!ctx) return VASE_ERR_INVALID;
     if (!check_layer(ctx, layer)) return fail(ctx, VASE_ERR_INVALID, "layer out of range");
+    if (ctx->plan.store)
+        return fail(ctx, VASE_ERR_UNSUPPORTED, "with the compressed value store, vase_decode_attention reads it");
     if (!q || !out || !mb || !mb->codes || !mb->qparams || !mb->rmask || !mb->hp_rows)
         return fail(ctx, VASE_ERR_INVALID, "null input, output or mixed buffer");
     if (!aligned(q, 16) || !aligned(out, 4)) return fail(ctx, VASE_ERR_ALIGN, "q must be 16-byte aligned, out 4-byte");
@@ -979,7 +1136,7 @@ int vase_decode_attention_mixed(vase_ctx* ctx, int32_t layer, int32_t bits, cons
         return fail(ctx, VASE_ERR_INVALID, "no codes of this bit width for the layer's current round");
     const Plan& P = ctx->plan;
     if (P.G > 16) return fail(ctx, VASE_ERR_UNSUPPORTED, "decode attention handles at most 16 query heads per KV head");
-    DecodeParams dp;
+    DecodeParams dp{};
     dp.q = static_cast<const uint4*>(q);
     dp.kc = kc_layer(ctx, layer);
     dp.vc = vc_layer(ctx, layer);
@@ -995,6 +1152,7 @@ int vase_decode_attention_mixed(vase_ctx* ctx, int32_t layer, int32_t bits, cons
     dp.codes = static_cast<const uint8_t*>(mb->codes);
     dp.qparams = mb->qparams;
     dp.rmask = mb->rmask;
+    dp.ring_state = nullptr;
     dp.bits = bits;
     dp.code_row = kHeadDim * bits / 8;
     dp.Kq = ctx->cfg.budget_k;
@@ -1161,11 +1319,32 @@ int vase_kv_view_get(const vase_ctx* ctx, int32_t layer, vase_kv_view* out) {
     if (!ctx || !out || layer < 0 || layer >= ctx->cfg.num_layers) return VASE_ERR_INVALID;
     vase_ctx* c = const_cast<vase_ctx*>(ctx);
     out->k = kc_layer(c, layer);
-    out->v = vc_layer(c, layer);
+    out->v = ctx->plan.store ? nullptr : vc_layer(c, layer);  // the store's values: vase_value_store_get
     out->positions = pos_layer(c, layer);
     out->value_scores = c->bufs.value_scores + static_cast<int64_t>(layer) * ctx->plan.units * ctx->plan.N;
     out->unit_stride = static_cast<int64_t>(ctx->plan.N) * kHeadDim;
     out->slots = ctx->plan.N;
+    out->fill = ctx->layers[layer].fill;
+    return VASE_OK;
+}
+
+int vase_value_store_get(const vase_ctx* ctx, int32_t layer, vase_value_store* out) {
+    if (!ctx || !out || layer < 0 || layer >= ctx->cfg.num_layers) return VASE_ERR_INVALID;
+    const Plan& P = ctx->plan;
+    if (!P.store) return VASE_ERR_UNSUPPORTED;
+    uint8_t* base = static_cast<uint8_t*>(ctx->bufs.v_cache) + static_cast<size_t>(layer) * P.st_layer_bytes;
+    out->codes = base + P.st_codes_off;
+    out->sz = reinterpret_cast<float*>(base + P.st_qp_off);
+    out->mask = reinterpret_cast<uint32_t*>(base + P.st_mask_off);
+    out->ring = base + P.st_ring_off;
+    out->state = reinterpret_cast<int32_t*>(base + P.st_state_off);
+    out->bits = ctx->cfg.value_bits;
+    out->code_row = P.st_code_row;
+    out->slots = P.N;
+    out->sz_stride = P.st_Np;
+    out->mask_stride = P.st_mask_stride;
+    out->ring_rows = P.st_H;
+    out->units = P.units;
     out->fill = ctx->layers[layer].fill;
     return VASE_OK;
 }
@@ -1312,6 +1491,10 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
     const char* why = nullptr;
     if (!make_plan(cfg, num_sms, &P, &why)) return cfg->head_dim != 128 ? VASE_ERR_UNSUPPORTED : VASE_ERR_INVALID;
     const vase_config& c = *cfg;
+    if (P.store) {
+        g_config_error = "the static-scratch eviction works on the bf16 value cache (value_bits = 0)";
+        return VASE_ERR_UNSUPPORTED;
+    }
     if (layer < 0 || layer >= c.num_layers) {
         g_config_error = "layer out of range";
         return VASE_ERR_INVALID;
@@ -1413,7 +1596,7 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
             return VASE_ERR_CUDA;
         }
     } else {
-        DkvParams dp;
+        DkvParams dp{};
         dp.batch = batch;
         dp.N = P.N;
         dp.K = c.budget_k;
@@ -1435,7 +1618,7 @@ extern "C" int vase_evict_static_scratch(const vase_config* cfg, const vase_buff
             return VASE_ERR_CUDA;
         }
     }
-    SelectParams sel;
+    SelectParams sel{};  // value-initialised: a field this path does not set is zero (pointers null)
     sel.batch = batch;
     sel.attn = attn;
     sel.dkv = dkv;

@@ -103,7 +103,7 @@ int mixed_cluster(int Gp, int bits, size_t smem, int units, int n_chunks) {
 
 }  // namespace
 
-// Returns cudaErrorInvalidValue when the unit's masks exceed kDecodeMaxMaskWords (K above 16384) or G > 8.
+// Returns cudaErrorInvalidValue when the unit's masks exceed kDecodeMaxMaskWords (more than 17408 slots) or G > 8.
 cudaError_t launch_decode_mixed(DecodeParams p, int num_sms, cudaStream_t s) {
     (void)num_sms;
     if (p.G > 8 || p.mask_words > kDecodeMaxMaskWords) return cudaErrorInvalidValue;

@@ -143,6 +143,7 @@ __global__ void __launch_bounds__(kThreads) decode_simt_kernel(const DecodeParam
         return c < p.mask_words ? mask_s[c] & low_mask(rq) : 0u;
     };
     int pre_val = 0, pre_upto = 0;  // producer: reserved rows of the unit before chunk pre_upto
+    int ring_head = 0;              // producer: compressed value store, the ring row of the unit's first bf16 value
     auto issue_bf16 = [&](int j) {
         const int s = j % kStages;
         const int c = rank + j * C;
@@ -157,9 +158,17 @@ __global__ void __launch_bounds__(kThreads) decode_simt_kernel(const DecodeParam
         }
         uint8_t* vdst = stage + s * kStageBytes + kChunkBytes;
         mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(n_res + rows - rq) * kRowBytes);
-        if (n_res > 0)
-            bulk_load(vdst, p.hp_rows + (static_cast<int64_t>(unit) * p.hp_cap + pre_val) * kVecPerRow,
-                      static_cast<uint32_t>(n_res) * kRowBytes, &full[s]);
+        if (n_res > 0) {
+            // the chunk's bf16 rows follow each other in the reserved cache; in the store's ring they may wrap
+            int at = pre_val + ring_head;
+            if (at >= p.hp_cap) at -= p.hp_cap;
+            const int first = min(n_res, p.hp_cap - at);
+            const int64_t row0 = static_cast<int64_t>(unit) * p.hp_cap;
+            bulk_load(vdst, p.hp_rows + (row0 + at) * kVecPerRow, static_cast<uint32_t>(first) * kRowBytes, &full[s]);
+            if (n_res > first)
+                bulk_load(vdst + first * kRowBytes, p.hp_rows + row0 * kVecPerRow,
+                          static_cast<uint32_t>(n_res - first) * kRowBytes, &full[s]);
+        }
         if (rows > rq)
             bulk_load(vdst + rq * kRowBytes, p.vc + (unit_row + s0 + rq) * kVecPerRow,
                       static_cast<uint32_t>(rows - rq) * kRowBytes, &full[s]);
@@ -231,6 +240,13 @@ __global__ void __launch_bounds__(kThreads) decode_simt_kernel(const DecodeParam
     if (warp == kConsumerWarps) {
         // ---- producer: the rest of the ring's chunks as the consumers free their stages
         if (lane == 0) {
+            if (kBits > 0 && p.ring_state) {
+                ring_head = p.ring_state[4 * unit];
+                if (ring_head < 0 || ring_head >= p.hp_cap) {  // not a state the store kernels wrote
+                    record_error(p.err, kErrDecodeMask);
+                    ring_head = 0;
+                }
+            }
             if (kBits > 0)
                 for (int j = 0; j < min(kStages, n_mine); ++j) issue_bf16(j);
             int issued = min(kStages, n_mine);

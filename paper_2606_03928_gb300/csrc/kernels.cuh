@@ -31,6 +31,8 @@ enum ErrSite : uint32_t {
     kErrSmallKFull = 65,
     kErrSmallKFree = 66,
     kErrSmallDone = 67,
+    kErrStoreOverflow = 80,  // VASE_SITE_STORE_OVERFLOW: an append would overflow the ring after an eviction
+    kErrStoreState = 81,     // VASE_SITE_STORE_STATE: ring state or masks out of range (a store not written here)
 };
 
 constexpr int kTileTokens = 128;   // tokens per MMA tile (M)
@@ -162,6 +164,7 @@ struct SelectParams {
     uint4* vc;              // V rows
     float* vscore_dbg;      // nullable, [slot][units][N]: the value magnitudes of this eviction
     int32_t* src;           // [slot][units][K]
+    uint8_t* resv;          // nullable, [slot][units][store_resv_stride(K)]: 1 = new slot j is in R_V u R_B (store)
     float* pooled_dbg;      // nullable, [slot][units][N]
     float* key_dbg;         // nullable
     uint8_t* keep_dbg;      // nullable
@@ -222,7 +225,36 @@ struct DecodeParams {
     const float* qparams;   // [units][Kp][2]
     const uint32_t* rmask;  // [units][mask_words]
     const uint4* hp_rows;   // [units][hp_cap][16]: the reserved rows below Kq in slot order
+    // compressed value store: hp_rows is a ring, its entry i at row (head + i) mod hp_cap, head = ring_state[4 u]
+    const int32_t* ring_state;  // nullable, [units][4]
     int32_t bits, code_row, Kq, Kp, mask_words, hp_cap;
+};
+
+// Bytes per unit of the selection's R_V u R_B flags (K rounded up to 16: whole 16-byte copies per unit).
+__host__ __device__ inline int store_resv_stride(int K) { return (K + 15) & ~15; }
+
+// Compressed value store of every layer (the mixed-precision cache Sec. 6 proposes): per layer and unit the
+// b-bit codes and (s, z) of every slot, one bit per slot set where the value is held in bf16, the ring of H bf16
+// rows holding those values in slot order, and (head, count) of the ring.
+struct StoreParams {
+    uint8_t* base;          // the store (the V buffer in this mode)
+    int64_t layer_bytes;    // bytes per layer
+    int64_t codes_off, qp_off, mask_off, ring_off, state_off;  // sub-arrays within a layer
+    int32_t units, N, Np, mask_stride, mask_words, H, bits, code_row, K, b, Hkv;
+    int32_t layer[kMaxLayerBatch];
+    int32_t fill[kMaxLayerBatch];   // append: fill before the call
+    int32_t round[kMaxLayerBatch];  // append: evictions so far
+    // append: value rows [slot][n][b][Hkv][16], layer slots kv_stride vectors apart
+    const uint4* v;
+    int64_t kv_stride;
+    int32_t n;
+    int32_t big;            // 1: the ring may overflow (a first fill past H): the launch carries the overflow's memory
+    int32_t n_v;            // N_v: the large-Range values the overflow keeps
+    const float* vmag;      // base of [L][units][N]: value magnitudes (appended rows included)
+    // eviction: the selection's kept list ([slot][units][K]) and R_V u R_B flags ([slot][units][resv stride])
+    const int32_t* src;
+    const uint8_t* resv;
+    uint32_t* err;
 };
 
 // ------------------------------------------------------------------ launchers (return cudaError_t)
@@ -239,6 +271,11 @@ cudaError_t evict_small_set_attributes(size_t smem_bytes);
 cudaError_t launch_evict_small(const CUtensorMap& kmap, const CUtensorMap& qmap, const SmallEvictParams& p, int units,
                                size_t smem_bytes, cudaStream_t s);
 cudaError_t launch_quantize(const QuantParams& p, int units, size_t smem_bytes, cudaStream_t s);
+cudaError_t launch_store_append(const StoreParams& p, int n_layers, cudaStream_t s);
+cudaError_t launch_store_evict(const StoreParams& p, int n_layers, cudaStream_t s);
+size_t store_evict_smem_bytes(int K, int mask_stride);
+size_t store_append_smem_bytes(int mask_stride, int H, int n, int K, bool big);
+cudaError_t store_set_attributes(size_t evict_smem, size_t append_smem);
 size_t quantize_smem_bytes(int K, int B);
 cudaError_t quantize_set_attributes(size_t smem_bytes);
 cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, DecodeParams p, size_t smem_bytes,
@@ -256,6 +293,6 @@ cudaError_t decode_set_attributes(int G, size_t smem_bytes);
 size_t decode_mixed_smem_bytes(int G, int bits, int mask_words);
 cudaError_t decode_mixed_set_attributes();
 cudaError_t launch_decode_mixed(DecodeParams p, int num_sms, cudaStream_t s);
-constexpr int kDecodeMaxMaskWords = 512;  // reserved-slot mask words of a unit the mixed-precision decode holds
+constexpr int kDecodeMaxMaskWords = 544;  // reserved-slot mask words of a unit the mixed-precision decode holds
 
 }  // namespace vase

@@ -6,6 +6,7 @@
 
 #include "kernels.cuh"
 #include "ptx.cuh"
+#include "quant.cuh"
 
 namespace vase {
 
@@ -86,7 +87,7 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
     const int64_t units = static_cast<int64_t>(p.b) * Hkv;
     const int64_t unit0 = static_cast<int64_t>(layer) * units + static_cast<int64_t>(s) * Hkv;  // unit of head 0
     uint4* const kc = p.kc + unit0 * N * kVecPerRow;
-    uint4* const vc = p.vc + unit0 * N * kVecPerRow;
+    uint4* const vc = p.vc ? p.vc + unit0 * N * kVecPerRow : nullptr;  // null: the values go to the compressed store
     int32_t* const pos = p.pos + unit0 * N;
     float* const vmag = p.vmag + unit0 * N;
     uint4* const qwin = p.qwin + (static_cast<int64_t>(layer) * p.b + s) * Hq * W * kVecPerRow;
@@ -112,7 +113,7 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendParams p) {
                 } else if (r < 2 * Hkv) {
                     is_v = true;
                     val = vin[(row_in * Hkv + (r - Hkv)) * kVecPerRow + seg];
-                    vc[(static_cast<int64_t>(r - Hkv) * N + fill + t) * kVecPerRow + seg] = val;
+                    if (vc) vc[(static_cast<int64_t>(r - Hkv) * N + fill + t) * kVecPerRow + seg] = val;
                 } else {
                     const int hq = r - 2 * Hkv;
                     qwin[(static_cast<int64_t>(hq) * W + slot) * kVecPerRow + seg] =
@@ -488,6 +489,7 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
     float* const vmag = p.vmag + static_cast<int64_t>(layer) * p.units * N;
     float* const vscore_dbg = p.vscore_dbg ? p.vscore_dbg + zs : nullptr;
     int32_t* const src_out = p.src + static_cast<int64_t>(z) * p.units * K;
+    uint8_t* const resv_out = p.resv ? p.resv + static_cast<int64_t>(z) * p.units * store_resv_stride(K) : nullptr;
     float* const pooled_dbg = p.pooled_dbg ? p.pooled_dbg + zs : nullptr;
     float* const key_dbg = p.key_dbg ? p.key_dbg + zs : nullptr;
     uint8_t* const keep_dbg = p.keep_dbg ? p.keep_dbg + zs : nullptr;
@@ -617,6 +619,9 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
                 src_out[static_cast<int64_t>(unit) * K + dst] = i;
                 src_s[dst] = i;
                 pos[base + dst] = pos_s[i];
+                // compressed value store: new slot dst keeps a reserved (bf16) value if it is in R_B or R_V
+                if (resv_out)
+                    resv_out[static_cast<int64_t>(unit) * store_resv_stride(K) + dst] = (i >= K || (flags[i] & kFlagValue)) ? 1 : 0;
             }
             ++dst;
         } else if (i < first_ev) {
@@ -692,7 +697,7 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     const int warp = tid >> 5;
-    if (warp < 2) {
+    if (warp == 0 || (warp == 1 && p.vc)) {  // no V rows here with the compressed value store
         const int64_t unit_row = (static_cast<int64_t>(layer) * p.units + unit) * N;
         uint8_t* const rows = reinterpret_cast<uint8_t*>((warp == 0 ? p.kc : p.vc) + unit_row * kVecPerRow);
         gather_rows(rows, src_s, sh.first_evicted, K, smem_raw + warp * Ly.gather_stages * kGatherChunkBytes,
@@ -1038,37 +1043,11 @@ __global__ void __launch_bounds__(kSelThreads) quantize_kernel(const QuantParams
         const uint2 row = reinterpret_cast<const uint2*>(p.vc + (base + j) * kVecPerRow)[lane];
         reinterpret_cast<uint2*>(p.hp_rows + (static_cast<int64_t>(unit) * p.hp_cap + idx) * kVecPerRow)[lane] = row;
     }
-    const float levels = static_cast<float>((1 << p.bits) - 1);
-    const int code_bytes = p.bits / 2;  // bytes of one lane's four codes
     for (int j = warp; j < C; j += kSelWarps) {
         if (flags[j]) continue;  // R_V keeps its bf16 row (uniform over the warp)
         const uint2 raw = reinterpret_cast<const uint2*>(p.vc + (base + j) * kVecPerRow)[lane];
-        const float v[4] = {__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xFFFF0000u),
-                            __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xFFFF0000u)};
-        float lo = fminf(fminf(v[0], v[1]), fminf(v[2], v[3]));
-        float hi = fmaxf(fmaxf(v[0], v[1]), fmaxf(v[2], v[3]));
-#pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) {
-            lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-            hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-        }
-        const float s = __fdiv_rn(__fsub_rn(hi, lo), levels);
-        uint32_t packed = 0;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float t = s > 0.f ? rintf(__fdiv_rn(__fsub_rn(v[e], lo), s)) : 0.f;
-            const uint32_t c = static_cast<uint32_t>(fminf(fmaxf(t, 0.f), levels));
-            packed |= c << (e * p.bits);
-        }
-        uint8_t* dst = p.codes + (static_cast<int64_t>(unit) * K + j) * p.row_bytes + lane * code_bytes;
-        if (code_bytes == 4) *reinterpret_cast<uint32_t*>(dst) = packed;
-        else if (code_bytes == 2) *reinterpret_cast<uint16_t*>(dst) = static_cast<uint16_t>(packed);
-        else *dst = static_cast<uint8_t>(packed);
-        if (lane == 0) {
-            float* qp = p.qparams + (static_cast<int64_t>(unit) * p.Kp + j) * 2;
-            qp[0] = s;
-            qp[1] = lo;
-        }
+        quantize_row_warp(raw, p.bits, lane, p.codes + (static_cast<int64_t>(unit) * K + j) * p.row_bytes,
+                          p.qparams + (static_cast<int64_t>(unit) * p.Kp + j) * 2);
     }
 }
 

@@ -27,6 +27,7 @@ VASE_ERR_UNSUPPORTED = -5
 VASE_ERR_ALIGN = -6
 VASE_ERR_DEVICE = -7
 VASE_SITE_SELF_TEST = 127  # error-word site of vase_self_test_wait_timeout
+VASE_SITE_STORE_OVERFLOW, VASE_SITE_STORE_STATE = 80, 81  # error-word sites of the compressed value store
 
 VASE_VARIANT_ATTNV = 0
 VASE_VARIANT_DKV = 1
@@ -42,15 +43,18 @@ EXPORTED = [
     "vase_append_all", "vase_append_all_strided", "vase_evict_all", "vase_self_test_wait_timeout", "vase_refresh_value_scores", "vase_evict_static_scratch",
     "vase_decode_attention", "vase_mixed_buffer_sizes", "vase_quantize_values", "vase_decode_attention_mixed",
     "vase_host_staging_bytes", "vase_stage_host_inputs", "vase_append_all_staged", "vase_read_positions_all",
+    "vase_value_store_get",
 ]
-KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "evict_small"]
+KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "evict_small", "store_append",
+                "store_evict"]
 
 
 class vase_config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "budget_k", "buffer_b", "window", "num_q_heads", "num_kv_heads", "head_dim", "num_layers", "batch",
         "variant", "n_v", "value_score", "pool_kernel", "dkv_rank", "stochastic", "dkv_fixed_g", "debug_outputs")] + [
-        ("seed", ctypes.c_uint64)] + [(n, ctypes.c_int32) for n in ("reserve_kind", "gqa_reduce", "dkv_shared_g")]
+        ("seed", ctypes.c_uint64)] + [(n, ctypes.c_int32) for n in ("reserve_kind", "gqa_reduce", "dkv_shared_g",
+                                                                     "value_bits")]
 
 
 class vase_buffer_sizes(ctypes.Structure):
@@ -77,6 +81,12 @@ class vase_kv_view(ctypes.Structure):
 class vase_mixed_buffers(ctypes.Structure):
     _fields_ = [("codes", ctypes.c_void_p), ("qparams", ctypes.c_void_p), ("rmask", ctypes.c_void_p),
                 ("hp_rows", ctypes.c_void_p)]
+
+
+class vase_value_store(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("codes", "sz", "mask", "ring", "state")] + [
+        (n, ctypes.c_int32) for n in ("bits", "code_row", "slots", "sz_stride", "mask_stride", "ring_rows", "units",
+                                      "fill")]
 
 
 class vase_debug_view(ctypes.Structure):
@@ -126,6 +136,7 @@ def load(path: str = LIB_PATH):
         "vase_set_layer_state": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_layer_state)]),
         "vase_kv_view_get": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_kv_view)]),
         "vase_debug_view_get": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_debug_view)]),
+        "vase_value_store_get": (ctypes.c_int, [P, I32, ctypes.POINTER(vase_value_store)]),
         "vase_check_device_error": (ctypes.c_int, [P, P, ctypes.POINTER(U32)]),
         "vase_launch_count": (I64, [P]),
         "vase_status_string": (ctypes.c_char_p, [ctypes.c_int]),
@@ -342,7 +353,7 @@ class VaseCache:
 
     def __init__(self, geometry: Geometry, *, variant="attnv", n_v=-1, value_score=VASE_VALUE_RANGE,
                  pool_kernel=7, dkv_rank=20, stochastic=True, dkv_fixed_g=False, debug_outputs=False, seed=0,
-                 reserve="value", gqa="mean", dkv_shared_g=False, device=None):
+                 reserve="value", gqa="mean", dkv_shared_g=False, value_bits=0, device=None):
         g = geometry
         self.geometry = g
         self.cfg = vase_config_default(
@@ -352,7 +363,8 @@ class VaseCache:
             value_score=value_score, pool_kernel=pool_kernel, dkv_rank=dkv_rank, stochastic=int(stochastic),
             dkv_fixed_g=int(dkv_fixed_g), debug_outputs=int(debug_outputs), seed=seed,
             reserve_kind={"value": VASE_RESERVE_VALUE, "random": VASE_RESERVE_RANDOM}[reserve],
-            gqa_reduce={"mean": VASE_GQA_MEAN, "max": VASE_GQA_MAX}[gqa], dkv_shared_g=int(dkv_shared_g))
+            gqa_reduce={"mean": VASE_GQA_MEAN, "max": VASE_GQA_MAX}[gqa], dkv_shared_g=int(dkv_shared_g),
+            value_bits=int(value_bits))
         sizes = vase_get_buffer_sizes(self.cfg)
         dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
         self.device = dev
@@ -360,7 +372,10 @@ class VaseCache:
         self.slots = N
         self.k_cache = torch.empty((g.num_layers, g.batch, g.num_kv_heads, N, g.head_dim), dtype=torch.bfloat16,
                                    device=dev)
-        self.v_cache = torch.empty_like(self.k_cache)
+        # the bf16 value cache, or (value_bits > 0) the compressed value store the library lays out itself
+        self.v_cache = (torch.empty(sizes.v_cache, dtype=torch.uint8, device=dev) if value_bits
+                        else torch.empty_like(self.k_cache))
+        self.value_bits = int(value_bits)
         self.q_window = torch.empty((g.num_layers, g.batch, g.num_q_heads, g.window, g.head_dim),
                                     dtype=torch.bfloat16, device=dev)
         self.positions = torch.full((g.num_layers, g.batch, g.num_kv_heads, N), -1, dtype=torch.int32, device=dev)
@@ -495,6 +510,28 @@ class VaseCache:
 
     def profile_collect(self):
         return vase_profile_collect(self.ctx)
+
+    def value_store(self, layer):
+        """One layer's compressed value store as torch views: codes [units, N, code_row] uint8, sz [units, Np, 2]
+        fp32, mask [units, mask_stride] int32, ring [units, H, d] bf16, state [units, 4] int32 (ring head, count)."""
+        vs = vase_value_store()
+        _check(self.ctx, load().vase_value_store_get(self.ctx, layer, ctypes.byref(vs)), "vase_value_store_get")
+        base = self.v_cache.data_ptr()
+        U = vs.units
+
+        def sl(ptr, nbytes, dtype):
+            off = ptr - base
+            return self.v_cache[off:off + nbytes].view(dtype)
+
+        d = self.geometry.head_dim
+        return {
+            "codes": sl(vs.codes, U * vs.slots * vs.code_row, torch.uint8).view(U, vs.slots, vs.code_row),
+            "sz": sl(vs.sz, U * vs.sz_stride * 8, torch.float32).view(U, vs.sz_stride, 2),
+            "mask": sl(vs.mask, U * vs.mask_stride * 4, torch.int32).view(U, vs.mask_stride),
+            "ring": sl(vs.ring, U * vs.ring_rows * d * 2, torch.bfloat16).view(U, vs.ring_rows, d),
+            "state": sl(vs.state, U * 16, torch.int32).view(U, 4),
+            "bits": vs.bits, "ring_rows": vs.ring_rows, "fill": vs.fill,
+        }
 
     def debug_view(self, slot=0):
         """Workspace results of the latest eviction call for its slot-th layer: attn, pooled, value_score, key

@@ -47,6 +47,7 @@ def test_struct_layouts_match_ctypes(lib):
     structs = {
         "vase_config": V.vase_config, "vase_buffer_sizes": V.vase_buffer_sizes, "vase_buffers": V.vase_buffers,
         "vase_layer_state": V.vase_layer_state, "vase_kv_view": V.vase_kv_view, "vase_debug_view": V.vase_debug_view,
+        "vase_mixed_buffers": V.vase_mixed_buffers, "vase_value_store": V.vase_value_store,
     }
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "vase.h"', "int main(void) {"]
     for name, cls in structs.items():
@@ -81,6 +82,26 @@ def test_config_validation_without_a_gpu(lib):
             V.vase_get_buffer_sizes(cfg)
 
 
+def test_value_store_configuration_without_a_gpu(lib):
+    """The compressed value store: bit widths 2, 4, 8 only, AttnV only; its V buffer is the layout of codes,
+    (s, z), masks, ring (N_v + 2B rows) and ring state per unit, smaller than the bf16 cache it replaces
+    (Qwen3-1.7B geometry, one layer, K 2048, B 128, N_v 512)."""
+    from oracle import vase_oracle as O
+    from paper_2606_03928_gb300 import vase as V
+    base = dict(budget_k=2048, buffer_b=128, window=32, num_q_heads=16, num_kv_heads=8, num_layers=1, batch=8)
+    bf = V.vase_get_buffer_sizes(V.vase_config_default(**base)).v_cache
+    units, N, words = 64, 2176, 68
+    for bits in (2, 4, 8):
+        st = V.vase_get_buffer_sizes(V.vase_config_default(value_bits=bits, **base)).v_cache
+        per_unit, bf_unit = O.store_bytes(N, O.store_capacity(2048, 128, 512), 128, bits)
+        assert bf == units * bf_unit
+        exact = units * (per_unit + 4 * words + 16)   # + the mask words and the ring state
+        assert exact <= st < exact + 5 * 256 and st < bf
+    for bad in (dict(value_bits=3), dict(value_bits=16), dict(value_bits=4, variant=V.VASE_VARIANT_DKV)):
+        with pytest.raises(V.VaseError):
+            V.vase_get_buffer_sizes(V.vase_config_default(**{**base, **bad}))
+
+
 def test_paper_defaults(lib):
     from paper_2606_03928_gb300 import vase as V
     c = V.vase_config_default()
@@ -89,4 +110,4 @@ def test_paper_defaults(lib):
 
 def test_status_strings(lib):
     assert lib.vase_status_string(-3) == b"cache not full"
-    assert lib.vase_abi_version() == 2
+    assert lib.vase_abi_version() == 3

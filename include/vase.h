@@ -225,10 +225,10 @@ int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream);
  * The caller owns q and out; the call uses no workspace (the slots of each KV head are split
  * over the CTAs of one thread-block cluster, whose states are folded in shared memory), so
  * calls may overlap with each other but not with an append or eviction of the same layer.
- * With the compressed value store (value_bits > 0) the values are read from it: bf16 rows from the
- * reserved ring, every other value as Q s + z from its codes (CUDA cores, at most 8 query heads per KV head).
+ * With the compressed value store (value_bits > 0) the values are read from it on the tensor cores: bf16 rows
+ * from the reserved ring, every other value as Q s + z from its codes.
  * Errors: VASE_ERR_INVALID (bad layer, null pointer, empty layer), VASE_ERR_ALIGN,
- * VASE_ERR_UNSUPPORTED (more than 16 query heads per KV head; more than 8 with the store). */
+ * VASE_ERR_UNSUPPORTED (more than 16 query heads per KV head). */
 int vase_decode_attention(vase_ctx* ctx, int32_t layer, const void* q, float* out, void* stream);
 
 /* ---- Mixed-precision values: the b-bit per-token quantizer of Sec. 4.4 and the reserved cache of Sec. 6.

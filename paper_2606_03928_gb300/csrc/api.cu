@@ -257,7 +257,7 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     p.off_staging = o;
     p.staging_bytes = static_cast<size_t>(c->buffer_b) * c->batch * (c->num_q_heads + 2 * c->num_kv_heads) * kRowBytes;
     o = align_up(o + p.staging_bytes, kAlign);
-    p.decode_smem = decode_smem_bytes(p.G);
+    p.decode_smem = decode_smem_bytes(p.G, c->value_bits != 0);
     p.ws_bytes = o;
     // fused small-unit eviction: AttnV, at most 128 window rows, every 128-token tile's S = K Q^T resident in TMEM
     p.small_tiles = p.n_tiles;
@@ -594,7 +594,7 @@ int vase_create(const vase_config* cfg, const vase_buffers* bufs, vase_ctx** out
     if ((e = score_attn_set_attributes(P.score_smem, P.cluster)) != cudaSuccess ||
         (e = dkv_set_attributes(P.dkv_smem)) != cudaSuccess ||
         (e = select_set_attributes(P.select_smem)) != cudaSuccess ||
-        (e = decode_set_attributes(P.G, P.decode_smem)) != cudaSuccess ||
+        (e = decode_set_attributes(P.G, P.decode_smem, P.store)) != cudaSuccess ||
         (e = decode_mixed_set_attributes()) != cudaSuccess ||
         (e = quantize_set_attributes(quantize_smem_bytes(cfg->budget_k, cfg->buffer_b))) != cudaSuccess ||
         (P.small_ok && (e = evict_small_set_attributes(P.small_smem)) != cudaSuccess) ||
@@ -980,7 +980,7 @@ namespace {
 // every slot, the ring of bf16 rows and its head).
 int decode_store(vase_ctx* ctx, int32_t layer, const void* q, float* out, cudaStream_t stream) {
     const Plan& P = ctx->plan;
-    if (P.G > 8) return fail(ctx, VASE_ERR_UNSUPPORTED, "decode over the compressed value store handles at most 8 query heads per KV head");
+    if (P.G > 16) return fail(ctx, VASE_ERR_UNSUPPORTED, "decode handles at most 16 query heads per KV head");
     uint8_t* base = static_cast<uint8_t*>(ctx->bufs.v_cache) + static_cast<size_t>(layer) * P.st_layer_bytes;
     DecodeParams dp{};
     dp.q = static_cast<const uint4*>(q);
@@ -1006,7 +1006,8 @@ int decode_store(vase_ctx* ctx, int32_t layer, const void* q, float* out, cudaSt
     dp.Kp = P.st_Np;
     dp.mask_words = P.st_mask_stride;
     dp.hp_cap = P.st_H;
-    cudaError_t e = launch_decode_mixed(dp, P.num_sms, stream);
+    // the tensor-core kernel, its V tiles written from the ring rows and the codes by builder warps
+    cudaError_t e = launch_decode(ctx->kmap_dec, ctx->vmap_dec, dp, P.decode_smem, P.num_sms, stream);
     if (e == cudaErrorInvalidValue) return fail(ctx, VASE_ERR_UNSUPPORTED, "too many slots for the mixed decode");
     if (e != cudaSuccess) return cuda_fail(ctx, e, "value store decode attention launch");
     ctx->launches += 1;

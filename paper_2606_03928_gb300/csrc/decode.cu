@@ -55,8 +55,13 @@ constexpr int kChunk = kDecodeTileRows;  // 64 slots: the M of the score MMA
 constexpr int kStages = 3;
 constexpr int kSoftWarps = 4;
 constexpr int kThreads = 32 * (2 + kSoftWarps);
+constexpr int kBuildWarps = 4;                             // store: the warps that write the V tiles
+constexpr int kThreadsStore = kThreads + 32 * kBuildWarps;
 constexpr uint32_t kBoxBytes = kChunk * 128;          // 64 rows x 64 dims bf16 (one TMA box)
 constexpr uint32_t kStageBytes = 4 * kBoxBytes;       // K dims 0-63, K dims 64-127, V dims 0-63, V dims 64-127
+// With the compressed value store the V tile of a stage is written by builder warps straight from the store (a
+// bf16 slot's row from the ring, a coded slot's codes expanded), so a stage has the same size in both forms.
+__host__ __device__ constexpr uint32_t stage_bytes_of(bool) { return kStageBytes; }
 constexpr int kNS = 16;                               // score columns (query heads, padded)
 constexpr float kLazyMax = 8.f;                       // log2 units
 
@@ -65,25 +70,28 @@ struct DecodeSmem {
     uint32_t q_off;      // Q as the score MMA's B operand: 2 panels x 16 rows x 128 B (K-major, 128-byte swizzle)
     uint32_t p_off;      // 2 buffers x NP rows x 128 B: P^T as the output MMA's B operand (K-major over slots)
     uint32_t red_off;    // [2][kSoftWarps][16] chunk maxima, [2][kSoftWarps] status flags (padded to 16),
-                         // [kSoftWarps][16] sums
+                         // [kSoftWarps][16] sums, [kSoftWarps][16] bias sums (store)
+    uint32_t mask_off;   // store: the unit's bf16 masks [kDecodeMaxMaskWords]
     uint32_t bar_off;
     uint32_t total;      // bytes from the 1024-aligned base
 };
 
-__host__ __device__ inline DecodeSmem decode_layout(int NP) {
+__host__ __device__ inline DecodeSmem decode_layout(int NP, bool store = false) {
     DecodeSmem L;
     uint32_t o = 0;
     L.stage_off = o;
-    o += kStages * kStageBytes;
+    o += kStages * stage_bytes_of(store);
     L.q_off = o;
     o += 2 * kNS * 128;
     L.p_off = o;
     o += 2u * NP * 128;
     L.red_off = o;
-    o += 4u * (3 * kSoftWarps * kNS + 16);
+    o += 4u * (4 * kSoftWarps * kNS + 16);
+    L.mask_off = o;
+    o += store ? 4u * kDecodeMaxMaskWords : 0u;
     L.bar_off = o;
-    o += 8u * (2 * kStages + 9) + 16;  // full, empty (x kStages), s_full, s_empty, p_full, o_full (x2), mma_done,
-                                       // TMEM slot
+    o += 8u * (3 * kStages + 9) + 16;  // full, empty, v_full (x kStages), s_full, s_empty, p_full, o_full (x2),
+                                       // mma_done, TMEM slot
     L.total = (o + 15u) & ~15u;
     return L;
 }
@@ -122,27 +130,50 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// The codes of dims 8q .. 8q+7 of a half row (kBits-bit fields, dim i at bit i*kBits of the little-endian words
+// cw) as eight bf16 values: the integers themselves (exact in bf16: their fp32 bits' top half).
+template <int kBits>
+__device__ __forceinline__ uint4 expand8(const uint32_t* cw, int q) {
+    uint32_t w[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const int b0 = (8 * q + 2 * e) * kBits, b1 = b0 + kBits;
+        const uint32_t c0 = (cw[b0 >> 5] >> (b0 & 31)) & ((1u << kBits) - 1u);
+        const uint32_t c1 = (cw[b1 >> 5] >> (b1 & 31)) & ((1u << kBits) - 1u);
+        w[e] = (__float_as_uint(static_cast<float>(c0)) >> 16) | (__float_as_uint(static_cast<float>(c1)) & 0xFFFF0000u);
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 // Byte offset of bf16 element (row, col) in a K-major panel of 128-byte rows with the 128-byte swizzle.
 __device__ __forceinline__ uint32_t sw128_offset(int row, int col) {
     return static_cast<uint32_t>(row * 128 + ((((col >> 3) ^ (row & 7)) & 7) << 4) + ((col & 7) << 1));
 }
 
-template <int NP>
-__global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_constant__ CUtensorMap kmap,
+// kStore: the values come from the compressed value store.  Four more warps (builders) write each stage's V
+// tile from the store, in the layout TMA gives the bf16 form (rows of 64 dims, 128-byte swizzle): a bf16 slot's
+// row read from the ring, a coded slot's row as its codes (integers, exact in bf16); they reuse a stage once its
+// output MMA has read it (empty) and signal v_full.  A coded slot's weight in P is p s and its p z joins a
+// per-head bias: o = sum p v' = sum (p s) Q + sum p z.
+template <int NP, bool kStore>
+__global__ void __launch_bounds__(kStore ? kThreadsStore : kThreads) decode_tc_kernel(const __grid_constant__ CUtensorMap kmap,
                                                                const __grid_constant__ CUtensorMap vmap,
                                                                const DecodeParams p) {
     constexpr int GH = NP / 2;  // query heads the instantiation handles
     constexpr uint32_t kTmemCols = NP == 16 ? 64 : 128;
+    constexpr uint32_t kSB = stage_bytes_of(kStore);
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const DecodeSmem Ly = decode_layout(NP);
+    const DecodeSmem Ly = decode_layout(NP, kStore);
+    uint32_t* mask_s = reinterpret_cast<uint32_t*>(smem + Ly.mask_off);
     uint8_t* stage = smem + Ly.stage_off;
     uint8_t* q_s = smem + Ly.q_off;
     uint8_t* p_s = smem + Ly.p_off;
     float* red = reinterpret_cast<float*>(smem + Ly.red_off);
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + Ly.bar_off);
     uint64_t* empty = full + kStages;
-    uint64_t* s_full = empty + kStages;
+    uint64_t* v_full = empty + kStages;  // store: the builders have written the stage's V tile
+    uint64_t* s_full = v_full + kStages;
     uint64_t* s_empty = s_full + 2;
     uint64_t* p_full = s_empty + 2;
     uint64_t* o_full = p_full + 2;
@@ -166,6 +197,7 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
+            mbar_init(&v_full[s], kBuildWarps);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
@@ -183,9 +215,10 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
             asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.kc + (unit_row + s0) * kVecPerRow),
                          "r"(bytes)
                          : "memory");
-            asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.vc + (unit_row + s0) * kVecPerRow),
-                         "r"(bytes)
-                         : "memory");
+            if (!kStore)
+                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p.vc + (unit_row + s0) * kVecPerRow),
+                             "r"(bytes)
+                             : "memory");
         }
     }
     if (warp == 1) {
@@ -193,15 +226,41 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
         tmem_relinquish();
     }
     asm volatile("griddepcontrol.wait;" ::: "memory");  // query and cache rows of preceding kernels are visible
-    auto load_chunk = [&](int j) {  // chunk j of this CTA into stage j % kStages
+    // store: the unit's bf16 masks and the ring row of its first bf16 value
+    int ring_head = 0;
+    if (kStore) {
+        for (int w = tid; w < p.mask_words; w += kThreadsStore) mask_s[w] = p.rmask[static_cast<int64_t>(unit) * p.mask_words + w];
+        ring_head = p.ring_state[4 * unit];
+        if (ring_head < 0 || ring_head >= p.hp_cap) {  // not a state the store kernels wrote
+            if (tid == 0) record_error(p.err, kErrDecodeMask);
+            ring_head = 0;
+        }
+        __syncthreads();
+    }
+    // bf16 mask of a chunk's slots (store), limited to its filled rows
+    auto chunk_bf16 = [&](int c, int rows) -> uint64_t {
+        const uint32_t w0 = 2 * c < p.mask_words ? mask_s[2 * c] : 0u;
+        const uint32_t w1 = 2 * c + 1 < p.mask_words ? mask_s[2 * c + 1] : 0u;
+        const uint64_t m = static_cast<uint64_t>(w0) | static_cast<uint64_t>(w1) << 32;
+        return rows >= 64 ? m : m & ((1ull << rows) - 1ull);
+    };
+    // chunk j of this CTA into stage j % kStages
+    auto load_chunk = [&](int j) {
         const int s = j % kStages;
-        const int32_t y = p.row_base + static_cast<int32_t>(unit_row) + (rank + j * C) * kChunk;
-        uint8_t* st = stage + s * kStageBytes;
-        mbar_arrive_expect_tx(&full[s], kStageBytes);
+        const int c = rank + j * C;
+        const int32_t y = p.row_base + static_cast<int32_t>(unit_row) + c * kChunk;
+        uint8_t* st = stage + s * kSB;
+        if (!kStore) {
+            mbar_arrive_expect_tx(&full[s], kStageBytes);
+            tma_load_2d(st, &kmap, 0, y, &full[s]);
+            tma_load_2d(st + kBoxBytes, &kmap, 64, y, &full[s]);
+            tma_load_2d(st + 2 * kBoxBytes, &vmap, 0, y, &full[s]);
+            tma_load_2d(st + 3 * kBoxBytes, &vmap, 64, y, &full[s]);
+            return;
+        }
+        mbar_arrive_expect_tx(&full[s], 2 * kBoxBytes);  // K only: the builders write the V tile
         tma_load_2d(st, &kmap, 0, y, &full[s]);
         tma_load_2d(st + kBoxBytes, &kmap, 64, y, &full[s]);
-        tma_load_2d(st + 2 * kBoxBytes, &vmap, 0, y, &full[s]);
-        tma_load_2d(st + 3 * kBoxBytes, &vmap, 64, y, &full[s]);
     };
     if (tid == 0)
         for (int j = 0; j < min(kStages, n_mine); ++j) load_chunk(j);  // the ring's first fill, before anything else
@@ -209,7 +268,7 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
     {
         const uint4* qrow =
             p.q + (static_cast<int64_t>(seq) * p.Hkv * G + static_cast<int64_t>(head) * G) * kVecPerRow;
-        for (int i = tid; i < kNS * kVecPerRow; i += kThreads) {
+        for (int i = tid; i < kNS * kVecPerRow; i += (kStore ? kThreadsStore : kThreads)) {
             const int n = i / kVecPerRow;
             const int c = i - n * kVecPerRow;  // 16-byte piece: dims 8c .. 8c+7
             const uint4 v = n < G ? qrow[n * kVecPerRow + c] : make_uint4(0, 0, 0, 0);
@@ -246,8 +305,9 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
             auto issue_o = [&](int jj) -> bool {
                 const int b = jj & 1;
                 if (!mbar_wait(&p_full[b], (jj >> 1) & 1, p.err, kErrDecodeFull)) return false;
+                if (kStore && !mbar_wait(&v_full[jj % kStages], (jj / kStages) & 1, p.err, kErrDecodeFull)) return false;
                 tc_fence_after();
-                const uint32_t v_addr = smem_u32(stage + (jj % kStages) * kStageBytes + 2 * kBoxBytes);
+                const uint32_t v_addr = smem_u32(stage + (jj % kStages) * kSB + 2 * kBoxBytes);
                 const uint32_t p_addr = smem_u32(p_s + b * NP * 128);
 #pragma unroll
                 for (int kk = 0; kk < kChunk / 16; ++kk)
@@ -266,7 +326,7 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
                     break;
                 }
                 tc_fence_after();
-                const uint32_t k_addr = smem_u32(stage + s * kStageBytes);
+                const uint32_t k_addr = smem_u32(stage + s * kSB);
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk)
                     tc_mma_bf16(t_s + b * kNS, sw128_kmajor_desc(k_addr + (kk >> 2) * kBoxBytes + (kk & 3) * 32),
@@ -288,13 +348,15 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
     float acc[GH];            // thread = output dimension 32 qd + lane
     float m_run[GH];
     float l_part[GH];         // this thread's slot share of the sum (threads with lane < 16 own a slot)
+    float b_part[GH];         // store: this thread's slot share of sum p z over coded slots
 #pragma unroll
     for (int g = 0; g < GH; ++g) {
         acc[g] = 0.f;
         m_run[g] = -INFINITY;
         l_part[g] = 0.f;
+        b_part[g] = 0.f;
     }
-    if (warp >= 2) {
+    if (warp >= 2 && warp < 2 + kSoftWarps) {
         const uint32_t lane_base = static_cast<uint32_t>(32 * qd) << 16;
         float alpha_prev[GH];
 #pragma unroll
@@ -323,6 +385,11 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
             const int b = j & 1;
             const int s0 = (rank + j * C) * kChunk;
             const int rows = min(kChunk, p.fill - s0);
+            // store: this slot's (s, z), requested before the wait for the scores so that its latency hides there
+            // (a bf16 slot's pair is read and ignored)
+            float2 szv = make_float2(1.f, 0.f);
+            if (kStore && lane < 16 && slot_l < rows)
+                szv = reinterpret_cast<const float2*>(p.qparams)[static_cast<int64_t>(unit) * p.Kp + s0 + slot_l];
             float sv[16];
             const bool got = ok && mbar_wait(&s_full[b], (j >> 1) & 1, p.err, kErrDecodeFull);
             if (got) {
@@ -365,8 +432,8 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
                 if (raise) m_run[g] = mc;
             }
             // the rows past the unit's fill in a ragged chunk hold stale bytes: zero their V rows (P is 0 there)
-            if (rows < kChunk) {
-                uint8_t* vt = stage + (j % kStages) * kStageBytes + 2 * kBoxBytes;
+            uint8_t* vt = stage + (j % kStages) * kSB + 2 * kBoxBytes;
+            if (!kStore && rows < kChunk) {  // (the store's builders write those rows themselves)
                 for (int i = tid - 64; i < (kChunk - rows) * 16; i += 32 * kSoftWarps) {
                     const int r = rows + (i >> 4);
                     const int c = i & 15;
@@ -374,13 +441,21 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
                         make_uint4(0, 0, 0, 0);
                 }
             }
-            // weights exp2(s - m) <= 2^8 as hi + lo bf16 pairs: P^T rows 2g and 2g + 1, column = slot
+            float sz_s = 1.f, sz_z = 0.f;  // store: (s, z) of this thread's slot if it is coded
+            if (kStore && lane < 16 && slot_l < rows && !((chunk_bf16(rank + j * C, rows) >> slot_l) & 1ull)) {
+                sz_s = szv.x;
+                sz_z = szv.y;
+            }
+            // weights exp2(s - m) <= 2^8 as hi + lo bf16 pairs: P^T rows 2g and 2g + 1, column = slot; a coded
+            // slot's column holds p s and its p z joins the head's bias
             if (lane < 16) {
                 uint8_t* pb = p_s + b * NP * 128;
 #pragma unroll
                 for (int g = 0; g < GH; ++g) {
-                    const float w = g < G ? ex2(sc[g] - m_run[g]) : 0.f;
-                    l_part[g] = fmaf(l_part[g], alpha[g], w);
+                    const float w0 = g < G ? ex2(sc[g] - m_run[g]) : 0.f;
+                    l_part[g] = fmaf(l_part[g], alpha[g], w0);
+                    if (kStore) b_part[g] = fmaf(b_part[g], alpha[g], w0 * sz_z);
+                    const float w = kStore ? w0 * sz_s : w0;
                     const __nv_bfloat16 hi = __float2bfloat16_rn(w);
                     const __nv_bfloat16 lo = __float2bfloat16_rn(w - __bfloat162float(hi));
                     *reinterpret_cast<__nv_bfloat16*>(pb + sw128_offset(2 * g, slot_l)) = hi;
@@ -396,6 +471,69 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
         }
         if (ok && !fold_o(n_mine - 1, alpha_prev)) ok = false;
         tc_fence_before();
+    } else if (kStore && warp >= 2 + kSoftWarps) {
+        // ---- builders (store): the V tile of every chunk of this CTA.  Thread (row r, half) writes dims
+        // 64 half .. 64 half + 63 of slot row r, 16 bytes (8 dims) at a time into the 128-byte swizzled row: a bf16
+        // slot's from its ring row (the k-th bf16 slot of the chunk is ring entry pre + k behind the head), a coded
+        // slot's as its codes, rows past the fill as zeros (P is 0 there)
+        const int t = tid - 32 * (2 + kSoftWarps);
+        const int r = t >> 1, half = t & 1;
+        int pre_val = 0, pre_upto = 0;  // bf16 values of the unit before mask word pre_upto
+        for (int j = 0; j < n_mine; ++j) {
+            const int s = j % kStages;
+            const int c = rank + j * C;
+            const int s0 = c * kChunk;
+            const int rows = min(kChunk, p.fill - s0);
+            // the stage's previous tile has been read by its output MMA
+            if (j >= kStages && !mbar_wait(&empty[s], ((j / kStages) - 1) & 1, p.err, kErrDecodeEmpty)) break;
+            const uint64_t m = chunk_bf16(c, rows);
+            while (pre_upto < 2 * c) {
+                if (pre_upto < p.mask_words) pre_val += __popc(mask_s[pre_upto]);
+                ++pre_upto;
+            }
+            uint4 v[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v[q] = make_uint4(0, 0, 0, 0);
+            if (r < rows && ((m >> r) & 1ull)) {
+                const int k = pre_val + __popcll(m & ((1ull << r) - 1ull));
+                if (k < p.hp_cap) {
+                    int at = ring_head + k;
+                    at -= at >= p.hp_cap ? p.hp_cap : 0;
+                    const uint4* src = p.hp_rows + (static_cast<int64_t>(unit) * p.hp_cap + at) * kVecPerRow + half * 8;
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) v[q] = src[q];
+                } else {  // masks that do not match the ring: a zero row
+                    record_error(p.err, kErrDecodeMask);
+                }
+            } else if (r < rows) {
+                const int bits = p.bits;
+                const uint4* cr = reinterpret_cast<const uint4*>(
+                    p.codes + (static_cast<int64_t>(unit) * p.Kq + s0 + r) * p.code_row + half * 8 * bits);
+                uint32_t cw[16];
+                if (bits == 8) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) *reinterpret_cast<uint4*>(cw + 4 * i) = cr[i];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) v[q] = expand8<8>(cw, q);
+                } else if (bits == 4) {
+#pragma unroll
+                    for (int i = 0; i < 2; ++i) *reinterpret_cast<uint4*>(cw + 4 * i) = cr[i];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) v[q] = expand8<4>(cw, q);
+                } else {
+                    *reinterpret_cast<uint4*>(cw) = cr[0];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) v[q] = expand8<2>(cw, q);
+                }
+            }
+
+            uint8_t* dst = stage + s * kSB + 2 * kBoxBytes + half * kBoxBytes + r * 128;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) *reinterpret_cast<uint4*>(dst + (((q ^ (r & 7)) & 7) << 4)) = v[q];
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // tile writes -> tensor-core reads
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&v_full[s]);
+        }
     }
     __syncthreads();  // every MMA read and TMEM load is done; the stage area is free
     if (warp == 1) tmem_dealloc(tmem, kTmemCols);
@@ -404,7 +542,8 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
     float* res_o = reinterpret_cast<float*>(stage);                       // [GH][d]
     float* res_ml = reinterpret_cast<float*>(stage + GH * kHeadDim * 4);  // [GH][2]
     float* red_l = red + 2 * kSoftWarps * kNS + 16;                       // [kSoftWarps][16] (after the flags)
-    if (warp >= 2) {
+    float* red_b = red_l + kSoftWarps * kNS;                              // [kSoftWarps][16] bias sums (store)
+    if (warp >= 2 && warp < 2 + kSoftWarps) {
 #pragma unroll
         for (int g = 0; g < GH; ++g) {
             float sum = l_part[g];
@@ -414,9 +553,26 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
             sum += __shfl_xor_sync(0xffffffffu, sum, 8);
             sum += __shfl_xor_sync(0xffffffffu, sum, 16);
             if (lane == 0) red_l[sw * kNS + g] = sum;
-            if (g < G) res_o[g * kHeadDim + 32 * qd + lane] = acc[g];
+            if (kStore) {
+                float bs = b_part[g];
+                bs += __shfl_xor_sync(0xffffffffu, bs, 1);
+                bs += __shfl_xor_sync(0xffffffffu, bs, 2);
+                bs += __shfl_xor_sync(0xffffffffu, bs, 4);
+                bs += __shfl_xor_sync(0xffffffffu, bs, 8);
+                bs += __shfl_xor_sync(0xffffffffu, bs, 16);
+                if (lane == 0) red_b[sw * kNS + g] = bs;
+            } else if (g < G) {
+                res_o[g * kHeadDim + 32 * qd + lane] = acc[g];
+            }
         }
         named_bar(1, 32 * kSoftWarps);
+        if (kStore) {  // the output rows with the heads' bias: sum p z over every coded slot, added to each dim
+#pragma unroll
+            for (int g = 0; g < GH; ++g)
+                if (g < G)
+                    res_o[g * kHeadDim + 32 * qd + lane] =
+                        acc[g] + ((red_b[g] + red_b[kNS + g]) + (red_b[2 * kNS + g] + red_b[3 * kNS + g]));
+        }
         if (tid - 64 < G) {
             const int g = tid - 64;
             res_ml[2 * g] = m_run[0];
@@ -432,7 +588,7 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
         const int total = G * kHeadDim;
         const int per = (total + C - 1) / C;
         const int end = min(total, (rank + 1) * per);
-        for (int i = rank * per + tid; i < end; i += kThreads) {
+        for (int i = rank * per + tid; i < end; i += (kStore ? kThreadsStore : kThreads)) {
             const int g = i / kHeadDim;
             const int d = i - g * kHeadDim;
             float2 ml[kDecodeMaxCluster];
@@ -462,12 +618,12 @@ __global__ void __launch_bounds__(kThreads) decode_tc_kernel(const __grid_consta
     cluster_sync();  // every CTA has read what it needs from the others' shared memory
 }
 
-template <int NP>
+template <int NP, bool kStore>
 cudaError_t launch_np(const CUtensorMap& kmap, const CUtensorMap& vmap, const DecodeParams& p, size_t smem_bytes,
                       cudaStream_t s) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(p.cluster), static_cast<unsigned>(p.units));
-    cfg.blockDim = dim3(kThreads);
+    cfg.blockDim = dim3(kStore ? kThreadsStore : kThreads);
     cfg.dynamicSmemBytes = smem_bytes;
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
@@ -479,12 +635,14 @@ cudaError_t launch_np(const CUtensorMap& kmap, const CUtensorMap& vmap, const De
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<NP>, kmap, vmap, p);
+    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<NP, kStore>, kmap, vmap, p);
 }
 
 }  // namespace tc
 
-bool use_tc(int G) { return G >= 3; }
+// The tensor cores from G = 3 on (below, the dot products are a small share of the work); the compressed value
+// store always, since its V tiles are written by the builder warps off the softmax path.
+bool use_tc(int G, bool store) { return store || G >= 3; }
 int tc_np(int G) { return G <= 8 ? 16 : 32; }
 // CTAs per unit: enough clusters to fill the GPU `per_sm` CTAs deep (the kernel's residency), at most
 // kDecodeMaxCluster and at most one CTA per chunk.
@@ -496,30 +654,37 @@ int cluster_for(int units, int n_chunks, int num_sms, int per_sm) {
 
 }  // namespace
 
-size_t decode_smem_bytes(int G) {
-    return use_tc(G) ? tc::decode_layout(tc_np(G)).total + 1024 : simt::decode_layout(2).total;
+size_t decode_smem_bytes(int G, bool store) {
+    return use_tc(G, store) ? tc::decode_layout(tc_np(G), store).total + 1024 : simt::decode_layout(2).total;
 }
 
-cudaError_t decode_set_attributes(int G, size_t smem_bytes) {
+cudaError_t decode_set_attributes(int G, size_t smem_bytes, bool store) {
     const int bytes = static_cast<int>(smem_bytes);
-    if (!use_tc(G))
+    if (!use_tc(G, store))
         return cudaFuncSetAttribute(simt::decode_simt_kernel<2, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (store)
+        return tc_np(G) == 16
+                   ? cudaFuncSetAttribute(tc::decode_tc_kernel<16, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)
+                   : cudaFuncSetAttribute(tc::decode_tc_kernel<32, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     return tc_np(G) == 16
-               ? cudaFuncSetAttribute(tc::decode_tc_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)
-               : cudaFuncSetAttribute(tc::decode_tc_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+               ? cudaFuncSetAttribute(tc::decode_tc_kernel<16, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)
+               : cudaFuncSetAttribute(tc::decode_tc_kernel<32, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
 cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, DecodeParams p, size_t smem_bytes,
                           int num_sms, cudaStream_t s) {
-    if (!use_tc(p.G)) {
+    if (!use_tc(p.G, p.ring_state != nullptr)) {
         p.n_chunks = (p.fill + simt::kChunk - 1) / simt::kChunk;
         p.cluster = cluster_for(p.units, p.n_chunks, num_sms, 4);
         return simt::launch_gp<2, 0>(p, smem_bytes, s);
     }
     p.n_chunks = (p.fill + tc::kChunk - 1) / tc::kChunk;
-    p.cluster = cluster_for(p.units, p.n_chunks, num_sms, 2);
-    return tc_np(p.G) == 16 ? tc::launch_np<16>(kmap, vmap, p, smem_bytes, s)
-                            : tc::launch_np<32>(kmap, vmap, p, smem_bytes, s);
+    p.cluster = cluster_for(p.units, p.n_chunks, num_sms, 2);  // two CTAs per SM
+    if (p.ring_state)  // the compressed value store
+        return tc_np(p.G) == 16 ? tc::launch_np<16, true>(kmap, vmap, p, smem_bytes, s)
+                                : tc::launch_np<32, true>(kmap, vmap, p, smem_bytes, s);
+    return tc_np(p.G) == 16 ? tc::launch_np<16, false>(kmap, vmap, p, smem_bytes, s)
+                            : tc::launch_np<32, false>(kmap, vmap, p, smem_bytes, s);
 }
 
 }  // namespace vase

@@ -288,8 +288,8 @@ size_t select_static_smem_bytes();  // the selection kernel's static shared memo
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster);
 cudaError_t dkv_set_attributes(size_t smem_bytes);
 cudaError_t select_set_attributes(size_t smem_bytes);
-size_t decode_smem_bytes(int G);
-cudaError_t decode_set_attributes(int G, size_t smem_bytes);
+size_t decode_smem_bytes(int G, bool store);
+cudaError_t decode_set_attributes(int G, size_t smem_bytes, bool store);
 size_t decode_mixed_smem_bytes(int G, int bits, int mask_words);
 cudaError_t decode_mixed_set_attributes();
 cudaError_t launch_decode_mixed(DecodeParams p, int num_sms, cudaStream_t s);

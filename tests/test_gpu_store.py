@@ -182,6 +182,8 @@ def _run_rounds(geo, n_v, bits, prefill, rounds, seed, decode=True, evict_all=Fa
         steps = [1, 1, 1, geo.buffer_b - 3]
         for i, n in enumerate(steps):
             _append(cache, models, rng, n, layers)
+            if i == 0 and decode and r == 0:  # a ragged last chunk, one slot past K
+                _check_decode(cache, 0, models[0], bits, rng)
             if i == 1:
                 for l in range(layers):
                     _check_store(cache, l, models[l], bits)
@@ -208,12 +210,30 @@ def test_store_batched_evictions_and_small_ring():
     _run_rounds(geo, 0, 4, [1] * 5 + [155], 3, seed=11, evict_all=True)
 
 
-def test_store_grouped_query_heads_decode():
-    """G = 4 and G = 8 query heads per KV head read the store (the CUDA-core mixed decode)."""
+@pytest.mark.parametrize("bits", [2, 4, 8])
+def test_store_grouped_query_heads_decode(bits):
+    """G = 4 and G = 8 query heads per KV head read the store on the tensor cores (as G = 1 and 2 do in the tests
+    above): bf16 rows from the ring and the other rows expanded from their codes into the V tile; a first fill of
+    256 in one call (80 quantized in it), K 192 (three whole 64-slot chunks) and ragged fills."""
     from paper_2606_03928_gb300.vase import Geometry
     for hq, seed in ((32, 21), (64, 22)):
         geo = Geometry(192, 64, 16, hq, 8, 1, 1)
-        _run_rounds(geo, 48, 4, [256], 2, seed=seed)
+        _run_rounds(geo, 48, bits, [256], 2, seed=seed + bits)
+
+
+def test_store_decode_sixteen_query_heads():
+    """G = 16 (64 query heads over 4 KV heads): the 32-column form of the tensor-core decode over the store."""
+    from paper_2606_03928_gb300.vase import Geometry
+    geo = Geometry(128, 32, 16, 64, 4, 1, 1)
+    _run_rounds(geo, 32, 4, [160], 2, seed=41)
+
+
+def test_store_decode_qwen3_8b_geometry_sampled():
+    """A larger unit on the tensor-core path: K 1024, B 128, 32/8 heads (G = 4), two sequences, 4 bits, the ring
+    wrapped by several rounds; a decode step after every eviction."""
+    from paper_2606_03928_gb300.vase import Geometry
+    geo = Geometry(1024, 128, 32, 32, 8, 2, 1)
+    _run_rounds(geo, 256, 4, [700, 452], 3, seed=31)
 
 
 def test_store_refuses_a_state_it_did_not_write():

@@ -261,3 +261,73 @@ def test_store_refuses_a_state_it_did_not_write():
     assert status != 0 and code & 0x80000000, (status, code)  # the decode's own site; the context stays usable
     assert cache.check_device_error()[0] == 0
 
+
+
+def test_store_qwen3_1p7b_geometry_batched_sampled_units():
+    """The bench's store configuration at full unit size: Qwen3-1.7B geometry (K 2048, B 128, W 32, 16/8 heads,
+    batch 8: 64 units per layer), two layers, 4 bits, appended and evicted through the batched all-layer calls
+    the bench times (vase_append_all, vase_evict_all).  The first fill of 2176 values in two pieces overflows the
+    768-row ring; then three rounds.  Eight sampled units of each layer are checked bit-exactly against the
+    oracle's store model after every eviction, and decoded."""
+    from paper_2606_03928_gb300.vase import Geometry, VaseCache
+    geo = Geometry(2048, 128, 32, 16, 8, 2, 8)
+    nv, bits, L = 512, 4, 2
+    cache = VaseCache(geo, n_v=nv, value_bits=bits, debug_outputs=True, seed=5)
+    rng = np.random.default_rng(55)
+    sample = sorted(rng.choice(64, 8, replace=False).tolist())
+    models = [Model(geo, nv) for _ in range(L)]
+    dev = cache.device
+
+    def append_all(n):
+        q, k, v = _stream(rng, n, geo, L)
+        cache.append_all(PU.bits_to_bf16_tensor(q, dev), PU.bits_to_bf16_tensor(k, dev),
+                         PU.bits_to_bf16_tensor(v, dev))
+        for l in range(L):
+            models[l].append(k[l], v[l])
+
+    def check_sampled(l, after_evict):
+        torch.cuda.synchronize()
+        vs = cache.value_store(l)
+        codes, sz = vs["codes"].cpu().numpy(), vs["sz"].cpu().numpy()
+        mask = vs["mask"].cpu().numpy().view(np.uint32)
+        ring = vs["ring"].view(torch.int16).cpu().numpy().view(np.uint16)
+        state = vs["state"].cpu().numpy()
+        m = models[l]
+        for u in sample:
+            st = m.store[u]
+            assert state[u, 0] == st["head"] and state[u, 1] == len(st["slots"]), f"layer {l} unit {u}: ring state"
+            bf = O.store_reserved_mask(st, m.N)
+            if after_evict:
+                assert bf[:m.fill].sum() == nv + geo.buffer_b
+            got = np.unpackbits(mask[u].view(np.uint8), bitorder="little")[:m.N].astype(bool)
+            assert np.array_equal(got, bf), f"layer {l} unit {u}: mask"
+            pos = O.store_ring_positions(st)
+            slots = np.array(st["slots"], dtype=np.int64)
+            assert np.array_equal(ring[u, [pos[s] for s in st["slots"]]], m.v[u, slots]), f"layer {l} unit {u}: ring"
+            coded = np.flatnonzero(~bf[:m.fill])
+            rc, rs, rz = O.quantize_values(O.bf16_bits_to_f64(m.v[u, coded]), bits)
+            assert np.array_equal(_unpack(codes[u, coded], bits), rc), f"layer {l} unit {u}: codes"
+            assert np.array_equal(sz[u, coded, 0], rs) and np.array_equal(sz[u, coded, 1], rz)
+
+    append_all(1500)
+    append_all(676)
+    for l in range(L):
+        check_sampled(l, False)
+    for r in range(3):
+        assert cache.evict_all() == L
+        for l in range(L):
+            models[l].evict(cache.debug_view(l)["src"].cpu().numpy())
+            check_sampled(l, True)
+        # decode of layer 1 on the sampled units
+        G = geo.num_q_heads // geo.num_kv_heads
+        q_bits = W.f32_to_bf16_bits(rng.standard_normal((geo.batch, geo.num_q_heads, 128)).astype(np.float32))
+        out = cache.decode_attention(1, PU.bits_to_bf16_tensor(q_bits, dev)).cpu().numpy()
+        m = models[1]
+        for u in sample:
+            s, h = divmod(u, geo.num_kv_heads)
+            ref, scale = O.decode_attention_mixed(O.bf16_bits_to_f64(q_bits[s, h * G:(h + 1) * G]),
+                                                  O.bf16_bits_to_f64(m.k[u, :m.fill]), O.bf16_bits_to_f64(m.v[u, :m.fill]),
+                                                  O.store_reserved_mask(m.store[u], m.N)[:m.fill], bits)
+            assert np.all(np.abs(out[s, h * G:(h + 1) * G] - ref) <= DEC_RTOL * scale + DEC_ATOL), f"unit {u}: decode"
+        append_all(geo.buffer_b)
+    assert cache.check_device_error()[0] == 0

@@ -372,8 +372,9 @@ class VaseCache:
         self.slots = N
         self.k_cache = torch.empty((g.num_layers, g.batch, g.num_kv_heads, N, g.head_dim), dtype=torch.bfloat16,
                                    device=dev)
-        # the bf16 value cache, or (value_bits > 0) the compressed value store the library lays out itself
-        self.v_cache = (torch.empty(sizes.v_cache, dtype=torch.uint8, device=dev) if value_bits
+        # the bf16 value cache, or (value_bits > 0) the compressed value store the library lays out itself (zeroed,
+        # so that the bytes the library never writes -- padding, unused ring rows -- compare equal across caches)
+        self.v_cache = (torch.zeros(sizes.v_cache, dtype=torch.uint8, device=dev) if value_bits
                         else torch.empty_like(self.k_cache))
         self.value_bits = int(value_bits)
         self.q_window = torch.empty((g.num_layers, g.batch, g.num_q_heads, g.window, g.head_dim),

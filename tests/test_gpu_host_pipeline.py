@@ -28,8 +28,8 @@ def _tensors(wl, L, r, n, dev=None):
     return out
 
 
-@pytest.mark.parametrize("variant", ["attnv", "dkv"])
-def test_staged_host_rounds_equal_device_appends(variant):
+@pytest.mark.parametrize("variant,value_bits", [("attnv", 0), ("dkv", 0), ("attnv", 4)])
+def test_staged_host_rounds_equal_device_appends(variant, value_bits):
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     from paper_2606_03928_gb300 import build
@@ -38,8 +38,8 @@ def test_staged_host_rounds_equal_device_appends(variant):
     L = 3
     wl = W.shrink(W.WORKLOADS["single_layer_k256"], num_layers=L, batch=2, budget_k=128, buffer_b=32, window=16)
     K, B = wl.budget_k, wl.buffer_b
-    ref = V.VaseCache(PU.geometry_of(wl, L), variant=variant, seed=11)
-    dut = V.VaseCache(PU.geometry_of(wl, L), variant=variant, seed=11)
+    ref = V.VaseCache(PU.geometry_of(wl, L), variant=variant, seed=11, value_bits=value_bits)
+    dut = V.VaseCache(PU.geometry_of(wl, L), variant=variant, seed=11, value_bits=value_bits)
     # the same prefill of K tokens per layer in both
     pre = [W.stream_chunk(wl, 31, layer, 0, K) for layer in range(L)]
     for layer in range(L):

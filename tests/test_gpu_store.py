@@ -331,3 +331,27 @@ def test_store_qwen3_1p7b_geometry_batched_sampled_units():
             assert np.all(np.abs(out[s, h * G:(h + 1) * G] - ref) <= DEC_RTOL * scale + DEC_ATOL), f"unit {u}: decode"
         append_all(geo.buffer_b)
     assert cache.check_device_error()[0] == 0
+
+
+def test_store_refuses_the_bf16_cache_calls():
+    """With the store, the calls that need bf16 value rows -- the magnitude refresh, the read path's quantizer
+    and its mixed decode -- return VASE_ERR_UNSUPPORTED and launch nothing; the view reports no V rows."""
+    from paper_2606_03928_gb300 import vase as V
+    from paper_2606_03928_gb300.vase import Geometry, VaseCache
+    cache = VaseCache(Geometry(128, 32, 16, 8, 8, 1, 1), n_v=16, value_bits=2, seed=1)
+    n0 = cache.launch_count()
+    for call in (lambda: cache.refresh_value_scores(0),
+                 lambda: cache.quantize_values(0, 2, cache.mixed_buffers(2)[0])):
+        with pytest.raises(V.VaseError) as exc:
+            call()
+        assert exc.value.status == V.VASE_ERR_UNSUPPORTED
+    mb, _ = cache.mixed_buffers(2)
+    q = torch.zeros((1, 8, 128), dtype=torch.bfloat16, device=cache.device)
+    with pytest.raises(V.VaseError) as exc:
+        cache.decode_attention_mixed(0, 2, mb, q)
+    assert exc.value.status == V.VASE_ERR_UNSUPPORTED
+    assert cache.launch_count() == n0
+    import ctypes
+    kv = V.vase_kv_view()
+    assert V.load().vase_kv_view_get(cache.ctx, 0, ctypes.byref(kv)) == 0
+    assert kv.k and not kv.v

@@ -86,3 +86,15 @@ def test_static_scratch_refuses_a_layer_larger_than_the_array():
         V.vase_evict_static_scratch(cfg, bufs, 0, wl.slots, 0)
     assert exc.value.status == V.VASE_ERR_UNSUPPORTED
     assert "VASE_STATIC_SCRATCH_BYTES" in str(exc.value)
+
+
+def test_static_scratch_refuses_the_compressed_value_store():
+    """The static-scratch eviction works on the bf16 value cache: with value_bits set it returns
+    VASE_ERR_UNSUPPORTED from the configuration alone."""
+    V = _lib()
+    cfg = V.vase_config_default(budget_k=256, buffer_b=64, window=32, num_q_heads=16, num_kv_heads=8, head_dim=128,
+                                num_layers=1, batch=1, value_bits=4)
+    bufs = V.vase_buffers(None, None, None, None, None, None)
+    with pytest.raises(V.VaseError) as exc:
+        V.vase_evict_static_scratch(cfg, bufs, 0, 320, 0)
+    assert exc.value.status == V.VASE_ERR_UNSUPPORTED

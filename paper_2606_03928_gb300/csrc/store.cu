@@ -422,57 +422,69 @@ __global__ void __launch_bounds__(kStoreThreads) store_evict_kernel(const StoreP
     }
     if (tid == 0) u.state[1] = total_ring;
 
-    // the moves, in phases of kStoreWarps * kStoreRowsPerWarp new slots
-    uint2* stage = reinterpret_cast<uint2*>(smem + Ly.stage_off) + warp * kStoreRowsPerWarp * kRowWords2;
-    float2* stage_sz = reinterpret_cast<float2*>(smem + Ly.sz_off) + warp * kStoreRowsPerWarp;
-    const int code_lanes = p.code_row / 8;  // lanes moving 8 code bytes each
+    // The moves, in phases of kPhase new slots.  Thread t < kPhase owns slot base + t and moves its whole row with
+    // 16-byte copies (a code row and its (s, z), or a 256-byte ring row); the rows to quantize are staged the same
+    // way and then quantized by the warps (one warp per row: the quantizer reduces over the row's lanes).  Row t's
+    // 16-byte piece c sits at piece c ^ (t % 16) of its 256 bytes, so that the threads of a warp, each on its own
+    // row, touch different banks.
     constexpr int kPhase = kStoreWarps * kStoreRowsPerWarp;
+    uint4* stage4 = reinterpret_cast<uint4*>(smem + Ly.stage_off);   // [kPhase][16] (row t at 256 t)
+    float2* stage_sz = reinterpret_cast<float2*>(smem + Ly.sz_off);  // [kPhase]
+    const int code_vecs = p.code_row / 16;  // 16-byte pieces of a code row (2, 4 or 8)
+    uint8_t* const codes = u.codes;
+    const uint4* const ring4 = reinterpret_cast<const uint4*>(u.ring);
     for (int base = 0; base < K; base += kPhase) {
-        // every read of the phase in flight at once (asynchronous copies into the warp's stage)
+        const int j = base + tid;
+        uint32_t kind = kKindRing;
+        int o = 0, rr = 0, s = j;
+        bool load = false;
+        if (tid < kPhase && j < K) {
+            const uint32_t info = info_s[j];
+            kind = info >> 30;
+            o = static_cast<int>((info >> 15) & 0x7FFFu);
+            rr = static_cast<int>(info & 0x7FFFu);
+            s = src_s[j];
+            uint4* dst = stage4 + tid * 16;
+            const int sw = tid & 15;
+            if (kind == kKindCoded) {
+                load = s != j;  // in place already otherwise
+                if (load) {
+                    const uint4* src = reinterpret_cast<const uint4*>(codes + static_cast<int64_t>(s) * p.code_row);
+                    for (int c = 0; c < code_vecs; ++c) cp_async<16>(dst + (c ^ sw), src + c);
+                    cp_async<8>(stage_sz + tid, u.sz + 2 * s);
+                }
+            } else {
+                load = kind == kKindSpill || o != rr;
+                if (load) {
+                    const uint4* src = ring4 + static_cast<int64_t>(wrap(head + o, H)) * 16;
 #pragma unroll
-        for (int i = 0; i < kStoreRowsPerWarp; ++i) {
-            const int j = base + warp * kStoreRowsPerWarp + i;
-            if (j < K) {
-                const uint32_t info = info_s[j];
-                const uint32_t kind = info >> 30;
-                const int o = static_cast<int>((info >> 15) & 0x7FFFu);
-                const int rr = static_cast<int>(info & 0x7FFFu);
-                if (kind == kKindCoded) {
-                    const int s = src_s[j];
-                    if (s != j) {  // (in place already otherwise)
-                        if (lane < code_lanes)
-                            cp_async<8>(stage + i * kRowWords2 + lane, u.codes + static_cast<int64_t>(s) * p.code_row + 8 * lane);
-                        if (lane == 31) cp_async<8>(stage_sz + i, u.sz + 2 * s);
-                    }
-                } else if (kind == kKindSpill || o != rr) {
-                    cp_async<8>(stage + i * kRowWords2 + lane, u.ring + wrap(head + o, H) * kRowWords2 + lane);
+                    for (int c = 0; c < 16; ++c) cp_async<16>(dst + (c ^ sw), src + c);
                 }
             }
         }
         cp_async_all();
         __syncthreads();  // every read of the phase precedes every write
-#pragma unroll 4
-        for (int i = 0; i < kStoreRowsPerWarp; ++i) {
-            const int j = base + warp * kStoreRowsPerWarp + i;
-            if (j >= K) break;
-            const uint32_t info = info_s[j];
-            const uint32_t kind = info >> 30;
-            const int o = static_cast<int>((info >> 15) & 0x7FFFu);
-            const int rr = static_cast<int>(info & 0x7FFFu);
+        if (load && kind != kKindSpill) {
+            const uint4* srow = stage4 + tid * 16;
+            const int sw = tid & 15;
             if (kind == kKindCoded) {
-                if (src_s[j] == j) continue;
-                if (lane < code_lanes)
-                    reinterpret_cast<uint2*>(u.codes + static_cast<int64_t>(j) * p.code_row)[lane] =
-                        stage[i * kRowWords2 + lane];
-                if (lane == 31) *reinterpret_cast<float2*>(u.sz + 2 * j) = stage_sz[i];
-            } else if (kind == kKindRing) {
-                if (o != rr) u.ring[wrap(head + rr, H) * kRowWords2 + lane] = stage[i * kRowWords2 + lane];
+                uint4* d = reinterpret_cast<uint4*>(codes + static_cast<int64_t>(j) * p.code_row);
+                for (int c = 0; c < code_vecs; ++c) d[c] = srow[c ^ sw];
+                *reinterpret_cast<float2*>(u.sz + 2 * j) = stage_sz[tid];
             } else {
-                quantize_row_warp(stage[i * kRowWords2 + lane], p.bits, lane,
-                                  u.codes + static_cast<int64_t>(j) * p.code_row, u.sz + 2 * j);
+                uint4* d = reinterpret_cast<uint4*>(u.ring) + static_cast<int64_t>(wrap(head + rr, H)) * 16;
+#pragma unroll
+                for (int c = 0; c < 16; ++c) d[c] = srow[c ^ sw];
             }
         }
-        __syncwarp();  // this warp's stage is read before its next phase refills it
+        // the rows to quantize: warp w takes the phase's slots w, w + kStoreWarps, ... (the test is uniform)
+        for (int t = warp; t < kPhase; t += kStoreWarps) {
+            const int jj = base + t;
+            if (jj >= K || (info_s[jj] >> 30) != kKindSpill) continue;
+            const uint2 raw = reinterpret_cast<const uint2*>(stage4 + t * 16 + ((lane >> 1) ^ (t & 15)))[lane & 1];
+            quantize_row_warp(raw, p.bits, lane, codes + static_cast<int64_t>(jj) * p.code_row, u.sz + 2 * jj);
+        }
+        __syncthreads();  // the stage is read before the next phase refills it
     }
 }
 

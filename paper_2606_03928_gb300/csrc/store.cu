@@ -22,6 +22,8 @@ constexpr int kStoreThreads = 256;
 constexpr int kStoreWarps = kStoreThreads / 32;
 constexpr int kStoreRowsPerWarp = 16;  // rows a warp has in flight per phase of the eviction sweep
 constexpr int kRowWords2 = 32;         // uint2 per 256-byte row
+constexpr int kEvictPhase = 64;        // new slots per phase of the eviction sweep
+constexpr int kEvictBufs = 2;          // phases of the sweep in flight
 
 struct StoreUnit {
     uint8_t* codes;
@@ -56,6 +58,13 @@ __device__ __forceinline__ void cp_async(void* smem_dst, const void* gsrc) {
 }
 __device__ __forceinline__ void cp_async_all() {
     asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+// The copies issued since the last commit form a group; cp_async_wait_prior<n>() waits for every group but the
+// latest n.
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int kPending>
+__device__ __forceinline__ void cp_async_wait_prior() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(kPending) : "memory");
 }
 
 // Exclusive scan of one value per thread over the block; *total gets the sum.  Starts and ends with a barrier
@@ -334,9 +343,9 @@ __host__ __device__ inline StoreEvictSmem store_evict_layout(int K, int mask_str
     o += 4u * mask_stride;
     o = (o + 15u) & ~15u;
     L.stage_off = o;
-    o += kStoreWarps * kStoreRowsPerWarp * 256u;
+    o += static_cast<uint32_t>(kEvictBufs * kEvictPhase) * 256u;
     L.sz_off = o;
-    o += kStoreWarps * kStoreRowsPerWarp * 8u;
+    o += static_cast<uint32_t>(kEvictBufs * kEvictPhase) * 8u;
     L.scan_off = o;
     o += 4u * (kStoreWarps + 1);
     L.total = (o + 15u) & ~15u;
@@ -355,8 +364,11 @@ __global__ void __launch_bounds__(kStoreThreads) store_evict_kernel(const StoreP
     extern __shared__ __align__(16) uint8_t smem[];
     const int K = p.K;
     const StoreEvictSmem Ly = store_evict_layout(K, p.mask_stride);
+    // the kept list src[j], and slot j's info word: kind << 30 | s for a coded value (s = src[j]), kind << 30 |
+    // o << 15 | r for a bf16 one (o its old ring rank, r its new one where it stays in the ring).  (One array could
+    // hold both and let a fifth CTA onto an SM; at the Qwen3-1.7B geometry that measured slower.)
     int32_t* src_s = reinterpret_cast<int32_t*>(smem + Ly.src_off);
-    uint32_t* info_s = reinterpret_cast<uint32_t*>(smem + Ly.info_off);  // kind << 30 | o << 15 | r
+    uint32_t* info_s = reinterpret_cast<uint32_t*>(smem + Ly.info_off);
     uint8_t* resv_s = smem + Ly.resv_off;
     uint32_t* mask_s = reinterpret_cast<uint32_t*>(smem + Ly.mask_off);
     uint32_t* pre_s = reinterpret_cast<uint32_t*>(smem + Ly.pre_off);
@@ -407,7 +419,7 @@ __global__ void __launch_bounds__(kStoreThreads) store_evict_kernel(const StoreP
         const uint32_t o = pre_s[s >> 5] + __popc(w & ((1u << (s & 31)) - 1u));
         const uint32_t kind = !bf ? kKindCoded : (resv_s[j] ? kKindRing : kKindSpill);
         n_ring += kind == kKindRing;
-        info_s[j] = kind << 30 | (o & 0x7FFFu) << 15;
+        info_s[j] = kind == kKindCoded ? static_cast<uint32_t>(s) : kind << 30 | (o & 0x7FFFu) << 15;
     }
     int total_ring;
     int r = block_scan(n_ring, scan_s, &total_ring);
@@ -422,69 +434,84 @@ __global__ void __launch_bounds__(kStoreThreads) store_evict_kernel(const StoreP
     }
     if (tid == 0) u.state[1] = total_ring;
 
-    // The moves, in phases of kPhase new slots.  Thread t < kPhase owns slot base + t and moves its whole row with
-    // 16-byte copies (a code row and its (s, z), or a 256-byte ring row); the rows to quantize are staged the same
-    // way and then quantized by the warps (one warp per row: the quantizer reduces over the row's lanes).  Row t's
-    // 16-byte piece c sits at piece c ^ (t % 16) of its 256 bytes, so that the threads of a warp, each on its own
-    // row, touch different banks.
-    constexpr int kPhase = kStoreWarps * kStoreRowsPerWarp;
-    uint4* stage4 = reinterpret_cast<uint4*>(smem + Ly.stage_off);   // [kPhase][16] (row t at 256 t)
-    float2* stage_sz = reinterpret_cast<float2*>(smem + Ly.sz_off);  // [kPhase]
+    // The moves, in phases of kEvictPhase new slots, kEvictBufs phases in flight: the reads of phase i + 1 ..
+    // i + kEvictBufs - 1 are issued before the writes of phase i.  That is safe because no phase reads what an earlier phase writes: codes and
+    // (s, z) are read at src[j] >= j and written at j, and a ring entry is read at its old rank o, which is at
+    // least every new rank r of the slots before it, where the earlier phases write.  Within a phase every read
+    // precedes every write (a barrier), and a buffer is refilled only after the phase that used it is done.
+    // Thread t < kEvictPhase owns slot base + t and moves its whole row with 16-byte copies (a code row and its
+    // (s, z), or a 256-byte ring row); the rows to quantize are staged the same way and then quantized by the
+    // warps (one warp per row: the quantizer reduces over the row's lanes).  Row t's 16-byte piece c sits at
+    // piece c ^ (t % 16) of its 256 bytes, so that the threads of a warp, each on its own row, touch different
+    // banks.
+    uint4* const stage4 = reinterpret_cast<uint4*>(smem + Ly.stage_off);   // [kEvictBufs][kEvictPhase][16]
+    float2* const stage_sz = reinterpret_cast<float2*>(smem + Ly.sz_off);  // [kEvictBufs][kEvictPhase]
     const int code_vecs = p.code_row / 16;  // 16-byte pieces of a code row (2, 4 or 8)
     uint8_t* const codes = u.codes;
     const uint4* const ring4 = reinterpret_cast<const uint4*>(u.ring);
-    for (int base = 0; base < K; base += kPhase) {
+    const int sw = tid & 15;
+    // this thread's slot of the phase at `base`: its reads into buffer `buf`
+    auto issue_reads = [&](int base, int buf) {
         const int j = base + tid;
-        uint32_t kind = kKindRing;
-        int o = 0, rr = 0, s = j;
-        bool load = false;
-        if (tid < kPhase && j < K) {
-            const uint32_t info = info_s[j];
-            kind = info >> 30;
-            o = static_cast<int>((info >> 15) & 0x7FFFu);
-            rr = static_cast<int>(info & 0x7FFFu);
-            s = src_s[j];
-            uint4* dst = stage4 + tid * 16;
-            const int sw = tid & 15;
-            if (kind == kKindCoded) {
-                load = s != j;  // in place already otherwise
-                if (load) {
-                    const uint4* src = reinterpret_cast<const uint4*>(codes + static_cast<int64_t>(s) * p.code_row);
-                    for (int c = 0; c < code_vecs; ++c) cp_async<16>(dst + (c ^ sw), src + c);
-                    cp_async<8>(stage_sz + tid, u.sz + 2 * s);
-                }
-            } else {
-                load = kind == kKindSpill || o != rr;
-                if (load) {
-                    const uint4* src = ring4 + static_cast<int64_t>(wrap(head + o, H)) * 16;
-#pragma unroll
-                    for (int c = 0; c < 16; ++c) cp_async<16>(dst + (c ^ sw), src + c);
-                }
+        if (tid >= kEvictPhase || j >= K) return;
+        const uint32_t info = info_s[j];
+        const uint32_t kind = info >> 30;
+        const int o = static_cast<int>((info >> 15) & 0x7FFFu);
+        const int rr = static_cast<int>(info & 0x7FFFu);
+        uint4* dst = stage4 + (buf * kEvictPhase + tid) * 16;
+        if (kind == kKindCoded) {
+            const int s = static_cast<int>(info & 0x3FFFFFFFu);
+            if (s != j) {  // in place already otherwise
+                const uint4* src = reinterpret_cast<const uint4*>(codes + static_cast<int64_t>(s) * p.code_row);
+                for (int c = 0; c < code_vecs; ++c) cp_async<16>(dst + (c ^ sw), src + c);
+                cp_async<8>(stage_sz + buf * kEvictPhase + tid, u.sz + 2 * s);
             }
+        } else if (kind == kKindSpill || o != rr) {
+            const uint4* src = ring4 + static_cast<int64_t>(wrap(head + o, H)) * 16;
+#pragma unroll
+            for (int c = 0; c < 16; ++c) cp_async<16>(dst + (c ^ sw), src + c);
         }
-        cp_async_all();
-        __syncthreads();  // every read of the phase precedes every write
-        if (load && kind != kKindSpill) {
-            const uint4* srow = stage4 + tid * 16;
-            const int sw = tid & 15;
+    };
+    const int n_phase = (K + kEvictPhase - 1) / kEvictPhase;
+    for (int ph = 0; ph < kEvictBufs - 1; ++ph) {
+        if (ph < n_phase) issue_reads(ph * kEvictPhase, ph);
+        cp_async_commit();
+    }
+    for (int ph = 0; ph < n_phase; ++ph) {
+        const int base = ph * kEvictPhase, buf = ph % kEvictBufs;
+        const int ahead = ph + kEvictBufs - 1;
+        if (ahead < n_phase) issue_reads(ahead * kEvictPhase, ahead % kEvictBufs);
+        cp_async_commit();
+        cp_async_wait_prior<kEvictBufs - 1>();  // this thread's reads of phase ph have landed
+        __syncthreads();        // every read of phase ph precedes every write
+        const int j = base + tid;
+        if (tid < kEvictPhase && j < K) {
+            const uint32_t info = info_s[j];
+            const uint32_t kind = info >> 30;
+            const int o = static_cast<int>((info >> 15) & 0x7FFFu);
+            const int rr = static_cast<int>(info & 0x7FFFu);
+            const uint4* srow = stage4 + (buf * kEvictPhase + tid) * 16;
             if (kind == kKindCoded) {
-                uint4* d = reinterpret_cast<uint4*>(codes + static_cast<int64_t>(j) * p.code_row);
-                for (int c = 0; c < code_vecs; ++c) d[c] = srow[c ^ sw];
-                *reinterpret_cast<float2*>(u.sz + 2 * j) = stage_sz[tid];
-            } else {
+                if (static_cast<int>(info & 0x3FFFFFFFu) != j) {
+                    uint4* d = reinterpret_cast<uint4*>(codes + static_cast<int64_t>(j) * p.code_row);
+                    for (int c = 0; c < code_vecs; ++c) d[c] = srow[c ^ sw];
+                    *reinterpret_cast<float2*>(u.sz + 2 * j) = stage_sz[buf * kEvictPhase + tid];
+                }
+            } else if (kind == kKindRing && o != rr) {
                 uint4* d = reinterpret_cast<uint4*>(u.ring) + static_cast<int64_t>(wrap(head + rr, H)) * 16;
 #pragma unroll
                 for (int c = 0; c < 16; ++c) d[c] = srow[c ^ sw];
             }
         }
         // the rows to quantize: warp w takes the phase's slots w, w + kStoreWarps, ... (the test is uniform)
-        for (int t = warp; t < kPhase; t += kStoreWarps) {
+        for (int t = warp; t < kEvictPhase; t += kStoreWarps) {
             const int jj = base + t;
             if (jj >= K || (info_s[jj] >> 30) != kKindSpill) continue;
-            const uint2 raw = reinterpret_cast<const uint2*>(stage4 + t * 16 + ((lane >> 1) ^ (t & 15)))[lane & 1];
+            const uint4* srow = stage4 + (buf * kEvictPhase + t) * 16;
+            const uint2 raw = reinterpret_cast<const uint2*>(srow + ((lane >> 1) ^ (t & 15)))[lane & 1];
             quantize_row_warp(raw, p.bits, lane, codes + static_cast<int64_t>(jj) * p.code_row, u.sz + 2 * jj);
         }
-        __syncthreads();  // the stage is read before the next phase refills it
+        __syncthreads();  // buffer `buf` is read before the reads of phase ph + kEvictBufs refill it
     }
 }
 

@@ -194,7 +194,8 @@ struct SmallEvictParams {
     float scale_log2;       // log2(e) / sqrt(d)
     float* attn;            // [slot][units][N]: the window score, written for the debug view (nullable)
 };
-constexpr int kSmallThreads = 256;
+constexpr int kSmallThreads = 512;
+constexpr int kSmallWarps = kSmallThreads / 32;
 constexpr int kSmallMaxTiles = 8;
 
 // Mixed-precision values of one layer: codes of the unreserved kept value rows, their (s, z), and the

@@ -277,23 +277,45 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
 }
 
 // The same selection as radix_top_k for n <= kT candidates, by rank: slot i is taken when fewer than k slots
-// outrank it (a larger key, or an equal key at a lower slot).  One candidate per thread, n comparisons each against
-// keys read as broadcasts; no histogram passes.  Ends with a barrier.
+// outrank it (a larger key, or an equal key at a lower slot).  Each candidate's count is split over P = 1, 2 or 4
+// neighbouring threads (as many as kT / n allows): part p compares against the groups of four keys g with
+// g % P == p, read as broadcasts (the parts of a warp read neighbouring 16-byte groups, so different banks), and
+// the parts' counts are summed by shuffles.  Groups wholly below i count keys >= x, groups wholly above it keys
+// > x (one comparison per key); only i's own group tests the slot order.  No histogram passes.  Ends with a
+// barrier.
 template <int kT>
 __device__ void rank_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, uint8_t flag) {
-    const int i = threadIdx.x;
-    if (k > 0 && i < n) {
-        const uint32_t x = ord[i];
-        int rank = 0;
-        const int n4 = n & ~3;
-        for (int j = 0; j < n4; j += 4) {
-            const uint4 y = *reinterpret_cast<const uint4*>(ord + j);
-            rank += (y.x > x) + (y.y > x) + (y.z > x) + (y.w > x);
-            rank += (y.x == x && j < i) + (y.y == x && j + 1 < i) + (y.z == x && j + 2 < i) + (y.w == x && j + 3 < i);
+    const int P = 4 * n <= kT ? 4 : (2 * n <= kT ? 2 : 1);
+    const int i = threadIdx.x / P, part = threadIdx.x - i * P;
+    int rank = 0;
+    uint32_t x = 0;
+    const bool live = k > 0 && i < n;
+    if (live) {
+        x = ord[i];
+        const uint4* ord4 = reinterpret_cast<const uint4*>(ord);
+        const int g4 = n >> 2, gi = i >> 2;  // groups of four keys; gi holds candidate i itself
+        int g = part;
+        for (; g < gi && g < g4; g += P) {  // every slot below i: an equal key outranks it too
+            const uint4 y = ord4[g];
+            rank += (y.x >= x) + (y.y >= x) + (y.z >= x) + (y.w >= x);
         }
-        for (int j = n4; j < n; ++j) rank += (ord[j] > x) + (ord[j] == x && j < i);
-        if (rank < k) flags[i] |= flag;
+        if (g == gi && g < g4) {  // the group of i: ties count for the slots below it only
+            const uint4 y = ord4[g];
+            const int j = 4 * g;
+            rank += (y.x > x) + (y.y > x) + (y.z > x) + (y.w > x);
+            rank += (y.x == x && j < i) + (y.y == x && j + 1 < i) + (y.z == x && j + 2 < i);
+            g += P;
+        }
+        for (; g < g4; g += P) {  // every slot above i: only a larger key outranks it
+            const uint4 y = ord4[g];
+            rank += (y.x > x) + (y.y > x) + (y.z > x) + (y.w > x);
+        }
+        if (part == 0)
+            for (int j = 4 * g4; j < n; ++j) rank += (ord[j] > x) + (ord[j] == x && j < i);
     }
+    // the parts of a candidate are P neighbouring lanes of one warp (P divides 32); all lanes take part
+    for (int o = 1; o < P; o <<= 1) rank += __shfl_xor_sync(0xffffffffu, rank, o);
+    if (live && part == 0 && rank < k) flags[i] |= flag;
     __syncthreads();
 }
 
@@ -467,6 +489,18 @@ __device__ void gather_rows(uint8_t* base, const int32_t* src, int j_first, int 
 // kT threads per CTA: 256 where four CTAs share an SM; 512 or 1024 where the unit's arrays leave room for two
 // or one, so that the selection phase, which no other CTA's gather hides there, runs on as many warps.
 //
+// The staged value magnitudes and positions of one unit, requested into the selection's shared-memory layout
+// (completion by cp_async_wait_all, which select_unit runs): the fused small-unit eviction issues them before
+// its window score, so that their memory latency passes under the score.
+__device__ __forceinline__ void select_stage_rows(const SelectParams& p, int unit, int z, uint8_t* smem_raw) {
+    const int N = p.N;
+    const SelLayout Ly = sel_layout(N, p.K, p.n_parts, true);
+    const int layer = p.batch.layer[z];
+    const int64_t base = static_cast<int64_t>(layer) * p.units * N + static_cast<int64_t>(unit) * N;
+    cp_async_words(smem_raw + Ly.vm_off, p.vmag + base, N);
+    cp_async_words(smem_raw + Ly.pos_off, p.pos + base, N);
+}
+
 // The body is select_unit, which the fused small-unit eviction (evict_small_kernel) runs too, on window scores it
 // has already written to shared memory (a_ready: the staging skips them; one part).
 template <int kT>
@@ -500,14 +534,15 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
     const int kseg_hi = min(K, seg_hi);
 
     // The unit's inputs: with `staged`, every array is requested at once (one memory latency for all),
-    // and the positions and value magnitudes are compacted from the staged copies at the end.
+    // and the positions and value magnitudes are compacted from the staged copies at the end.  With a_ready the
+    // caller has written the window scores and requested the value magnitudes and positions itself
+    // (select_stage_rows) before its own work.
     float* vm_s = staged ? reinterpret_cast<float*>(smem_raw + Ly.vm_off) : nullptr;
     int32_t* pos_s = staged ? reinterpret_cast<int32_t*>(smem_raw + Ly.pos_off) : nullptr;
-    if (staged) {
+    if (staged && !a_ready) {
         if (p.variant == 0) {
-            if (!a_ready)
-                for (int part = 0; part < p.n_parts; ++part)
-                    cp_async_words(a_s + part * N, attn + (static_cast<int64_t>(part) * p.units + unit) * N, N);
+            for (int part = 0; part < p.n_parts; ++part)
+                cp_async_words(a_s + part * N, attn + (static_cast<int64_t>(part) * p.units + unit) * N, N);
         } else {
             cp_async_words(a_s, dkv + base, K);
         }
@@ -819,6 +854,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1)
         tmem_alloc(tmem_slot, static_cast<uint32_t>(p.tmem_cols));
         tmem_relinquish();
     }
+    if (sp.staged) select_stage_rows(sp, unit, z, smem);  // lands under the score (the region is free until then)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -885,12 +921,12 @@ __global__ void __launch_bounds__(kSmallThreads, 1)
     tc_fence_after();
 
     // ---- softmax statistics of the window rows: warp w reads the lanes of quadrant w % 4 (32 tokens) of the
-    // tiles t = w / 4, w / 4 + 2, ...; every column c is a window row
+    // tiles t = w / 4, w / 4 + kSmallWarps / 4, ...; every column c is a window row
     const int quad = warp & 3;
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
     const float cs = p.scale_log2;
     const int nch = GWp / 32;
-    for (int t = warp >> 2; t < T; t += 2) {
+    for (int t = warp >> 2; t < T; t += kSmallWarps / 4) {
         const bool valid = t * kTileTokens + quad * 32 + lane < N;
         for (int ch = 0; ch < nch; ++ch) {
             float v[32];
@@ -909,7 +945,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1)
         row_m[r] = m * cs;
     }
     __syncthreads();
-    for (int t = warp >> 2; t < T; t += 2) {
+    for (int t = warp >> 2; t < T; t += kSmallWarps / 4) {
         const bool valid = t * kTileTokens + quad * 32 + lane < N;
         for (int ch = 0; ch < nch; ++ch) {
             float v[32];
@@ -932,7 +968,7 @@ __global__ void __launch_bounds__(kSmallThreads, 1)
     const SelLayout SL = sel_layout(N, sp.K, 1, true);
     float* a_s = reinterpret_cast<float*>(smem + SL.a_off);
     float* attn_out = p.attn ? p.attn + (static_cast<int64_t>(z) * sp.units + unit) * N : nullptr;
-    for (int t = warp >> 2; t < T; t += 2) {
+    for (int t = warp >> 2; t < T; t += kSmallWarps / 4) {
         const int token = t * kTileTokens + quad * 32 + lane;
         float acc = 0.f, head_sum = 0.f;
         int head_end = p.head_rows;

@@ -830,3 +830,43 @@ def test_bounded_wait_runs_out_and_the_host_reads_its_site():
     assert code & 0x80000000 and (code & 0xFFFF) == V.VASE_SITE_SELF_TEST
     assert cache.check_device_error() == (0, 0)  # read and cleared
     _run_layer(SMALL, cache=cache)
+
+
+# Ties in the selection go to the lower slot: R_V over equal value magnitudes, the sampled set (noise off) over
+# equal keys.  Value rows are drawn from three distinct rows and three quarters of the key rows are one row, so
+# both thresholds fall inside runs of bit-identical scores.  The kept set must be exactly the rule applied to the
+# GPU's own scores (its debug outputs): on the fused small-unit kernel (rank count), the selection kernel's rank
+# count (K = 256) and its radix select (K = 1024).
+@pytest.mark.parametrize("K,B,batch", [(256, 64, 2), (256, 64, 24), (1024, 64, 24)])
+def test_selection_ties_go_to_the_lower_slot(K, B, batch):
+    wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=16, num_q_heads=16, num_kv_heads=8, batch=batch,
+                  num_layers=1)
+    N = K + B
+    st = W.layer_state(wl, 3, 0, 0, "dense")
+    rng = np.random.default_rng(11)
+    for s in range(batch):
+        for h in range(wl.num_kv_heads):
+            rows = st["v_bits"][s, h, rng.integers(0, N, size=3)].copy()
+            st["v_bits"][s, h] = rows[rng.integers(0, 3, size=N)]
+            st["k_bits"][s, h, : 3 * N // 4] = st["k_bits"][s, h, 0]
+    cache = _cache(wl, 1, stochastic=False)
+    PU.upload_layer(cache, 0, st, 0)
+    assert cache.evict(0) == 0
+    status, code = cache.check_device_error()
+    assert status == 0, f"device error word {code:#x}"
+    got = PU.download(cache, 0)
+    n_v = K // 4
+    m = K - n_v - B
+    tied_v = tied_k = 0
+    for u in range(batch * wl.num_kv_heads):
+        vm = np.asarray(got["value_score"][u][:K], dtype=np.float32)  # the magnitudes the kernel ranked
+        order = sorted(range(K), key=lambda i: (-vm[i], i))
+        r_v = set(order[:n_v])
+        key = np.asarray(got["key"][u][:K], dtype=np.float32)
+        cand = [i for i in range(K) if i not in r_v]
+        korder = sorted(cand, key=lambda i: (-key[i], i))
+        kept = sorted(r_v | set(korder[:m]) | set(range(K, N)))
+        assert got["src"][u].tolist() == kept, f"unit {u}: kept set differs from the lower-slot tie rule"
+        tied_v += int(np.sum(vm == vm[order[n_v - 1]]) > 1)
+        tied_k += int(np.sum(key[cand] == key[korder[m - 1]]) > 1)
+    assert tied_v > 0 and tied_k > 0, (tied_v, tied_k)

@@ -276,17 +276,17 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
     __syncthreads();
 }
 
-// The same selection as radix_top_k for n <= kT candidates, by rank: slot i is taken when fewer than k slots
-// outrank it (a larger key, or an equal key at a lower slot).  Each candidate's count is split over P = 1, 2 or 4
-// neighbouring threads (as many as kT / n allows): part p compares against the groups of four keys g with
-// g % P == p, read as broadcasts (the parts of a warp read neighbouring 16-byte groups, so different banks), and
-// the parts' counts are summed by shuffles.  Groups wholly below i count keys >= x, groups wholly above it keys
-// > x (one comparison per key); only i's own group tests the slot order.  No histogram passes.  Ends with a
-// barrier.
-template <int kT>
-__device__ void rank_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, uint8_t flag) {
-    const int P = 4 * n <= kT ? 4 : (2 * n <= kT ? 2 : 1);
-    const int i = threadIdx.x / P, part = threadIdx.x - i * P;
+// The same selection as radix_top_k for n candidates, by rank, by a team of nt >= n threads (t = 0 .. nt - 1,
+// whole warps): slot i is taken when fewer than k slots outrank it (a larger key, or an equal key at a lower slot).
+// Each candidate's count is split over P = 1, 2 or 4 neighbouring threads (as many as nt / n allows): part p
+// compares against the groups of four keys g with g % P == p, read as broadcasts (the parts of a warp read
+// neighbouring 16-byte groups, so different banks), and the parts' counts are summed by shuffles.  Groups wholly
+// below i count keys >= x, groups wholly above it keys > x (one comparison per key); only i's own group tests
+// the slot order.  No histogram passes and no barrier (rank_top_k: the whole block, then a barrier).
+__device__ __forceinline__ void rank_top_k_team(const uint32_t* ord, int n, int k, uint8_t* flags, uint8_t flag,
+                                                int t, int nt) {
+    const int P = 4 * n <= nt ? 4 : (2 * n <= nt ? 2 : 1);
+    const int i = t / P, part = t - i * P;
     int rank = 0;
     uint32_t x = 0;
     const bool live = k > 0 && i < n;
@@ -316,6 +316,11 @@ __device__ void rank_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, ui
     // the parts of a candidate are P neighbouring lanes of one warp (P divides 32); all lanes take part
     for (int o = 1; o < P; o <<= 1) rank += __shfl_xor_sync(0xffffffffu, rank, o);
     if (live && part == 0 && rank < k) flags[i] |= flag;
+}
+
+template <int kT>
+__device__ void rank_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, uint8_t flag) {
+    rank_top_k_team(ord, n, k, flags, flag, threadIdx.x, kT);
     __syncthreads();
 }
 
@@ -333,22 +338,26 @@ __device__ __forceinline__ void top_k_select(const uint32_t* ord, int n, int k, 
 // (exponential race); with stochastic = 0 the key is the pooled score itself
 // (Sec. 4.1).  DKV: the K - B largest leverage products.  Writes the ascending
 // list of kept slots.
-// Asynchronous copy of `count` 32-bit words from global to shared memory by the whole block, in 16-byte
-// pieces when both ends allow it; completion by cp_async_wait_all().
-__device__ __forceinline__ void cp_async_words(void* smem_dst, const void* gsrc, int count) {
+// Asynchronous copy of `count` 32-bit words from global to shared memory by the whole block (or by the team of
+// threads t = 0 .. nt - 1), in 16-byte pieces when both ends allow it; completion by cp_async_wait_all().
+__device__ __forceinline__ void cp_async_words(void* smem_dst, const void* gsrc, int count, int t = -1, int nt = 0) {
+    if (t < 0) {  // the whole block
+        t = threadIdx.x;
+        nt = blockDim.x;
+    }
     const bool vec = ((reinterpret_cast<uintptr_t>(gsrc) | smem_u32(smem_dst)) & 15u) == 0;
     if (vec) {
         const int n4 = count >> 2;
-        for (int i = threadIdx.x; i < n4; i += blockDim.x)
+        for (int i = t; i < n4; i += nt)
             asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst) + 16u * i),
                          "l"(static_cast<const uint8_t*>(gsrc) + 16 * i)
                          : "memory");
-        for (int i = 4 * n4 + threadIdx.x; i < count; i += blockDim.x)
+        for (int i = 4 * n4 + t; i < count; i += nt)
             asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(smem_dst) + 4u * i),
                          "l"(static_cast<const uint8_t*>(gsrc) + 4 * i)
                          : "memory");
     } else {
-        for (int i = threadIdx.x; i < count; i += blockDim.x)
+        for (int i = t; i < count; i += nt)
             asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(smem_dst) + 4u * i),
                          "l"(static_cast<const uint8_t*>(gsrc) + 4 * i)
                          : "memory");
@@ -492,20 +501,64 @@ __device__ void gather_rows(uint8_t* base, const int32_t* src, int j_first, int 
 // The staged value magnitudes and positions of one unit, requested into the selection's shared-memory layout
 // (completion by cp_async_wait_all, which select_unit runs): the fused small-unit eviction issues them before
 // its window score, so that their memory latency passes under the score.
-__device__ __forceinline__ void select_stage_rows(const SelectParams& p, int unit, int z, uint8_t* smem_raw) {
+__device__ __forceinline__ void select_stage_rows(const SelectParams& p, int unit, int z, uint8_t* smem_raw,
+                                                  int t = -1, int nt = 0) {
     const int N = p.N;
     const SelLayout Ly = sel_layout(N, p.K, p.n_parts, true);
     const int layer = p.batch.layer[z];
     const int64_t base = static_cast<int64_t>(layer) * p.units * N + static_cast<int64_t>(unit) * N;
-    cp_async_words(smem_raw + Ly.vm_off, p.vmag + base, N);
-    cp_async_words(smem_raw + Ly.pos_off, p.pos + base, N);
+    cp_async_words(smem_raw + Ly.vm_off, p.vmag + base, N, t, nt);
+    cp_async_words(smem_raw + Ly.pos_off, p.pos + base, N, t, nt);
+}
+
+// The reservation key of slot i (orderable; the N_v largest are R_V): its value magnitude vm (Eq. (5), Sec. 3.1),
+// or with random reservation a Philox uniform keyed by the slot's position, the round and the unit.
+__device__ __forceinline__ uint32_t reserve_ord(const SelectParams& p, int layer, int rnd, int unit, float vm,
+                                                int32_t pi) {
+    if (p.reserve_random) {  // the N_v largest reservation uniforms: a uniformly random N_v-subset
+        const uint32_t c2_res = static_cast<uint32_t>(layer) | (kTagReserve << 24);
+        const Philox4 w = philox4x32_10(
+            Philox4{static_cast<uint32_t>(pi), static_cast<uint32_t>(rnd), c2_res, static_cast<uint32_t>(unit)},
+            p.seed_lo, p.seed_hi);
+        return (w.x >> 9) + 1u;
+    }
+    return __float_as_uint(vm) + 1u;
+}
+
+// R_V of one AttnV unit (the N_v largest reservation keys among the slots below K, ties to the lower slot) by a
+// team of threads t = 0 .. nt - 1 (whole warps, K <= nt, using named barrier bar_id) while the rest of the block
+// does other work, on inputs the team itself staged (select_stage_rows with the same team): the flags cleared,
+// the keys, then the rank count.  select_unit(..., rv_ready = true) then skips these steps; the caller orders
+// the two with a block barrier.
+__device__ void select_reserve_team(const SelectParams& p, int unit, int z, uint8_t* smem_raw, int t, int nt,
+                                    uint32_t bar_id) {
+    const int N = p.N, K = p.K;
+    const SelLayout Ly = sel_layout(N, K, p.n_parts, true);
+    const float* vm_s = reinterpret_cast<const float*>(smem_raw + Ly.vm_off);
+    const int32_t* pos_s = reinterpret_cast<const int32_t*>(smem_raw + Ly.pos_off);
+    uint32_t* ord = reinterpret_cast<uint32_t*>(smem_raw + Ly.ord_off);
+    uint8_t* flags = smem_raw + Ly.flag_off;
+    const int layer = p.batch.layer[z], rnd = p.batch.rnd[z];
+    float* const vscore_dbg =
+        p.vscore_dbg ? p.vscore_dbg + (static_cast<int64_t>(z) * p.units + unit) * N : nullptr;
+    cp_async_wait_all();
+    named_bar(bar_id, static_cast<uint32_t>(nt));
+    for (int i = t; i < N; i += nt) flags[i] = 0;
+    for (int i = t; i < K; i += nt) {
+        const float vm = vm_s[i];
+        ord[i] = reserve_ord(p, layer, rnd, unit, vm, p.reserve_random ? pos_s[i] : 0);
+        if (vscore_dbg) vscore_dbg[i] = vm;
+    }
+    named_bar(bar_id, static_cast<uint32_t>(nt));
+    rank_top_k_team(ord, K, p.n_v, flags, kFlagValue, t, nt);
 }
 
 // The body is select_unit, which the fused small-unit eviction (evict_small_kernel) runs too, on window scores it
 // has already written to shared memory (a_ready: the staging skips them; one part).
 template <int kT>
 __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int z, uint8_t* smem_raw, SelShared& sh,
-                                            bool a_ready, uint4* gbuf = nullptr, int gbuf_rows = 0) {
+                                            bool a_ready, uint4* gbuf = nullptr, int gbuf_rows = 0,
+                                            bool rv_ready = false) {
     const int N = p.N, K = p.K;
     const bool staged = p.staged != 0;
     const SelLayout Ly = sel_layout(N, K, p.n_parts, staged);
@@ -549,7 +602,8 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
         cp_async_words(vm_s, vmag + base, N);
         cp_async_words(pos_s, pos + base, N);
     }
-    for (int i = tid; i < N; i += kT) flags[i] = 0;
+    if (!rv_ready)
+        for (int i = tid; i < N; i += kT) flags[i] = 0;
     if (tid == 0) sh.first_evicted = K;
     if (staged) {
         cp_async_wait_all();
@@ -579,22 +633,16 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
             __syncthreads();
             for (int i = tid; i < N; i += kT) const_cast<float*>(attn)[base + i] = a_s[i];
         }
-        const uint32_t c2_res = static_cast<uint32_t>(layer) | (kTagReserve << 24);
-        for (int i = tid; i < K; i += kT) {
-            const float vm = staged ? vm_s[i] : vmag[base + i];
-            if (p.reserve_random) {  // the N_v largest reservation uniforms: a uniformly random N_v-subset
-                const int32_t pi = staged ? pos_s[i] : pos[base + i];
-                const Philox4 w = philox4x32_10(
-                    Philox4{static_cast<uint32_t>(pi), static_cast<uint32_t>(rnd), c2_res, static_cast<uint32_t>(unit)},
-                    p.seed_lo, p.seed_hi);
-                ord[i] = (w.x >> 9) + 1u;
-            } else {
-                ord[i] = __float_as_uint(vm) + 1u;
+        if (!rv_ready) {  // (otherwise select_reserve_team has set the R_V flags)
+            for (int i = tid; i < K; i += kT) {
+                const float vm = staged ? vm_s[i] : vmag[base + i];
+                const int32_t pi = p.reserve_random ? (staged ? pos_s[i] : pos[base + i]) : 0;
+                ord[i] = reserve_ord(p, layer, rnd, unit, vm, pi);
+                if (vscore_dbg) vscore_dbg[base + i] = vm;
             }
-            if (vscore_dbg) vscore_dbg[base + i] = vm;
+            __syncthreads();
+            top_k_select<kT>(ord, K, p.n_v, flags, kFlagValue, kseg_lo, kseg_hi, sh);
         }
-        __syncthreads();
-        top_k_select<kT>(ord, K, p.n_v, flags, kFlagValue, kseg_lo, kseg_hi, sh);
         // keys over the candidates C
         const int h = p.pool / 2;
         const float inv_pool = 1.0f / static_cast<float>(p.pool);
@@ -854,7 +902,15 @@ __global__ void __launch_bounds__(kSmallThreads, 1)
         tmem_alloc(tmem_slot, static_cast<uint32_t>(p.tmem_cols));
         tmem_relinquish();
     }
-    if (sp.staged) select_stage_rows(sp, unit, z, smem);  // lands under the score (the region is free until then)
+    // The selection's staged inputs land under the score (their region is free until then).  Where K fits the
+    // rank count of warps 1.., those warps also rank R_V (it needs only the value magnitudes) while thread 0
+    // issues the loads and products.
+    constexpr int kTeam = kSmallThreads - 32;
+    const bool rv_early = sp.staged && sp.variant == 0 && sp.K <= kTeam;
+    if (sp.staged) {
+        if (!rv_early) select_stage_rows(sp, unit, z, smem);
+        else if (warp > 0) select_stage_rows(sp, unit, z, smem, tid - 32, kTeam);
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -915,6 +971,8 @@ __global__ void __launch_bounds__(kSmallThreads, 1)
         if (!q_ok) mbar_wait(q_full, 0, sp.err, kErrSmallQ);
         for (int t = landed; t < issued && !ok; ++t) mbar_wait(&k_full[t % S], (t / S) & 1, sp.err, kErrSmallKFull);
         if (!ok) *loads_ok = 0u;
+    } else if (rv_early && warp > 0) {
+        select_reserve_team(sp, unit, z, smem, tid - 32, kTeam, 1);
     }
     __syncwarp();
     if (!mbar_wait(all_done, 0, sp.err, kErrSmallDone)) atomicAnd(const_cast<uint32_t*>(loads_ok), 0u);
@@ -1019,7 +1077,8 @@ __global__ void __launch_bounds__(kSmallThreads, 1)
         return;
     }
     // ---- selection and gather on the scores just written (the selection's buffers sit below the score's)
-    select_unit<kSmallThreads>(sp, unit, z, smem, sh, true, reinterpret_cast<uint4*>(smem + Ly.q_off), sp.K);
+    select_unit<kSmallThreads>(sp, unit, z, smem, sh, true, reinterpret_cast<uint4*>(smem + Ly.q_off), sp.K,
+                               rv_early);
 }
 
 

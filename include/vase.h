@@ -210,6 +210,18 @@ int vase_evict(vase_ctx* ctx, int32_t layer, void* stream);
  * or a negative error. */
 int vase_evict_all(vase_ctx* ctx, void* stream);
 
+/* One whole step of the periodic eviction (Sec. 2): vase_append_all_strided of
+ * n_tokens decode steps (arguments, layout, checks and errors as there), then
+ * vase_evict_all, with the same results.  Where the append makes every layer full
+ * and the eviction of all of them fits one wave of the fused small-unit kernel
+ * (AttnV, bf16 values, one CTA per unit), both run in that kernel's one launch:
+ * each CTA appends its unit's key, value and window-query rows, then scores,
+ * selects and compacts the unit.  Returns the number of layers evicted (>= 0) or
+ * a negative error.  If the fused launch itself fails (VASE_ERR_CUDA) the layers'
+ * states already count the append. */
+int vase_append_evict_all(vase_ctx* ctx, const void* q, const void* k, const void* v, int32_t n_tokens,
+                          int64_t q_layer_stride, int64_t kv_layer_stride, void* stream);
+
 /* The value magnitude (Range, L2 or Var of the value row, Eq. (5) / App. A) of every cached
  * token is computed once, by the append that writes the row, and kept per slot in
  * value_scores; the AttnV eviction reads it instead of the V cache.  A caller that writes

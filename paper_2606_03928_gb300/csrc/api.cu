@@ -621,8 +621,9 @@ namespace {
 
 // Appends n_tokens to each layer of `layers` in one launch; the inputs of consecutive layer slots are q_stride
 // and kv_stride bytes apart (0: packed, one slot's [n][b][H][d] after the other).
-int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void* q, const void* k, const void* v,
-                 int32_t n_tokens, cudaStream_t stream, int64_t q_stride = 0, int64_t kv_stride = 0) {
+// Checks of an append's arguments (the same for every append entry point); VASE_OK or the failure.
+int check_append(vase_ctx* ctx, const int32_t* layers, int n_layers, const void* q, const void* k, const void* v,
+                 int32_t n_tokens, int64_t q_stride, int64_t kv_stride) {
     if (n_tokens < 1) return fail(ctx, VASE_ERR_INVALID, "n_tokens must be >= 1");
     if (!q || !k || !v) return fail(ctx, VASE_ERR_INVALID, "null input");
     if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16))
@@ -632,38 +633,66 @@ int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void*
     for (int z = 0; z < n_layers; ++z)
         if (ctx->layers[layers[z]].fill + n_tokens > ctx->plan.N)
             return fail(ctx, VASE_ERR_FULL, "append would exceed K + B slots");
+    return VASE_OK;
+}
+
+// The append kernel's parameter block for layers[z0 .. z0 + nz - 1] (inputs of layer slot z at q + z * q_stride and
+// k, v + z * kv_stride; a stride of 0 means packed), from the layers' states before the append.
+AppendParams append_params(vase_ctx* ctx, const int32_t* layers, int z0, int nz, const void* q, const void* k,
+                           const void* v, int32_t n_tokens, int64_t q_stride, int64_t kv_stride) {
     const vase_config& c = ctx->cfg;
     const size_t q_slot = q_stride > 0 ? static_cast<size_t>(q_stride) / 16
                                        : static_cast<size_t>(n_tokens) * c.batch * c.num_q_heads * kVecPerRow;
     const size_t kv_slot = kv_stride > 0 ? static_cast<size_t>(kv_stride) / 16
                                          : static_cast<size_t>(n_tokens) * c.batch * c.num_kv_heads * kVecPerRow;
+    AppendParams p{};
+    p.q = static_cast<const uint4*>(q) + z0 * q_slot;
+    p.k = static_cast<const uint4*>(k) + z0 * kv_slot;
+    p.v = static_cast<const uint4*>(v) + z0 * kv_slot;
+    p.q_stride = static_cast<int64_t>(q_slot);
+    p.kv_stride = static_cast<int64_t>(kv_slot);
+    p.qwin = static_cast<uint4*>(ctx->bufs.q_window);
+    p.kc = static_cast<uint4*>(ctx->bufs.k_cache);
+    p.vc = ctx->plan.store ? nullptr : static_cast<uint4*>(ctx->bufs.v_cache);  // store: values go below
+    p.pos = ctx->bufs.positions;
+    p.vmag = ctx->bufs.value_scores;
+    p.kind = c.value_score;
+    p.n = n_tokens;
+    p.b = c.batch;
+    p.Hq = c.num_q_heads;
+    p.Hkv = c.num_kv_heads;
+    p.W = c.window;
+    p.N = ctx->plan.N;
+    for (int z = 0; z < nz; ++z) {
+        const vase_layer_state& st = ctx->layers[layers[z0 + z]];
+        p.layer[z] = layers[z0 + z];
+        p.fill[z] = st.fill;
+        p.next_pos[z] = st.next_position;
+        p.q_ring[z] = static_cast<int32_t>(st.queries_seen % c.window);
+    }
+    return p;
+}
+
+// The layers' states after an append of n_tokens; true when one of them is full (an eviction is due).
+bool advance_after_append(vase_ctx* ctx, const int32_t* layers, int n_layers, int32_t n_tokens) {
+    bool due = false;
+    for (int z = 0; z < n_layers; ++z) {
+        vase_layer_state& st = ctx->layers[layers[z]];
+        st.fill += n_tokens;
+        st.next_position += n_tokens;
+        st.queries_seen += n_tokens;
+        due |= st.fill == ctx->plan.N;
+    }
+    return due;
+}
+
+int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void* q, const void* k, const void* v,
+                 int32_t n_tokens, cudaStream_t stream, int64_t q_stride = 0, int64_t kv_stride = 0) {
+    const int chk = check_append(ctx, layers, n_layers, q, k, v, n_tokens, q_stride, kv_stride);
+    if (chk != VASE_OK) return chk;
     for (int z0 = 0; z0 < n_layers; z0 += kMaxLayerBatch) {
         const int nz = n_layers - z0 < kMaxLayerBatch ? n_layers - z0 : kMaxLayerBatch;
-        AppendParams p{};
-        p.q = static_cast<const uint4*>(q) + z0 * q_slot;
-        p.k = static_cast<const uint4*>(k) + z0 * kv_slot;
-        p.v = static_cast<const uint4*>(v) + z0 * kv_slot;
-        p.q_stride = static_cast<int64_t>(q_slot);
-        p.kv_stride = static_cast<int64_t>(kv_slot);
-        p.qwin = static_cast<uint4*>(ctx->bufs.q_window);
-        p.kc = static_cast<uint4*>(ctx->bufs.k_cache);
-        p.vc = ctx->plan.store ? nullptr : static_cast<uint4*>(ctx->bufs.v_cache);  // store: values go below
-        p.pos = ctx->bufs.positions;
-        p.vmag = ctx->bufs.value_scores;
-        p.kind = c.value_score;
-        p.n = n_tokens;
-        p.b = c.batch;
-        p.Hq = c.num_q_heads;
-        p.Hkv = c.num_kv_heads;
-        p.W = c.window;
-        p.N = ctx->plan.N;
-        for (int z = 0; z < nz; ++z) {
-            const vase_layer_state& st = ctx->layers[layers[z0 + z]];
-            p.layer[z] = layers[z0 + z];
-            p.fill[z] = st.fill;
-            p.next_pos[z] = st.next_position;
-            p.q_ring[z] = static_cast<int32_t>(st.queries_seen % c.window);
-        }
+        const AppendParams p = append_params(ctx, layers, z0, nz, q, k, v, n_tokens, q_stride, kv_stride);
         cudaError_t e = timed_launch(ctx, VASE_KERNEL_APPEND, stream, [&] { return launch_append(p, nz, stream); });
         if (e != cudaSuccess) return cuda_fail(ctx, e, "append launch");
         ctx->launches += 1;
@@ -687,15 +716,7 @@ int append_batch(vase_ctx* ctx, const int32_t* layers, int n_layers, const void*
             ctx->launches += 1;
         }
     }
-    bool due = false;
-    for (int z = 0; z < n_layers; ++z) {
-        vase_layer_state& st = ctx->layers[layers[z]];
-        st.fill += n_tokens;
-        st.next_position += n_tokens;
-        st.queries_seen += n_tokens;
-        due |= st.fill == ctx->plan.N;
-    }
-    return due ? VASE_EVICT_DUE : VASE_OK;
+    return advance_after_append(ctx, layers, n_layers, n_tokens) ? VASE_EVICT_DUE : VASE_OK;
 }
 
 LayerBatch make_batch(vase_ctx* ctx, const int32_t* layers, int nz) {
@@ -746,8 +767,14 @@ void fill_select_params(vase_ctx* ctx, const LayerBatch& batch, float* attn, flo
     sel.err = err;
 }
 
-// One eviction step for up to kMaxLayerBatch full layers: every kernel covers all of them in one launch.
-int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
+// True when a batched eviction of nz layers runs the fused small-unit kernel: every unit of every layer in one
+// wave, one CTA each, and units small enough for it.
+bool fused_small(const Plan& P, int nz) { return P.small_ok && static_cast<long>(P.units) * nz <= P.num_sms; }
+
+// One eviction step for up to kMaxLayerBatch full layers: every kernel covers all of them in one launch.  With
+// fused_append (only where fused_small holds) the fused kernel first appends the step's rows of every unit.
+int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s,
+                const AppendParams* fused_append = nullptr) {
     const Plan& P = ctx->plan;
     const vase_config& c = ctx->cfg;
     const LayerBatch batch = make_batch(ctx, layers, nz);
@@ -764,8 +791,12 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
     fill_select_params(ctx, batch, attn, vscore, src, err, &sel);
     // Launch-bound batches (every unit of every layer in one wave, one CTA each) whose units are small enough for
     // the fused kernel: score, selection and gather in one launch
-    if (P.small_ok && static_cast<long>(P.units) * nz <= P.num_sms) {
+    if (fused_small(P, nz)) {
         SmallEvictParams sm{};
+        if (fused_append) {
+            sm.append = 1;
+            sm.ap = *fused_append;
+        }
         sm.sel = sel;
         sm.sel.n_parts = 1;
         sm.sel.staged = 1;
@@ -796,6 +827,7 @@ int evict_batch(vase_ctx* ctx, const int32_t* layers, int nz, cudaStream_t s) {
         }
         return VASE_OK;
     }
+    if (fused_append) return fail(ctx, VASE_ERR_INVALID, "a fused append needs the fused small-unit eviction");
     if (c.variant == VASE_VARIANT_ATTNV) {
         const ScoreAttnParams sp = score_params(P, c, batch, nz, attn, err);
         if ((e = timed_launch(ctx, VASE_KERNEL_SCORE, s, [&] {
@@ -949,6 +981,32 @@ int vase_evict_all(vase_ctx* ctx, void* stream) {
     }
     ctx->last_batch = done;
     return static_cast<int>(due.size());
+}
+
+int vase_append_evict_all(vase_ctx* ctx, const void* q, const void* k, const void* v, int32_t n_tokens,
+                          int64_t q_layer_stride, int64_t kv_layer_stride, void* stream) {
+    if (!ctx) return VASE_ERR_INVALID;
+    const Plan& P = ctx->plan;
+    const int L = ctx->cfg.num_layers;
+    // one launch where the append makes every layer full and the eviction of all of them is the fused kernel's
+    bool fused = !P.store && L <= P.slots && fused_small(P, L) && n_tokens >= 1;
+    for (int l = 0; l < L && fused; ++l) fused = ctx->layers[l].fill + n_tokens == P.N;
+    if (!fused) {
+        const int r = vase_append_all_strided(ctx, q, k, v, n_tokens, q_layer_stride, kv_layer_stride, stream);
+        if (r < 0) return r;
+        return vase_evict_all(ctx, stream);
+    }
+    if (q_layer_stride <= 0 || kv_layer_stride <= 0) return fail(ctx, VASE_ERR_INVALID, "layer strides must be > 0");
+    std::vector<int32_t> all(static_cast<size_t>(L));
+    for (int32_t l = 0; l < L; ++l) all[l] = l;
+    const int chk = check_append(ctx, all.data(), L, q, k, v, n_tokens, q_layer_stride, kv_layer_stride);
+    if (chk != VASE_OK) return chk;
+    const AppendParams ap = append_params(ctx, all.data(), 0, L, q, k, v, n_tokens, q_layer_stride, kv_layer_stride);
+    advance_after_append(ctx, all.data(), L, n_tokens);
+    const int r = evict_batch(ctx, all.data(), L, static_cast<cudaStream_t>(stream), &ap);
+    if (r != VASE_OK) return r;
+    ctx->last_batch = all;
+    return L;
 }
 
 int vase_refresh_value_scores(vase_ctx* ctx, int32_t layer, void* stream) {

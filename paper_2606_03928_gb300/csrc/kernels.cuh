@@ -193,6 +193,8 @@ struct SmallEvictParams {
     int64_t q_layer_rows;   // window rows per layer
     float scale_log2;       // log2(e) / sqrt(d)
     float* attn;            // [slot][units][N]: the window score, written for the debug view (nullable)
+    int32_t append;         // 1: each CTA first appends its unit's rows of `ap` (the step's append, fused)
+    AppendParams ap;        // the append of every layer slot of the launch (same slot order as sel.batch)
 };
 constexpr int kSmallThreads = 512;
 constexpr int kSmallWarps = kSmallThreads / 32;

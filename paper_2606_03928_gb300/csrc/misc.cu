@@ -859,6 +859,58 @@ __device__ __forceinline__ float ex2_approx(float x) {
     return y;
 }
 
+// The append of one unit (sequence s, KV head h) of layer slot z, the unit's share of what append_kernel does for
+// a whole sequence: the key and value rows of the n new decode steps into slots fill .. fill + n - 1, with their
+// positions and value magnitudes, and the query rows of its G heads for the steps that stay in the window ring
+// (the last W).  A half warp moves one 256-byte row; every thread of the block calls it.
+__device__ void append_unit(const AppendParams& p, int z, int s, int h) {
+    const int layer = p.layer[z], fill = p.fill[z], n = p.n, W = p.W, N = p.N;
+    const int G = p.Hq / p.Hkv;
+    const int64_t unit = (static_cast<int64_t>(layer) * p.b + s) * p.Hkv + h;
+    uint4* const kc = p.kc + unit * N * kVecPerRow;
+    uint4* const vc = p.vc ? p.vc + unit * N * kVecPerRow : nullptr;
+    int32_t* const pos = p.pos + unit * N;
+    float* const vmag = p.vmag + unit * N;
+    uint4* const qwin =
+        p.qwin + ((static_cast<int64_t>(layer) * p.b + s) * p.Hq + static_cast<int64_t>(h) * G) * W * kVecPerRow;
+    const uint4* const qin = p.q + static_cast<int64_t>(z) * p.q_stride;
+    const uint4* const kin = p.k + static_cast<int64_t>(z) * p.kv_stride;
+    const uint4* const vin = p.v + static_cast<int64_t>(z) * p.kv_stride;
+    const int nq = min(n, W);          // steps n - nq .. n - 1 keep their queries
+    const int rows = 2 * n + nq * G;   // key and value rows of every step (alternating), then the query rows
+    // the trip count is the same for every thread of the block, so the half-warp shuffles see full warps
+    for (int e0 = 0; e0 < rows * 16; e0 += blockDim.x) {
+        const int e = e0 + static_cast<int>(threadIdx.x);
+        const int r = e >> 4, seg = e & 15;
+        uint4 val = make_uint4(0, 0, 0, 0);
+        bool is_v = false;
+        int t = 0;
+        if (r < 2 * n) {
+            t = r >> 1;
+            const int64_t row_in = (static_cast<int64_t>(t) * p.b + s) * p.Hkv + h;
+            if ((r & 1) == 0) {
+                kc[static_cast<int64_t>(fill + t) * kVecPerRow + seg] = kin[row_in * kVecPerRow + seg];
+            } else {
+                is_v = true;
+                val = vin[row_in * kVecPerRow + seg];
+                if (vc) vc[static_cast<int64_t>(fill + t) * kVecPerRow + seg] = val;
+            }
+        } else if (r < rows) {
+            const int qi = r - 2 * n;
+            const int g = qi % G;
+            t = n - nq + qi / G;
+            const int slot = (p.q_ring[z] + t) % W;
+            qwin[(static_cast<int64_t>(g) * W + slot) * kVecPerRow + seg] =
+                qin[((static_cast<int64_t>(t) * p.b + s) * p.Hq + static_cast<int64_t>(h) * G + g) * kVecPerRow + seg];
+        }
+        if (__any_sync(0xffffffffu, is_v)) {
+            const float mag = half_warp_value_magnitude(val, p.kind);
+            if (is_v && seg == 0) vmag[fill + t] = mag;
+        }
+    }
+    for (int t = threadIdx.x; t < n; t += blockDim.x) pos[fill + t] = static_cast<int32_t>(p.next_pos[z] + t);
+}
+
 __global__ void __launch_bounds__(kSmallThreads, 1)
     evict_small_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
                        const SmallEvictParams p) {
@@ -901,6 +953,11 @@ __global__ void __launch_bounds__(kSmallThreads, 1)
     if (warp == 0) {
         tmem_alloc(tmem_slot, static_cast<uint32_t>(p.tmem_cols));
         tmem_relinquish();
+    }
+    if (p.append) {  // the step's append of this unit, then every row it wrote is visible to the loads below
+        append_unit(p.ap, z, seq, head);
+        asm volatile("fence.proxy.async.global;" ::: "memory");  // generic writes -> the TMA loads of K and Q
+        __syncthreads();
     }
     // The selection's staged inputs land under the score (their region is free until then).  Where K fits the
     // rank count of warps 1.., those warps also rank R_V (it needs only the value magnitudes) while thread 0

@@ -43,7 +43,7 @@ EXPORTED = [
     "vase_append_all", "vase_append_all_strided", "vase_evict_all", "vase_self_test_wait_timeout", "vase_refresh_value_scores", "vase_evict_static_scratch",
     "vase_decode_attention", "vase_mixed_buffer_sizes", "vase_quantize_values", "vase_decode_attention_mixed",
     "vase_host_staging_bytes", "vase_stage_host_inputs", "vase_append_all_staged", "vase_read_positions_all",
-    "vase_value_store_get",
+    "vase_value_store_get", "vase_append_evict_all",
 ]
 KERNEL_NAMES = ["append", "score_attn", "value_score", "dkv_score", "select_compact", "evict_small", "store_append",
                 "store_evict"]
@@ -119,6 +119,7 @@ def load(path: str = LIB_PATH):
         "vase_self_test_wait_timeout": (ctypes.c_int, [P, P]),
         "vase_evict": (ctypes.c_int, [P, I32, P]),
         "vase_evict_all": (ctypes.c_int, [P, P]),
+        "vase_append_evict_all": (ctypes.c_int, [P, P, P, P, I32, I64, I64, P]),
         "vase_refresh_value_scores": (ctypes.c_int, [P, I32, P]),
         "vase_evict_static_scratch": (ctypes.c_int, [ctypes.POINTER(vase_config), ctypes.POINTER(vase_buffers), I32,
                                                      ctypes.POINTER(vase_layer_state), ctypes.POINTER(U32), P]),
@@ -232,6 +233,12 @@ def vase_evict(ctx, layer, stream=None):
 
 def vase_evict_all(ctx, stream=None):
     return _check(ctx, load().vase_evict_all(ctx, _stream_ptr(stream)), "vase_evict_all")
+
+
+def vase_append_evict_all(ctx, q_ptr, k_ptr, v_ptr, n_tokens, q_layer_stride, kv_layer_stride, stream=None):
+    return _check(ctx, load().vase_append_evict_all(ctx, q_ptr, k_ptr, v_ptr, n_tokens, q_layer_stride,
+                                                    kv_layer_stride, _stream_ptr(stream)),
+                  "vase_append_evict_all")
 
 
 def vase_refresh_value_scores(ctx, layer, stream=None):
@@ -429,6 +436,14 @@ class VaseCache:
     def evict_all(self, stream=None):
         """Evicts every full layer in batched launches; returns how many layers were evicted."""
         return vase_evict_all(self.ctx, stream)
+
+    def append_evict_all(self, q, k, v, stream=None):
+        """One step: q [L, n, b, Hq, d], k/v [L, n, b, Hkv, d] bf16 CUDA tensors appended to every layer, then every
+        full layer evicted (one fused launch where that applies); returns how many layers were evicted."""
+        for t in (q, k, v):
+            assert t.is_cuda and t.dtype == torch.bfloat16 and t.is_contiguous()
+        return vase_append_evict_all(self.ctx, q.data_ptr(), k.data_ptr(), v.data_ptr(), q.shape[1],
+                                     q[0].numel() * 2, k[0].numel() * 2, stream)
 
     def decode_attention(self, layer, q: torch.Tensor, out: torch.Tensor = None, stream=None):
         """Attention output of one decode step over the layer's cached pairs: q [b, Hq, d] bf16 CUDA tensor,

@@ -870,3 +870,48 @@ def test_selection_ties_go_to_the_lower_slot(K, B, batch):
         tied_v += int(np.sum(vm == vm[order[n_v - 1]]) > 1)
         tied_k += int(np.sum(key[cand] == key[korder[m - 1]]) > 1)
     assert tied_v > 0 and tied_k > 0, (tied_v, tied_k)
+
+
+# ----------------------------------------------------------------------------- the fused step (append + eviction)
+
+# vase_append_evict_all is vase_append_all_strided then vase_evict_all: bit-identical caches, positions, value
+# magnitudes, window rings and layer states over chained steps, in one launch per step where every unit of every
+# layer fits one wave of the fused kernel, and as the two calls where it does not (384 units).
+@pytest.mark.parametrize("L,K,B,Wn,Hq,Hkv,batch,kw,fused", [
+    (1, 256, 64, 32, 16, 8, 1, {}, True),                     # the single-layer geometry
+    (2, 200, 40, 16, 32, 8, 2, {"gqa": "max"}, True),         # G = 4, a ragged last tile, GQA max
+    (2, 256, 64, 16, 16, 8, 2, {"reserve": "random"}, True),  # random reservation (keys from positions)
+    (3, 192, 64, 16, 16, 8, 16, {}, False),                   # 384 units: the two calls
+])
+def test_append_evict_all_equals_append_all_then_evict_all(L, K, B, Wn, Hq, Hkv, batch, kw, fused):
+    from paper_2606_03928_gb300 import vase as V
+    wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=Wn, num_q_heads=Hq, num_kv_heads=Hkv, batch=batch,
+                  num_layers=L)
+    a, b = _cache(wl, L, **kw), _cache(wl, L, **kw)
+    dev = a.device
+
+    def inputs(first, n):
+        chunks = [W.stream_chunk(wl, 21, layer, first, n) for layer in range(L)]
+        return [torch.stack([PU.bits_to_bf16_tensor(c[key], dev) for c in chunks])
+                for key in ("q_bits", "k_bits", "v_bits")]
+
+    q, k, v = inputs(0, K)
+    for c in (a, b):
+        c.append_all(q, k, v)
+    for step in range(3):
+        q, k, v = inputs(K + step * B, B)
+        before = a.launch_count()
+        assert a.append_evict_all(q, k, v) == L
+        assert a.launch_count() - before == (1 if fused else 3)
+        b.append_all(q, k, v)
+        assert b.evict_all() == L
+        torch.cuda.synchronize()
+        for c in (a, b):
+            status, code = c.check_device_error()
+            assert status == 0, f"device error word {code:#x}"
+        assert torch.equal(a.k_cache, b.k_cache) and torch.equal(a.v_cache, b.v_cache)
+        assert torch.equal(a.positions, b.positions) and torch.equal(a.q_window, b.q_window)
+        assert torch.equal(a.value_scores[..., :K], b.value_scores[..., :K])
+        for layer in range(L):
+            assert a.layer_state(layer) == b.layer_state(layer)
+            assert a.layer_state(layer)["fill"] == K

@@ -617,9 +617,7 @@ def run_ours(args):
 
     # the oracle pool is started before the first CUDA work of this process
     from paper_2606_03928_gb300 import workloads as Wm
-    wl = Wm.WORKLOADS[args.workload]
-    if args.layers:
-        wl = Wm.shrink(wl, num_layers=args.layers)
+    wl = workload_by_name(Wm, args.workload, args.layers)
     pool = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         pool, cores, n_units = oracle_pool(wl, args.variant)

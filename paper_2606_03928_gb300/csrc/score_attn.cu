@@ -13,7 +13,9 @@
 // swizzle).  Two passes over the tiles, each on the tensor cores:
 //   pass A  S^T = Q K_tile^T (M = 128 window rows, N = 128 tokens): TMEM lane =
 //           window row, so every consumer thread keeps an online (max, sum of
-//           exp2) of its own row with no cross-lane traffic.  Short windows
+//           exp2) of its own row with no cross-lane traffic.  The reference of the
+//           sum is the maximum of the row's first chunk; it is raised only for a
+//           chunk whose sum against it passes 2^64, so most chunks take no maximum.  Short windows
 //           (G*W < 128) are replicated across the 128 lanes and each copy takes
 //           a slice of the tile's tokens.  The per-row statistics are then
 //           merged across copies, warps and (through distributed shared
@@ -489,6 +491,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                                 for (int q = 0; q < 64; ++q)
                                     if (q >= nvalid) v[q] = -INFINITY;
+                            }
+                            // Once the row has a reference m (the maximum of its first chunk), a chunk is summed
+                            // against it with no chunk maximum: (m, l) stays a valid pair as long as no exp2
+                            // overflows, and a sum above 2^64 (or inf) sends the chunk through the exact path below.
+                            if (m != -INFINITY) {
+                                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+                                for (int q = 0; q < 64; q += 4) {
+                                    s0 += ex2(fmaf(v[q], cs, -m));
+                                    s1 += ex2(fmaf(v[q + 1], cs, -m));
+                                    s2 += ex2(fmaf(v[q + 2], cs, -m));
+                                    s3 += ex2(fmaf(v[q + 3], cs, -m));
+                                }
+                                const float sum = (s0 + s1) + (s2 + s3);
+                                if (sum <= 0x1p64f) {
+                                    l += sum;
+                                    continue;
+                                }
                             }
                             float cm0 = v[0], cm1 = v[1], cm2 = v[2], cm3 = v[3];
 #pragma unroll

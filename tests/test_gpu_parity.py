@@ -33,7 +33,8 @@ def _cache(wl, num_layers, variant="attnv", debug=True, **kw):
 
 
 def _run_layer(wl, *, variant="attnv", layer=1, num_layers=2, round_index=3, seed=0, data_seed=0, units=None,
-               debug=True, positions="gapped", cache_kw=None, oracle_kw=None, state_round=None, cache=None):
+               debug=True, positions="gapped", cache_kw=None, oracle_kw=None, state_round=None, cache=None,
+               edit=None):
     """Uploads one layer, evicts it through the C ABI and checks `units` (default all) against the oracle.
 
     round_index is the eviction counter (it keys the noise); state_round (default round_index) draws the data.
@@ -43,6 +44,8 @@ def _run_layer(wl, *, variant="attnv", layer=1, num_layers=2, round_index=3, see
     if cache is None:
         cache = _cache(wl, num_layers, variant=variant, debug=debug, seed=seed, **cache_kw)
     st = W.layer_state(wl, data_seed, layer, round_index if state_round is None else state_round, positions)
+    if edit is not None:
+        edit(st)
     PU.upload_layer(cache, layer, st, round_index)
     other = None
     if num_layers > 1:
@@ -770,6 +773,34 @@ def test_dkv_shared_g_matches_oracle_and_is_shared():
 
 
 # ----------------------------------------------------------------------------- maximum sizes and degenerate cases
+
+def _lift_keys(wl, st, units, alphas=(4.0, 5.0, 8.0)):
+    """Plants key rows far above the rest of a window row's logits: key = alpha * q_r for one window query r
+    of the unit, so that q_r . k / sqrt(d) in log2 units sits about 60 (alpha 4), 80 (5) and 130 (8) above
+    the other keys of that row.  They sit in later tiles than the first, among the candidates."""
+    N, G, Wn = wl.slots, wl.group, wl.window
+    for n, (s, h) in enumerate(units):
+        for i, a in enumerate(alphas):
+            r = (n * 7 + i * 5) % (G * Wn)
+            g, w = divmod(r, Wn)
+            q = O.bf16_bits_to_f64(st["q_bits"][s, h * G + g, w])
+            j = 130 + (70 + i * 397 + n * 131) % (wl.budget_k - 130)  # past the first 128-token tile
+            st["k_bits"][s, h, j] = W.f32_to_bf16_bits(a * q)
+
+
+# The window score sums each row's exponentials against the maximum of the row's first chunk and raises that
+# reference only for a chunk whose sum against it passes 2^64.  Keys planted far above the first chunk make some
+# rows take that path (sums of about 2^60, 2^80 and an overflow to inf); every score, kept set and moved row still
+# follows the oracle.  Geometries: the persistent schedule with replicated 64-row windows, cluster mode with 128
+# rows, and 512 window rows (two 256-column pass-B accumulators).
+@pytest.mark.parametrize("K,B,Wn,Hq,Hkv,batch", [(256, 64, 32, 16, 8, 20), (1024, 128, 32, 32, 8, 2),
+                                                 (1024, 256, 64, 64, 8, 1)])
+def test_window_score_with_keys_far_above_the_first_chunk(K, B, Wn, Hq, Hkv, batch):
+    wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=Wn, num_q_heads=Hq, num_kv_heads=Hkv, batch=batch,
+                  num_layers=2)
+    units = [(0, 0), (0, Hkv - 1), (batch - 1, 3)]
+    _, _, _, flips = _run_layer(wl, units=units, edit=lambda st: _lift_keys(wl, st, units))
+    assert flips <= 2
 
 def test_largest_supported_unit_matches_oracle():
     """K = 16384, B = 256 (N = 16640, inputs read unstaged by the single-CTA selection), one unit, the score

@@ -435,7 +435,8 @@ int vase_profile_collect(vase_ctx* ctx, double* total_ms, int64_t* launches);
  *              by the next call made with a non-NULL device_error, so a caller that passes
  *              NULL on its hot path can ask now and then.
  * Layers needing more scratch than the array holds (256 + (b*Hkv) * (K+B) * 4 * (1 + parts)
- * + (b*Hkv) * K * 4 bytes, parts = 2 when G*W > 256, else 1, each term rounded up to 256)
+ * + (b*Hkv) * K * 4 bytes, parts = 4 when G*W > 256 (2 with GQA max-aggregation and a window
+ * that does not divide 128), else 1, each term rounded up to 256)
  * are rejected with VASE_ERR_UNSUPPORTED before any buffer is looked at; the Qwen3-32B
  * geometry at batch 16 (about 17 MB) is one.  The first call on a device looks up the array's
  * device address (cudaGetSymbolAddress) with that device current; make that first call before

@@ -23,7 +23,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
 struct Plan {
-    int N, units, G, GW, GWp, NB, n_rb, n_rbA, rep, q_rows, q_box, buf_cols, nbuf;
+    int N, units, G, GW, GWp, NB, n_rb, n_rbA, rep, q_rows, q_box, buf_cols, nbuf, cgroups;
     int n_tiles, cluster, stages, stages_p, tmem_cols, n_v, m, num_sms;
     int cluster_for[kMaxLayerBatch + 1];  // CTAs per unit of the score kernel, by layers per launch
     bool persist_for[kMaxLayerBatch + 1]; // one CTA per SM taking several units (interleaved passes)
@@ -104,7 +104,10 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
         return false;
     }
     p.GWp = p.GW <= 256 ? (p.GW + 31) / 32 * 32 : (p.GW + 255) / 256 * 256;
-    p.NB = p.GWp < 256 ? p.GWp : 256;
+    // At 512 window rows four consumer groups each own one 128-column accumulator and one 128-row block, in
+    // both passes (pass B in four parts); GQA max then needs whole query heads per 128-row block.
+    p.cgroups = p.GWp == 512 && (c->gqa_reduce != VASE_GQA_MAX || 128 % c->window == 0) ? 4 : 2;
+    p.NB = p.cgroups == 4 ? 128 : (p.GWp < 256 ? p.GWp : 256);
     p.n_rb = p.GWp / p.NB;
     if (c->gqa_reduce == VASE_GQA_MAX && p.n_rb > 1 && p.NB % c->window) {
         *why = "GQA max-aggregation with G * window > 256 needs window to divide 256";
@@ -139,7 +142,7 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
         for (int C = 1; C <= 16 && C <= p.n_tiles; ++C) {
             const int T = ceil_div(p.n_tiles, C);
             if (ceil_div(p.n_tiles, T) != C) continue;
-            if (score_attn_smem_bytes(p.q_rows, 1, p.n_rbA, p.GWp, C, 2) > kMaxDynSmem) continue;
+            if (score_attn_smem_bytes(p.q_rows, 1, p.n_rbA, p.GWp, C, 2, p.cgroups) > kMaxDynSmem) continue;
             const long ctas = static_cast<long>(p.units) * C * nz;
             const long waves = (ctas + num_sms - 1) / num_sms;
             const long cost = waves * (T + 1);
@@ -160,7 +163,7 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     // items on: batch-1 launches of 288 units); this needs two window-row buffers.
     p.stages_p = 0;
     for (int s = 4; s >= 2; --s) {
-        if (score_attn_smem_bytes(p.q_rows, 2, p.n_rbA, p.GWp, 1, s) <= kMaxDynSmem) {
+        if (score_attn_smem_bytes(p.q_rows, 2, p.n_rbA, p.GWp, 1, s, p.cgroups) <= kMaxDynSmem) {
             p.stages_p = s;
             break;
         }
@@ -177,14 +180,14 @@ bool make_plan_impl(const vase_config* c, int num_sms, Plan* P, const char** why
     p.cluster = c_max > 0 ? c_max : 1;  // shared memory is sized for the largest cluster used
     p.stages = 0;
     for (int s = 6; s >= 2; --s) {
-        if (score_attn_smem_bytes(p.q_rows, 1, p.n_rbA, p.GWp, p.cluster, s) <= kMaxDynSmem) {
+        if (score_attn_smem_bytes(p.q_rows, 1, p.n_rbA, p.GWp, p.cluster, s, p.cgroups) <= kMaxDynSmem) {
             p.stages = s;
             break;
         }
     }
-    p.score_smem = score_attn_smem_bytes(p.q_rows, 1, p.n_rbA, p.GWp, p.cluster, p.stages);
+    p.score_smem = score_attn_smem_bytes(p.q_rows, 1, p.n_rbA, p.GWp, p.cluster, p.stages, p.cgroups);
     if (any_persist) {
-        const size_t sp = score_attn_smem_bytes(p.q_rows, 2, p.n_rbA, p.GWp, 1, p.stages_p);
+        const size_t sp = score_attn_smem_bytes(p.q_rows, 2, p.n_rbA, p.GWp, 1, p.stages_p, p.cgroups);
         if (sp > p.score_smem) p.score_smem = sp;
     }
     if (p.tmem_cols > 256 && p.score_smem < 120 * 1024) p.score_smem = 120 * 1024;  // one CTA per SM owns TMEM
@@ -330,6 +333,7 @@ ScoreAttnParams score_params(const Plan& P, const vase_config& c, const LayerBat
     sp.tiles_per_cta = ceil_div(P.n_tiles, sp.cluster);
     sp.buf_cols = P.buf_cols;
     sp.nbuf = P.nbuf;
+    sp.cgroups = P.cgroups;
     sp.units = P.units;
     sp.tmem_cols = P.tmem_cols;
     sp.Hq = c.num_q_heads;

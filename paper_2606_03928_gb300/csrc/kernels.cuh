@@ -122,6 +122,7 @@ struct ScoreAttnParams {
     int32_t stages;         // tile ring depth
     int32_t buf_cols;       // TMEM columns per accumulator buffer
     int32_t nbuf;           // accumulator buffers in TMEM (2 or 4)
+    int32_t cgroups;        // consumer warpgroups (2, or 4 with one buffer and one row block each)
     int32_t units;          // units per layer
     int32_t tmem_cols;
     int32_t Hq, Hkv, W, G;
@@ -284,7 +285,7 @@ cudaError_t quantize_set_attributes(size_t smem_bytes);
 cudaError_t launch_decode(const CUtensorMap& kmap, const CUtensorMap& vmap, DecodeParams p, size_t smem_bytes,
                           int num_sms, cudaStream_t s);
 
-size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages);
+size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages, int groups);
 size_t dkv_smem_bytes(int stages);
 size_t select_smem_bytes(int N, int K, int n_parts, bool staged);
 size_t select_static_smem_bytes();  // the selection kernel's static shared memory

@@ -24,6 +24,11 @@
 //           token, so each thread accumulates sum_r exp2(s_ri - m'_r) of its token
 //           alone, m'_r = m_r + log2(l_r * G*W) folding the softmax denominator
 //           and the 1/(G*W) mean into the exponent.
+// With 512 window rows (G*W > 256) a tile's products fill all 512 TMEM columns in either
+// pass, so four consumer warpgroups each own one 128-column accumulator and one 128-row
+// block of the window, in both passes (pass B writes four partial scores that the
+// selection adds): a group's next product waits only for that group, and sixteen
+// consumer warps cover the TMEM-load and exp2 latencies that eight left exposed.
 // A single-CTA group that takes several items runs them as phases: phase k
 // interleaves pass B of item k-1 (K re-read from L2, kept there by an
 // evict-last hint on the pass-A read) with pass A of item k (K read from HBM),
@@ -37,9 +42,11 @@ namespace vase {
 
 namespace {
 
-constexpr int kGroups = 2;                      // consumer warpgroups; group g takes the items i with i % 2 == g
-constexpr int kConsumers = 128 * kGroups;
-constexpr int kThreads = kConsumers + 96;       // + a TMA warp and two MMA-issue warps (even / odd items)
+// Consumer warpgroups: kG = 2 (group g takes the items i with i % 2 == g, alternating over the accumulator
+// buffers) or kG = 4 (one buffer each: at 512 window rows a tile's products are four 128 x 128 items in both
+// passes, and group g always takes row block g).  Plus a TMA warp and two MMA-issue warps (even / odd items).
+constexpr int kMaxGroups = 4;
+__host__ __device__ constexpr int score_threads(int groups) { return 128 * groups + 96; }
 constexpr int kMaxBufs = 4;
 constexpr int kMaxStages = 8;
 constexpr uint32_t kTileBytes = kTileTokens * kRowBytes;  // 32 KB: two 64-column panels of 128 rows
@@ -50,7 +57,7 @@ struct ScoreSmem {
 };
 
 __host__ __device__ inline ScoreSmem score_layout(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster,
-                                                   int stages, int stage_bytes) {
+                                                   int stages, int stage_bytes, int groups) {
     ScoreSmem L;
     uint32_t o = 0;
     L.q_off = o;
@@ -58,14 +65,14 @@ __host__ __device__ inline ScoreSmem score_layout(int q_rows, int q_bufs, int n_
     L.k_off = o;
     o += static_cast<uint32_t>(stages) * stage_bytes;
     L.bar_off = o;
-    o += 8 * (6 + 3 * stages + 2 * kMaxBufs);
+    o += 8 * (2 + 2 * kMaxGroups + 3 * stages + 2 * kMaxBufs);
     o = (o + 15u) & ~15u;
     L.slot_off = o;
     o += 16;
     L.pm_off = o;
-    o += 4u * n_rbA * kConsumers;  // [group][sub][128 lanes]
+    o += 4u * n_rbA * 128 * groups;  // [group][sub][128 lanes]
     L.pl_off = o;
-    o += 4u * n_rbA * kConsumers;
+    o += 4u * n_rbA * 128 * groups;
     L.xm_off = o;
     o += 4u * cluster * GWp;
     L.xl_off = o;
@@ -89,6 +96,49 @@ __device__ __forceinline__ void merge_ml(float& m, float& l, float m2, float l2)
     if (mn == -INFINITY) return;
     l = l * exp2f(m - mn) + l2 * exp2f(m2 - mn);
     m = mn;
+}
+
+// One chunk of a row's online (max, sum of exp2) in pass A.  Once the row has a reference m (the maximum of
+// its first chunk), a chunk is summed against it with no chunk maximum: (m, l) stays a valid pair as long as
+// no exp2 overflows, and a sum above 2^64 (or inf) sends the chunk through the exact path, which raises m.
+template <int CW>
+__device__ __forceinline__ void row_stats_chunk(const float (&v)[CW], float cs, float& m, float& l) {
+    if (m != -INFINITY) {
+        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+        for (int q = 0; q < CW; q += 4) {
+            s0 += ex2(fmaf(v[q], cs, -m));
+            s1 += ex2(fmaf(v[q + 1], cs, -m));
+            s2 += ex2(fmaf(v[q + 2], cs, -m));
+            s3 += ex2(fmaf(v[q + 3], cs, -m));
+        }
+        const float sum = (s0 + s1) + (s2 + s3);
+        if (sum <= 0x1p64f) {
+            l += sum;
+            return;
+        }
+    }
+    float cm0 = v[0], cm1 = v[1], cm2 = v[2], cm3 = v[3];
+#pragma unroll
+    for (int q = 4; q < CW; q += 4) {
+        cm0 = fmaxf(cm0, v[q]);
+        cm1 = fmaxf(cm1, v[q + 1]);
+        cm2 = fmaxf(cm2, v[q + 2]);
+        cm3 = fmaxf(cm3, v[q + 3]);
+    }
+    const float mn = fmaxf(m, fmaxf(fmaxf(cm0, cm1), fmaxf(cm2, cm3)) * cs);
+    if (mn != -INFINITY) {
+        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+        for (int q = 0; q < CW; q += 4) {
+            s0 += ex2(fmaf(v[q], cs, -mn));
+            s1 += ex2(fmaf(v[q + 1], cs, -mn));
+            s2 += ex2(fmaf(v[q + 2], cs, -mn));
+            s3 += ex2(fmaf(v[q + 3], cs, -mn));
+        }
+        l = l * ex2(m - mn) + ((s0 + s1) + (s2 + s3));
+        m = mn;
+    }
 }
 
 // Work item w of the launch: layer slot w / units, unit w % units.
@@ -141,21 +191,23 @@ __device__ __forceinline__ bool phase_tile(int t, int nA, int nB, int lead, int&
 // the buffer is released as soon as the item's last TMEM load has landed; with four, each group already has a
 // second buffer in flight and the release follows the item's arithmetic (measured faster there).  A template
 // argument so that each form compiles to its own loop.
-template <bool kHeadMax, bool kEarly>
-__global__ void __launch_bounds__(kThreads, 1)
+template <bool kHeadMax, bool kEarly, int kG>
+__global__ void __launch_bounds__(score_threads(kG), 1)
     score_attn_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap qmap,
                       const ScoreAttnParams p) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     constexpr int stage_bytes = kTileBytes;
-    const ScoreSmem Ly = score_layout(p.q_rows, p.q_bufs, p.n_rbA, p.GWp, p.cluster, p.stages, stage_bytes);
+    constexpr int kConsumers = 128 * kG;
+    constexpr int kThreads = score_threads(kG);
+    const ScoreSmem Ly = score_layout(p.q_rows, p.q_bufs, p.n_rbA, p.GWp, p.cluster, p.stages, stage_bytes, kG);
 
     uint8_t* q_s = smem + Ly.q_off;
     uint8_t* st_s = smem + Ly.k_off;
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Ly.bar_off);
     uint64_t* q_full = bars;                      // [2]
-    uint64_t* q_empty = bars + 2;                 // [2][group]
-    uint64_t* k_full = bars + 6;                  // [stages]
+    uint64_t* q_empty = bars + 2;                 // [2][kG]
+    uint64_t* k_full = bars + 2 + 2 * kMaxGroups; // [stages]
     uint64_t* k_empty = k_full + p.stages;        // [stages][group]
     uint64_t* t_full = k_empty + 2 * p.stages;    // [nbuf]
     uint64_t* t_empty = t_full + kMaxBufs;        // [nbuf]
@@ -204,8 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // seen the last of its items that read it); the TMA warp waits for the owners of each.
         for (int b = 0; b < 2; ++b) {
             mbar_init(&q_full[b], 1);
-            mbar_init(&q_empty[2 * b], 128);
-            mbar_init(&q_empty[2 * b + 1], 128);
+            for (int g = 0; g < kG; ++g) mbar_init(&q_empty[kG * b + g], 128);
         }
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&k_full[s], 1);
@@ -244,8 +295,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_prefetch_desc(&qmap);
             const uint64_t keep = l2_policy_evict_last();   // pass-A reads: read again by pass B
             const uint64_t drop = l2_policy_evict_first();  // pass-B reads: last use
-            // Owner groups (bit g = consumer group g) of the tile in each stage and of the pass-B items that read
-            // each window-row buffer, and the parity of the next phase of every per-group empty barrier.
+            // Owners of the tile in each stage (bit x = MMA warp x, two bits per stage) and of the pass-B items that
+            // read each window-row buffer (bit g = consumer group g, kG bits per buffer), and the parity of the next
+            // phase of every per-owner empty barrier.
             uint32_t slot_owners = 0, kpar = 0, q_owners = 0, qpar = 0;
             int slot_item[kMaxStages];  // item of the tile in each stage (stage release by MMA completion)
             int ld = 0, g = 0, st_pos = 0;
@@ -260,7 +312,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const bool isA = phase_tile(t, nA, nB, lead, j);
                     const int n_sub = isA ? n_rbA : n_rb;
                     const uint32_t owners = n_sub > 1 ? 3u : (1u << (g & 1));
-                    if (!isA) b_owners |= owners;
+                    if (!isA)
+                        for (int i = 0; i < n_sub; ++i) b_owners |= 1u << ((g + i) & (kG - 1));
                     const int ls = st_pos;
                     if (ld >= p.stages && mma_release) {
                         const int i = slot_item[ls];
@@ -280,10 +333,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         // window rows of item k: R copies of the GWp rows (pass A lanes), or q_rows rows
                         const int qb = k & (p.q_bufs - 1);
                         if (k >= 2) {  // item k - 2 is done with the buffer
-                            const uint32_t prev = (q_owners >> (2 * qb)) & 3u;
-                            for (int grp = 0; grp < 2; ++grp) {
+                            const uint32_t prev = (q_owners >> (kG * qb)) & ((1u << kG) - 1u);
+                            for (int grp = 0; grp < kG; ++grp) {
                                 if (!((prev >> grp) & 1u)) continue;
-                                const int bit = 2 * qb + grp;
+                                const int bit = kG * qb + grp;
                                 if (ok) ok = mbar_wait(&q_empty[bit], (qpar >> bit) & 1u, p.err, kErrScoreQ);
                                 qpar ^= 1u << bit;
                             }
@@ -316,7 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // the pass-B items of this phase read item k - 1's window rows; item k + 1 takes that buffer
                 if (k >= 1 && k + 1 < n_w) {
                     const int qb = (k - 1) & (p.q_bufs - 1);
-                    q_owners = (q_owners & ~(3u << (2 * qb))) | (b_owners << (2 * qb));
+                    q_owners = (q_owners & ~(((1u << kG) - 1u) << (kG * qb))) | (b_owners << (kG * qb));
                 }
             }
             // drain: every load has been consumed (and so has landed) before the CTA leaves
@@ -432,7 +485,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (C > 1) cluster_wait();
     } else {
         // ---------------------------------------------------------------- consumer warpgroups
-        const int grp = tid >> 7;   // 0 or 1: group g takes the items i with i % 2 == g
+        const int grp = tid >> 7;   // group g takes the items i with i % kG == g
         const int L = tid & 127;    // TMEM lane
         const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
         const float cs = p.scale_log2;
@@ -444,6 +497,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         float* pmg = pm + grp * n_rbA * 128;
         float* plg = pl + grp * n_rbA * 128;
         constexpr bool early = kEarly;
+        constexpr int kCW = kG == 4 ? 32 : 64;  // pass-A columns per TMEM load (registers are scarcer at kG = 4)
         int st_pos = 0;  // K stage ring position
         int item = 0;    // accumulator counter
         for (int k = 0; k <= n_w; ++k) {
@@ -461,76 +515,42 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // ------------------------------------ pass A: row statistics
                     const int tok0 = tile * kTileTokens;
                     for (int sub = 0; sub < n_rbA; ++sub, ++item) {
-                        if ((item & 1) != grp) continue;
+                        if ((item & (kG - 1)) != grp) continue;
                         const int buf = item & bmask;
                         if (ok) ok = mbar_wait(&t_full[buf], (item >> bshift) & 1, p.err, kErrScoreTFull);
                         tc_fence_after();
                         float m = pmg[sub * 128 + L];
                         float l = plg[sub * 128 + L];
-                        // online (max, sum of exp2) over this lane's token columns, 64 (or 32) at a time
-                        for (int c = 0; c < cw; c += 64) {
-                            float v[64];
-                            const int width = cw - c >= 64 ? 64 : 32;
-                            if (width == 64) {
-                                tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), v);
-                            } else {
-                                float h[32];
-                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), h);
+                        // online (max, sum of exp2) over this lane's token columns, kCW (or 32) at a time
+                        for (int c = 0; c < cw; c += kCW) {
+                            float v[kCW];
+                            const int width = cw - c >= kCW ? kCW : 32;
+                            if constexpr (kCW == 64) {
+                                if (width == 64) {
+                                    tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), v);
+                                } else {
+                                    float h[32];
+                                    tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), h);
 #pragma unroll
-                                for (int q = 0; q < 32; ++q) {
-                                    v[q] = h[q];
-                                    v[q + 32] = -INFINITY;
+                                    for (int q = 0; q < 32; ++q) {
+                                        v[q] = h[q];
+                                        v[q + 32] = -INFINITY;
+                                    }
                                 }
+                            } else {
+                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), v);
                             }
-                            if (early && c + 64 >= cw) {  // the item's last load has landed
+                            if (early && c + kCW >= cw) {  // the item's last load has landed
                                 tc_fence_before();
                                 mbar_arrive(&t_empty[buf]);
                             }
                             const int nvalid = min(width, p.N - (tok0 + c0 + c));
-                            if (nvalid < 64) {
+                            if (nvalid < kCW) {
 #pragma unroll
-                                for (int q = 0; q < 64; ++q)
+                                for (int q = 0; q < kCW; ++q)
                                     if (q >= nvalid) v[q] = -INFINITY;
                             }
-                            // Once the row has a reference m (the maximum of its first chunk), a chunk is summed
-                            // against it with no chunk maximum: (m, l) stays a valid pair as long as no exp2
-                            // overflows, and a sum above 2^64 (or inf) sends the chunk through the exact path below.
-                            if (m != -INFINITY) {
-                                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-                                for (int q = 0; q < 64; q += 4) {
-                                    s0 += ex2(fmaf(v[q], cs, -m));
-                                    s1 += ex2(fmaf(v[q + 1], cs, -m));
-                                    s2 += ex2(fmaf(v[q + 2], cs, -m));
-                                    s3 += ex2(fmaf(v[q + 3], cs, -m));
-                                }
-                                const float sum = (s0 + s1) + (s2 + s3);
-                                if (sum <= 0x1p64f) {
-                                    l += sum;
-                                    continue;
-                                }
-                            }
-                            float cm0 = v[0], cm1 = v[1], cm2 = v[2], cm3 = v[3];
-#pragma unroll
-                            for (int q = 4; q < 64; q += 4) {
-                                cm0 = fmaxf(cm0, v[q]);
-                                cm1 = fmaxf(cm1, v[q + 1]);
-                                cm2 = fmaxf(cm2, v[q + 2]);
-                                cm3 = fmaxf(cm3, v[q + 3]);
-                            }
-                            const float mn = fmaxf(m, fmaxf(fmaxf(cm0, cm1), fmaxf(cm2, cm3)) * cs);
-                            if (mn != -INFINITY) {
-                                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-                                for (int q = 0; q < 64; q += 4) {
-                                    s0 += ex2(fmaf(v[q], cs, -mn));
-                                    s1 += ex2(fmaf(v[q + 1], cs, -mn));
-                                    s2 += ex2(fmaf(v[q + 2], cs, -mn));
-                                    s3 += ex2(fmaf(v[q + 3], cs, -mn));
-                                }
-                                l = l * ex2(m - mn) + ((s0 + s1) + (s2 + s3));
-                                m = mn;
-                            }
+                            row_stats_chunk<kCW>(v, cs, m, l);
                         }
                         pmg[sub * 128 + L] = m;
                         plg[sub * 128 + L] = l;
@@ -548,14 +568,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     float acc = 0.f;
                     bool mine = false;
                     for (int sub = 0; sub < n_rb; ++sub, ++item) {
-                        if ((item & 1) != grp) continue;
+                        if ((item & (kG - 1)) != grp) continue;
                         mine = true;
                         const int buf = item & bmask;
                         if (ok) ok = mbar_wait(&t_full[buf], (item >> bshift) & 1, p.err, kErrScoreTFull);
                         owned_b = true;
-                        if (sub >= n_rb - 2) {
+                        if (sub >= n_rb - kG) {
                             // item k - 1's last pass-B tile: this group is done with its window rows
-                            if (j == nB - 1 && k + 1 < n_w) mbar_arrive(&q_empty[2 * ((k - 1) & (p.q_bufs - 1)) + grp]);
+                            if (j == nB - 1 && k + 1 < n_w) mbar_arrive(&q_empty[kG * ((k - 1) & (p.q_bufs - 1)) + grp]);
                         }
                         tc_fence_after();
                         if (!kHeadMax) {
@@ -583,6 +603,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 tc_fence_before();
                                 mbar_arrive(&t_empty[buf]);
                             };
+                            if constexpr (kG == 4) {
+                                // one register set (the 608-thread block leaves 96 registers a thread); the other
+                                // groups' warps cover the load latency
+                                for (int ch = 0; ch < nch; ++ch) {
+                                    tmem_ld32_issue(col0 + 32 * ch, ra);
+                                    tmem_wait_ld32(ra);
+                                    if (ch + 1 == nch) release();
+                                    sum32(ra, 32 * ch);
+                                }
+                            } else {
                             tmem_ld32_issue(col0, ra);
                             tmem_wait_ld32(ra);
                             if (nch == 1) release();
@@ -600,29 +630,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     }
                                 }
                             }
+                            }
                         } else {
                         // GQA max-aggregation: the sum runs per query head (W consecutive window rows, whole
                         // heads per row block) and the token keeps the largest head sum
                         float head_sum = 0.f;
                         int head_end = kHeadMax ? sub * NB + head_rows : 0;
-                        for (int c = 0; c < NB; c += 64) {
-                            float v[64];
-                            const int width = NB - c >= 64 ? 64 : 32;
-                            if (width == 64) {
-                                tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), v);
-                            } else {
-                                float h[32];
-                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), h);
+                        for (int c = 0; c < NB; c += kCW) {
+                            float v[kCW];
+                            const int width = NB - c >= kCW ? kCW : 32;
+                            if constexpr (kCW == 64) {
+                                if (width == 64) {
+                                    tmem_ld64(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), v);
+                                } else {
+                                    float h[32];
+                                    tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), h);
 #pragma unroll
-                                for (int q = 0; q < 32; ++q) v[q] = h[q];
+                                    for (int q = 0; q < 32; ++q) v[q] = h[q];
+                                }
+                            } else {
+                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), v);
                             }
-                            if (early && c + 64 >= NB) {  // the item's last load has landed
+                            if (early && c + kCW >= NB) {  // the item's last load has landed
                                 tc_fence_before();
                                 mbar_arrive(&t_empty[buf]);
                             }
                             const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
 #pragma unroll
-                            for (int q = 0; q < 16; ++q) {
+                            for (int q = 0; q < kCW / 4; ++q) {
                                 if (q < width / 4) {
                                     if (sub * NB + c + 4 * q == head_end) {  // the same in every thread
                                         acc = fmaxf(acc, head_sum);
@@ -644,7 +679,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     // no item in the last pass-B tile: the group's last one (if any) was waited for earlier
                     if (!mine && owned_b && j == nB - 1 && k + 1 < n_w)
-                        mbar_arrive(&q_empty[2 * ((k - 1) & (p.q_bufs - 1)) + grp]);
+                        mbar_arrive(&q_empty[kG * ((k - 1) & (p.q_bufs - 1)) + grp]);
                     if (mine && token < p.N) {
                         const int part = n_rb > 1 ? grp : 0;
                         attn_out[(static_cast<int64_t>(part) * p.units + itB.unit) * p.N + token] = acc;
@@ -658,7 +693,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             named_bar(1, kConsumers);
             for (int r = tid; r < GWp; r += kConsumers) {
                 float m = -INFINITY, l = 0.f;
-                for (int g = 0; g < kGroups; ++g) {
+                for (int g = 0; g < kG; ++g) {
                     const float* gm = pm + g * n_rbA * 128;
                     const float* gl = pl + g * n_rbA * 128;
                     if (R > 1) {
@@ -704,13 +739,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages) {
-    return score_layout(q_rows, q_bufs, n_rbA, GWp, cluster, stages, kTileBytes).total + 1024;
+size_t score_attn_smem_bytes(int q_rows, int q_bufs, int n_rbA, int GWp, int cluster, int stages, int groups) {
+    return score_layout(q_rows, q_bufs, n_rbA, GWp, cluster, stages, kTileBytes, groups).total + 1024;
 }
 
 cudaError_t score_attn_set_attributes(size_t smem_bytes, int cluster) {
-    for (auto fn : {score_attn_kernel<false, false>, score_attn_kernel<true, false>, score_attn_kernel<false, true>,
-                    score_attn_kernel<true, true>}) {
+    for (auto fn : {score_attn_kernel<false, false, 2>, score_attn_kernel<true, false, 2>,
+                    score_attn_kernel<false, true, 2>, score_attn_kernel<true, true, 2>,
+                    score_attn_kernel<false, true, 4>, score_attn_kernel<true, true, 4>}) {
         cudaError_t e =
             cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem_bytes));
         if (e == cudaSuccess && cluster > 8) e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
@@ -723,7 +759,7 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
                               size_t smem_bytes, cudaStream_t s) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(p.cluster) * static_cast<unsigned>(p.groups), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.blockDim = dim3(static_cast<unsigned>(score_threads(p.cgroups)), 1, 1);
     cfg.dynamicSmemBytes = smem_bytes;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
@@ -733,11 +769,16 @@ cudaError_t launch_score_attn(const CUtensorMap& kmap, const CUtensorMap& qmap, 
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    // four groups own one buffer each (their next product waits for them: early release); two groups with two
+    // buffers each release after the arithmetic, with one buffer each as soon as the last load has landed
+    if (p.cgroups == 4)
+        return p.head_rows > 0 ? cudaLaunchKernelEx(&cfg, score_attn_kernel<true, true, 4>, kmap, qmap, p)
+                               : cudaLaunchKernelEx(&cfg, score_attn_kernel<false, true, 4>, kmap, qmap, p);
     if (p.nbuf == 2)
-        return p.head_rows > 0 ? cudaLaunchKernelEx(&cfg, score_attn_kernel<true, true>, kmap, qmap, p)
-                               : cudaLaunchKernelEx(&cfg, score_attn_kernel<false, true>, kmap, qmap, p);
-    return p.head_rows > 0 ? cudaLaunchKernelEx(&cfg, score_attn_kernel<true, false>, kmap, qmap, p)
-                           : cudaLaunchKernelEx(&cfg, score_attn_kernel<false, false>, kmap, qmap, p);
+        return p.head_rows > 0 ? cudaLaunchKernelEx(&cfg, score_attn_kernel<true, true, 2>, kmap, qmap, p)
+                               : cudaLaunchKernelEx(&cfg, score_attn_kernel<false, true, 2>, kmap, qmap, p);
+    return p.head_rows > 0 ? cudaLaunchKernelEx(&cfg, score_attn_kernel<true, false, 2>, kmap, qmap, p)
+                           : cudaLaunchKernelEx(&cfg, score_attn_kernel<false, false, 2>, kmap, qmap, p);
 }
 
 }  // namespace vase

@@ -514,7 +514,7 @@ def test_evict_all_with_several_units_per_cta_matches_oracle(K, B, Wn, Hq, Hkv):
 
 def test_sixteen_layers_of_512_window_rows_match_oracle():
     """G*W = 512 window rows (the Qwen3-32B group and window) on sixteen layers in one batched launch, one CTA
-    per unit scoring four 128-row blocks in pass A and two 256-row items in pass B: every layer's workspace
+    per unit whose four consumer groups each score one 128-row block in both passes: every layer's workspace
     slot, kept set and compacted rows are checked on sampled units, and every layer's counters advance."""
     wl = W.shrink(W.WORKLOADS["qwen3_32b_k8192"], budget_k=192, buffer_b=64, batch=2, num_layers=16)
     L = wl.num_layers
@@ -706,9 +706,10 @@ def test_random_reservation_differs_from_value_reservation():
 
 
 # (K, B, W, Hq, Hkv): heads of 16 rows four to a 64-column chunk; 12-row heads that straddle chunks and a
-# padded tail; G*W = 512 in two 256-row blocks (parts combined by max); one query head per KV head
+# padded tail; G*W = 512 in four 128-row blocks (parts combined by max); G*W = 512 with 256-row heads, two
+# 256-row blocks; one query head per KV head
 @pytest.mark.parametrize("K,B,Wn,Hq,Hkv", [(256, 64, 16, 32, 8), (200, 40, 12, 24, 8), (256, 64, 64, 32, 4),
-                                          (192, 64, 32, 8, 8)])
+                                          (512, 128, 256, 16, 8), (192, 64, 32, 8, 8)])
 def test_gqa_max_aggregation_matches_oracle(K, B, Wn, Hq, Hkv):
     wl = W.shrink(SMALL, budget_k=K, buffer_b=B, window=Wn, num_q_heads=Hq, num_kv_heads=Hkv, batch=2,
                   num_layers=2)

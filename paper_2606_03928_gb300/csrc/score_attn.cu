@@ -46,7 +46,11 @@ namespace {
 // buffers) or kG = 4 (one buffer each: at 512 window rows a tile's products are four 128 x 128 items in both
 // passes, and group g always takes row block g).  Plus a TMA warp and two MMA-issue warps (even / odd items).
 constexpr int kMaxGroups = 4;
-__host__ __device__ constexpr int score_threads(int groups) { return 128 * groups + 96; }
+constexpr int kMaxMma = 4;
+// MMA-issue warps: warp x issues the items i with i % mma_warps == x, so each accumulator buffer (item i uses
+// buffer i % nbuf) is only ever issued into by one warp.
+__host__ __device__ constexpr int score_mma_warps(int) { return 2; }
+__host__ __device__ constexpr int score_threads(int groups) { return 128 * groups + 32 + 32 * score_mma_warps(groups); }
 constexpr int kMaxBufs = 4;
 constexpr int kMaxStages = 8;
 constexpr uint32_t kTileBytes = kTileTokens * kRowBytes;  // 32 KB: two 64-column panels of 128 rows
@@ -65,7 +69,7 @@ __host__ __device__ inline ScoreSmem score_layout(int q_rows, int q_bufs, int n_
     L.k_off = o;
     o += static_cast<uint32_t>(stages) * stage_bytes;
     L.bar_off = o;
-    o += 8 * (2 + 2 * kMaxGroups + 3 * stages + 2 * kMaxBufs);
+    o += 8 * (2 + 2 * kMaxGroups + (1 + kMaxMma) * stages + 2 * kMaxBufs);
     o = (o + 15u) & ~15u;
     L.slot_off = o;
     o += 16;
@@ -200,6 +204,7 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
     constexpr int stage_bytes = kTileBytes;
     constexpr int kConsumers = 128 * kG;
     constexpr int kThreads = score_threads(kG);
+    constexpr int kM = score_mma_warps(kG);
     const ScoreSmem Ly = score_layout(p.q_rows, p.q_bufs, p.n_rbA, p.GWp, p.cluster, p.stages, stage_bytes, kG);
 
     uint8_t* q_s = smem + Ly.q_off;
@@ -208,8 +213,8 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
     uint64_t* q_full = bars;                      // [2]
     uint64_t* q_empty = bars + 2;                 // [2][kG]
     uint64_t* k_full = bars + 2 + 2 * kMaxGroups; // [stages]
-    uint64_t* k_empty = k_full + p.stages;        // [stages][group]
-    uint64_t* t_full = k_empty + 2 * p.stages;    // [nbuf]
+    uint64_t* k_empty = k_full + p.stages;        // [stages][kM]
+    uint64_t* t_full = k_empty + kM * p.stages;   // [nbuf]
     uint64_t* t_empty = t_full + kMaxBufs;        // [nbuf]
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Ly.slot_off);
     float* pm = reinterpret_cast<float*>(smem + Ly.pm_off);      // [group][n_rbA][128] running max per lane
@@ -260,8 +265,7 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
         }
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&k_full[s], 1);
-            mbar_init(&k_empty[2 * s], 1);      // MMA warp 0's commit after its last product of the tile
-            mbar_init(&k_empty[2 * s + 1], 1);  // MMA warp 1's
+            for (int x = 0; x < kM; ++x) mbar_init(&k_empty[kM * s + x], 1);  // MMA warp x's commit after its last product of the tile
         }
         for (int b = 0; b < nbuf; ++b) {
             mbar_init(&t_full[b], 1);     // the MMA warp's commit
@@ -274,7 +278,7 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
         pl[i] = 0.f;
     }
     const int tma_warp = kConsumers / 32;
-    const int mma_warp = tma_warp + 1;  // and mma_warp + 1
+    const int mma_warp = tma_warp + 1;  // .. mma_warp + kM - 1
     if (warp == tma_warp) {
         tmem_alloc(tmem_slot, static_cast<uint32_t>(p.tmem_cols));
         tmem_relinquish();
@@ -299,7 +303,6 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
             // read each window-row buffer (bit g = consumer group g, kG bits per buffer), and the parity of the next
             // phase of every per-owner empty barrier.
             uint32_t slot_owners = 0, kpar = 0, q_owners = 0, qpar = 0;
-            int slot_item[kMaxStages];  // item of the tile in each stage (stage release by MMA completion)
             int ld = 0, g = 0, st_pos = 0;
             for (int k = 0; k <= n_w; ++k) {
                 const int nA = k < n_w ? n_my : 0;
@@ -311,24 +314,24 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                     int j;
                     const bool isA = phase_tile(t, nA, nB, lead, j);
                     const int n_sub = isA ? n_rbA : n_rb;
-                    const uint32_t owners = n_sub > 1 ? 3u : (1u << (g & 1));
+                    uint32_t owners = 0;  // MMA warps with an item of the tile
+                    for (int i = 0; i < n_sub; ++i) owners |= 1u << ((g + i) & (kM - 1));
                     if (!isA)
                         for (int i = 0; i < n_sub; ++i) b_owners |= 1u << ((g + i) & (kG - 1));
                     const int ls = st_pos;
                     if (ld >= p.stages && mma_release) {
-                        const int i = slot_item[ls];
+                        const int i = ld - p.stages;  // one item per tile: the item of the stage's last load
                         if (ok) ok = mbar_wait(&t_full[i & bmask], (i >> bshift) & 1, p.err, kErrScoreKEmpty);
                     } else if (ld >= p.stages) {
-                        const uint32_t prev = (slot_owners >> (2 * ls)) & 3u;
-                        for (int grp = 0; grp < 2; ++grp) {
-                            if (!((prev >> grp) & 1u)) continue;
-                            const int bit = 2 * ls + grp;
+                        const uint32_t prev = (slot_owners >> (kM * ls)) & ((1u << kM) - 1u);
+                        for (int x = 0; x < kM; ++x) {
+                            if (!((prev >> x) & 1u)) continue;
+                            const int bit = kM * ls + x;
                             if (ok) ok = mbar_wait(&k_empty[bit], (kpar >> bit) & 1u, p.err, kErrScoreKEmpty);
                             kpar ^= 1u << bit;
                         }
                     }
-                    slot_owners = (slot_owners & ~(3u << (2 * ls))) | (owners << (2 * ls));
-                    slot_item[ls] = g;
+                    slot_owners = (slot_owners & ~(((1u << kM) - 1u) << (kM * ls))) | (owners << (kM * ls));
                     if (isA && j == 0) {
                         // window rows of item k: R copies of the GWp rows (pass A lanes), or q_rows rows
                         const int qb = k & (p.q_bufs - 1);
@@ -375,20 +378,20 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
             // drain: every load has been consumed (and so has landed) before the CTA leaves
             for (int ls = 0; ls < p.stages && ls < ld; ++ls) {
                 if (mma_release) {
-                    const int i = slot_item[ls];
+                    const int i = ls + (ld - 1 - ls) / p.stages * p.stages;  // the stage's last load
                     mbar_wait(&t_full[i & bmask], (i >> bshift) & 1, p.err, kErrScoreDrain);
                     continue;
                 }
-                const uint32_t prev = (slot_owners >> (2 * ls)) & 3u;
-                for (int grp = 0; grp < 2; ++grp) {
-                    const int bit = 2 * ls + grp;
-                    if ((prev >> grp) & 1u) mbar_wait(&k_empty[bit], (kpar >> bit) & 1u, p.err, kErrScoreDrain);
+                const uint32_t prev = (slot_owners >> (kM * ls)) & ((1u << kM) - 1u);
+                for (int x = 0; x < kM; ++x) {
+                    const int bit = kM * ls + x;
+                    if ((prev >> x) & 1u) mbar_wait(&k_empty[bit], (kpar >> bit) & 1u, p.err, kErrScoreDrain);
                 }
             }
         }
         __syncwarp();
         if (C > 1) cluster_wait();
-    } else if (warp == mma_warp || warp == mma_warp + 1) {
+    } else if (warp >= mma_warp && warp < mma_warp + kM) {
         // ---------------------------------------------------------------- MMA warps: one elected lane issues
         // Warp mma_warp + x issues the items i with i % 2 == x (the items of consumer group x).  Each issuing
         // thread runs a serial wait / issue / commit loop whose overhead exceeds the MMAs' own time on the tensor
@@ -424,12 +427,14 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                     const int qb = (isA ? k : k - 1) & (p.q_bufs - 1);
                     if (isA && j == 0 && ok) ok = mbar_wait(&q_full[qb], (k >> 1) & 1, p.err, kErrScoreQ);
                     if (ok) ok = mbar_wait(&k_full[s], s_phase, p.err, kErrScoreKFull);
-                    if (n_sub > 1 || (g & 1) == mine) {  // this warp owns an item of the tile
+                    bool owns = false;
+                    for (int i = 0; i < n_sub; ++i) owns |= ((g + i) & (kM - 1)) == mine;
+                    if (owns) {  // this warp owns an item of the tile
                         const uint64_t qdesc = qdesc0 + ((static_cast<uint32_t>(qb) * q_bytes) >> 4);
                         const uint64_t kt = kdesc + ((static_cast<uint32_t>(s) * stage_bytes) >> 4);
                         for (int sub = 0; sub < n_sub; ++sub) {
                             const int gi = g + sub;
-                            if ((gi & 1) != mine) continue;
+                            if ((gi & (kM - 1)) != mine) continue;
                             const int buf = gi & bmask;
                             const int use = gi >> bshift;
                             if (use > 0 && ok) ok = mbar_wait(&t_empty[buf], (use - 1) & 1, p.err, kErrScoreTEmpty);
@@ -462,8 +467,8 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                         if (!mma_release) {
                             // the stage is free once this warp's products of the tile have read it
                             if (elect_one()) {
-                                if (ok) tc_commit(&k_empty[2 * s + mine]);
-                                else mbar_arrive(&k_empty[2 * s + mine]);
+                                if (ok) tc_commit(&k_empty[kM * s + mine]);
+                                else mbar_arrive(&k_empty[kM * s + mine]);
                             }
                             __syncwarp();
                         }
@@ -476,7 +481,7 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                 }
             }
             // drain: the consumers have read every accumulator of this warp, so its MMAs have completed
-            for (int b = mine; b < nbuf; b += 2) {
+            for (int b = mine; b < nbuf; b += kM) {
                 const int uses = (n_items - b + nbuf - 1) / nbuf;
                 if (uses > 0) mbar_wait(&t_empty[b], (uses - 1) & 1, p.err, kErrScoreDrain);
             }
@@ -498,6 +503,7 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
         float* plg = pl + grp * n_rbA * 128;
         constexpr bool early = kEarly;
         constexpr int kCW = kG == 4 ? 32 : 64;  // pass-A columns per TMEM load (registers are scarcer at kG = 4)
+
         int st_pos = 0;  // K stage ring position
         int item = 0;    // accumulator counter
         for (int k = 0; k <= n_w; ++k) {
@@ -514,10 +520,14 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                 if (isA) {
                     // ------------------------------------ pass A: row statistics
                     const int tok0 = tile * kTileTokens;
-                    for (int sub = 0; sub < n_rbA; ++sub, ++item) {
-                        if ((item & (kG - 1)) != grp) continue;
-                        const int buf = item & bmask;
-                        if (ok) ok = mbar_wait(&t_full[buf], (item >> bshift) & 1, p.err, kErrScoreTFull);
+                    // (kG = 4: a tile's four items are this group's row block and three others')
+                    const int item0 = item;
+                    item += n_rbA;
+                    for (int sub = kG == 4 ? grp : 0; sub < n_rbA; sub += kG == 4 ? kG : 1) {
+                        const int it = item0 + sub;
+                        if (kG != 4 && (it & (kG - 1)) != grp) continue;
+                        const int buf = it & bmask;
+                        if (ok) ok = mbar_wait(&t_full[buf], (it >> bshift) & 1, p.err, kErrScoreTFull);
                         tc_fence_after();
                         float m = pmg[sub * 128 + L];
                         float l = plg[sub * 128 + L];
@@ -567,11 +577,14 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                     const int token = tile * kTileTokens + L;
                     float acc = 0.f;
                     bool mine = false;
-                    for (int sub = 0; sub < n_rb; ++sub, ++item) {
-                        if ((item & (kG - 1)) != grp) continue;
+                    const int item0 = item;
+                    item += n_rb;
+                    for (int sub = kG == 4 ? grp : 0; sub < n_rb; sub += kG == 4 ? kG : 1) {
+                        const int it = item0 + sub;
+                        if (kG != 4 && (it & (kG - 1)) != grp) continue;
                         mine = true;
-                        const int buf = item & bmask;
-                        if (ok) ok = mbar_wait(&t_full[buf], (item >> bshift) & 1, p.err, kErrScoreTFull);
+                        const int buf = it & bmask;
+                        if (ok) ok = mbar_wait(&t_full[buf], (it >> bshift) & 1, p.err, kErrScoreTFull);
                         owned_b = true;
                         if (sub >= n_rb - kG) {
                             // item k - 1's last pass-B tile: this group is done with its window rows

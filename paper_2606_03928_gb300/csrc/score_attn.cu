@@ -105,9 +105,25 @@ __device__ __forceinline__ void merge_ml(float& m, float& l, float m2, float l2)
 // One chunk of a row's online (max, sum of exp2) in pass A.  Once the row has a reference m (the maximum of
 // its first chunk), a chunk is summed against it with no chunk maximum: (m, l) stays a valid pair as long as
 // no exp2 overflows, and a sum above 2^64 (or inf) sends the chunk through the exact path, which raises m.
-template <int CW>
+template <int CW, bool kPacked>
 __device__ __forceinline__ void row_stats_chunk(const float (&v)[CW], float cs, float& m, float& l) {
     if (m != -INFINITY) {
+        if constexpr (kPacked) {  // (the four-group consumers) packed pairs: fewer issued instructions
+            const float2 cs2 = make_float2(cs, cs), nm2 = make_float2(-m, -m);
+            float2 b0 = make_float2(0.f, 0.f), b1 = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int q = 0; q < CW; q += 4) {
+                const float2 x0 = __ffma2_rn(make_float2(v[q], v[q + 1]), cs2, nm2);
+                const float2 x1 = __ffma2_rn(make_float2(v[q + 2], v[q + 3]), cs2, nm2);
+                b0 = __fadd2_rn(b0, make_float2(ex2(x0.x), ex2(x0.y)));
+                b1 = __fadd2_rn(b1, make_float2(ex2(x1.x), ex2(x1.y)));
+            }
+            const float sum = (b0.x + b0.y) + (b1.x + b1.y);
+            if (sum <= 0x1p64f) {
+                l += sum;
+                return;
+            }
+        } else {
         float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
         for (int q = 0; q < CW; q += 4) {
@@ -120,6 +136,7 @@ __device__ __forceinline__ void row_stats_chunk(const float (&v)[CW], float cs, 
         if (sum <= 0x1p64f) {
             l += sum;
             return;
+        }
         }
     }
     float cm0 = v[0], cm1 = v[1], cm2 = v[2], cm3 = v[3];
@@ -548,7 +565,8 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                                     }
                                 }
                             } else {
-                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c), v);
+                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c0 + c),
+                                          *reinterpret_cast<float(*)[32]>(v));
                             }
                             if (early && c + kCW >= cw) {  // the item's last load has landed
                                 tc_fence_before();
@@ -560,7 +578,7 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                                 for (int q = 0; q < kCW; ++q)
                                     if (q >= nvalid) v[q] = -INFINITY;
                             }
-                            row_stats_chunk<kCW>(v, cs, m, l);
+                            row_stats_chunk<kCW, kG == 4>(v, cs, m, l);
                         }
                         pmg[sub * 128 + L] = m;
                         plg[sub * 128 + L] = l;
@@ -599,6 +617,20 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                             uint32_t ra[32], rb[32];
                             auto sum32 = [&](const uint32_t (&r)[32], int c) {
                                 const float4* m4 = reinterpret_cast<const float4*>(rowm + sub * NB + c);
+                                if constexpr (kG == 4) {  // packed pairs (FFMA2, FADD2): fewer issued instructions
+                                    const float2 cs2 = make_float2(cs, cs);
+                                    float2 b0 = make_float2(0.f, 0.f), b1 = make_float2(0.f, 0.f);
+#pragma unroll
+                                    for (int q = 0; q < 8; ++q) {
+                                        const float4 mm = m4[q];
+                                        const float2 x0 = __ffma2_rn(make_float2(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1])), cs2, make_float2(-mm.x, -mm.y));
+                                        const float2 x1 = __ffma2_rn(make_float2(__uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3])), cs2, make_float2(-mm.z, -mm.w));
+                                        b0 = __fadd2_rn(b0, make_float2(ex2(x0.x), ex2(x0.y)));
+                                        b1 = __fadd2_rn(b1, make_float2(ex2(x1.x), ex2(x1.y)));
+                                    }
+                                    acc += (b0.x + b0.y) + (b1.x + b1.y);
+                                    return;
+                                }
                                 float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
                                 for (int q = 0; q < 8; ++q) {
@@ -662,7 +694,8 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                                     for (int q = 0; q < 32; ++q) v[q] = h[q];
                                 }
                             } else {
-                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c), v);
+                                tmem_ld32(taddr + lane_base + static_cast<uint32_t>(buf * bufcols + c),
+                                          *reinterpret_cast<float(*)[32]>(v));
                             }
                             if (early && c + kCW >= NB) {  // the item's last load has landed
                                 tc_fence_before();

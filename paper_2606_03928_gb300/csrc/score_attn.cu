@@ -24,11 +24,13 @@
 //           token, so each thread accumulates sum_r exp2(s_ri - m'_r) of its token
 //           alone, m'_r = m_r + log2(l_r * G*W) folding the softmax denominator
 //           and the 1/(G*W) mean into the exponent.
-// With 512 window rows (G*W > 256) a tile's products fill all 512 TMEM columns in either
-// pass, so four consumer warpgroups each own one 128-column accumulator and one 128-row
-// block of the window, in both passes (pass B writes four partial scores that the
-// selection adds): a group's next product waits only for that group, and sixteen
-// consumer warps cover the TMEM-load and exp2 latencies that eight left exposed.
+// Consumers: four warpgroups, each owning one 128-column TMEM accumulator, wherever the
+// window fits 128 rows (each tile is one item per pass, dealt to the groups in turn) or
+// has 512 rows (a tile's products then fill all 512 TMEM columns in either pass, and each
+// group owns one 128-row block in both passes; pass B writes four partial scores that
+// the selection adds).  A group's next product waits only for that group, and sixteen
+// consumer warps cover the TMEM-load and exp2 latencies that eight left exposed.  In
+// between (256 window rows) two groups share two 256-column accumulators.
 // A single-CTA group that takes several items runs them as phases: phase k
 // interleaves pass B of item k-1 (K re-read from L2, kept there by an
 // evict-last hint on the pass-A read) with pass A of item k (K read from HBM),
@@ -520,6 +522,7 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
         float* plg = pl + grp * n_rbA * 128;
         constexpr bool early = kEarly;
         constexpr int kCW = kG == 4 ? 32 : 64;  // pass-A columns per TMEM load (registers are scarcer at kG = 4)
+        const bool own_block = kG == 4 && n_rbA == kG;  // one row block per group in both passes (n_rb == n_rbA)
 
         int st_pos = 0;  // K stage ring position
         int item = 0;    // accumulator counter
@@ -537,12 +540,12 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                 if (isA) {
                     // ------------------------------------ pass A: row statistics
                     const int tok0 = tile * kTileTokens;
-                    // (kG = 4: a tile's four items are this group's row block and three others')
+                    // (kG = 4 with four row blocks: a tile's four items are this group's row block and three others')
                     const int item0 = item;
                     item += n_rbA;
-                    for (int sub = kG == 4 ? grp : 0; sub < n_rbA; sub += kG == 4 ? kG : 1) {
+                    for (int sub = own_block ? grp : 0; sub < n_rbA; sub += own_block ? kG : 1) {
                         const int it = item0 + sub;
-                        if (kG != 4 && (it & (kG - 1)) != grp) continue;
+                        if (!own_block && (it & (kG - 1)) != grp) continue;
                         const int buf = it & bmask;
                         if (ok) ok = mbar_wait(&t_full[buf], (it >> bshift) & 1, p.err, kErrScoreTFull);
                         tc_fence_after();
@@ -597,9 +600,9 @@ __global__ void __launch_bounds__(score_threads(kG), 1)
                     bool mine = false;
                     const int item0 = item;
                     item += n_rb;
-                    for (int sub = kG == 4 ? grp : 0; sub < n_rb; sub += kG == 4 ? kG : 1) {
+                    for (int sub = own_block ? grp : 0; sub < n_rb; sub += own_block ? kG : 1) {
                         const int it = item0 + sub;
-                        if (kG != 4 && (it & (kG - 1)) != grp) continue;
+                        if (!own_block && (it & (kG - 1)) != grp) continue;
                         mine = true;
                         const int buf = it & bmask;
                         if (ok) ok = mbar_wait(&t_full[buf], (it >> bshift) & 1, p.err, kErrScoreTFull);

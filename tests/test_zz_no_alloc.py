@@ -5,7 +5,7 @@ forbids allocation after start-up) hand the library their caches but no workspac
 vase_evict_static_scratch then keeps its scratch in a static device array.  This
 file checks, through the C ABI, that two such calls in a row give what vase_evict
 gives on an identical copy of the caches -- for both scoring variants, and for a
-window of more than 256 rows, whose score comes in two parts -- and that a layer
+window of more than 256 rows, whose score comes in four parts -- and that a layer
 needing more scratch than the array holds is refused before anything runs.  It is
 collected last on purpose.
 """
@@ -33,8 +33,8 @@ CASES = {
     # (workload, shrink arguments, variant)
     "attnv_k256": ("single_layer_k256", dict(num_layers=2, batch=2), "attnv"),
     "dkv_k256": ("single_layer_k256", dict(num_layers=2, batch=2), "dkv"),
-    # G*W = 8 * 64 = 512 window rows: the window score is written as two parts that the selection adds
-    "attnv_two_parts": ("qwen3_32b_k8192", dict(num_layers=2, batch=1, budget_k=256, buffer_b=64), "attnv"),
+    # G*W = 8 * 64 = 512 window rows: the window score is written as four parts that the selection adds
+    "attnv_four_parts": ("qwen3_32b_k8192", dict(num_layers=2, batch=1, budget_k=256, buffer_b=64), "attnv"),
 }
 
 

@@ -165,6 +165,9 @@ struct SelShared {
     int warp_tot[32];  // one per warp of the block (up to 1024 threads)
     uint32_t bcast[4];
     int first_evicted;  // lowest evicted slot (slots below it keep their place)
+    uint32_t small_x[32];  // radix_top_k: the keys of a boundary digit with at most 32 members ...
+    int small_i[32];       // ... and their slots
+    int n_small;
 };
 
 // Exclusive prefix over threads of `v` in thread order; returns the offset and
@@ -249,15 +252,45 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
                     if (above < static_cast<uint32_t>(remain) && above + cj >= static_cast<uint32_t>(remain)) {
                         sh.bcast[0] = static_cast<uint32_t>(8 * lane + j);
                         sh.bcast[1] = above;
+                        sh.bcast[2] = cj;
                     }
                     above += cj;
                 }
             }
+            if (lane == 0) sh.n_small = 0;
         }
         __syncthreads();
         remain -= static_cast<int>(sh.bcast[1]);
         prefix |= sh.bcast[0] << shift;
         mask |= 0xFFu << shift;
+        if (shift > 0 && sh.bcast[2] <= 32u) {
+            // At most 32 keys share the digits so far: every key above them is taken, and they are ranked among
+            // themselves by one warp (larger key, or equal key at a lower slot) instead of the remaining passes.
+            for (int i = tid; i < n; i += kT) {
+                const uint32_t x = ord[i];
+                if ((x & mask) == prefix) {
+                    const int j = atomicAdd(&sh.n_small, 1);
+                    sh.small_x[j] = x;
+                    sh.small_i[j] = i;
+                } else if ((x & mask) > prefix) {
+                    flags[i] |= flag;
+                }
+            }
+            __syncthreads();
+            const int ns = sh.n_small;
+            if (tid < ns) {
+                const uint32_t x = sh.small_x[tid];
+                const int xi = sh.small_i[tid];
+                int rank = 0;
+                for (int j = 0; j < ns; ++j) {
+                    const uint32_t y = sh.small_x[j];
+                    rank += (y > x) || (y == x && sh.small_i[j] < xi);
+                }
+                if (rank < remain) flags[xi] |= flag;
+            }
+            __syncthreads();
+            return;
+        }
     }
     const uint32_t thr = prefix;
     int eq = 0;
@@ -778,6 +811,9 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
         }
         return;
     }
+#ifdef VASE_PROBE_NOGATHER
+    return;
+#endif
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     const int warp = tid >> 5;
     if (warp == 0 || (warp == 1 && p.vc)) {  // no V rows here with the compressed value store

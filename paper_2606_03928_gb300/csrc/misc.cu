@@ -811,9 +811,6 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
         }
         return;
     }
-#ifdef VASE_PROBE_NOGATHER
-    return;
-#endif
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     const int warp = tid >> 5;
     if (warp == 0 || (warp == 1 && p.vc)) {  // no V rows here with the compressed value store

@@ -731,14 +731,7 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
     for (int i = seg_lo; i < seg_hi; ++i) {
         const bool keep = (i >= K) || flags[i];
         if (keep) {
-            if (dst < K) {
-                src_out[static_cast<int64_t>(unit) * K + dst] = i;
-                src_s[dst] = i;
-                pos[base + dst] = pos_s[i];
-                // compressed value store: new slot dst keeps a reserved (bf16) value if it is in R_B or R_V
-                if (resv_out)
-                    resv_out[static_cast<int64_t>(unit) * store_resv_stride(K) + dst] = (i >= K || (flags[i] & kFlagValue)) ? 1 : 0;
-            }
+            if (dst < K) src_s[dst] = i;
             ++dst;
         } else if (i < first_ev) {
             first_ev = i;
@@ -747,24 +740,30 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
         if (key_dbg && i >= K) key_dbg[base + i] = -1.f;
     }
     if (first_ev < K) atomicMin(&sh.first_evicted, first_ev);
+    if (total != K) {  // cannot happen for a consistent state; the rows stay where they are
+        if (tid == 0) record_error(p.err, kErrSelectCount);
+        return;
+    }
+    __syncthreads();  // the kept list is complete
+    // The kept list, positions and value magnitudes of the new slots, written slot by slot (coalesced) from the
+    // old slots' copies in shared memory; the compressed value store also gets each new slot's reserved flag.
+    int32_t* const src_u = src_out + static_cast<int64_t>(unit) * K;
+    for (int j = tid; j < K; j += kT) {
+        const int i = src_s[j];
+        src_u[j] = i;
+        pos[base + j] = pos_s[i];
+        if (staged) vmag[base + j] = vm_s[i];
+        // compressed value store: new slot j keeps a reserved (bf16) value if it is in R_B or R_V
+        if (resv_out)
+            resv_out[static_cast<int64_t>(unit) * store_resv_stride(K) + j] = (i >= K || (flags[i] & kFlagValue)) ? 1 : 0;
+    }
     for (int i = K + tid; i < N; i += kT) pos[base + i] = -1;
-    // value magnitudes move with their rows too
-    if (!staged) {
+    if (!staged) {  // value magnitudes through the same shared-memory array as the positions
         __syncthreads();
         vm_s = a_s;
         for (int i = tid; i < N; i += kT) vm_s[i] = vmag[base + i];
         __syncthreads();
-    }
-    dst = dst0;
-    for (int i = seg_lo; i < seg_hi; ++i) {
-        if ((i >= K) || flags[i]) {
-            if (dst < K) vmag[base + dst] = vm_s[i];
-            ++dst;
-        }
-    }
-    if (total != K) {  // cannot happen for a consistent state; the rows stay where they are
-        if (tid == 0) record_error(p.err, kErrSelectCount);
-        return;
+        for (int j = tid; j < K; j += kT) vmag[base + j] = vm_s[src_s[j]];
     }
     __syncthreads();  // the kept list and the lowest evicted slot are complete; the selection data is dead
 

@@ -634,14 +634,17 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
         }
         cp_async_words(vm_s, vmag + base, N);
         cp_async_words(pos_s, pos + base, N);
+    } else if (!staged) {
+        // unstaged: the first score part into a_s and the value magnitudes (as raw words) into ord, all requested
+        // at once; ord turns into the reservation keys in place below
+        if (p.variant == 0 && !a_ready) cp_async_words(a_s, attn + base, N);
+        if (p.variant == 0 && !rv_ready) cp_async_words(ord, vmag + base, K);
     }
     if (!rv_ready)
         for (int i = tid; i < N; i += kT) flags[i] = 0;
     if (tid == 0) sh.first_evicted = K;
-    if (staged) {
-        cp_async_wait_all();
-        __syncthreads();
-    }
+    cp_async_wait_all();
+    __syncthreads();
     if (p.variant == 0) {
         if (staged) {
             if (p.n_parts > 1) {
@@ -652,13 +655,16 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
                     a_s[i] = a;
                 }
             }
-        } else if (!a_ready) {
+        } else if (!a_ready && p.n_parts > 1) {
             for (int i = tid; i < N; i += kT) {
-                float a = attn[base + i];
-                for (int part = 1; part < p.n_parts; ++part) {
-                    const float b = attn[(static_cast<int64_t>(part) * p.units + unit) * N + i];
-                    a = p.gqa_max ? fmaxf(a, b) : a + b;
-                }
+                float b[3];  // the other parts (at most four in all), loaded before any is used
+#pragma unroll
+                for (int part = 1; part < 4; ++part)
+                    b[part - 1] = part < p.n_parts ? attn[(static_cast<int64_t>(part) * p.units + unit) * N + i] : 0.f;
+                float a = a_s[i];
+#pragma unroll
+                for (int part = 1; part < 4; ++part)
+                    if (part < p.n_parts) a = p.gqa_max ? fmaxf(a, b[part - 1]) : a + b[part - 1];
                 a_s[i] = a;
             }
         }
@@ -668,7 +674,7 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
         }
         if (!rv_ready) {  // (otherwise select_reserve_team has set the R_V flags)
             for (int i = tid; i < K; i += kT) {
-                const float vm = staged ? vm_s[i] : vmag[base + i];
+                const float vm = staged ? vm_s[i] : __uint_as_float(ord[i]);
                 const int32_t pi = p.reserve_random ? (staged ? pos_s[i] : pos[base + i]) : 0;
                 ord[i] = reserve_ord(p, layer, rnd, unit, vm, pi);
                 if (vscore_dbg) vscore_dbg[base + i] = vm;
@@ -718,7 +724,9 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
     // positions move with the kept rows (unstaged: copy the old ones into shared memory, a_s is free now)
     if (!staged) {
         pos_s = reinterpret_cast<int32_t*>(a_s);
-        for (int i = tid; i < N; i += kT) pos_s[i] = pos[base + i];
+        __syncthreads();  // every read of the scores in a_s is done
+        cp_async_words(pos_s, pos + base, N);
+        cp_async_wait_all();  // (block_exclusive_scan below is the barrier)
     }
     // keep = R_B u R_V u sampled; ascending list of kept slots (also kept in shared memory for the gather)
     int32_t* src_s = reinterpret_cast<int32_t*>(smem_raw + Ly.src_off);
@@ -761,7 +769,8 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
     if (!staged) {  // value magnitudes through the same shared-memory array as the positions
         __syncthreads();
         vm_s = a_s;
-        for (int i = tid; i < N; i += kT) vm_s[i] = vmag[base + i];
+        cp_async_words(vm_s, vmag + base, N);
+        cp_async_wait_all();
         __syncthreads();
         for (int j = tid; j < K; j += kT) vmag[base + j] = vm_s[src_s[j]];
     }

@@ -635,11 +635,14 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
         cp_async_words(vm_s, vmag + base, N);
         cp_async_words(pos_s, pos + base, N);
     } else if (!staged) {
-        // unstaged: the first score part into a_s and the value magnitudes (as raw words) into ord, all requested
-        // at once; ord turns into the reservation keys in place below
+        // unstaged: the first score part into a_s, the value magnitudes (as raw words) into ord and the candidates'
+        // positions into the kept list's region (free until the kept list), all requested at once; ord turns into
+        // the reservation keys in place below
         if (p.variant == 0 && !a_ready) cp_async_words(a_s, attn + base, N);
         if (p.variant == 0 && !rv_ready) cp_async_words(ord, vmag + base, K);
+        if (p.variant == 0 && (p.stochastic || p.reserve_random)) cp_async_words(smem_raw + Ly.src_off, pos + base, K);
     }
+    const int32_t* const pos_k = staged ? pos_s : reinterpret_cast<const int32_t*>(smem_raw + Ly.src_off);
     if (!rv_ready)
         for (int i = tid; i < N; i += kT) flags[i] = 0;
     if (tid == 0) sh.first_evicted = K;
@@ -675,7 +678,7 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
         if (!rv_ready) {  // (otherwise select_reserve_team has set the R_V flags)
             for (int i = tid; i < K; i += kT) {
                 const float vm = staged ? vm_s[i] : __uint_as_float(ord[i]);
-                const int32_t pi = p.reserve_random ? (staged ? pos_s[i] : pos[base + i]) : 0;
+                const int32_t pi = p.reserve_random ? pos_k[i] : 0;
                 ord[i] = reserve_ord(p, layer, rnd, unit, vm, pi);
                 if (vscore_dbg) vscore_dbg[base + i] = vm;
             }
@@ -699,7 +702,7 @@ __device__ __forceinline__ void select_unit(const SelectParams& p, int unit, int
             } else {
                 key = pooled;
                 if (p.stochastic) {
-                    const int32_t pi = staged ? pos_s[i] : pos[base + i];
+                    const int32_t pi = pos_k[i];
                     const Philox4 w = philox4x32_10(
                         Philox4{static_cast<uint32_t>(pi), static_cast<uint32_t>(rnd), c2,
                                 static_cast<uint32_t>(unit)},

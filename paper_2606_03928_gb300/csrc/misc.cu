@@ -165,8 +165,8 @@ struct SelShared {
     int warp_tot[32];  // one per warp of the block (up to 1024 threads)
     uint32_t bcast[4];
     int first_evicted;  // lowest evicted slot (slots below it keep their place)
-    uint32_t small_x[32];  // radix_top_k: the keys of a boundary digit with at most 32 members ...
-    int small_i[32];       // ... and their slots
+    uint32_t small_x[64];  // radix_top_k: the keys of a boundary digit with at most 64 members ...
+    int small_i[64];       // ... and their slots
     int n_small;
 };
 
@@ -263,9 +263,9 @@ __device__ void radix_top_k(const uint32_t* ord, int n, int k, uint8_t* flags, u
         remain -= static_cast<int>(sh.bcast[1]);
         prefix |= sh.bcast[0] << shift;
         mask |= 0xFFu << shift;
-        if (shift > 0 && sh.bcast[2] <= 32u) {
-            // At most 32 keys share the digits so far: every key above them is taken, and they are ranked among
-            // themselves by one warp (larger key, or equal key at a lower slot) instead of the remaining passes.
+        if (shift > 0 && sh.bcast[2] <= 64u) {
+            // At most 64 keys share the digits so far: every key above them is taken, and they are ranked among
+            // themselves by two warps (larger key, or equal key at a lower slot) instead of the remaining passes.
             for (int i = tid; i < n; i += kT) {
                 const uint32_t x = ord[i];
                 if ((x & mask) == prefix) {

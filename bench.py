@@ -4,17 +4,18 @@
 One step = one eviction round of every layer of the workload: for each layer
 the B new decode tokens of the stream are appended (window ring + cache) and
 the layer is evicted (score, value magnitude, selection, compaction), all
-through the C ABI.  The default workload is the Qwen3-1.7B attention geometry
-(28 layers, 16/8 heads, d = 128, batch 8, K = 2048, B = 128, W = 32, an
-8192-token seeded synthetic decode stream: 48 rounds per layer, replayed
-cyclically when more steps are asked for).  Every step touches about 3.9 GB
-of cache, far more than the 129 MB L2, so no L2 flush is needed between steps.
+through the C ABI.  The default workload is the largest configuration, the
+Qwen3-32B attention geometry (64 layers, 64/8 heads, d = 128, batch 16,
+K = 8192, B = 256, W = 64; seeded synthetic decode tokens, a few distinct
+rounds replayed cyclically); the same run also measures the other
+configurations (the `configs` records).  Every step touches about 71 GB of
+cache, far more than the 129 MB L2, so no L2 flush is needed between steps.
 
 Metric: eviction-step KV token-heads per second = (layers * batch * Hkv * (K+B))
 per step / step time.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-  python bench.py --workload qwen3_8b_k4096|qwen3_32b_k8192 [--layers L] [--variant dkv]
+  python bench.py --workload qwen3_1p7b_k2048|qwen3_8b_k4096|sweep:K:B:batch:rate [--layers L] [--variant dkv]
   python bench.py --sweep [--sweep-full]     # the Qwen3-8B-geometry grid over K, B, batch, outlier rate
   python bench.py --decode [--mixed-bits b]  # decode attention over the kept cache
 
